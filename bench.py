@@ -1,0 +1,438 @@
+#!/usr/bin/env python
+"""Verify-step benchmark of the TSS target-side verification path on GB300.
+
+Default workload: Llama-2-7B-shaped decoder (32 layers, d 4096, 32 x 128 heads, MLP 11008,
+vocab 32000), random-init bf16 weights, batch 1, context 1024 (synthetic KV), chain draft k = 5
+(uniform random ids; 20% of steps start with a greedy prefix of length 0-5), skip set
+{20, 24, 27, 30}, greedy acceptance.  One step = one tss_verify (controller, embedding, every
+active layer, LM head + argmax, acceptance, KV compaction).
+
+Prints one JSON line (rank 0).  `value` is verified tokens/s (rows scored per second, B*(k+1)
+per step) with inputs resident in HBM; `e2e` is the same metric through the C ABI with host
+buffers (token upload and result read-back inside the timed region, one synchronisation per
+step).  `--impl reference` times the CPU oracle on a bounded sample of the same workload.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "7B verify-step latency (us) & tokens/s at k=5, 4 skipped layers; % HBM roofline"
+NOMINAL_HBM_GBS = 8000.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", default="tss", choices=["tss", "reference"])
+    p.add_argument("--workload", default="7b_chain", choices=["7b_chain", "7b_dense", "7b_tree", "13b_mixed", "7b_long", "tiny"])
+    p.add_argument("--skip", type=int, default=None, help="7b_long: number of skipped layers (sweep point)")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-profile", action="store_true")
+    return p.parse_args()
+
+
+def make_workload(name, skip=None):
+    from paper_2609_26100_gb300 import synth
+    if name == "7b_chain":
+        return synth.workload_7b_chain()
+    if name == "7b_dense":
+        return synth.workload_7b_chain(mask_layers=())
+    if name == "7b_tree":
+        return synth.workload_7b_tree()
+    if name == "13b_mixed":
+        return synth.workload_13b_mixed()
+    if name == "7b_long":
+        return synth.workload_7b_long(n_skip=8 if skip is None else skip)
+    if name == "tiny":
+        return synth.config_chain(synth.TINY, "tiny_bench", 1, [128], 4, {0: synth.mask_of([2])}, [0])
+    raise ValueError(name)
+
+
+def workload_config(w, args):
+    a = w.arch
+    ks = sorted({len(r.parents) - 1 for r in w.requests})
+    return {
+        "workload": f"{w.name}: L{a.n_layers} d{a.d_model} H{a.n_heads}x{a.head_dim} F{a.d_mlp} V{a.vocab}, "
+                    f"B={len(w.requests)}, ctx={sorted({r.ctx_len for r in w.requests})[:4]}, "
+                    f"rows={w.n_rows}, k={ks}, active_union={len(w.active_union())}/{a.n_layers}, mode={w.mode}",
+        "batch": len(w.requests), "rows_per_step": w.n_rows,
+        "skip_sets": {str(d): [l for l in range(64) if (m >> l) & 1] for d, m in w.phi.items()},
+        "parallelism": f"replicas x{args.gpus}" if args.gpus > 1 else "single GPU",
+        "l2": "inputs larger than L2: every step streams the active-layer weights (GBs) from HBM",
+    }
+
+
+def measured_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of this GPU's clocks and throttle reasons during the timed region."""
+    FIELDS = ("pci.bus_id,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, bus_id):
+        self.bus_id = bus_id.lower()
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+        return False
+
+    def summary(self):
+        rows = []
+        for ln in (self.out or "").splitlines():
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            if self.bus_id and not f[0].lower().endswith(self.bus_id[-12:]):
+                continue
+            rows.append(f)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": float(rows[0][2]) if rows[0][2].replace(".", "").isdigit() else None,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max(float(r[3]) for r in rows if r[3].replace(".", "").isdigit())}
+
+
+def kernel_bytes(w):
+    """Algorithmic bytes per launch of each kernel kind (weights + activations in and out + KV)."""
+    a = w.arch
+    d, f, V, M = a.d_model, a.d_mlp, a.vocab, w.n_rows
+    kv_read = sum(r.ctx_len for r in w.requests) * a.kv_bytes_per_token  # per layer, all requests
+    return {
+        "qkv_gemm": 3 * d * d * 2 + M * d * 2 + M * d * 2 + M * 2 * d * 2,
+        "attention": kv_read + M * d * 2 * 2 + M * 2 * d * 2,
+        "o_gemm": d * d * 2 + M * d * 2 + M * d * 4 * 2,
+        "gate_up_gemm": 2 * f * d * 2 + M * d * 2 + M * f * 2,
+        "down_gemm": d * f * 2 + M * f * 2 + M * d * 4 * 2,
+        "lm_head_gemm": V * d * 2 + M * d * 2 + M * V * 4,
+    }
+
+
+# ----------------------------------------------------------------------------------------------
+# CPU oracle sample (cpu_baseline leg and --impl reference)
+# ----------------------------------------------------------------------------------------------
+class OracleSample:
+    """The oracle on a bounded sample of the workload: embedding + LM head with every layer
+    skipped (t0), and with one sampled active layer (t1); a full step is estimated as
+    t0 + n_active * (t1 - t0)."""
+
+    def __init__(self, w, device):
+        import numpy as np
+        import torch
+        from paper_2609_26100_gb300 import synth
+        self.w = w
+        a = w.arch
+        self.union = w.active_union()
+        self.sample_layers = self.union[:2]
+        gen = synth.make_weights(a, w.seed, device=device, layers=self.sample_layers)
+        f32 = lambda t: t.float().cpu().numpy()  # noqa: E731
+        self.weights = {"embed": f32(gen["embed"]), "lm_head": f32(gen["lm_head"]), "final_norm": f32(gen["final_norm"]),
+                        "layers": [None if lw is None else {k: f32(v) for k, v in lw.items()} for lw in gen["layers"]]}
+        del gen
+        r = w.requests[0]
+        self.kv = [None] * a.n_layers
+        for l in self.sample_layers:
+            blk = synth.kv_block(a, l, 0, r.ctx_len, w.seed, device=device).float().cpu().numpy()
+            self.kv[l] = (blk[0], blk[1])
+        if device != "cpu":
+            torch.cuda.empty_cache()
+        self.np = np
+
+    def _run(self, active):
+        from oracle import tss_oracle as O
+        a, r = self.w.arch, self.w.requests[0]
+        skip = frozenset(l for l in range(a.n_layers) if l not in active)
+        t = time.perf_counter()
+        O.verify_request(self.weights, a, skip, r.tokens, r.parents, r.ctx_len, self.kv)
+        return time.perf_counter() - t
+
+    def step_seconds(self, i=0):
+        """Estimated oracle seconds for one full step of request 0 (median-free single sample)."""
+        if not hasattr(self, "t0"):
+            self.t0 = min(self._run([]) for _ in range(2))
+        t1 = self._run([self.sample_layers[i % len(self.sample_layers)]])
+        n_act = sum(1 for l in range(self.w.arch.n_layers) if not (self.w.skip_mask(0) >> l) & 1)
+        per_req = self.t0 + n_act * max(t1 - self.t0, 0.0)
+        return per_req * len(self.w.requests)
+
+    def describe(self, n):
+        return (f"oracle (NumPy fp32) verify of request 0 with all layers skipped and with 1 sampled active layer, "
+                f"extrapolated to its active layers and scaled by the batch; {n} sample(s)")
+
+
+def cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count()
+
+
+# ----------------------------------------------------------------------------------------------
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import torch
+    w = make_workload(args.workload, args.skip)
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    s = OracleSample(w, dev)
+    for i in range(args.warmup):
+        s.step_seconds(i)
+    times = [s.step_seconds(i) for i in range(args.steps)]
+    sec = statistics.median(times)
+    value = w.n_rows / sec
+    cb = {"value": value, "unit": "tokens/s", "cores": cores(), "kind": "oracle", "sample": s.describe(args.steps)}
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": workload_config(w, args), "cpu_baseline": cb,
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))
+
+
+def run_tss(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_26100_gb300 import build as _build
+    from paper_2609_26100_gb300 import native, synth
+    from paper_2609_26100_gb300.runner import TssRunner
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if rank == 0 or world == 1:
+        _build.build()
+    if world > 1:
+        dist.barrier()
+    _build.build()  # no-op when up to date
+    w = make_workload(args.workload, args.skip)
+    a = w.arch
+    union = w.active_union()
+    max_ctx = max(r.ctx_len for r in w.requests)
+    max_n = max(len(r.parents) for r in w.requests)
+
+    # cpu baseline sample needs host copies of a few layers; take them before the GPU run
+    sample = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        sample = OracleSample(w, "cuda")
+
+    weights = synth.make_weights(a, w.seed, device="cuda", layers=union)
+    for l in range(a.n_layers):  # layers no request runs still need (unused) tensors for the ABI
+        if weights["layers"][l] is None:
+            weights["layers"][l] = {k: torch.zeros(s, dtype=torch.bfloat16, device="cuda")
+                                    for k, s in synth.layer_shapes(a).items()}
+    run = TssRunner(a, weights, n_slots=len(w.requests), kv_cap=max_ctx + max_n + 8, max_batch=len(w.requests),
+                    max_rows=max(16, w.n_rows), max_nodes=max_n, kv_layers=union)
+    del weights
+    torch.cuda.empty_cache()
+    run.set_phi(w.phi)
+    run.fill_synthetic(w)
+    stream = torch.cuda.current_stream()
+
+    # Per-step drafts.  7B chain: 20% of steps carry a greedy prefix of length 0-5, built from the
+    # model's own greedy continuation (obtained through the library during setup).
+    sample_mode = w.mode == "sample"
+    probs = None
+    if sample_mode:
+        probs = torch.cat([r.draft_probs for r in w.requests], 0).cuda()
+    n_var = 10
+    token_sets = []
+    for v in range(n_var):
+        toks = []
+        for b, r in enumerate(w.requests):
+            if sample_mode or v == 0:
+                toks.extend(r.tokens)
+            else:
+                toks.extend(synth.draft_tokens(r.parents, a.vocab, w.seed + v, f"bench.{v}.{b}"))
+        token_sets.append(toks)
+    if w.name == "7b_chain":
+        r = w.requests[0]
+        greedy = []
+        res = run.alloc_results(1, w.n_rows, logits=False)
+        toks = list(token_sets[0])
+        for i in range(len(r.parents) - 1):
+            b = run.batch([synth.Request(r.ctx_len, r.parents, toks, r.domain)])
+            run.verify(b, res)
+            torch.cuda.synchronize()
+            g = int(res["bonus"][0])
+            greedy.append(g)
+            toks[i + 1] = g
+        sel = synth.uniform_ints(n_var, 5, w.seed, "bench.prefix").tolist()
+        for v in range(n_var):
+            if v % 5 == 4:  # one step in five
+                lp = sel[v] + 1
+                token_sets[v][1:1 + lp] = greedy[:lp]
+    batches = []
+    for v in range(n_var):
+        tt = torch.tensor(token_sets[v], dtype=torch.int32, device="cuda")
+        batches.append(run.batch(w.requests, tokens=tt,
+                                 mode=native.TSS_MODE_SAMPLE if sample_mode else native.TSS_MODE_GREEDY,
+                                 temperature=w.temperature, draft_probs=probs, philox_seed=w.seed, philox_offset=v))
+    res = run.alloc_results(len(w.requests), w.n_rows, logits=False)
+    for i in range(args.warmup):
+        run.verify(batches[i % n_var], res)
+    if run.sync_status() != native.TSS_OK:
+        raise RuntimeError("device status error during warm-up")
+
+    # ---------------- timed region (device-resident inputs) ----------------
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    accepts = []
+    bus = torch.cuda.get_device_properties(local).pci_bus_id if hasattr(torch.cuda.get_device_properties(local), "pci_bus_id") else ""
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(str(bus)) as clk:
+        ev[0].record(stream)
+        for i in range(args.steps):
+            run.verify(batches[i % n_var], res)
+            ev[i + 1].record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
+    total_ms = ev[0].elapsed_time(ev[-1])
+    status = run.sync_status()
+    if status != native.TSS_OK:
+        raise RuntimeError(f"device status {status} in the timed region")
+    accepts.append(res["accept_len"].float().mean().item())
+    if world > 1:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms = total_ms / args.steps
+    value = world * w.n_rows * args.steps / (total_ms / 1e3)
+
+    # ---------------- e2e: host buffers through the C ABI, one sync per step ----------------
+    e2e = None
+    if not args.no_e2e and not sample_mode:
+        hres = run.alloc_results(len(w.requests), w.n_rows, logits=False, host=True)
+        htoks = [torch.tensor(token_sets[v], dtype=torch.int32).pin_memory() for v in range(n_var)]
+        hb = [run.batch(w.requests, tokens=htoks[v], io_host=True) for v in range(n_var)]
+        for i in range(3):
+            run.verify(hb[i % n_var], hres)
+        torch.cuda.synchronize()
+        n_e2e = max(10, min(args.steps, 100))
+        acc_sum = 0
+        t0 = time.perf_counter()
+        for i in range(n_e2e):
+            run.verify(hb[i % n_var], hres)
+            stream.synchronize()
+            acc_sum += int(hres["accept_len"].sum())
+        e2e_s = time.perf_counter() - t0
+        e2e = {"value": world * w.n_rows * n_e2e / e2e_s, "unit": "tokens/s",
+               "h2d_bytes_per_step": 4 * w.n_rows,
+               "d2h_bytes_per_step": 4 * (3 * len(w.requests) + hres["path"].numel()),
+               "ms_per_step": e2e_s / n_e2e * 1e3, "steps": n_e2e}
+
+    # ---------------- per-kernel device times (CUDA events around every launch) ----------------
+    roofline = None
+    kernels = None
+    peak, peak_kind = measured_peak()
+    if not args.no_profile:
+        times = native.TssKernelTimes()
+        n_prof = max(5, min(args.steps, 20))
+        for i in range(n_prof):
+            run.v.verify_profiled(batches[i % n_var], run.kv_struct, res["_struct"], times, stream.cuda_stream)
+        kb = kernel_bytes(w)
+        kernels = {}
+        for k, name in enumerate(native.KERNEL_KINDS):
+            if times.launches[k]:
+                avg = times.ms[k] / times.launches[k]
+                kernels[name] = {"launches_per_step": times.launches[k] / n_prof, "ms_per_step": times.ms[k] / n_prof,
+                                 "avg_launch_us": avg * 1e3}
+                if name in kb:
+                    kernels[name]["gbs"] = kb[name] / (avg * 1e-3) / 1e9
+        tot = sum(v["ms_per_step"] for v in kernels.values())
+        for v in kernels.values():
+            v["share"] = v["ms_per_step"] / tot
+        dom = max((n for n in kernels if n in kb), key=lambda n: kernels[n]["ms_per_step"])
+        ach = kernels[dom]["gbs"]
+        roofline = {"kernel": dom, "bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
+                    "frac": ach / peak, "peak_source": f"{peak_kind} copy bandwidth",
+                    "bytes_per_launch": kb[dom], "traffic": None}
+
+    ab = synth.algorithmic_bytes(w)
+    step_gbs = ab["total"] / (ms * 1e-3) / 1e9
+    launches_per_step = 6 + 7 * len(union)
+    out = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights, synthetic KV)",
+        "config": workload_config(w, args),
+        "latency_us": {"mean": ms * 1e3, "median": statistics.median(step_ms) * 1e3,
+                       "p10": sorted(step_ms)[len(step_ms) // 10] * 1e3, "p90": sorted(step_ms)[(9 * len(step_ms)) // 10] * 1e3},
+        "committed_tokens_per_s": None,
+        "step_roofline": {"bytes_per_step": ab["total"], "weights": ab["weights"], "kv_read": ab["kv_read"],
+                          "achieved_gbs": step_gbs, "frac_of_measured": step_gbs / peak,
+                          "frac_of_nominal_8TBs": step_gbs / NOMINAL_HBM_GBS},
+        "roofline": roofline, "kernels": kernels, "e2e": e2e,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk.summary(),
+    }
+    mean_acc = statistics.mean(accepts) if accepts else 0.0
+    out["committed_tokens_per_s"] = world * len(w.requests) * (1 + mean_acc) * args.steps / (total_ms / 1e3)
+    if sample is not None:
+        n_s = 3
+        secs = [sample.step_seconds(i) for i in range(n_s)]
+        sec = statistics.median(secs)
+        out["cpu_baseline"] = {"value": w.n_rows / sec, "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+                               "sample": sample.describe(n_s), "seconds_per_step": sec}
+    run.close()
+    if rank == 0:
+        print(json.dumps(out))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_tss(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,224 @@
+/*
+ * tss.h -- C ABI of the GB300 (sm_103a) TSS target-side verification library (libtss.so).
+ *
+ * The library runs one verification step of speculative decoding on the *target* model, as the
+ * paper "TSS: Target-Side Sparsification for Speculative Decoding in Domain-Specific Large
+ * Language Models" states the problem:
+ *
+ *   - Sec. "Problem Formulation": the target has L blocks; a skip configuration S_d is a subset of
+ *     them, and S_d = {} is the dense verifier.  The draft proposes candidate tokens that the
+ *     target scores in parallel.
+ *   - Sec. "Domain-to-Configuration Mapping": Phi maps each supported domain to its skip set;
+ *     one complete target model serves every domain's sparse path.
+ *   - Sec. "Domain-Aware Skip Controller", first equation: S(x) = Phi(d(x)) for a supported
+ *     domain and the empty set otherwise, fixed for the whole request; second equation:
+ *     h_{l+1} = f_l(h_l) for l not in S(x), h_{l+1} = h_l for l in S(x).
+ *   - Sec. "Models and speculative decoding methods": the accept/reject rule is the base
+ *     method's, unchanged (greedy at temperature 0; speculative sampling otherwise).
+ *
+ * f_l is a LLaMA block (App. "Models"): RMSNorm, rotary multi-head attention (rotate-half
+ * pairing), SwiGLU MLP.  Weights are bf16; residual and accumulation are fp32.
+ *
+ * Conventions for every entry point:
+ *   - Pointers are plain addresses.  "device" means CUDA device memory of the current device,
+ *     "host" means host memory (pinned memory recommended where copies are asynchronous).
+ *   - A stream is a cudaStream_t passed as void* (NULL = the legacy default stream).
+ *   - Every call returns tss_status.  Errors the host can detect are reported before any work is
+ *     enqueued and leave all caller buffers untouched; tss_last_error() then gives a message.
+ *   - Kernels never trap.  A check that fails on the device records a code in a device status
+ *     word and the kernel continues with a safe value; the code is reported by
+ *     tss_sync_status() (TSS_ERR_DEVICE_CHECK or TSS_ERR_TIMEOUT).
+ *   - Layer indices are 0-based: bit l of a skip mask names layer l.
+ */
+#ifndef TSS_H
+#define TSS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int tss_status;
+#define TSS_OK 0
+#define TSS_ERR_INVALID_ARG 1     /* an argument failed host-side validation */
+#define TSS_ERR_OUT_OF_MEMORY 2   /* a device allocation at tss_create failed */
+#define TSS_ERR_KV_CAPACITY 3     /* ctx_len + n_nodes exceeds the KV cache capacity */
+#define TSS_ERR_CUDA 4            /* a CUDA runtime/driver call failed */
+#define TSS_ERR_UNSUPPORTED_ARCH 5 /* model shape or GPU (not sm_103) unsupported */
+#define TSS_ERR_TIMEOUT 6         /* a bounded device-side wait gave up */
+#define TSS_ERR_DEVICE_CHECK 7    /* a device-side input check failed (e.g. token id range) */
+
+#define TSS_MODE_GREEDY 0 /* temperature 0: argmax acceptance, chain or tree */
+#define TSS_MODE_SAMPLE 1 /* speculative sampling at temperature > 0, chain drafts */
+
+typedef struct tss_ctx tss_ctx; /* opaque; owns repacked weights and all workspaces */
+
+/* Model shape and capacity limits.
+ *   n_layers <= 64; head_dim 64 or 128; d_model = n_heads * head_dim and a multiple of 128.
+ *   max_batch: requests per verify (<= 64).  max_rows: total draft-block rows per verify
+ *   (<= 256).  max_nodes: rows per request, root included (<= 64).  max_domains: size of the
+ *   domain table Phi.  max_positions: RoPE positions must be < max_positions. */
+typedef struct {
+  int n_layers, d_model, n_heads, head_dim, d_mlp, vocab;
+  float rms_eps, rope_theta;
+  int max_batch, max_rows, max_nodes, max_domains, max_positions;
+} tss_arch;
+
+/* Caller-owned bf16 weights in device memory, row-major [out][in] (PyTorch nn.Linear layout).
+ * Per-layer fields are HOST arrays of n_layers device pointers.
+ *   embed [vocab][d_model], lm_head [vocab][d_model], final_norm / attn_norm / mlp_norm
+ *   [d_model], wq wk wv wo [d_model][d_model], w_gate w_up [d_mlp][d_model],
+ *   w_down [d_model][d_mlp].
+ * tss_create copies and repacks them; the caller may free its buffers when it returns. */
+typedef struct {
+  const void* embed;
+  const void* lm_head;
+  const void* final_norm;
+  const void* const* attn_norm;
+  const void* const* wq;
+  const void* const* wk;
+  const void* const* wv;
+  const void* const* wo;
+  const void* const* mlp_norm;
+  const void* const* w_gate;
+  const void* const* w_up;
+  const void* const* w_down;
+} tss_weights;
+
+/* One verification step for n_req requests.  Rows are the requests' draft blocks concatenated
+ * in request order; M = sum(n_nodes).  Row 0 of each block is the root (the last committed
+ * token, whose KV is not yet cached); rows 1.. are draft nodes.
+ *   n_nodes, ctx_len, domain_id, kv_slot, parent_idx, positions: HOST arrays.
+ *     n_nodes[b]   in [1, max_nodes]
+ *     ctx_len[b]   tokens of request b already in its KV cache (>= 0)
+ *     domain_id[b] key into Phi; an id never configured (or out of range) means dense
+ *     kv_slot[b]   cache slot of request b (distinct); NULL means slot b
+ *     parent_idx[M] request-local parent: -1 for row 0 only, otherwise in [0, own index)
+ *                  (a chain is i-1)
+ *     positions[M] RoPE positions; NULL means ctx_len + depth, otherwise must equal it
+ *   tokens[M] (int32), draft_probs, uniforms: DEVICE arrays, or HOST arrays when io_host != 0.
+ *     draft_probs (SAMPLE): [M][vocab] fp32; row i is the draft distribution that proposed the
+ *       token of row i (row 0 unused).
+ *     uniforms (SAMPLE, optional): [n_req][uniform_stride] fp32 in [0,1); for a chain of k
+ *       drafts slot i-1 is the accept test of draft i (i=1..k) and slot k+i-1 the residual draw
+ *       at draft i or the bonus draw (i=k+1).  NULL: the library draws them with
+ *       Philox4x32-10, key (seed lo, seed hi), counter (slot, request, offset lo, offset hi),
+ *       u = (first word >> 8) * 2^-24.
+ *   io_host != 0: the inputs above and every result array are HOST pointers; the library
+ *     copies them in and out on the stream (results are valid after the stream synchronises). */
+typedef struct {
+  int n_req;
+  const int32_t* n_nodes;
+  const int32_t* ctx_len;
+  const int32_t* domain_id;
+  const int32_t* kv_slot;
+  const int32_t* parent_idx;
+  const int32_t* positions;
+  const int32_t* tokens;
+  int mode;
+  float temperature;
+  const float* draft_probs;
+  const float* uniforms;
+  int uniform_stride;
+  uint64_t philox_seed;
+  uint64_t philox_offset;
+  int io_host;
+} tss_verify_batch;
+
+/* Caller-owned KV cache.  layer is a HOST array of n_layers device pointers; layer l points to a
+ * bf16 buffer [n_slots][2][n_heads][cap][head_dim] (K then V).  An entry may be NULL for a
+ * layer that no request of a batch runs.  The library reads rows [0, ctx_len) and writes rows
+ * [ctx_len, ctx_len + n_nodes) of every layer a request runs, and never touches the layers it
+ * skips. */
+typedef struct {
+  void* const* layer;
+  int n_slots;
+  int cap;
+} tss_kv_cache;
+
+/* Caller-owned results (DEVICE arrays, or HOST arrays when io_host != 0).
+ *   accept_len[n_req]       accepted draft tokens a
+ *   bonus[n_req]            token emitted after the accepted ones
+ *   path[n_req][path_stride] request-local rows of the accepted path: path[0] = 0 (root),
+ *                           path[1..a] the accepted nodes, -1 after; path_stride > max depth
+ *   new_ctx_len[n_req]      ctx_len + 1 + a (root and accepted drafts are now cached)
+ *   logits[M][vocab]        fp32 target logits of every row, or NULL */
+typedef struct {
+  int32_t* accept_len;
+  int32_t* bonus;
+  int32_t* path;
+  int path_stride;
+  int32_t* new_ctx_len;
+  float* logits;
+} tss_verify_result;
+
+/* Build a verifier on the current CUDA device (must be sm_103).  Copies and repacks the weights
+ * into library-owned device memory, allocates every workspace for the limits in *arch, and
+ * returns an opaque context.  Errors: INVALID_ARG, UNSUPPORTED_ARCH, OUT_OF_MEMORY, CUDA. */
+tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx** out);
+
+/* Phi(domain_id) = the set of layers whose bit is set in layer_bitmask (bit l = skip layer l;
+ * 0 = dense).  Sec. "Domain-to-Configuration Mapping".  Bits >= n_layers must be clear.
+ * Synchronous; affects verifies enqueued after it returns.  domain_id in [0, max_domains). */
+tss_status tss_set_skip_config(tss_ctx* ctx, int domain_id, uint64_t layer_bitmask);
+
+/* Remove domain_id from Phi: its requests then run the dense path (unsupported domain). */
+tss_status tss_clear_skip_config(tss_ctx* ctx, int domain_id);
+
+/* Sparsity ratio R_d = |S_d| / L of a configured domain (0 for an unconfigured one), and the
+ * number of layers the union of a batch's skip sets leaves active.  Host-only queries. */
+tss_status tss_sparsity_ratio(const tss_ctx* ctx, int domain_id, double* out);
+tss_status tss_active_layer_count(const tss_ctx* ctx, const tss_verify_batch* batch, int* out);
+
+/* One verification step, enqueued on `stream`: skip controller (per-request S(x), union of
+ * active layers, per-layer compacted row lists) -> embedding -> for every layer in the union:
+ * RMSNorm+QKV GEMM with RoPE and KV append, split-KV attention with the chain/tree mask,
+ * O projection, RMSNorm+SwiGLU MLP -> final norm + LM head with fused argmax -> acceptance
+ * (greedy walk or speculative sampling) -> KV compaction of the accepted path.  A skipped layer
+ * gets no launch, reads no weight byte and no KV row.  Asynchronous; steps on one context must
+ * not overlap on different streams (they share workspaces). */
+tss_status tss_verify(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
+                      const tss_verify_result* result, void* stream);
+
+/* Synchronise `stream`, then return and clear the device status word (TSS_OK if no device-side
+ * check failed since the last call). */
+tss_status tss_sync_status(tss_ctx* ctx, void* stream);
+
+/* Release everything the context owns (after the caller's streams are idle). NULL is a no-op. */
+void tss_destroy(tss_ctx* ctx);
+
+/* Plain bf16 weight-streaming linear layer on the library's GEMM kernel:
+ *   y[m][o] = sum_k x[m][k] * w[o][k], x [m_rows][k_dim] bf16, w [n_out][k_dim] bf16,
+ *   y [m_rows][n_out] fp32, all device, row-major; m_rows in [1, 256]; k_dim a multiple of 64;
+ *   n_out a multiple of 128; rows of x and w 16-byte aligned.  The projections inside f_l
+ *   (App. "Models") run on this kernel.  Uses the context's workspaces: do not overlap with a
+ *   tss_verify of the same context. */
+tss_status tss_linear(tss_ctx* ctx, const void* x, const void* w, float* y, int m_rows, int k_dim,
+                      int n_out, void* stream);
+
+/* Per-kernel device times of one verification step, by kernel kind:
+ *   0 controller + embedding + RMSNorms, 1 QKV GEMM (+RoPE, KV append), 2 attention,
+ *   3 O-projection GEMM, 4 gate/up GEMM (+SwiGLU), 5 down GEMM, 6 LM head GEMM (+argmax),
+ *   7 acceptance + KV compaction. */
+#define TSS_KERNEL_KINDS 8
+typedef struct {
+  float ms[TSS_KERNEL_KINDS];     /* summed device time of the kind's launches */
+  int launches[TSS_KERNEL_KINDS]; /* launches of the kind */
+} tss_kernel_times;
+
+/* Diagnostic twin of tss_verify: the same kernels, launched one by one (no graph, no
+ * programmatic overlap) with a CUDA event pair around each launch on `stream`; synchronises the
+ * stream and ADDS the step's per-kind times into *times.  Results are written as by tss_verify. */
+tss_status tss_verify_profiled(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
+                               const tss_verify_result* result, void* stream, tss_kernel_times* times);
+
+const char* tss_status_string(tss_status s);
+/* Message of the last error reported to the calling thread ("" if none). */
+const char* tss_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TSS_H */

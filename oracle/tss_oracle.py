@@ -45,7 +45,7 @@ from .philox import verify_uniforms
 
 GREEDY_MARGIN = 0.05  # top-2 logit margin below which a greedy decision is flagged
 SAMPLE_LOG_BAND = 0.05  # |ln(r q(x)) - ln p(x)| below which an accept test is flagged
-SAMPLE_CDF_BAND = 1e-3  # distance of u from a CDF boundary (in normalised mass) that is flagged
+SAMPLE_CDF_BAND = 2e-4  # slack (normalised mass) allowed when a drawn token is checked for validity
 
 
 # ----------------------------------------------------------------------------------------------
@@ -363,7 +363,7 @@ def uniform_slots(k: int):
     return (lambda i: i - 1), (lambda i: k + i - 1), 2 * k + 1
 
 
-def spec_sample_accept(logits, tokens, q, uniforms, temperature: float = 1.0):
+def spec_sample_accept(logits, tokens, q, uniforms, temperature: float = 1.0, return_draw: bool = False):
     """Speculative sampling on a chain draft (rule of the cited speculative-decoding works).
 
     logits: [k+1, V] target logits of rows 0..k; tokens: [k+1] (row 0 the root);
@@ -373,7 +373,8 @@ def spec_sample_accept(logits, tokens, q, uniforms, temperature: float = 1.0):
     (r_i < min(1, p/q) without a division); at the first rejection sample the bonus from
     normalise(max(0, p_{i-1} - q_i)) by inverse CDF with u_i and stop; if all k are accepted
     sample the bonus from p_k with u_{k+1}.
-    Returns (a, bonus, path, flagged) where flagged marks a decision within the tie bands.
+    Returns (a, bonus, path, flagged): flagged marks an accept/reject decision within
+    SAMPLE_LOG_BAND of its boundary.  With return_draw, also (weights, u) of the bonus draw.
     """
     k = len(tokens) - 1
     r_slot, u_slot, _ = uniform_slots(k)
@@ -391,15 +392,27 @@ def spec_sample_accept(logits, tokens, q, uniforms, temperature: float = 1.0):
         if lhs < rhs:
             continue
         res = np.maximum(p - np.asarray(q[i], dtype=np.float64), 0.0)
-        v, t, lo, hi = inverse_cdf(res, float(uniforms[u_slot(i)]))
-        if min(t - lo, hi - t) < SAMPLE_CDF_BAND:
-            flagged = True
-        return i - 1, v, list(range(i)), flagged
+        u = float(uniforms[u_slot(i)])
+        v = inverse_cdf(res, u)[0]
+        out = (i - 1, v, list(range(i)), flagged)
+        return out + ((res, u),) if return_draw else out
     p = softmax_t(logits[k], temperature)
-    v, t, lo, hi = inverse_cdf(p, float(uniforms[u_slot(k + 1)]))
-    if min(t - lo, hi - t) < SAMPLE_CDF_BAND:
-        flagged = True
-    return k, v, list(range(k + 1)), flagged
+    u = float(uniforms[u_slot(k + 1)])
+    v = inverse_cdf(p, u)[0]
+    out = (k, v, list(range(k + 1)), flagged)
+    return out + ((p, u),) if return_draw else out
+
+
+def draw_consistent(weights, u: float, v: int, band: float = SAMPLE_CDF_BAND) -> bool:
+    """True if token v is the inverse-CDF draw of u from ``weights`` up to ``band`` of normalised
+    mass at its interval edges (a drawn token whose boundary moved by rounding is still valid),
+    and v carries positive mass."""
+    w = np.asarray(weights, dtype=np.float64)
+    if not (0 <= v < len(w)) or w[v] <= 0.0:
+        return False
+    c = np.cumsum(w) / w.sum()
+    lo = c[v - 1] if v > 0 else 0.0
+    return lo - band <= u <= c[v] + band
 
 
 def philox_uniforms(seed: int, offset: int, req: int, k: int):

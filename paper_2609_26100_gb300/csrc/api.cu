@@ -1,0 +1,860 @@
+// C ABI and host runtime of the TSS verification library: weight repacking, workspace
+// management, host-side validation, the per-step launch plan over the union of active layers,
+// and CUDA-graph capture of that plan.
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <map>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "internal.h"
+
+using namespace tss;
+
+namespace {
+
+thread_local std::string g_err;
+
+tss_status fail(tss_status s, const std::string& msg) {
+  g_err = msg;
+  return s;
+}
+
+#define TSS_CU(call)                                                                           \
+  do {                                                                                         \
+    cudaError_t e_ = (call);                                                                   \
+    if (e_ != cudaSuccess) return fail(TSS_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// bf16 tensor [d2][d1][d0] (d0 innermost), box (64, rows, 1), 128-byte swizzle.  Weights use
+// rank 3 (d2 = layer, loaded with 3-D TMA); activations use rank 2.
+bool make_tmap(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint32_t box_rows,
+               int rank = 3) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {d0 * 2, d0 * d1 * 2};
+  cuuint32_t box[3] = {64, box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, static_cast<cuuint32_t>(rank), const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int pad_to(int x, int m) { return (x + m - 1) / m * m; }
+
+struct GraphKey {
+  int B, M, n_act, mode, splits;
+  bool operator<(const GraphKey& o) const {
+    return std::tie(B, M, n_act, mode, splits) < std::tie(o.B, o.M, o.n_act, o.mode, o.splits);
+  }
+};
+
+constexpr int kRing = 4;
+constexpr int kMaxPathStride = 1024;
+
+}  // namespace
+
+struct tss_ctx {
+  tss_arch a{};
+  int dev = 0, num_sms = 0;
+  int L = 0, d = 0, H = 0, D = 0, F = 0, V = 0;
+  int F_pad = 0, Ft = 0, V_pad = 0;
+  // repacked weights
+  __nv_bfloat16 *wqkv = nullptr, *wo = nullptr, *wgu = nullptr, *wdown = nullptr, *embed = nullptr, *lm = nullptr;
+  float *g_attn = nullptr, *g_mlp = nullptr, *g_final = nullptr;
+  float *rope_cos = nullptr, *rope_sin = nullptr;
+  // workspaces
+  float* h = nullptr;
+  __nv_bfloat16 *xn = nullptr, *qbuf = nullptr, *obuf = nullptr, *act = nullptr;
+  float* logits_ws = nullptr;
+  float* partials = nullptr;
+  size_t partials_floats = 0;
+  int* counters = nullptr;
+  float* amax_val = nullptr;
+  int* amax_idx = nullptr;
+  float *attn_po = nullptr, *attn_pml = nullptr;
+  int* attn_cnt = nullptr;
+  int max_splits = 16;
+  StepDesc* d_step = nullptr;
+  StepDesc* h_ring[kRing] = {};
+  cudaEvent_t ring_ev[kRing] = {};
+  bool ring_used[kRing] = {};
+  int ring_i = 0;
+  PlanDev* d_plan = nullptr;
+  unsigned long long* d_phi = nullptr;
+  int* d_phi_valid = nullptr;
+  std::vector<unsigned long long> phi;
+  std::vector<int> phi_valid;
+  int* d_status = nullptr;
+  int* h_status = nullptr;
+  // staging for host-pointer I/O
+  int* io_tokens = nullptr;
+  float* io_probs = nullptr;
+  float* io_unif = nullptr;
+  int* io_res = nullptr;  // accept[kMaxBatch] bonus[kMaxBatch] new_ctx[kMaxBatch] path[kMaxBatch*kMaxPathStride]
+  // tensor maps
+  CUtensorMap tm_wqkv, tm_wo, tm_wgu, tm_wdown, tm_lm;
+  std::map<int, CUtensorMap> tm_xn, tm_o, tm_act;
+  // graphs
+  std::map<GraphKey, cudaGraphExec_t> graphs;
+  cudaStream_t cap_stream = nullptr;
+  bool use_graphs = true;
+  int gemm_ctas_per_sm = 2;
+  std::vector<void*> allocs;
+
+  template <typename T>
+  tss_status alloc(T** p, size_t count) {
+    void* q = nullptr;
+    if (cudaMalloc(&q, count * sizeof(T) + 16) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(TSS_ERR_OUT_OF_MEMORY, "cudaMalloc of " + std::to_string(count * sizeof(T)) + " bytes failed");
+    }
+    allocs.push_back(q);
+    *p = static_cast<T*>(q);
+    return TSS_OK;
+  }
+};
+
+namespace {
+
+#define TSS_TRY(expr)              \
+  do {                             \
+    tss_status s_ = (expr);        \
+    if (s_ != TSS_OK) return s_;   \
+  } while (0)
+
+struct GemmShape {
+  int epi, n_tiles, kb;
+  const CUtensorMap* tmW;
+  const CUtensorMap* tmX;
+};
+
+void gemm_config(const tss_ctx* c, int n_pad, int n_tiles, int kb, int* grid, int* stages, size_t* smem, int* bufs) {
+  const int per_sm = n_pad <= 64 ? c->gemm_ctas_per_sm : 1;
+  const size_t budget = per_sm >= 2 ? 110 * 1024 : 220 * 1024;
+  int s = 2;
+  while (s < 12 && gemm_smem_bytes(n_pad, s + 1) <= budget) ++s;
+  *stages = s;
+  *smem = gemm_smem_bytes(n_pad, s);
+  *bufs = n_pad <= 128 ? 2 : 1;
+  long long T = static_cast<long long>(n_tiles) * kb;
+  long long g = static_cast<long long>(c->num_sms) * per_sm;
+  *grid = static_cast<int>(g < T ? g : T);
+}
+
+tss_status get_xmap(tss_ctx* c, std::map<int, CUtensorMap>& cache, const void* buf, int k, int n_pad,
+                    const CUtensorMap** out) {
+  auto it = cache.find(n_pad);
+  if (it == cache.end()) {
+    CUtensorMap m;
+    if (!make_tmap(&m, buf, static_cast<uint64_t>(k), kMaxRows, 1, static_cast<uint32_t>(n_pad), 2))
+      return fail(TSS_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
+    it = cache.emplace(n_pad, m).first;
+  }
+  *out = &it->second;
+  return TSS_OK;
+}
+
+MiscParams misc_params(tss_ctx* c) {
+  MiscParams p{};
+  p.step = c->d_step;
+  p.plan = c->d_plan;
+  p.phi_mask = c->d_phi;
+  p.phi_valid = c->d_phi_valid;
+  p.max_domains = c->a.max_domains;
+  p.n_layers = c->L;
+  p.d_model = c->d;
+  p.n_heads = c->H;
+  p.head_dim = c->D;
+  p.vocab = c->V;
+  p.rms_eps = c->a.rms_eps;
+  p.embed = c->embed;
+  p.h = c->h;
+  p.xn = c->xn;
+  p.g_attn = c->g_attn;
+  p.g_mlp = c->g_mlp;
+  p.g_final = c->g_final;
+  p.amax_val = c->amax_val;
+  p.amax_idx = c->amax_idx;
+  p.n_vtiles = c->V_pad / 128;
+  p.status = c->d_status;
+  return p;
+}
+
+GemmParams gemm_base(tss_ctx* c, int n_pad) {
+  GemmParams g{};
+  g.n_pad = n_pad;
+  g.plan = c->d_plan;
+  g.step = c->d_step;
+  g.partials = c->partials;
+  g.counters = c->counters;
+  g.status = c->d_status;
+  g.h = c->h;
+  g.q_out = c->qbuf;
+  g.act_out = c->act;
+  g.act_ld = c->F_pad;
+  g.rope_cos = c->rope_cos;
+  g.rope_sin = c->rope_sin;
+  g.amax_val = c->amax_val;
+  g.amax_idx = c->amax_idx;
+  g.d_model = c->d;
+  g.n_heads = c->H;
+  g.head_dim = c->D;
+  g.vocab = c->V;
+  g.layer_fixed = -1;
+  return g;
+}
+
+tss_status run_gemm(tss_ctx* c, int epi, const CUtensorMap& tmW, const CUtensorMap& tmX, GemmParams g, int n_tiles,
+                    int kb, cudaStream_t s, bool pdl) {
+  int grid, stages, bufs;
+  size_t smem;
+  gemm_config(c, g.n_pad, n_tiles, kb, &grid, &stages, &smem, &bufs);
+  g.n_tiles = n_tiles;
+  g.kb = kb;
+  g.stages = stages;
+  g.n_acc_bufs = bufs;
+  if (static_cast<size_t>(grid + n_tiles) * 128 * g.n_pad > c->partials_floats)
+    return fail(TSS_ERR_INVALID_ARG, "GEMM partial workspace too small");
+  TSS_CU(launch_gemm(epi, tmW, tmX, g, grid, smem, s, pdl));
+  return TSS_OK;
+}
+
+struct StepPlan {
+  int B, M, n_act, mode, splits, n_pad;
+};
+
+// Optional per-launch event timing (tss_verify_profiled).
+struct Prof {
+  std::vector<cudaEvent_t> ev;
+  std::vector<int> kind;
+  cudaStream_t s = nullptr;
+  tss_status begin(int k) {
+    cudaEvent_t e;
+    TSS_CU(cudaEventCreate(&e));
+    ev.push_back(e);
+    kind.push_back(k);
+    TSS_CU(cudaEventRecord(e, s));
+    return TSS_OK;
+  }
+  tss_status end() {
+    cudaEvent_t e;
+    TSS_CU(cudaEventCreate(&e));
+    ev.push_back(e);
+    kind.push_back(-1);
+    TSS_CU(cudaEventRecord(e, s));
+    return TSS_OK;
+  }
+};
+
+// Enqueue every kernel of one verification step (also used under stream capture).  With a Prof,
+// every launch is bracketed by events and launched without programmatic overlap.
+tss_status enqueue_step(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* prof = nullptr) {
+  const bool pdl = prof == nullptr;
+#define TSS_K(kind, expr)                       \
+  do {                                          \
+    if (prof) TSS_TRY(prof->begin(kind));       \
+    expr;                                       \
+    if (prof) TSS_TRY(prof->end());             \
+  } while (0)
+  MiscParams mp = misc_params(c);
+  const int n_pad = sp.n_pad;
+  const CUtensorMap *txn, *to, *tact;
+  TSS_TRY(get_xmap(c, c->tm_xn, c->xn, c->d, n_pad, &txn));
+  TSS_TRY(get_xmap(c, c->tm_o, c->obuf, c->d, n_pad, &to));
+  TSS_TRY(get_xmap(c, c->tm_act, c->act, c->F_pad, n_pad, &tact));
+
+  TSS_K(0, TSS_CU(launch_controller(mp, s, false)));
+  TSS_K(0, TSS_CU(launch_embed(mp, sp.M, s, pdl)));
+  AttnParams ap{};
+  ap.n_splits = sp.splits;
+  ap.n_heads = c->H;
+  ap.d_model = c->d;
+  ap.head_dim = c->D;
+  ap.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->D)));
+  ap.plan = c->d_plan;
+  ap.step = c->d_step;
+  ap.q = c->qbuf;
+  ap.o = c->obuf;
+  ap.part_o = c->attn_po;
+  ap.part_ml = c->attn_pml;
+  ap.counters = c->attn_cnt;
+  ap.status = c->d_status;
+  const int kbd = c->d / 64;
+  for (int j = 0; j < sp.n_act; ++j) {
+    // attention sub-block: h_{l+1} = f_l(h_l) only for layers in the union; others get no launch
+    TSS_K(0, TSS_CU(launch_rmsnorm(mp, j, 0, sp.M, s, pdl)));
+    GemmParams g = gemm_base(c, n_pad);
+    g.slot = j;
+    TSS_K(1, TSS_TRY(run_gemm(c, kEpiQkv, c->tm_wqkv, *txn, g, 3 * c->d / 128, kbd, s, pdl)));
+    ap.slot = j;
+    TSS_K(2, TSS_CU(launch_attention(ap, sp.B, s, pdl)));
+    TSS_K(3, TSS_TRY(run_gemm(c, kEpiResid, c->tm_wo, *to, g, c->d / 128, kbd, s, pdl)));
+    // feed-forward sub-block
+    TSS_K(0, TSS_CU(launch_rmsnorm(mp, j, 1, sp.M, s, pdl)));
+    TSS_K(4, TSS_TRY(run_gemm(c, kEpiSwiglu, c->tm_wgu, *txn, g, c->Ft, kbd, s, pdl)));
+    TSS_K(5, TSS_TRY(run_gemm(c, kEpiResid, c->tm_wdown, *tact, g, c->d / 128, c->F_pad / 64, s, pdl)));
+  }
+  TSS_K(0, TSS_CU(launch_rmsnorm(mp, kFinalSlot, 2, sp.M, s, pdl)));
+  GemmParams g = gemm_base(c, n_pad);
+  g.slot = kFinalSlot;
+  g.layer_fixed = 0;
+  TSS_K(6, TSS_TRY(run_gemm(c, kEpiLmHead, c->tm_lm, *txn, g, c->V_pad / 128, kbd, s, pdl)));
+  if (sp.mode == TSS_MODE_SAMPLE) {
+    TSS_K(7, TSS_CU(launch_accept_sample(mp, sp.B, s, pdl)));
+  } else {
+    TSS_K(7, TSS_CU(launch_accept_greedy(mp, sp.B, s, pdl)));
+  }
+  TSS_K(7, TSS_CU(launch_compact(mp, sp.B, sp.n_act, s, pdl)));
+#undef TSS_K
+  return TSS_OK;
+}
+
+tss_status validate_arch(const tss_arch* a) {
+  if (!a) return fail(TSS_ERR_INVALID_ARG, "arch is NULL");
+  if (a->n_layers < 1 || a->n_layers > kMaxLayers) return fail(TSS_ERR_UNSUPPORTED_ARCH, "n_layers must be in [1, 64]");
+  if (a->head_dim != 64 && a->head_dim != 128) return fail(TSS_ERR_UNSUPPORTED_ARCH, "head_dim must be 64 or 128");
+  if (a->n_heads < 1 || a->d_model != a->n_heads * a->head_dim)
+    return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_model must equal n_heads * head_dim");
+  if (a->d_model % 128 != 0) return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_model must be a multiple of 128");
+  if (a->d_mlp < 1 || a->vocab < 1) return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_mlp and vocab must be positive");
+  if (a->d_mlp % 8 != 0) return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_mlp must be a multiple of 8");
+  if (a->max_batch < 1 || a->max_batch > kMaxBatch) return fail(TSS_ERR_INVALID_ARG, "max_batch must be in [1, 64]");
+  if (a->max_rows < 1 || a->max_rows > kMaxRows) return fail(TSS_ERR_INVALID_ARG, "max_rows must be in [1, 256]");
+  if (a->max_nodes < 1 || a->max_nodes > kMaxNodes) return fail(TSS_ERR_INVALID_ARG, "max_nodes must be in [1, 64]");
+  if (a->max_domains < 1 || a->max_domains > (1 << 20)) return fail(TSS_ERR_INVALID_ARG, "max_domains out of range");
+  if (a->max_positions < 1) return fail(TSS_ERR_INVALID_ARG, "max_positions must be positive");
+  if (!(a->rms_eps >= 0.f) || !(a->rope_theta > 0.f)) return fail(TSS_ERR_INVALID_ARG, "rms_eps / rope_theta invalid");
+  return TSS_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+tss_status build_weights(tss_ctx* c, const tss_weights* w) {
+  const int L = c->L, d = c->d, F = c->F, V = c->V;
+  if (!w || !w->embed || !w->lm_head || !w->final_norm || !w->attn_norm || !w->wq || !w->wk || !w->wv || !w->wo ||
+      !w->mlp_norm || !w->w_gate || !w->w_up || !w->w_down)
+    return fail(TSS_ERR_INVALID_ARG, "a weight pointer is NULL");
+  for (int l = 0; l < L; ++l)
+    if (!w->attn_norm[l] || !w->wq[l] || !w->wk[l] || !w->wv[l] || !w->wo[l] || !w->mlp_norm[l] || !w->w_gate[l] ||
+        !w->w_up[l] || !w->w_down[l])
+      return fail(TSS_ERR_INVALID_ARG, "weights of layer " + std::to_string(l) + " incomplete");
+  const size_t dd = static_cast<size_t>(d) * d;
+  TSS_TRY(c->alloc(&c->wqkv, static_cast<size_t>(L) * 3 * dd));
+  TSS_TRY(c->alloc(&c->wo, static_cast<size_t>(L) * dd));
+  TSS_TRY(c->alloc(&c->wgu, static_cast<size_t>(L) * c->Ft * 128 * d));
+  TSS_TRY(c->alloc(&c->wdown, static_cast<size_t>(L) * d * c->F_pad));
+  TSS_TRY(c->alloc(&c->embed, static_cast<size_t>(V) * d));
+  TSS_TRY(c->alloc(&c->lm, static_cast<size_t>(c->V_pad) * d));
+  TSS_TRY(c->alloc(&c->g_attn, static_cast<size_t>(L) * d));
+  TSS_TRY(c->alloc(&c->g_mlp, static_cast<size_t>(L) * d));
+  TSS_TRY(c->alloc(&c->g_final, d));
+  const size_t b2 = sizeof(__nv_bfloat16);
+  TSS_CU(cudaMemset(c->wgu, 0, static_cast<size_t>(L) * c->Ft * 128 * d * b2));
+  TSS_CU(cudaMemset(c->wdown, 0, static_cast<size_t>(L) * d * c->F_pad * b2));
+  TSS_CU(cudaMemset(c->lm, 0, static_cast<size_t>(c->V_pad) * d * b2));
+  TSS_CU(cudaMemcpy(c->embed, w->embed, static_cast<size_t>(V) * d * b2, cudaMemcpyDeviceToDevice));
+  TSS_CU(cudaMemcpy(c->lm, w->lm_head, static_cast<size_t>(V) * d * b2, cudaMemcpyDeviceToDevice));
+  TSS_CU(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(w->final_norm), c->g_final, d, 0));
+  for (int l = 0; l < L; ++l) {
+    __nv_bfloat16* q = c->wqkv + static_cast<size_t>(l) * 3 * dd;
+    TSS_CU(cudaMemcpy(q, w->wq[l], dd * b2, cudaMemcpyDeviceToDevice));
+    TSS_CU(cudaMemcpy(q + dd, w->wk[l], dd * b2, cudaMemcpyDeviceToDevice));
+    TSS_CU(cudaMemcpy(q + 2 * dd, w->wv[l], dd * b2, cudaMemcpyDeviceToDevice));
+    TSS_CU(cudaMemcpy(c->wo + static_cast<size_t>(l) * dd, w->wo[l], dd * b2, cudaMemcpyDeviceToDevice));
+    // gate/up interleaved per 64 features: tile t = [gate rows 64t..64t+63 ; up rows 64t..64t+63]
+    __nv_bfloat16* gu = c->wgu + static_cast<size_t>(l) * c->Ft * 128 * d;
+    for (int t = 0; t < c->Ft; ++t) {
+      const int rows = F - 64 * t < 64 ? F - 64 * t : 64;
+      const size_t src_off = static_cast<size_t>(64) * t * d;
+      TSS_CU(cudaMemcpy(gu + static_cast<size_t>(t) * 128 * d, static_cast<const __nv_bfloat16*>(w->w_gate[l]) + src_off,
+                        static_cast<size_t>(rows) * d * b2, cudaMemcpyDeviceToDevice));
+      TSS_CU(cudaMemcpy(gu + (static_cast<size_t>(t) * 128 + 64) * d,
+                        static_cast<const __nv_bfloat16*>(w->w_up[l]) + src_off, static_cast<size_t>(rows) * d * b2,
+                        cudaMemcpyDeviceToDevice));
+    }
+    TSS_CU(cudaMemcpy2D(c->wdown + static_cast<size_t>(l) * d * c->F_pad, static_cast<size_t>(c->F_pad) * b2, w->w_down[l],
+                        static_cast<size_t>(F) * b2, static_cast<size_t>(F) * b2, d, cudaMemcpyDeviceToDevice));
+    TSS_CU(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(w->attn_norm[l]), c->g_attn + static_cast<size_t>(l) * d, d, 0));
+    TSS_CU(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(w->mlp_norm[l]), c->g_mlp + static_cast<size_t>(l) * d, d, 0));
+  }
+  TSS_CU(cudaDeviceSynchronize());
+  if (!make_tmap(&c->tm_wqkv, c->wqkv, d, 3 * d, L, 128) || !make_tmap(&c->tm_wo, c->wo, d, d, L, 128) ||
+      !make_tmap(&c->tm_wgu, c->wgu, d, static_cast<uint64_t>(c->Ft) * 128, L, 128) ||
+      !make_tmap(&c->tm_wdown, c->wdown, c->F_pad, d, L, 128) || !make_tmap(&c->tm_lm, c->lm, d, c->V_pad, 1, 128))
+    return fail(TSS_ERR_CUDA, "cuTensorMapEncodeTiled failed for a weight tensor");
+  return TSS_OK;
+}
+
+tss_status build_workspaces(tss_ctx* c) {
+  const int d = c->d;
+  const size_t R = kMaxRows;
+  TSS_TRY(c->alloc(&c->h, R * d));
+  TSS_TRY(c->alloc(&c->xn, R * d));
+  TSS_TRY(c->alloc(&c->qbuf, R * d));
+  TSS_TRY(c->alloc(&c->obuf, R * d));
+  TSS_TRY(c->alloc(&c->act, R * c->F_pad));
+  TSS_TRY(c->alloc(&c->logits_ws, static_cast<size_t>(c->a.max_rows) * c->V));
+  TSS_CU(cudaMemset(c->xn, 0, R * d * 2));
+  TSS_CU(cudaMemset(c->obuf, 0, R * d * 2));
+  TSS_CU(cudaMemset(c->act, 0, R * c->F_pad * 2));
+  const int max_tiles = std::max(std::max(3 * d / 128, c->Ft), c->V_pad / 128);
+  const size_t max_grid = static_cast<size_t>(c->num_sms) * 2;
+  c->partials_floats = (max_grid + max_tiles) * 128 * static_cast<size_t>(pad_to(c->a.max_rows, 16));
+  TSS_TRY(c->alloc(&c->partials, c->partials_floats));
+  TSS_TRY(c->alloc(&c->counters, max_tiles + 64));
+  TSS_CU(cudaMemset(c->counters, 0, (max_tiles + 64) * sizeof(int)));
+  TSS_TRY(c->alloc(&c->amax_val, static_cast<size_t>(c->V_pad / 128) * kMaxRows));
+  TSS_TRY(c->alloc(&c->amax_idx, static_cast<size_t>(c->V_pad / 128) * kMaxRows));
+  const size_t ph = static_cast<size_t>(c->a.max_batch) * c->H * c->max_splits * kMaxNodes;
+  TSS_TRY(c->alloc(&c->attn_po, ph * c->D));
+  TSS_TRY(c->alloc(&c->attn_pml, ph * 2));
+  TSS_TRY(c->alloc(&c->attn_cnt, static_cast<size_t>(c->a.max_batch) * c->H));
+  TSS_CU(cudaMemset(c->attn_cnt, 0, static_cast<size_t>(c->a.max_batch) * c->H * sizeof(int)));
+  TSS_TRY(c->alloc(&c->d_step, 1));
+  TSS_TRY(c->alloc(&c->d_plan, 1));
+  TSS_CU(cudaMemset(c->d_plan, 0, sizeof(PlanDev)));
+  TSS_TRY(c->alloc(&c->d_phi, c->a.max_domains));
+  TSS_TRY(c->alloc(&c->d_phi_valid, c->a.max_domains));
+  TSS_CU(cudaMemset(c->d_phi, 0, sizeof(unsigned long long) * c->a.max_domains));
+  TSS_CU(cudaMemset(c->d_phi_valid, 0, sizeof(int) * c->a.max_domains));
+  c->phi.assign(c->a.max_domains, 0ull);
+  c->phi_valid.assign(c->a.max_domains, 0);
+  TSS_TRY(c->alloc(&c->d_status, 1));
+  TSS_CU(cudaMemset(c->d_status, 0, sizeof(int)));
+  TSS_CU(cudaMallocHost(&c->h_status, sizeof(int)));
+  for (int i = 0; i < kRing; ++i) {
+    TSS_CU(cudaMallocHost(&c->h_ring[i], sizeof(StepDesc)));
+    TSS_CU(cudaEventCreateWithFlags(&c->ring_ev[i], cudaEventDisableTiming));
+  }
+  TSS_TRY(c->alloc(&c->io_tokens, kMaxRows));
+  TSS_TRY(c->alloc(&c->io_probs, static_cast<size_t>(c->a.max_rows) * c->V));
+  TSS_TRY(c->alloc(&c->io_unif, static_cast<size_t>(c->a.max_batch) * 4 * kMaxNodes));
+  TSS_TRY(c->alloc(&c->io_res, static_cast<size_t>(kMaxBatch) * (3 + kMaxPathStride)));
+  // RoPE tables in float64, stored as float32: angle(pos, i) = pos * theta^(-2i/D)
+  const int half = c->D / 2;
+  std::vector<float> hc(static_cast<size_t>(c->a.max_positions) * half), hs(hc.size());
+  for (int pos = 0; pos < c->a.max_positions; ++pos)
+    for (int i = 0; i < half; ++i) {
+      const double inv = std::pow(static_cast<double>(c->a.rope_theta), -2.0 * i / c->D);
+      const double ang = static_cast<double>(pos) * inv;
+      hc[static_cast<size_t>(pos) * half + i] = static_cast<float>(std::cos(ang));
+      hs[static_cast<size_t>(pos) * half + i] = static_cast<float>(std::sin(ang));
+    }
+  TSS_TRY(c->alloc(&c->rope_cos, hc.size()));
+  TSS_TRY(c->alloc(&c->rope_sin, hs.size()));
+  TSS_CU(cudaMemcpy(c->rope_cos, hc.data(), hc.size() * 4, cudaMemcpyHostToDevice));
+  TSS_CU(cudaMemcpy(c->rope_sin, hs.data(), hs.size() * 4, cudaMemcpyHostToDevice));
+  TSS_CU(cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking));
+  size_t max_smem = gemm_smem_bytes(16, 12);
+  for (int n = 16; n <= 256; n += 16) max_smem = std::max(max_smem, gemm_smem_bytes(n, 2));
+  max_smem = std::max<size_t>(max_smem, 220 * 1024 + 16 * 1024);
+  if (max_smem > 232448) max_smem = 232448;
+  TSS_CU(gemm_prepare(max_smem));
+  TSS_CU(attn_prepare());
+  return TSS_OK;
+}
+
+void destroy_ctx(tss_ctx* c) {
+  if (!c) return;
+  for (auto& kv : c->graphs) cudaGraphExecDestroy(kv.second);
+  for (void* p : c->allocs) cudaFree(p);
+  for (int i = 0; i < kRing; ++i) {
+    if (c->h_ring[i]) cudaFreeHost(c->h_ring[i]);
+    if (c->ring_ev[i]) cudaEventDestroy(c->ring_ev[i]);
+  }
+  if (c->h_status) cudaFreeHost(c->h_status);
+  if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+  delete c;
+}
+
+// Host-side per-step checks and the descriptor contents.  Nothing is enqueued here.
+tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache* kv,
+                        const tss_verify_result* res, StepDesc* sd, StepPlan* sp) {
+  if (!bt || !kv || !res) return fail(TSS_ERR_INVALID_ARG, "batch, kv or result is NULL");
+  const int B = bt->n_req;
+  if (B < 1 || B > c->a.max_batch) return fail(TSS_ERR_INVALID_ARG, "n_req must be in [1, max_batch]");
+  if (!bt->n_nodes || !bt->ctx_len || !bt->domain_id || !bt->parent_idx || !bt->tokens)
+    return fail(TSS_ERR_INVALID_ARG, "n_nodes, ctx_len, domain_id, parent_idx and tokens are required");
+  if (bt->mode != TSS_MODE_GREEDY && bt->mode != TSS_MODE_SAMPLE) return fail(TSS_ERR_INVALID_ARG, "unknown mode");
+  if (!kv->layer || kv->n_slots < 1 || kv->cap < 1) return fail(TSS_ERR_INVALID_ARG, "KV cache descriptor invalid");
+  if (!res->accept_len || !res->bonus || !res->path || !res->new_ctx_len)
+    return fail(TSS_ERR_INVALID_ARG, "result arrays accept_len, bonus, path and new_ctx_len are required");
+  std::memset(sd, 0, sizeof(StepDesc));
+  int M = 0, max_depth = 0, max_t = 0;
+  std::vector<int> slot_used(kv->n_slots, 0);
+  unsigned long long all_runs = 0ull;  // layers some request runs
+  for (int b = 0; b < B; ++b) {
+    const int n = bt->n_nodes[b], ctx = bt->ctx_len[b];
+    if (n < 1 || n > c->a.max_nodes) return fail(TSS_ERR_INVALID_ARG, "n_nodes out of [1, max_nodes]");
+    if (M + n > c->a.max_rows) return fail(TSS_ERR_INVALID_ARG, "total rows exceed max_rows");
+    if (ctx < 0) return fail(TSS_ERR_INVALID_ARG, "ctx_len negative");
+    if (static_cast<long long>(ctx) + n > kv->cap) return fail(TSS_ERR_KV_CAPACITY, "ctx_len + n_nodes exceeds KV capacity");
+    const int slot = bt->kv_slot ? bt->kv_slot[b] : b;
+    if (slot < 0 || slot >= kv->n_slots) return fail(TSS_ERR_INVALID_ARG, "kv_slot out of range");
+    if (slot_used[slot]++) return fail(TSS_ERR_INVALID_ARG, "two requests share a kv_slot");
+    const int dom = bt->domain_id[b];
+    const bool configured = dom >= 0 && dom < c->a.max_domains && c->phi_valid[dom];
+    const unsigned long long mask = configured ? c->phi[dom] : 0ull;  // S(x) or dense fallback
+    for (int l = 0; l < c->L; ++l)
+      if (!((mask >> l) & 1ull)) all_runs |= 1ull << l;
+    sd->req_ctx[b] = ctx;
+    sd->req_nodes[b] = n;
+    sd->req_rowoff[b] = M;
+    sd->req_slot[b] = slot;
+    sd->req_domain[b] = dom;
+    unsigned long long anc[kMaxNodes];
+    int depth[kMaxNodes];
+    for (int i = 0; i < n; ++i) {
+      const int par = bt->parent_idx[M + i];
+      if (i == 0 ? par != -1 : (par < 0 || par >= i))
+        return fail(TSS_ERR_INVALID_ARG, "parent_idx must be -1 for row 0 and in [0, i) otherwise");
+      if (bt->mode == TSS_MODE_SAMPLE && i > 0 && par != i - 1)
+        return fail(TSS_ERR_INVALID_ARG, "speculative sampling verifies chain drafts only");
+      depth[i] = i == 0 ? 0 : depth[par] + 1;
+      anc[i] = (i == 0 ? 0ull : anc[par]) | (1ull << i);
+      const int pos = ctx + depth[i];
+      if (bt->positions && bt->positions[M + i] != pos)
+        return fail(TSS_ERR_INVALID_ARG, "positions must equal ctx_len + depth");
+      if (pos >= c->a.max_positions) return fail(TSS_ERR_INVALID_ARG, "position beyond max_positions");
+      sd->row_req[M + i] = b;
+      sd->row_pos[M + i] = pos;
+      sd->row_parent[M + i] = par;
+      sd->row_anc[M + i] = anc[i];
+      if (depth[i] > max_depth) max_depth = depth[i];
+    }
+    max_t = std::max(max_t, ctx + n);
+    M += n;
+  }
+  if (res->path_stride < max_depth + 1 || res->path_stride > kMaxPathStride)
+    return fail(TSS_ERR_INVALID_ARG, "path_stride must be in [max depth + 1, 1024]");
+  for (int l = 0; l < c->L; ++l)
+    if (((all_runs >> l) & 1ull)) {
+      if (!kv->layer[l]) return fail(TSS_ERR_INVALID_ARG, "KV buffer of an active layer is NULL");
+      if (!aligned16(kv->layer[l])) return fail(TSS_ERR_INVALID_ARG, "KV buffers must be 16-byte aligned");
+    }
+  if (bt->mode == TSS_MODE_SAMPLE) {
+    if (!(bt->temperature > 0.f) || !std::isfinite(bt->temperature))
+      return fail(TSS_ERR_INVALID_ARG, "temperature must be positive and finite");
+    if (!bt->draft_probs) return fail(TSS_ERR_INVALID_ARG, "draft_probs required for speculative sampling");
+    if (bt->uniforms) {
+      int need = 0;
+      for (int b = 0; b < B; ++b) need = std::max(need, 2 * (bt->n_nodes[b] - 1) + 1);
+      if (bt->uniform_stride < need) return fail(TSS_ERR_INVALID_ARG, "uniform_stride < 2k + 1");
+      if (bt->io_host && bt->uniform_stride > 4 * kMaxNodes)
+        return fail(TSS_ERR_INVALID_ARG, "uniform_stride too large for host I/O");
+    }
+  }
+  int n_act = 0;
+  for (int l = 0; l < c->L; ++l) n_act += (all_runs >> l) & 1ull;
+  sd->B = B;
+  sd->M = M;
+  sd->n_act_host = n_act;
+  sd->mode = bt->mode;
+  sd->inv_temperature = bt->mode == TSS_MODE_SAMPLE ? 1.f / bt->temperature : 1.f;
+  sd->uniform_stride = bt->uniform_stride;
+  sd->path_stride = res->path_stride;
+  sd->kv_cap = kv->cap;
+  sd->seed_lo = static_cast<uint32_t>(bt->philox_seed);
+  sd->seed_hi = static_cast<uint32_t>(bt->philox_seed >> 32);
+  sd->off_lo = static_cast<uint32_t>(bt->philox_offset);
+  sd->off_hi = static_cast<uint32_t>(bt->philox_offset >> 32);
+  for (int l = 0; l < c->L; ++l) sd->kv_layer[l] = static_cast<__nv_bfloat16*>(kv->layer[l]);
+  // attention splits: aim for ~2 CTAs per SM; bucketed so graphs are reused as contexts grow
+  int tiles = (max_t + 63) / 64, tb = 1;
+  while (tb < tiles) tb <<= 1;
+  const int want = (2 * c->num_sms + B * c->H - 1) / (B * c->H);
+  int splits = std::max(1, std::min(std::min(want, c->max_splits), tb));
+  sp->B = B;
+  sp->M = M;
+  sp->n_act = n_act;
+  sp->mode = bt->mode;
+  sp->splits = splits;
+  sp->n_pad = pad_to(M, 16);
+  return TSS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* tss_status_string(tss_status s) {
+  switch (s) {
+    case TSS_OK: return "ok";
+    case TSS_ERR_INVALID_ARG: return "invalid argument";
+    case TSS_ERR_OUT_OF_MEMORY: return "out of device memory";
+    case TSS_ERR_KV_CAPACITY: return "KV cache capacity exceeded";
+    case TSS_ERR_CUDA: return "CUDA error";
+    case TSS_ERR_UNSUPPORTED_ARCH: return "unsupported model shape or GPU";
+    case TSS_ERR_TIMEOUT: return "device wait timed out";
+    case TSS_ERR_DEVICE_CHECK: return "device-side check failed";
+    default: return "unknown status";
+  }
+}
+
+const char* tss_last_error(void) { return g_err.c_str(); }
+
+tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx** out) {
+  if (!out) return fail(TSS_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  TSS_TRY(validate_arch(arch));
+  int dev = 0;
+  TSS_CU(cudaGetDevice(&dev));
+  cudaDeviceProp prop;
+  TSS_CU(cudaGetDeviceProperties(&prop, dev));
+  if (prop.major != 10 || prop.minor != 3)
+    return fail(TSS_ERR_UNSUPPORTED_ARCH, "this library is built for sm_103 (GB300); device is sm_" +
+                                               std::to_string(prop.major) + std::to_string(prop.minor));
+  if (!encode_fn()) return fail(TSS_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+  tss_ctx* c = new tss_ctx();
+  c->a = *arch;
+  c->dev = dev;
+  c->num_sms = prop.multiProcessorCount;
+  c->L = arch->n_layers;
+  c->d = arch->d_model;
+  c->H = arch->n_heads;
+  c->D = arch->head_dim;
+  c->F = arch->d_mlp;
+  c->V = arch->vocab;
+  c->Ft = (c->F + 63) / 64;
+  c->F_pad = c->Ft * 64;
+  c->V_pad = pad_to(c->V, 128);
+  if (const char* e = std::getenv("TSS_NO_GRAPH")) c->use_graphs = std::atoi(e) == 0;
+  if (const char* e = std::getenv("TSS_GEMM_CTAS_PER_SM")) c->gemm_ctas_per_sm = std::max(1, std::min(2, std::atoi(e)));
+  tss_status s = build_workspaces(c);
+  if (s == TSS_OK) s = build_weights(c, weights);
+  if (s != TSS_OK) {
+    const std::string msg = g_err;
+    destroy_ctx(c);
+    cudaGetLastError();
+    g_err = msg;
+    return s;
+  }
+  *out = c;
+  return TSS_OK;
+}
+
+void tss_destroy(tss_ctx* ctx) {
+  if (!ctx) return;
+  cudaDeviceSynchronize();
+  destroy_ctx(ctx);
+}
+
+tss_status tss_set_skip_config(tss_ctx* c, int domain_id, uint64_t mask) {
+  if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
+  if (domain_id < 0 || domain_id >= c->a.max_domains) return fail(TSS_ERR_INVALID_ARG, "domain_id out of range");
+  if (c->L < 64 && (mask >> c->L) != 0ull) return fail(TSS_ERR_INVALID_ARG, "skip mask names a layer >= n_layers");
+  c->phi[domain_id] = mask;
+  c->phi_valid[domain_id] = 1;
+  const int one = 1;
+  const unsigned long long m = mask;
+  TSS_CU(cudaMemcpy(c->d_phi + domain_id, &m, sizeof(m), cudaMemcpyHostToDevice));
+  TSS_CU(cudaMemcpy(c->d_phi_valid + domain_id, &one, sizeof(int), cudaMemcpyHostToDevice));
+  return TSS_OK;
+}
+
+tss_status tss_clear_skip_config(tss_ctx* c, int domain_id) {
+  if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
+  if (domain_id < 0 || domain_id >= c->a.max_domains) return fail(TSS_ERR_INVALID_ARG, "domain_id out of range");
+  c->phi[domain_id] = 0ull;
+  c->phi_valid[domain_id] = 0;
+  const int zero = 0;
+  TSS_CU(cudaMemcpy(c->d_phi_valid + domain_id, &zero, sizeof(int), cudaMemcpyHostToDevice));
+  return TSS_OK;
+}
+
+tss_status tss_sparsity_ratio(const tss_ctx* c, int domain_id, double* out) {
+  if (!c || !out) return fail(TSS_ERR_INVALID_ARG, "ctx or out is NULL");
+  if (domain_id < 0 || domain_id >= c->a.max_domains) return fail(TSS_ERR_INVALID_ARG, "domain_id out of range");
+  const unsigned long long m = c->phi_valid[domain_id] ? c->phi[domain_id] : 0ull;
+  *out = static_cast<double>(__builtin_popcountll(m)) / c->L;
+  return TSS_OK;
+}
+
+tss_status tss_active_layer_count(const tss_ctx* c, const tss_verify_batch* bt, int* out) {
+  if (!c || !bt || !out || !bt->domain_id) return fail(TSS_ERR_INVALID_ARG, "NULL argument");
+  if (bt->n_req < 1 || bt->n_req > c->a.max_batch) return fail(TSS_ERR_INVALID_ARG, "n_req out of range");
+  unsigned long long runs = 0ull;
+  for (int b = 0; b < bt->n_req; ++b) {
+    const int dom = bt->domain_id[b];
+    const unsigned long long m = (dom >= 0 && dom < c->a.max_domains && c->phi_valid[dom]) ? c->phi[dom] : 0ull;
+    for (int l = 0; l < c->L; ++l)
+      if (!((m >> l) & 1ull)) runs |= 1ull << l;
+  }
+  *out = __builtin_popcountll(runs);
+  return TSS_OK;
+}
+
+}  // extern "C"
+
+namespace {
+
+tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache* kv, const tss_verify_result* res,
+                       cudaStream_t s, Prof* prof) {
+  if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
+  const int ri = c->ring_i;
+  if (c->ring_used[ri]) TSS_CU(cudaEventSynchronize(c->ring_ev[ri]));
+  StepDesc* sd = c->h_ring[ri];
+  StepPlan sp;
+  TSS_TRY(prepare_step(c, bt, kv, res, sd, &sp));
+  const int M = sp.M, B = sp.B;
+  const bool host_io = bt->io_host != 0;
+  if (host_io) {
+    sd->tokens = c->io_tokens;
+    sd->draft_probs = bt->mode == TSS_MODE_SAMPLE ? c->io_probs : nullptr;
+    sd->uniforms = (bt->mode == TSS_MODE_SAMPLE && bt->uniforms) ? c->io_unif : nullptr;
+    sd->accept_len = c->io_res;
+    sd->bonus = c->io_res + kMaxBatch;
+    sd->new_ctx = c->io_res + 2 * kMaxBatch;
+    sd->path = c->io_res + 3 * kMaxBatch;
+  } else {
+    sd->tokens = bt->tokens;
+    sd->draft_probs = bt->draft_probs;
+    sd->uniforms = bt->uniforms;
+    sd->accept_len = res->accept_len;
+    sd->bonus = res->bonus;
+    sd->new_ctx = res->new_ctx_len;
+    sd->path = res->path;
+  }
+  // logits: the caller's buffer, else (sampling needs them) the workspace, else none
+  float* logits_dev = (res->logits && !host_io) ? res->logits : nullptr;
+  if (!logits_dev && (bt->mode == TSS_MODE_SAMPLE || (host_io && res->logits))) logits_dev = c->logits_ws;
+  sd->logits = logits_dev;
+
+  TSS_CU(cudaMemcpyAsync(c->d_step, sd, sizeof(StepDesc), cudaMemcpyHostToDevice, s));
+  TSS_CU(cudaEventRecord(c->ring_ev[ri], s));
+  c->ring_used[ri] = true;
+  c->ring_i = (ri + 1) % kRing;
+  if (host_io) {
+    TSS_CU(cudaMemcpyAsync(c->io_tokens, bt->tokens, sizeof(int) * M, cudaMemcpyHostToDevice, s));
+    if (bt->mode == TSS_MODE_SAMPLE) {
+      TSS_CU(cudaMemcpyAsync(c->io_probs, bt->draft_probs, sizeof(float) * M * c->V, cudaMemcpyHostToDevice, s));
+      if (bt->uniforms)
+        TSS_CU(cudaMemcpyAsync(c->io_unif, bt->uniforms, sizeof(float) * B * bt->uniform_stride, cudaMemcpyHostToDevice, s));
+    }
+  }
+  if (prof) {
+    prof->s = s;
+    TSS_TRY(enqueue_step(c, sp, s, prof));
+  } else if (c->use_graphs) {
+    const GraphKey key{sp.B, sp.M, sp.n_act, sp.mode, sp.splits};
+    auto it = c->graphs.find(key);
+    if (it == c->graphs.end()) {
+      cudaGraph_t graph = nullptr;
+      TSS_CU(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal));
+      tss_status st = enqueue_step(c, sp, c->cap_stream);
+      cudaError_t ce = cudaStreamEndCapture(c->cap_stream, &graph);
+      if (st != TSS_OK) {
+        if (graph) cudaGraphDestroy(graph);
+        return st;
+      }
+      if (ce != cudaSuccess) return fail(TSS_ERR_CUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
+      cudaGraphExec_t exec = nullptr;
+      ce = cudaGraphInstantiate(&exec, graph, 0);
+      cudaGraphDestroy(graph);
+      if (ce != cudaSuccess) return fail(TSS_ERR_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
+      it = c->graphs.emplace(key, exec).first;
+    }
+    TSS_CU(cudaGraphLaunch(it->second, s));
+  } else {
+    TSS_TRY(enqueue_step(c, sp, s));
+  }
+  if (host_io) {
+    TSS_CU(cudaMemcpyAsync(res->accept_len, c->io_res, sizeof(int) * B, cudaMemcpyDeviceToHost, s));
+    TSS_CU(cudaMemcpyAsync(res->bonus, c->io_res + kMaxBatch, sizeof(int) * B, cudaMemcpyDeviceToHost, s));
+    TSS_CU(cudaMemcpyAsync(res->new_ctx_len, c->io_res + 2 * kMaxBatch, sizeof(int) * B, cudaMemcpyDeviceToHost, s));
+    TSS_CU(cudaMemcpyAsync(res->path, c->io_res + 3 * kMaxBatch, sizeof(int) * B * res->path_stride,
+                           cudaMemcpyDeviceToHost, s));
+    if (res->logits)
+      TSS_CU(cudaMemcpyAsync(res->logits, c->logits_ws, sizeof(float) * M * c->V, cudaMemcpyDeviceToHost, s));
+  }
+  return TSS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+tss_status tss_verify(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache* kv, const tss_verify_result* res,
+                      void* stream) {
+  return verify_impl(c, bt, kv, res, static_cast<cudaStream_t>(stream), nullptr);
+}
+
+tss_status tss_verify_profiled(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache* kv,
+                               const tss_verify_result* res, void* stream, tss_kernel_times* times) {
+  if (!times) return fail(TSS_ERR_INVALID_ARG, "times is NULL");
+  Prof prof;
+  tss_status st = verify_impl(c, bt, kv, res, static_cast<cudaStream_t>(stream), &prof);
+  if (st == TSS_OK) {
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) st = fail(TSS_ERR_CUDA, std::string("cudaStreamSynchronize: ") + cudaGetErrorString(e));
+  }
+  for (size_t i = 0; st == TSS_OK && i + 1 < prof.ev.size(); i += 2) {
+    float ms = 0.f;
+    cudaError_t e = cudaEventElapsedTime(&ms, prof.ev[i], prof.ev[i + 1]);
+    if (e != cudaSuccess) {
+      st = fail(TSS_ERR_CUDA, std::string("cudaEventElapsedTime: ") + cudaGetErrorString(e));
+      break;
+    }
+    const int k = prof.kind[i];
+    if (k >= 0 && k < TSS_KERNEL_KINDS) {
+      times->ms[k] += ms;
+      times->launches[k] += 1;
+    }
+  }
+  for (cudaEvent_t e : prof.ev) cudaEventDestroy(e);
+  return st;
+}
+
+tss_status tss_sync_status(tss_ctx* c, void* stream) {
+  if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  TSS_CU(cudaMemcpyAsync(c->h_status, c->d_status, sizeof(int), cudaMemcpyDeviceToHost, s));
+  TSS_CU(cudaMemsetAsync(c->d_status, 0, sizeof(int), s));
+  TSS_CU(cudaStreamSynchronize(s));
+  const int v = *c->h_status;
+  if (v != 0) return fail(v, std::string("device status: ") + tss_status_string(v));
+  return TSS_OK;
+}
+
+tss_status tss_linear(tss_ctx* c, const void* x, const void* w, float* y, int m_rows, int k_dim, int n_out, void* stream) {
+  if (!c || !x || !w || !y) return fail(TSS_ERR_INVALID_ARG, "NULL argument");
+  if (m_rows < 1 || m_rows > kMaxRows || m_rows > c->a.max_rows) return fail(TSS_ERR_INVALID_ARG, "m_rows out of range");
+  if (k_dim < 64 || k_dim % 64 != 0) return fail(TSS_ERR_INVALID_ARG, "k_dim must be a positive multiple of 64");
+  if (n_out < 128 || n_out % 128 != 0) return fail(TSS_ERR_INVALID_ARG, "n_out must be a positive multiple of 128");
+  if (!aligned16(x) || !aligned16(w)) return fail(TSS_ERR_INVALID_ARG, "x and w must be 16-byte aligned");
+  const int n_pad = pad_to(m_rows, 16);
+  CUtensorMap tx, tw;
+  if (!make_tmap(&tx, x, k_dim, m_rows, 1, n_pad, 2) || !make_tmap(&tw, w, k_dim, n_out, 1, 128, 3))
+    return fail(TSS_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+  GemmParams g = gemm_base(c, n_pad);
+  g.slot = -1;
+  g.m_raw = m_rows;
+  g.layer_fixed = 0;
+  g.out = y;
+  g.out_ld = n_out;
+  g.o_real = n_out;
+  g.step = nullptr;
+  return run_gemm(c, kEpiStore, tw, tx, g, n_out / 128, k_dim / 64, static_cast<cudaStream_t>(stream), false);
+}
+
+}  // extern "C"

@@ -1,0 +1,115 @@
+// Host-visible launch interfaces shared by the library's translation units.
+#pragma once
+
+#include <utility>
+
+#include "common.cuh"
+
+namespace tss {
+
+// Fused epilogues of the weight-streaming GEMM.
+enum Epi : int {
+  kEpiStore = 0,   // y[row][o] = acc (fp32), plain linear layer
+  kEpiQkv = 1,     // RoPE on q/k, q -> bf16 buffer, k/v -> bf16 KV cache rows (KV append)
+  kEpiResid = 2,   // h[row][o] += acc (O projection, down projection)
+  kEpiSwiglu = 3,  // act[row][f] = bf16(silu(gate) * up) for interleaved gate/up tiles
+  kEpiLmHead = 4,  // logits[row][v] (fp32, optional) + per-tile argmax partials
+};
+
+struct GemmParams {
+  int n_tiles;      // output tiles of 128 weight rows
+  int kb;           // k-blocks of 64 per tile
+  int n_pad;        // MMA N = token rows padded to a multiple of 16 (<= 256)
+  int stages;       // smem pipeline depth
+  int n_acc_bufs;   // TMEM accumulator buffers (1 or 2)
+  int slot;         // plan slot whose compacted rows feed the GEMM; -1: plain rows [0, m_raw)
+  int m_raw;
+  int layer_fixed;  // >= 0: TMA layer coordinate; -1: plan->act_layer[slot]
+  const PlanDev* plan;
+  const StepDesc* step;
+  float* partials;  // stream-K partial tiles [(grid + n_tiles) * 128 * n_pad]
+  int* counters;    // per-tile arrival counters (self-resetting)
+  int* status;
+  float* out;       // kEpiStore
+  int out_ld;
+  int o_real;
+  float* h;         // kEpiResid: residual [kMaxRows][d_model]
+  __nv_bfloat16* q_out;    // kEpiQkv: [kMaxRows][d_model]
+  __nv_bfloat16* act_out;  // kEpiSwiglu: [kMaxRows][act_ld]
+  int act_ld;
+  const float* rope_cos;   // [max_positions][head_dim / 2]
+  const float* rope_sin;
+  float* amax_val;  // kEpiLmHead: [n_tiles][kMaxRows]
+  int* amax_idx;
+  int d_model, n_heads, head_dim, vocab;
+};
+
+size_t gemm_smem_bytes(int n_pad, int stages);
+__host__ __device__ uint32_t gemm_tmem_cols(int n_pad, int n_acc_bufs);
+cudaError_t gemm_prepare(size_t max_smem);
+cudaError_t launch_gemm(int epi, const CUtensorMap& tmW, const CUtensorMap& tmX, const GemmParams& p, int grid,
+                        size_t smem, cudaStream_t s, bool pdl);
+
+struct AttnParams {
+  int slot, n_splits, n_heads, d_model, head_dim;
+  float scale_log2;  // log2(e) / sqrt(head_dim)
+  const PlanDev* plan;
+  const StepDesc* step;
+  const __nv_bfloat16* q;  // [kMaxRows][d_model] compacted rows of the slot
+  __nv_bfloat16* o;        // [kMaxRows][d_model]
+  float* part_o;           // [B][H][n_splits][kMaxNodes][head_dim]
+  float* part_ml;          // [B][H][n_splits][kMaxNodes][2]
+  int* counters;           // [B][H], self-resetting
+  int* status;
+};
+size_t attn_smem_bytes(int head_dim);
+cudaError_t attn_prepare();
+cudaError_t launch_attention(const AttnParams& p, int B, cudaStream_t s, bool pdl);
+
+struct MiscParams {
+  const StepDesc* step;
+  PlanDev* plan;
+  const unsigned long long* phi_mask;
+  const int* phi_valid;
+  int max_domains, n_layers, d_model, n_heads, head_dim, vocab;
+  float rms_eps;
+  const __nv_bfloat16* embed;   // [vocab][d]
+  float* h;                     // [kMaxRows][d]
+  __nv_bfloat16* xn;            // [kMaxRows][d]
+  const float* g_attn;          // [L][d]
+  const float* g_mlp;           // [L][d]
+  const float* g_final;         // [d]
+  const float* amax_val;        // [n_vtiles][kMaxRows]
+  const int* amax_idx;
+  int n_vtiles;
+  int* status;
+};
+
+cudaError_t launch_controller(const MiscParams& p, cudaStream_t s, bool pdl);
+cudaError_t launch_embed(const MiscParams& p, int M, cudaStream_t s, bool pdl);
+// which: 0 = attention norm of the slot's layer, 1 = MLP norm, 2 = final norm (slot ignored)
+cudaError_t launch_rmsnorm(const MiscParams& p, int slot, int which, int M, cudaStream_t s, bool pdl);
+cudaError_t launch_accept_greedy(const MiscParams& p, int B, cudaStream_t s, bool pdl);
+cudaError_t launch_accept_sample(const MiscParams& p, int B, cudaStream_t s, bool pdl);
+cudaError_t launch_compact(const MiscParams& p, int B, int n_act, cudaStream_t s, bool pdl);
+cudaError_t launch_bf16_to_f32(const __nv_bfloat16* src, float* dst, size_t n, cudaStream_t s);
+
+// Launch with optional programmatic dependent launch (the kernel may start while the previous
+// kernel in the stream finishes; it calls griddepcontrol.wait before touching its outputs).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl,
+                     Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+}  // namespace tss

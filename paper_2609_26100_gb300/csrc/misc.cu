@@ -1,0 +1,395 @@
+// Row-wise and per-request kernels of the verification step: the skip controller, embedding
+// gather, RMSNorm, acceptance (greedy walk or speculative sampling) and KV compaction.
+#include "internal.h"
+
+namespace tss {
+
+// ------------------------------------------------------------------------------------------
+// Skip controller (Sec. "Domain-Aware Skip Controller", first equation; Sec.
+// "Domain-to-Configuration Mapping"): S(x) = Phi(d(x)) if the domain is configured, else the
+// empty set.  From the requests' skip sets it builds, on the device, the ascending list of layers
+// that at least one request runs (the only layers that get launches) and, per layer, the
+// compacted list of rows of the requests that run it.
+// ------------------------------------------------------------------------------------------
+__global__ void controller_kernel(const MiscParams p) {
+  griddep_wait();
+  griddep_launch();
+  const StepDesc* st = p.step;
+  PlanDev* pl = p.plan;
+  __shared__ unsigned long long smask[kMaxBatch];
+  __shared__ int sact[kMaxLayers];
+  __shared__ int s_n;
+  const int B = st->B, L = p.n_layers;
+  for (int b = threadIdx.x; b < B; b += blockDim.x) {
+    const int dom = st->req_domain[b];
+    const unsigned long long m =
+        (dom >= 0 && dom < p.max_domains && p.phi_valid[dom]) ? p.phi_mask[dom] : 0ull;  // dense fallback
+    smask[b] = m;
+    pl->req_mask[b] = m;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int n = 0;
+    for (int l = 0; l < L; ++l) {
+      bool any = false;
+      for (int b = 0; b < B; ++b) any = any || !((smask[b] >> l) & 1ull);
+      if (any) sact[n++] = l;
+    }
+    s_n = n;
+    pl->n_act = n;
+    for (int j = 0; j < n; ++j) pl->act_layer[j] = sact[j];
+    if (n != st->n_act_host) report(p.status, kStatusCheck);
+  }
+  __syncthreads();
+  for (int j = threadIdx.x; j <= s_n; j += blockDim.x) {
+    const bool final_slot = j == s_n;
+    const int slot = final_slot ? kFinalSlot : j;
+    const int l = final_slot ? -1 : sact[j];
+    int crow = 0;
+    for (int b = 0; b < B; ++b) {
+      const bool runs = final_slot || !((smask[b] >> l) & 1ull);
+      if (runs) {
+        pl->slot_crow[slot][b] = crow;
+        const int n = st->req_nodes[b], r0 = st->req_rowoff[b];
+        for (int i = 0; i < n; ++i) pl->slot_rows[slot][crow + i] = r0 + i;
+        crow += n;
+      } else {
+        pl->slot_crow[slot][b] = -1;
+      }
+    }
+    pl->slot_M[slot] = crow;
+  }
+}
+
+// h[m] = E[token[m]] (fp32 residual stream).
+__global__ void embed_kernel(const MiscParams p) {
+  griddep_wait();
+  griddep_launch();
+  const StepDesc* st = p.step;
+  const int m = blockIdx.x;
+  if (m >= st->M) return;
+  int tok = st->tokens[m];
+  if (tok < 0 || tok >= p.vocab) {
+    if (threadIdx.x == 0) report(p.status, kStatusCheck);
+    tok = 0;
+  }
+  const __nv_bfloat16* e = p.embed + static_cast<size_t>(tok) * p.d_model;
+  float* h = p.h + static_cast<size_t>(m) * p.d_model;
+  for (int i = threadIdx.x; i < p.d_model; i += blockDim.x) h[i] = __bfloat162float(e[i]);
+}
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  if (lane == 0) red[w] = v;
+  __syncthreads();
+  float t = 0.f;
+  for (int i = 0; i < nw; ++i) t += red[i];
+  __syncthreads();
+  return t;
+}
+
+// xn[n] = bf16(h[row_n] / sqrt(mean(h^2) + eps) * g) for the compacted rows n of a slot.
+__global__ void rmsnorm_kernel(const MiscParams p, int slot, int which) {
+  griddep_wait();
+  griddep_launch();
+  __shared__ float red[32];
+  const PlanDev* pl = p.plan;
+  const int n = blockIdx.x;
+  const bool final_slot = which == 2;
+  const int sl = final_slot ? kFinalSlot : slot;
+  if (!final_slot && slot >= pl->n_act) return;
+  if (n >= pl->slot_M[sl]) return;
+  const int m = pl->slot_rows[sl][n];
+  const int d = p.d_model;
+  const float* g = final_slot ? p.g_final : (which == 0 ? p.g_attn : p.g_mlp) + static_cast<size_t>(pl->act_layer[slot]) * d;
+  const float* h = p.h + static_cast<size_t>(m) * d;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) ss += h[i] * h[i];
+  ss = block_sum(ss, red);
+  const float rs = rsqrtf(ss / static_cast<float>(d) + p.rms_eps);
+  __nv_bfloat16* x = p.xn + static_cast<size_t>(n) * d;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) x[i] = __float2bfloat16_rn(h[i] * rs * g[i]);
+}
+
+// ------------------------------------------------------------------------------------------
+// Acceptance.  Greedy (temperature 0, Sec. "Evaluation Protocol"): from the root, step to the
+// lowest-index child whose token equals the argmax of the current row while one exists; the
+// bonus is the argmax of the last row reached.  Argmax ties go to the lowest token id.
+// ------------------------------------------------------------------------------------------
+__device__ void write_result(const MiscParams& p, int b, int a, int bonus, const int* path) {
+  const StepDesc* st = p.step;
+  st->accept_len[b] = a;
+  st->bonus[b] = bonus;
+  st->new_ctx[b] = st->req_ctx[b] + 1 + a;
+  for (int i = 0; i < st->path_stride; ++i) st->path[static_cast<size_t>(b) * st->path_stride + i] = i <= a ? path[i] : -1;
+  p.plan->res_accept[b] = a;
+  for (int i = 0; i <= a; ++i) p.plan->res_path[b][i] = path[i];
+}
+
+__global__ void accept_greedy_kernel(const MiscParams p) {
+  griddep_wait();
+  griddep_launch();
+  const StepDesc* st = p.step;
+  const int b = blockIdx.x;
+  if (b >= st->B) return;
+  __shared__ int am[kMaxNodes];
+  __shared__ int path[kMaxNodes];
+  const int N = st->req_nodes[b], off = st->req_rowoff[b];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  for (int i = warp; i < N; i += nw) {
+    float bv = -INFINITY;
+    int bi = 0x7fffffff;
+    for (int t = lane; t < p.n_vtiles; t += 32) {
+      const float v = p.amax_val[static_cast<size_t>(t) * kMaxRows + off + i];
+      const int ix = p.amax_idx[static_cast<size_t>(t) * kMaxRows + off + i];
+      if (v > bv || (v == bv && ix < bi)) {
+        bv = v;
+        bi = ix;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (ov > bv || (ov == bv && oi < bi)) {
+        bv = ov;
+        bi = oi;
+      }
+    }
+    if (lane == 0) am[i] = bi;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int cur = 0, a = 0;
+    path[0] = 0;
+    while (true) {
+      const int want = am[cur];
+      int nxt = -1;
+      for (int c = cur + 1; c < N; ++c) {
+        if (st->row_parent[off + c] == cur && st->tokens[off + c] == want) {
+          nxt = c;
+          break;
+        }
+      }
+      if (nxt < 0) break;
+      cur = nxt;
+      path[++a] = cur;
+    }
+    write_result(p, b, a, am[cur], path);
+  }
+}
+
+// Philox4x32-10 (Salmon et al., SC'11): 10 rounds of the 4x32 Philox round with key bumps.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+__device__ __forceinline__ double draw_uniform(const StepDesc* st, int b, int slot) {
+  if (st->uniforms) return static_cast<double>(st->uniforms[static_cast<size_t>(b) * st->uniform_stride + slot]);
+  const uint4 x = philox4x32_10(make_uint4(static_cast<uint32_t>(slot), static_cast<uint32_t>(b), st->off_lo, st->off_hi),
+                                st->seed_lo, st->seed_hi);
+  return static_cast<double>(x.x >> 8) * (1.0 / 16777216.0);
+}
+
+template <typename T, typename Op>
+__device__ __forceinline__ T block_reduce(T v, T* red, Op op) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v = op(v, __shfl_xor_sync(0xffffffffu, v, off));
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  if (lane == 0) red[w] = v;
+  __syncthreads();
+  T t = red[0];
+  for (int i = 1; i < nw; ++i) t = op(t, red[i]);
+  __syncthreads();
+  return t;
+}
+
+// Inverse CDF over token ids in ascending order: the smallest v whose running sum of w exceeds
+// u * sum(w).  Each thread owns a contiguous chunk; chunk sums are scanned in thread order.
+template <typename WFn>
+__device__ int inverse_cdf_block(int V, double u, WFn w, double* scan) {
+  const int nt = blockDim.x, t = threadIdx.x;
+  const int C = (V + nt - 1) / nt;
+  const int v0 = min(V, t * C), v1 = min(V, v0 + C);
+  double local = 0.0;
+  for (int v = v0; v < v1; ++v) local += w(v);
+  scan[t] = local;
+  __syncthreads();
+  if (t == 0) {
+    double run = 0.0;
+    for (int i = 0; i < nt; ++i) {
+      const double x = scan[i];
+      scan[i] = run;
+      run += x;
+    }
+    scan[nt] = run;
+  }
+  __syncthreads();
+  __shared__ int sel;
+  if (t == 0) sel = -1;
+  __syncthreads();
+  const double total = scan[nt];
+  const double target = u * total;
+  const double lo = scan[t], hi = (t + 1 < nt) ? scan[t + 1] : total;
+  if (local > 0.0 && lo <= target && (target < hi || t + 1 == nt || hi >= total)) {
+    double run = lo;
+    int pick = -1, last_pos = -1;
+    for (int v = v0; v < v1; ++v) {
+      const double x = w(v);
+      if (x > 0.0) last_pos = v;
+      run += x;
+      if (run > target && x > 0.0) {
+        pick = v;
+        break;
+      }
+    }
+    if (pick < 0) pick = last_pos;
+    atomicCAS(&sel, -1, pick);
+  }
+  __syncthreads();
+  int r = sel;
+  if (r < 0) {  // target at or beyond the total: the last token with positive mass
+    __shared__ int lastv;
+    if (t == 0) lastv = -1;
+    __syncthreads();
+    for (int v = v1 - 1; v >= v0; --v)
+      if (w(v) > 0.0) {
+        atomicMax(&lastv, v);
+        break;
+      }
+    __syncthreads();
+    r = lastv < 0 ? 0 : lastv;
+  }
+  __syncthreads();
+  return r;
+}
+
+// Speculative sampling on a chain draft (rule of the speculative-decoding works the paper cites
+// as its base methods): p_i = softmax(logits_i / T); accept draft x_i iff r_i * q_i(x_i) <
+// p_{i-1}(x_i); at the first rejection draw the bonus from normalise(max(0, p_{i-1} - q_i));
+// if every draft is accepted draw it from p_k.  Uniform slots: r_i at i-1, u_i at k+i-1.
+__global__ void accept_sample_kernel(const MiscParams p) {
+  griddep_wait();
+  griddep_launch();
+  const StepDesc* st = p.step;
+  const int b = blockIdx.x;
+  if (b >= st->B) return;
+  __shared__ double scan[1025];
+  __shared__ double redd[32];
+  __shared__ int path[kMaxNodes];
+  const int N = st->req_nodes[b], off = st->req_rowoff[b], k = N - 1, V = p.vocab;
+  const double invT = static_cast<double>(st->inv_temperature);
+  auto dmax = [](double a, double c) { return a > c ? a : c; };
+  auto dsum = [](double a, double c) { return a + c; };
+  int a = 0, bonus = 0;
+  for (int i = 0; i < N; ++i) path[i] = i;
+  for (int i = 1; i <= k + 1; ++i) {
+    const float* lg = st->logits + static_cast<size_t>(off + i - 1) * V;
+    double mx = -INFINITY;
+    for (int v = threadIdx.x; v < V; v += blockDim.x) mx = dmax(mx, static_cast<double>(lg[v]));
+    mx = block_reduce(mx, redd, dmax);
+    double z = 0.0;
+    for (int v = threadIdx.x; v < V; v += blockDim.x) z += exp((static_cast<double>(lg[v]) - mx) * invT);
+    z = block_reduce(z, redd, dsum);
+    auto pr = [&](int v) { return exp((static_cast<double>(lg[v]) - mx) * invT) / z; };
+    if (i <= k) {
+      const int x = st->tokens[off + i];
+      const float* q = st->draft_probs + static_cast<size_t>(off + i) * V;
+      if (x < 0 || x >= V) {
+        if (threadIdx.x == 0) report(p.status, kStatusCheck);
+        a = i - 1;
+        bonus = 0;
+        break;
+      }
+      const double qx = static_cast<double>(q[x]);
+      if (!(qx > 0.0) && threadIdx.x == 0) report(p.status, kStatusCheck);
+      const double r = draw_uniform(st, b, i - 1);
+      if (r * qx < pr(x)) continue;  // accept draft i
+      const double u = draw_uniform(st, b, k + i - 1);
+      bonus = inverse_cdf_block(V, u, [&](int v) {
+        const double d = pr(v) - static_cast<double>(q[v]);
+        return d > 0.0 ? d : 0.0;
+      }, scan);
+      a = i - 1;
+      break;
+    }
+    const double u = draw_uniform(st, b, 2 * k);
+    bonus = inverse_cdf_block(V, u, pr, scan);
+    a = k;
+  }
+  if (threadIdx.x == 0) write_result(p, b, a, bonus, path);
+}
+
+// ------------------------------------------------------------------------------------------
+// KV compaction: for every layer the request ran, cache rows ctx + path[j] move to ctx + j,
+// j = 1..a (the root's row stays).  path[j] > j - 1 and increasing, so copying j in increasing
+// order never overwrites a row that a later j still reads.  Chains leave the cache unchanged.
+// ------------------------------------------------------------------------------------------
+__global__ void compact_kernel(const MiscParams p) {
+  griddep_wait();
+  griddep_launch();
+  const StepDesc* st = p.step;
+  const PlanDev* pl = p.plan;
+  const int head = blockIdx.x, b = blockIdx.y, j = blockIdx.z;
+  if (b >= st->B || j >= pl->n_act || pl->slot_crow[j][b] < 0) return;
+  const int a = pl->res_accept[b];
+  if (a <= 0) return;
+  const int D = p.head_dim, H = p.n_heads;
+  const size_t cap = static_cast<size_t>(st->kv_cap);
+  __nv_bfloat16* K = st->kv_layer[pl->act_layer[j]] + ((static_cast<size_t>(st->req_slot[b]) * 2) * H + head) * cap * D;
+  __nv_bfloat16* Vv = K + static_cast<size_t>(H) * cap * D;
+  const size_t ctx = static_cast<size_t>(st->req_ctx[b]);
+  for (int jj = 1; jj <= a; ++jj) {
+    const int src = pl->res_path[b][jj];
+    if (src == jj) continue;
+    for (int dd = threadIdx.x; dd < D; dd += blockDim.x) {
+      K[(ctx + jj) * D + dd] = K[(ctx + src) * D + dd];
+      Vv[(ctx + jj) * D + dd] = Vv[(ctx + src) * D + dd];
+    }
+  }
+}
+
+__global__ void bf16_to_f32_kernel(const __nv_bfloat16* src, float* dst, size_t n) {
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x)
+    dst[i] = __bfloat162float(src[i]);
+}
+
+cudaError_t launch_controller(const MiscParams& p, cudaStream_t s, bool pdl) {
+  return launch_k(controller_kernel, dim3(1), dim3(128), 0, s, pdl, p);
+}
+cudaError_t launch_embed(const MiscParams& p, int M, cudaStream_t s, bool pdl) {
+  return launch_k(embed_kernel, dim3(M), dim3(256), 0, s, pdl, p);
+}
+cudaError_t launch_rmsnorm(const MiscParams& p, int slot, int which, int M, cudaStream_t s, bool pdl) {
+  return launch_k(rmsnorm_kernel, dim3(M), dim3(256), 0, s, pdl, p, slot, which);
+}
+cudaError_t launch_accept_greedy(const MiscParams& p, int B, cudaStream_t s, bool pdl) {
+  return launch_k(accept_greedy_kernel, dim3(B), dim3(256), 0, s, pdl, p);
+}
+cudaError_t launch_accept_sample(const MiscParams& p, int B, cudaStream_t s, bool pdl) {
+  return launch_k(accept_sample_kernel, dim3(B), dim3(1024), 0, s, pdl, p);
+}
+cudaError_t launch_compact(const MiscParams& p, int B, int n_act, cudaStream_t s, bool pdl) {
+  if (n_act <= 0) n_act = 1;
+  return launch_k(compact_kernel, dim3(p.n_heads, B, n_act), dim3(128), 0, s, pdl, p);
+}
+cudaError_t launch_bf16_to_f32(const __nv_bfloat16* src, float* dst, size_t n, cudaStream_t s) {
+  const int blocks = static_cast<int>((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
+  bf16_to_f32_kernel<<<blocks > 0 ? blocks : 1, 256, 0, s>>>(src, dst, n);
+  return cudaGetLastError();
+}
+
+}  // namespace tss

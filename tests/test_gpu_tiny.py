@@ -1,0 +1,391 @@
+"""GPU parity on the tiny decoder (4 layers, d 256, 4 heads x 64, MLP 688, vocab 2048): the CUDA
+path through the C ABI against the CPU oracle on the same seeded inputs."""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import tss_oracle as O
+from paper_2609_26100_gb300 import native, synth
+from tests.conftest import oracle_weights
+from tests.parity_util import assert_logits, greedy_valid, gpu_path, kv_to_torch, to_device_weights
+
+pytestmark = pytest.mark.gpu
+
+ARCH = synth.TINY
+SEED = synth.DEFAULT_SEED
+
+
+@pytest.fixture(scope="module")
+def weights():
+    from paper_2609_26100_gb300 import build
+    build.build()
+    w = synth.make_weights(ARCH)
+    return w, oracle_weights(w), to_device_weights(w)
+
+
+def make_runner(wg, n_slots=4, cap=512, **kw):
+    from paper_2609_26100_gb300.runner import TssRunner
+    return TssRunner(ARCH, wg, n_slots=n_slots, kv_cap=cap, max_batch=8, **kw)
+
+
+def upload_context(run, kv, slot):
+    for l, layer in enumerate(kv):
+        if layer is not None:
+            k, v = kv_to_torch(layer)
+            run.write_kv(l, slot, k, v)
+
+
+def greedy_ar(wo, skip, kv, root, C, n):
+    out, tok = [], root
+    for s in range(n):
+        lg, nk = O.verify_request(wo, ARCH, skip, [tok], [-1], C + s, kv)
+        kv = O.append_kv(kv, nk, [0])
+        tok = O.argmax_lowest(lg[0])
+        out.append(tok)
+    return out
+
+
+def run_step(run, reqs, **kw):
+    res = run.alloc_results(len(reqs), sum(len(r.parents) for r in reqs))
+    b = run.batch(reqs, **kw)
+    run.verify(b, res)
+    st = run.sync_status()
+    torch.cuda.synchronize()
+    return res, st
+
+
+@pytest.mark.parametrize("mask_layers", [(2,), ()])
+def test_chain_greedy_16_steps_lockstep(weights, mask_layers):
+    """Tiny config: 128-token context (oracle prefill under the mask), chain k=4 = oracle greedy
+    continuation with the token at a seeded position replaced, 16 verify steps."""
+    w, wo, wg = weights
+    wl = synth.workload_tiny(mask_layers)
+    skip = O.mask_to_set(wl.phi[0])
+    ctx = synth.uniform_ints(128, ARCH.vocab, SEED, "tiny.ctx").tolist()
+    kv = O.prefill(wo, ARCH, skip, ctx)
+    run = make_runner(wg, n_slots=1, cap=256)
+    run.set_phi(wl.phi)
+    upload_context(run, kv, 0)
+    C, k = len(ctx), 4
+    root = int(synth.uniform_ints(1, ARCH.vocab, SEED, "tiny.root").item())
+    flagged = exact = 0
+    pos_draws = synth.uniform_ints(16, k, SEED, "tiny.pos").tolist()
+    for step in range(16):
+        greedy = greedy_ar(wo, skip, kv, root, C, k)
+        j = 1 + pos_draws[step]
+        toks = [root] + greedy
+        toks[j] = (toks[j] + 1 + step) % ARCH.vocab
+        parents = synth.chain_parents(k)
+        ref, nk = O.verify_request(wo, ARCH, skip, toks, parents, C, kv)
+        a, bonus, path = O.greedy_accept(ref, toks, parents)
+        assert a == j - 1  # the replaced draft is the first mismatch
+        res, st = run_step(run, [synth.Request(C, parents, toks, 0)])
+        assert st == native.TSS_OK
+        gl = res["logits"].cpu().numpy()
+        assert_logits(gl, ref, f"step {step}")
+        ga, gb = int(res["accept_len"][0]), int(res["bonus"][0])
+        gp = gpu_path(res, 0, ga)
+        if O.greedy_flagged(ref, path):
+            flagged += 1
+            assert greedy_valid(ref, toks, parents, gp, gb)
+        else:
+            exact += 1
+            assert (ga, gb, gp) == (a, bonus, path)
+        assert int(res["new_ctx_len"][0]) == C + 1 + ga
+        # KV rows the GPU appended for the block, every layer the request runs
+        for l in nk:
+            gk = run.kv[l][0, 0, :, C:C + k + 1].float().cpu().numpy()
+            np.testing.assert_allclose(gk, np.transpose(nk[l][0], (1, 0, 2)), atol=3e-2, rtol=2e-2)
+        for l in skip:
+            assert torch.count_nonzero(run.kv[l]) == 0  # a skipped layer's cache is never written
+        # lockstep on the oracle's state
+        kv = O.append_kv(kv, nk, path)
+        for l in nk:
+            kk, vv = kv_to_torch((np.transpose(nk[l][0][path], (1, 0, 2)), np.transpose(nk[l][1][path], (1, 0, 2))))
+            run.write_kv(l, 0, kk, vv, pos0=C)
+        C += 1 + a
+        root = bonus
+    assert exact + flagged == 16 and exact >= 4
+    run.close()
+
+
+def test_tree_greedy_and_compaction(weights):
+    """60-node draft tree (branching 4,3,2,2,1,1) with a planted greedy path: per-node logits,
+    longest matching root path, and the KV compacted to that path."""
+    w, wo, wg = weights
+    skip = frozenset({1})
+    ctx = synth.uniform_ints(96, ARCH.vocab, SEED, "tree.ctx").tolist()
+    kv = O.prefill(wo, ARCH, skip, ctx)
+    run = make_runner(wg, n_slots=2, cap=256)
+    run.set_phi({3: O.set_to_mask(skip)})
+    upload_context(run, kv, 1)
+    parents = synth.eagle_tree(60, (4, 3, 2, 2, 1, 1))
+    C = len(ctx)
+    root = 11
+    greedy = greedy_ar(wo, skip, kv, root, C, 6)
+    toks = synth.draft_tokens(parents, ARCH.vocab, SEED, "tree.tok")
+    toks[0] = root
+    ch = O.children_of(parents)
+    cur = 0
+    for rank, g in zip((2, 1, 0, 1, 0, 0), greedy):
+        if len(ch[cur]) <= rank:
+            break
+        nxt = ch[cur][rank]
+        for sib in ch[cur]:
+            if toks[sib] == g:
+                toks[sib] = (g + 7) % ARCH.vocab
+        toks[nxt] = g
+        cur = nxt
+    ref, nk = O.verify_request(wo, ARCH, skip, toks, parents, C, kv)
+    a, bonus, path = O.greedy_accept(ref, toks, parents)
+    res, st = run_step(run, [synth.Request(C, parents, toks, 3)], slots=[1])
+    assert st == native.TSS_OK
+    assert_logits(res["logits"].cpu().numpy(), ref, "tree")
+    ga, gb = int(res["accept_len"][0]), int(res["bonus"][0])
+    gp = gpu_path(res, 0, ga)
+    if O.greedy_flagged(ref, path):
+        assert greedy_valid(ref, toks, parents, gp, gb)
+    else:
+        assert (ga, gb, gp) == (a, bonus, path)
+        assert a >= 2
+    for l in nk:
+        comp_k = O.compact_block_rows(nk[l][0], gp)  # oracle rows in the GPU's accepted order
+        comp_v = O.compact_block_rows(nk[l][1], gp)
+        gk = run.kv[l][1, 0, :, C:C + ga + 1].float().cpu().numpy()
+        gv = run.kv[l][1, 1, :, C:C + ga + 1].float().cpu().numpy()
+        np.testing.assert_allclose(gk, np.transpose(comp_k, (1, 0, 2)), atol=3e-2, rtol=2e-2)
+        np.testing.assert_allclose(gv, np.transpose(comp_v, (1, 0, 2)), atol=3e-2, rtol=2e-2)
+    assert torch.count_nonzero(run.kv[1][1]) == 0 and torch.count_nonzero(run.kv[0][0]) == 0
+    run.close()
+
+
+def test_mixed_domain_batch_and_untouched_skipped_kv(weights):
+    """Four requests with different skip sets (one domain never configured = dense), different
+    context lengths and draft lengths in one batch; skipped layers' KV keeps a sentinel."""
+    w, wo, wg = weights
+    phi = {0: O.set_to_mask({2}), 1: O.set_to_mask({0, 3}), 2: 0}
+    doms = [0, 1, 2, 7]
+    ctxs = [128, 77, 200, 5]
+    ks = [4, 2, 0, 3]
+    run = make_runner(wg, n_slots=4, cap=256)
+    run.set_phi(phi)
+    sentinel = 7.0
+    for t in run.kv:
+        t.fill_(sentinel)
+    reqs, kvs, skips = [], [], []
+    for b in range(4):
+        skip = O.skip_set({d: O.mask_to_set(m) for d, m in phi.items()}, doms[b])
+        ctx = synth.uniform_ints(ctxs[b], ARCH.vocab, SEED, f"mix.ctx{b}").tolist()
+        kv = O.prefill(wo, ARCH, skip, ctx)
+        upload_context(run, kv, b)
+        parents = synth.chain_parents(ks[b])
+        toks = synth.draft_tokens(parents, ARCH.vocab, SEED, f"mix.tok{b}")
+        reqs.append(synth.Request(ctxs[b], parents, toks, doms[b]))
+        kvs.append(kv)
+        skips.append(skip)
+    res, st = run_step(run, reqs)
+    assert st == native.TSS_OK
+    gl = res["logits"].cpu().numpy()
+    off = 0
+    for b, r in enumerate(reqs):
+        n = len(r.parents)
+        ref, nk = O.verify_request(wo, ARCH, skips[b], r.tokens, r.parents, r.ctx_len, kvs[b])
+        assert_logits(gl[off:off + n], ref, f"request {b}")
+        a, bonus, path = O.greedy_accept(ref, r.tokens, r.parents)
+        if not O.greedy_flagged(ref, path):
+            assert (int(res["accept_len"][b]), int(res["bonus"][b])) == (a, bonus)
+        for l in range(ARCH.n_layers):
+            region = run.kv[l][b]
+            if l in skips[b]:
+                assert bool((region == sentinel).all()), f"request {b} skipped layer {l} was touched"
+            else:
+                assert bool((region[:, :, r.ctx_len + n:] == sentinel).all())
+        off += n
+    run.close()
+
+
+def test_all_layers_skipped_is_embedding_norm_lm_head(weights):
+    w, wo, wg = weights
+    run = make_runner(wg, n_slots=1, cap=64)
+    run.set_phi({0: (1 << ARCH.n_layers) - 1})
+    parents = synth.chain_parents(3)
+    toks = [5, 17, 2047, 0]
+    res, st = run_step(run, [synth.Request(10, parents, toks, 0)])
+    assert st == native.TSS_OK
+    ref, nk = O.verify_request(wo, ARCH, frozenset(range(ARCH.n_layers)), toks, parents, 10, [None] * 4)
+    assert nk == {}
+    assert_logits(res["logits"].cpu().numpy(), ref, "all skipped")
+    for t in run.kv:
+        assert torch.count_nonzero(t) == 0
+    run.close()
+
+
+def test_root_only_and_empty_context(weights):
+    w, wo, wg = weights
+    run = make_runner(wg, n_slots=2, cap=64)
+    reqs = [synth.Request(0, [-1], [42], 0), synth.Request(0, synth.chain_parents(2), [1, 2, 3], 0)]
+    res, st = run_step(run, reqs)
+    assert st == native.TSS_OK
+    gl = res["logits"].cpu().numpy()
+    empty = [O.empty_kv(ARCH) for _ in range(4)]
+    r0, _ = O.verify_request(wo, ARCH, frozenset(), [42], [-1], 0, empty)
+    r1, _ = O.verify_request(wo, ARCH, frozenset(), [1, 2, 3], [-1, 0, 1], 0, empty)
+    assert_logits(gl[:1], r0, "root only")
+    assert_logits(gl[1:], r1, "empty context")
+    assert int(res["accept_len"][0]) == 0 and int(res["new_ctx_len"][0]) == 1
+    run.close()
+
+
+def test_speculative_sampling_chain(weights):
+    """B=3 chains (k=4, 1, 3) at temperature 1 with Philox uniforms and with caller uniforms."""
+    w, wo, wg = weights
+    run = make_runner(wg, n_slots=3, cap=256)
+    run.set_phi({0: O.set_to_mask({1}), 1: 0})
+    ks, ctxs, doms = [4, 1, 3], [64, 33, 90], [0, 1, 0]
+    reqs, kvs, skips, qs = [], [], [], []
+    for b in range(3):
+        skip = frozenset({1}) if doms[b] == 0 else frozenset()
+        ctx = synth.uniform_ints(ctxs[b], ARCH.vocab, SEED, f"samp.ctx{b}").tolist()
+        kv = O.prefill(wo, ARCH, skip, ctx)
+        upload_context(run, kv, b)
+        q, samp = synth.draft_probs_and_samples(ks[b] + 1, ARCH.vocab, SEED, f"samp.q{b}")
+        toks = [int(synth.uniform_ints(1, ARCH.vocab, SEED, f"samp.root{b}").item())] + samp[1:]
+        reqs.append(synth.Request(ctxs[b], synth.chain_parents(ks[b]), toks, doms[b], q))
+        kvs.append(kv)
+        skips.append(skip)
+        qs.append(q)
+    probs = torch.cat(qs, 0).cuda()
+    checked = exact = 0
+    for trial in range(6):
+        use_unif = trial % 2 == 1
+        stride = 2 * max(ks) + 1
+        unif = synth.uniform01(3 * stride, SEED, f"samp.u{trial}").float().view(3, stride)
+        kw = dict(mode=native.TSS_MODE_SAMPLE, temperature=1.0, draft_probs=probs, philox_seed=1234,
+                  philox_offset=trial)
+        if use_unif:
+            kw["uniforms"] = unif.cuda()
+        res, st = run_step(run, reqs, **kw)
+        assert st == native.TSS_OK
+        gl = res["logits"].cpu().numpy()
+        off = 0
+        for b, r in enumerate(reqs):
+            n = len(r.parents)
+            ref, _ = O.verify_request(wo, ARCH, skips[b], r.tokens, r.parents, r.ctx_len, kvs[b])
+            assert_logits(gl[off:off + n], ref, f"sample request {b}")
+            u = unif[b].double().numpy() if use_unif else O.philox_uniforms(1234, trial, b, ks[b])
+            a, bonus, path, flagged, (dw, du) = O.spec_sample_accept(ref, r.tokens, qs[b].numpy(), u, 1.0,
+                                                                      return_draw=True)
+            ga, gb = int(res["accept_len"][b]), int(res["bonus"][b])
+            if not flagged:
+                assert ga == a, f"trial {trial} req {b}: accept_len {ga} != {a}"
+                assert gb == bonus or O.draw_consistent(dw, du, gb), f"trial {trial} req {b}: bonus {gb} vs {bonus}"
+                checked += 1
+                exact += gb == bonus
+            off += n
+    assert checked >= 9 and exact >= checked // 2
+    run.close()
+
+
+def test_graph_and_eager_paths_agree_bitwise(weights):
+    w, wo, wg = weights
+    reqs = [synth.Request(40, synth.chain_parents(4), [3, 1, 4, 1, 5], 0)]
+    outs = []
+    for eager in (False, True):
+        os.environ["TSS_NO_GRAPH"] = "1" if eager else "0"
+        try:
+            run = make_runner(wg, n_slots=1, cap=64)
+        finally:
+            os.environ.pop("TSS_NO_GRAPH", None)
+        run.set_phi({0: O.set_to_mask({3})})
+        for l in range(4):
+            run.kv[l].copy_(synth.normal_bf16(run.kv[l].shape, SEED, f"ge{l}", 0.5).cuda())
+        r1, _ = run_step(run, reqs)
+        r2, _ = run_step(run, reqs)
+        assert torch.equal(r1["logits"], r2["logits"])  # deterministic
+        outs.append(r1["logits"].clone())
+        run.close()
+    assert torch.equal(outs[0], outs[1])
+
+
+def test_host_io_matches_device_io(weights):
+    w, wo, wg = weights
+    run = make_runner(wg, n_slots=2, cap=64)
+    for l in range(4):
+        run.kv[l].copy_(synth.normal_bf16(run.kv[l].shape, SEED, f"io{l}", 0.5).cuda())
+    reqs = [synth.Request(30, synth.chain_parents(3), [9, 8, 7, 6], 0), synth.Request(12, [-1, 0, 0], [1, 2, 3], 0)]
+    dev, _ = run_step(run, reqs)
+    hres = run.alloc_results(2, 7, host=True)
+    b = run.batch(reqs, io_host=True)
+    run.verify(b, hres)
+    assert run.sync_status() == native.TSS_OK
+    for key in ("accept_len", "bonus", "new_ctx_len", "path"):
+        assert torch.equal(hres[key], dev[key].cpu())
+    assert torch.equal(hres["logits"], dev["logits"].cpu())
+    run.close()
+
+
+def test_linear_matches_matmul(weights):
+    w, wo, wg = weights
+    run = make_runner(wg, n_slots=1, cap=16)
+    for m, k, n in [(1, 64, 128), (6, 256, 384), (61, 512, 640), (144, 128, 256), (256, 192, 128), (17, 4096, 1024)]:
+        x = synth.normal_bf16((m, k), SEED, f"lx{m}", 1.0).cuda()
+        wt = synth.normal_bf16((n, k), SEED, f"lw{n}", 0.05).cuda()
+        y = torch.empty((m, n), dtype=torch.float32, device="cuda")
+        run.v.linear(x, wt, y)
+        torch.cuda.synchronize()
+        ref = x.double().cpu().numpy() @ wt.double().cpu().numpy().T
+        np.testing.assert_allclose(y.cpu().numpy(), ref, rtol=1e-4, atol=1e-4, err_msg=f"{m}x{k}x{n}")
+    run.close()
+
+
+def test_host_validation_errors(weights):
+    w, wo, wg = weights
+    run = make_runner(wg, n_slots=2, cap=32)
+    res = run.alloc_results(2, 8)
+
+    def status(reqs, **kw):
+        b = run.batch(reqs, **kw)
+        try:
+            run.verify(b, res)
+            return native.TSS_OK
+        except native.TssError as e:
+            return e.status
+
+    good = synth.Request(4, [-1, 0], [1, 2], 0)
+    assert status([synth.Request(4, [-1, 1], [1, 2], 0)]) == native.TSS_ERR_INVALID_ARG  # parent not before child
+    assert status([synth.Request(4, [0, 0], [1, 2], 0)]) == native.TSS_ERR_INVALID_ARG  # root must be -1
+    assert status([synth.Request(31, [-1, 0], [1, 2], 0)]) == native.TSS_ERR_KV_CAPACITY
+    assert status([good, good], slots=[1, 1]) == native.TSS_ERR_INVALID_ARG  # shared slot
+    assert status([synth.Request(4, [-1, 0, 0], [1, 2, 3], 0)], mode=native.TSS_MODE_SAMPLE,
+                  draft_probs=torch.ones(3, ARCH.vocab, device="cuda")) == native.TSS_ERR_INVALID_ARG  # tree
+    assert status([good], mode=native.TSS_MODE_SAMPLE) == native.TSS_ERR_INVALID_ARG  # no draft probs
+    with pytest.raises(native.TssError):
+        run.v.set_skip_config(0, 1 << ARCH.n_layers)
+    assert status([good]) == native.TSS_OK
+    assert run.sync_status() == native.TSS_OK
+    run.close()
+
+
+def test_device_check_reports_bad_token(weights):
+    w, wo, wg = weights
+    run = make_runner(wg, n_slots=1, cap=32)
+    res = run.alloc_results(1, 2)
+    b = run.batch([synth.Request(4, [-1, 0], [1, ARCH.vocab + 5], 0)])
+    run.verify(b, res)
+    assert run.sync_status() == native.TSS_ERR_DEVICE_CHECK
+    assert run.sync_status() == native.TSS_OK  # cleared
+    run.close()
+
+
+def test_sparsity_ratio_and_active_layers(weights):
+    w, wo, wg = weights
+    run = make_runner(wg, n_slots=2, cap=32)
+    run.set_phi({0: O.set_to_mask({1, 3}), 1: O.set_to_mask({1})})
+    assert run.v.sparsity_ratio(0) == 0.5 and run.v.sparsity_ratio(5) == 0.0
+    b = run.batch([synth.Request(1, [-1], [1], 0), synth.Request(1, [-1], [1], 1)])
+    assert run.v.active_layer_count(b) == 3  # union: layer 1 skipped by both
+    run.v.clear_skip_config(1)
+    assert run.v.active_layer_count(b) == 4
+    run.close()

@@ -277,3 +277,10 @@ def test_stored_kv_rows_are_bf16_values(tiny_oracle_weights):
     for k, v in nk.values():
         assert np.array_equal(O.round_to_bf16(k), k) and np.array_equal(O.round_to_bf16(v), v)
         assert np.any(k != 0)
+
+
+def test_draw_consistency_check():
+    w = np.array([0.1, 0.0, 0.4, 0.5])
+    assert O.draw_consistent(w, 0.3, 2) and O.draw_consistent(w, 0.05, 0)
+    assert not O.draw_consistent(w, 0.3, 3) and not O.draw_consistent(w, 0.1, 1)  # zero mass
+    assert O.draw_consistent(w, 0.10005, 0, band=1e-4) and not O.draw_consistent(w, 0.2, 0, band=1e-4)
