@@ -36,6 +36,8 @@ def parse_args():
     p.add_argument("--impl", default="tss", choices=["tss", "reference"])
     p.add_argument("--workload", default="7b_chain", choices=["7b_chain", "7b_dense", "7b_tree", "13b_mixed", "7b_long", "tiny"])
     p.add_argument("--skip", type=int, default=None, help="7b_long: number of skipped layers (sweep point)")
+    p.add_argument("--layers", type=int, default=None,
+                   help="truncate the model to its first N layers (small profiling case; not a bench workload)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-profile", action="store_true")
@@ -248,6 +250,10 @@ def run_tss(args):
         dist.barrier()
     _build.build()  # no-op when up to date
     w = make_workload(args.workload, args.skip)
+    if args.layers:
+        import dataclasses
+        w.arch = dataclasses.replace(w.arch, n_layers=args.layers)
+        w.phi = {d: m & ((1 << args.layers) - 1) for d, m in w.phi.items()}
     a = w.arch
     union = w.active_union()
     max_ctx = max(r.ctx_len for r in w.requests)

@@ -208,9 +208,10 @@ typedef struct {
   int launches[TSS_KERNEL_KINDS]; /* launches of the kind */
 } tss_kernel_times;
 
-/* Diagnostic twin of tss_verify: the same kernels, launched one by one (no graph, no
- * programmatic overlap) with a CUDA event pair around each launch on `stream`; synchronises the
- * stream and ADDS the step's per-kind times into *times.  Results are written as by tss_verify. */
+/* Diagnostic twin of tss_verify: the same kernels without programmatic overlap, each bracketed by
+ * a CUDA event pair, captured into a one-off graph and launched on `stream` (so the events time
+ * device work only); synchronises the stream and ADDS the step's per-kind times into *times.
+ * Results are written as by tss_verify. */
 tss_status tss_verify_profiled(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
                                const tss_verify_result* result, void* stream, tss_kernel_times* times);
 

@@ -253,7 +253,7 @@ struct Prof {
     TSS_CU(cudaEventCreate(&e));
     ev.push_back(e);
     kind.push_back(k);
-    TSS_CU(cudaEventRecord(e, s));
+    TSS_CU(cudaEventRecordWithFlags(e, s, cudaEventRecordExternal));  // a record node under capture
     return TSS_OK;
   }
   tss_status end() {
@@ -261,7 +261,7 @@ struct Prof {
     TSS_CU(cudaEventCreate(&e));
     ev.push_back(e);
     kind.push_back(-1);
-    TSS_CU(cudaEventRecord(e, s));
+    TSS_CU(cudaEventRecordWithFlags(e, s, cudaEventRecordExternal));  // a record node under capture
     return TSS_OK;
   }
 };
@@ -471,6 +471,7 @@ tss_status build_workspaces(tss_ctx* c) {
   if (max_smem > 232448) max_smem = 232448;
   TSS_CU(gemm_prepare(max_smem));
   TSS_CU(attn_prepare());
+  TSS_CU(misc_prepare());
   return TSS_OK;
 }
 
@@ -753,8 +754,26 @@ tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cach
     }
   }
   if (prof) {
-    prof->s = s;
-    TSS_TRY(enqueue_step(c, sp, s, prof));
+    // Launches bracketed by events, captured into a graph so that the device runs them back to
+    // back: the events then time device work only, not host launch latency.
+    prof->s = c->cap_stream;
+    cudaGraph_t graph = nullptr;
+    TSS_CU(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal));
+    tss_status st = enqueue_step(c, sp, c->cap_stream, prof);
+    cudaError_t ce = cudaStreamEndCapture(c->cap_stream, &graph);
+    if (st != TSS_OK) {
+      if (graph) cudaGraphDestroy(graph);
+      return st;
+    }
+    if (ce != cudaSuccess) return fail(TSS_ERR_CUDA, std::string("profile capture: ") + cudaGetErrorString(ce));
+    cudaGraphExec_t exec = nullptr;
+    ce = cudaGraphInstantiate(&exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (ce != cudaSuccess) return fail(TSS_ERR_CUDA, std::string("profile instantiate: ") + cudaGetErrorString(ce));
+    ce = cudaGraphLaunch(exec, s);
+    if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
+    cudaGraphExecDestroy(exec);
+    if (ce != cudaSuccess) return fail(TSS_ERR_CUDA, std::string("profile launch: ") + cudaGetErrorString(ce));
   } else if (c->use_graphs) {
     const GraphKey key{sp.B, sp.M, sp.n_act, sp.mode, sp.splits};
     auto it = c->graphs.find(key);

@@ -421,9 +421,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   }
 }
 
+template <int EPI>
+cudaError_t gemm_max_carveout() {
+  return cudaFuncSetAttribute(gemm_kernel<EPI>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                              cudaSharedmemCarveoutMaxShared);
+}
+
 cudaError_t gemm_prepare(size_t max_smem) {
   cudaError_t e;
   const int bytes = static_cast<int>(max_smem);
+  // One shared-memory carveout for every kernel of the step: no L1/shared reconfiguration at
+  // kernel boundaries.
+  if ((e = gemm_max_carveout<kEpiStore>()) || (e = gemm_max_carveout<kEpiQkv>()) || (e = gemm_max_carveout<kEpiResid>()) ||
+      (e = gemm_max_carveout<kEpiSwiglu>()) || (e = gemm_max_carveout<kEpiLmHead>()))
+    return e;
   if ((e = cudaFuncSetAttribute(gemm_kernel<kEpiStore>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
   if ((e = cudaFuncSetAttribute(gemm_kernel<kEpiQkv>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;
   if ((e = cudaFuncSetAttribute(gemm_kernel<kEpiResid>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes))) return e;

@@ -85,6 +85,7 @@ struct MiscParams {
   int* status;
 };
 
+cudaError_t misc_prepare();
 cudaError_t launch_controller(const MiscParams& p, cudaStream_t s, bool pdl);
 cudaError_t launch_embed(const MiscParams& p, int M, cudaStream_t s, bool pdl);
 // which: 0 = attention norm of the slot's layer, 1 = MLP norm, 2 = final norm (slot ignored)

@@ -367,6 +367,17 @@ __global__ void bf16_to_f32_kernel(const __nv_bfloat16* src, float* dst, size_t 
     dst[i] = __bfloat162float(src[i]);
 }
 
+cudaError_t misc_prepare() {
+  const int c = cudaSharedmemCarveoutMaxShared;
+  const cudaFuncAttribute a = cudaFuncAttributePreferredSharedMemoryCarveout;
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(controller_kernel, a, c)) || (e = cudaFuncSetAttribute(embed_kernel, a, c)) ||
+      (e = cudaFuncSetAttribute(rmsnorm_kernel, a, c)) || (e = cudaFuncSetAttribute(accept_greedy_kernel, a, c)) ||
+      (e = cudaFuncSetAttribute(accept_sample_kernel, a, c)) || (e = cudaFuncSetAttribute(compact_kernel, a, c)))
+    return e;
+  return cudaSuccess;
+}
+
 cudaError_t launch_controller(const MiscParams& p, cudaStream_t s, bool pdl) {
   return launch_k(controller_kernel, dim3(1), dim3(128), 0, s, pdl, p);
 }
