@@ -215,6 +215,25 @@ typedef struct {
 tss_status tss_verify_profiled(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
                                const tss_verify_result* result, void* stream, tss_kernel_times* times);
 
+/* Allocation-free twin of tss_linear.  The paper has no counterpart: this entry point exists for
+ * callers that cannot allocate device memory when they run the layer -- a plugin inside a host
+ * framework that owns the whole device memory pool, a process with a memory budget fixed at
+ * start-up, or a latency-critical loop that must not call cudaMalloc/cudaFree (they can
+ * synchronise the device and stall unrelated streams).  It needs no tss_ctx and allocates
+ * nothing: the stream-K scratch (partial tiles, per-tile counters) is a file-scope device array
+ * of the library, 8 MiB + 1 KiB, held on every GPU that loads libtss.so until the process exits.
+ *   y[m][o] = sum_k x[m][k] * w[o][k]; x [m_rows][k_dim] bf16, w [n_out][k_dim] bf16,
+ *   y [m_rows][n_out] fp32, device, row-major, 16-byte aligned; m_rows in [1, 64]; k_dim a
+ *   multiple of 64; n_out a multiple of 128, at most 32768; and the scratch a problem needs,
+ *   (min(#SMs, n_out/128 * k_dim/64) + n_out/128) * 128 * pad16(m_rows) * 4 bytes, at most 8 MiB
+ *   -- larger requests return TSS_ERR_INVALID_ARG with a message.
+ * The first call on a device (per process) looks up the array's device address and sets the
+ * kernel's shared-memory limit; make that first call before any stream capture.  Every call on a
+ * device shares the one array and the next call overwrites it (the counters are cleared on
+ * `stream` at each call): calls that overlap on the GPU race, so serialise them on one stream.
+ * Asynchronous on `stream`; no device status word is reported. */
+tss_status tss_linear_static(const void* x, const void* w, float* y, int m_rows, int k_dim, int n_out, void* stream);
+
 const char* tss_status_string(tss_status s);
 /* Message of the last error reported to the calling thread ("" if none). */
 const char* tss_last_error(void);

@@ -73,6 +73,8 @@ constexpr int kMaxPathStride = 1024;
 
 }  // namespace
 
+void tss::set_last_error(const std::string& msg) { g_err = msg; }
+
 struct tss_ctx {
   tss_arch a{};
   int dev = 0, num_sms = 0;

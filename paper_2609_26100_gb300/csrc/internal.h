@@ -1,6 +1,7 @@
 // Host-visible launch interfaces shared by the library's translation units.
 #pragma once
 
+#include <string>
 #include <utility>
 
 #include "common.cuh"
@@ -94,6 +95,9 @@ cudaError_t launch_accept_greedy(const MiscParams& p, int B, cudaStream_t s, boo
 cudaError_t launch_accept_sample(const MiscParams& p, int B, cudaStream_t s, bool pdl);
 cudaError_t launch_compact(const MiscParams& p, int B, int n_act, cudaStream_t s, bool pdl);
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* src, float* dst, size_t n, cudaStream_t s);
+
+// Records the message tss_last_error() returns on the calling thread.
+void set_last_error(const std::string& msg);
 
 // Launch with optional programmatic dependent launch (the kernel may start while the previous
 // kernel in the stream finishes; it calls griddepcontrol.wait before touching its outputs).

@@ -26,7 +26,7 @@ TSS_MODE_SAMPLE = 1
 EXPORTS = (
     "tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_sync_status", "tss_destroy", "tss_linear",
-    "tss_status_string", "tss_last_error",
+    "tss_linear_static", "tss_status_string", "tss_last_error",
 )
 
 _P = ctypes.c_void_p
@@ -92,15 +92,24 @@ def lib() -> ctypes.CDLL:
         L.tss_destroy.argtypes = [_P]
         L.tss_destroy.restype = None
         L.tss_linear.argtypes = [_P, _P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P]
+        L.tss_linear_static.argtypes = [_P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P]
         L.tss_status_string.argtypes = [ctypes.c_int]
         L.tss_status_string.restype = ctypes.c_char_p
         L.tss_last_error.argtypes = []
         L.tss_last_error.restype = ctypes.c_char_p
         for name in ("tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
-                     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_sync_status", "tss_linear"):
+                     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_sync_status", "tss_linear",
+                     "tss_linear_static"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
+
+
+def linear_static(x, w, y, stream=None) -> None:
+    """y = x @ w^T through tss_linear_static (no context, no device allocation)."""
+    m, k = x.shape
+    check(lib().tss_linear_static(x.data_ptr(), w.data_ptr(), y.data_ptr(), m, k, w.shape[0], stream),
+          "tss_linear_static")
 
 
 class TssError(RuntimeError):
