@@ -199,10 +199,11 @@ tss_status tss_linear(tss_ctx* ctx, const void* x, const void* w, float* y, int 
                       int n_out, void* stream);
 
 /* Per-kernel device times of one verification step, by kernel kind:
- *   0 controller + embedding + RMSNorms, 1 QKV GEMM (+RoPE, KV append), 2 attention,
- *   3 O-projection GEMM, 4 gate/up GEMM (+SwiGLU), 5 down GEMM, 6 LM head GEMM (+argmax),
- *   7 acceptance + KV compaction. */
-#define TSS_KERNEL_KINDS 8
+ *   0 controller + embedding (+ RMSNorms on the multi-kernel path), 1 QKV GEMM (+RoPE, KV
+ *   append), 2 attention, 3 O-projection GEMM, 4 gate/up GEMM (+SwiGLU), 5 down GEMM, 6 LM head
+ *   GEMM (+argmax), 7 acceptance + KV compaction, 8 the persistent verify kernel (every active
+ *   layer and the LM head in one launch; kinds 1-6 are then empty). */
+#define TSS_KERNEL_KINDS 9
 typedef struct {
   float ms[TSS_KERNEL_KINDS];     /* summed device time of the kind's launches */
   int launches[TSS_KERNEL_KINDS]; /* launches of the kind */

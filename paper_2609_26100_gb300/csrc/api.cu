@@ -121,6 +121,15 @@ struct tss_ctx {
   cudaStream_t cap_stream = nullptr;
   bool use_graphs = true;
   int gemm_ctas_per_sm = 2;
+  // persistent verify kernel
+  bool use_mk = true;
+  unsigned long long epoch = 0;
+  float* ssp = nullptr;
+  unsigned long long* flags = nullptr;  // hflag | qkvflag | guflag | attflag
+  int* mk_zero = nullptr;               // counters [7][max_tiles] | abort word | attention counters
+  int mk_max_tiles = 0, mk_n_zero = 0;
+  float *mk_part0 = nullptr, *mk_part1 = nullptr;
+  size_t mk_part_floats = 0;
   std::vector<void*> allocs;
 
   template <typename T>
@@ -331,6 +340,96 @@ tss_status enqueue_step(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* pr
   return TSS_OK;
 }
 
+// Stages of the persistent kernel's ring that fit next to its attention buffers; 0 if none.
+int mk_stages(const tss_ctx* c, int n_pad) {
+  int s = 0;
+  while (s < 12 && mk_smem_bytes(n_pad, s + 1, c->D) <= 232448) ++s;
+  return s >= 2 ? s : 0;
+}
+
+// One verification step on the persistent path: prologue (controller, embedding, sums of
+// squares), the persistent verify kernel (all layers + LM head), finish (acceptance + KV
+// compaction).
+tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* prof) {
+  MiscParams mp = misc_params(c);
+  const int n_pad = sp.n_pad;
+  const CUtensorMap *to, *tact;
+  TSS_TRY(get_xmap(c, c->tm_o, c->obuf, c->d, n_pad, &to));
+  TSS_TRY(get_xmap(c, c->tm_act, c->act, c->F_pad, n_pad, &tact));
+  const int stages = mk_stages(c, n_pad);
+  const size_t smem = mk_smem_bytes(n_pad, stages, c->D);
+  const int nt = c->d / 128;
+  MkParams p{};
+  p.n_act = sp.n_act;
+  p.d = c->d;
+  p.H = c->H;
+  p.D = c->D;
+  p.F_pad = c->F_pad;
+  p.Ft = c->Ft;
+  p.V = c->V;
+  p.V_pad = c->V_pad;
+  p.n_pad = n_pad;
+  p.stages = stages;
+  p.attn_splits = sp.splits;
+  p.B = sp.B;
+  p.max_tiles = c->mk_max_tiles;
+  p.eps = c->a.rms_eps;
+  p.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->D)));
+  p.seq_base = ++c->epoch * 1024ull;
+  p.step = c->d_step;
+  p.plan = c->d_plan;
+  p.h = c->h;
+  p.qbuf = c->qbuf;
+  p.obuf = c->obuf;
+  p.act = c->act;
+  p.partials0 = c->mk_part0;
+  p.partials1 = c->mk_part1;
+  p.counters = c->mk_zero;
+  p.abort_word = c->mk_zero + 7 * c->mk_max_tiles;
+  p.ssp = c->ssp;
+  p.hflag = c->flags;
+  p.qkvflag = c->flags + nt;
+  p.guflag = c->flags + 4 * nt;
+  p.attflag = c->flags + 4 * nt + c->Ft;
+  p.amax_val = c->amax_val;
+  p.amax_idx = c->amax_idx;
+  p.attn_po = c->attn_po;
+  p.attn_pml = c->attn_pml;
+  p.attn_cnt = c->attn_cnt;
+  p.g_attn = c->g_attn;
+  p.g_mlp = c->g_mlp;
+  p.g_final = c->g_final;
+  p.rope_cos = c->rope_cos;
+  p.rope_sin = c->rope_sin;
+  p.status = c->d_status;
+  MkTensorMaps tm;
+  tm.qkv = c->tm_wqkv;
+  tm.o = c->tm_wo;
+  tm.gu = c->tm_wgu;
+  tm.down = c->tm_wdown;
+  tm.lm = c->tm_lm;
+  tm.xo = *to;
+  tm.xact = *tact;
+#define TSS_MK(kind, expr)                 \
+  do {                                     \
+    if (prof) TSS_TRY(prof->begin(kind));  \
+    expr;                                  \
+    if (prof) TSS_TRY(prof->end());        \
+  } while (0)
+  TSS_MK(0, TSS_CU(launch_prologue(mp, c->ssp, c->mk_zero, c->mk_n_zero, sp.M, s, false)));
+  TSS_MK(8, TSS_CU(launch_verify_mk(tm, p, c->num_sms, smem, s)));
+  TSS_MK(7, TSS_CU(launch_finish(mp, sp.B, s, false)));
+#undef TSS_MK
+  return TSS_OK;
+}
+
+bool mk_supported(const tss_ctx* c, const StepPlan& sp) {
+  if (!c->use_mk) return false;
+  const int stages = mk_stages(c, sp.n_pad);
+  if (stages < 2) return false;
+  return mk_max_blocks_per_sm(c->D, mk_smem_bytes(sp.n_pad, stages, c->D)) >= 1;
+}
+
 tss_status validate_arch(const tss_arch* a) {
   if (!a) return fail(TSS_ERR_INVALID_ARG, "arch is NULL");
   if (a->n_layers < 1 || a->n_layers > kMaxLayers) return fail(TSS_ERR_UNSUPPORTED_ARCH, "n_layers must be in [1, 64]");
@@ -473,6 +572,22 @@ tss_status build_workspaces(tss_ctx* c) {
   if (max_smem > 232448) max_smem = 232448;
   TSS_CU(gemm_prepare(max_smem));
   TSS_CU(attn_prepare());
+  TSS_CU(mk_prepare());
+  {
+    const int nt = d / 128;
+    c->mk_max_tiles = max_tiles;
+    TSS_TRY(c->alloc(&c->ssp, static_cast<size_t>(nt) * kMaxRows));
+    TSS_CU(cudaMemset(c->ssp, 0, static_cast<size_t>(nt) * kMaxRows * sizeof(float)));
+    const size_t nflags = static_cast<size_t>(nt) + 3 * nt + c->Ft + static_cast<size_t>(c->a.max_batch) * c->H;
+    TSS_TRY(c->alloc(&c->flags, nflags));
+    TSS_CU(cudaMemset(c->flags, 0, nflags * sizeof(unsigned long long)));
+    c->mk_n_zero = 7 * max_tiles + 1;
+    TSS_TRY(c->alloc(&c->mk_zero, static_cast<size_t>(c->mk_n_zero)));
+    TSS_CU(cudaMemset(c->mk_zero, 0, static_cast<size_t>(c->mk_n_zero) * sizeof(int)));
+    c->mk_part_floats = (static_cast<size_t>(c->num_sms) + max_tiles) * 128 * static_cast<size_t>(pad_to(c->a.max_rows, 16));
+    TSS_TRY(c->alloc(&c->mk_part0, c->mk_part_floats));
+    TSS_TRY(c->alloc(&c->mk_part1, c->mk_part_floats));
+  }
   TSS_CU(misc_prepare());
   return TSS_OK;
 }
@@ -643,6 +758,7 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   c->V_pad = pad_to(c->V, 128);
   if (const char* e = std::getenv("TSS_NO_GRAPH")) c->use_graphs = std::atoi(e) == 0;
   if (const char* e = std::getenv("TSS_GEMM_CTAS_PER_SM")) c->gemm_ctas_per_sm = std::max(1, std::min(2, std::atoi(e)));
+  if (const char* e = std::getenv("TSS_PATH")) c->use_mk = std::string(e) != "multi";
   tss_status s = build_workspaces(c);
   if (s == TSS_OK) s = build_weights(c, weights);
   if (s != TSS_OK) {
@@ -755,7 +871,12 @@ tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cach
         TSS_CU(cudaMemcpyAsync(c->io_unif, bt->uniforms, sizeof(float) * B * bt->uniform_stride, cudaMemcpyHostToDevice, s));
     }
   }
-  if (prof) {
+  if (mk_supported(c, sp)) {
+    // Persistent path: three launches per step (the verify kernel is a cooperative launch), so no
+    // graph is needed; with a Prof the events bracket each launch directly.
+    if (prof) prof->s = s;
+    TSS_TRY(enqueue_step_mk(c, sp, s, prof));
+  } else if (prof) {
     // Launches bracketed by events, captured into a graph so that the device runs them back to
     // back: the events then time device work only, not host launch latency.
     prof->s = c->cap_stream;

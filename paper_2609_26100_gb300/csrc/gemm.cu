@@ -26,13 +26,6 @@ namespace tss {
 constexpr int kGemmThreads = 192;  // warp 0: TMA, warp 1: MMA + TMEM alloc, warps 2-5: epilogue
 constexpr uint32_t kWTileBytes = 128 * 64 * 2;
 
-__host__ __device__ uint32_t gemm_tmem_cols(int n_pad, int n_acc_bufs) {
-  uint32_t need = static_cast<uint32_t>(n_pad * n_acc_bufs);
-  uint32_t c = 32;
-  while (c < need) c <<= 1;
-  return c;
-}
-
 size_t gemm_smem_bytes(int n_pad, int stages) {
   const size_t x_bytes = static_cast<size_t>(n_pad) * 128;
   return 1024                                          // alignment slack

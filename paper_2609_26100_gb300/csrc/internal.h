@@ -46,7 +46,13 @@ struct GemmParams {
 };
 
 size_t gemm_smem_bytes(int n_pad, int stages);
-__host__ __device__ uint32_t gemm_tmem_cols(int n_pad, int n_acc_bufs);
+// TMEM columns for n_acc_bufs accumulators of n_pad fp32 columns (a power of two >= 32).
+__host__ __device__ inline uint32_t gemm_tmem_cols(int n_pad, int n_acc_bufs) {
+  uint32_t need = static_cast<uint32_t>(n_pad * n_acc_bufs);
+  uint32_t c = 32;
+  while (c < need) c <<= 1;
+  return c;
+}
 cudaError_t gemm_prepare(size_t max_smem);
 cudaError_t launch_gemm(int epi, const CUtensorMap& tmW, const CUtensorMap& tmX, const GemmParams& p, int grid,
                         size_t smem, cudaStream_t s, bool pdl);
@@ -87,6 +93,8 @@ struct MiscParams {
 };
 
 cudaError_t misc_prepare();
+cudaError_t launch_prologue(const MiscParams& p, float* ssp, int* zero_ints, int n_zero, int M, cudaStream_t s, bool pdl);
+cudaError_t launch_finish(const MiscParams& p, int B, cudaStream_t s, bool pdl);
 cudaError_t launch_controller(const MiscParams& p, cudaStream_t s, bool pdl);
 cudaError_t launch_embed(const MiscParams& p, int M, cudaStream_t s, bool pdl);
 // which: 0 = attention norm of the slot's layer, 1 = MLP norm, 2 = final norm (slot ignored)
@@ -95,6 +103,46 @@ cudaError_t launch_accept_greedy(const MiscParams& p, int B, cudaStream_t s, boo
 cudaError_t launch_accept_sample(const MiscParams& p, int B, cudaStream_t s, bool pdl);
 cudaError_t launch_compact(const MiscParams& p, int B, int n_act, cudaStream_t s, bool pdl);
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* src, float* dst, size_t n, cudaStream_t s);
+
+// Persistent verify kernel (verify_mk.cu).
+struct MkParams {
+  int n_act, d, H, D, F_pad, Ft, V, V_pad, n_pad, stages, attn_splits, B, max_tiles;
+  float eps, scale_log2;
+  unsigned long long seq_base;  // epoch * 1024: flag values grow over steps, never reset
+  const StepDesc* step;
+  const PlanDev* plan;
+  float* h;
+  __nv_bfloat16* qbuf;
+  __nv_bfloat16* obuf;
+  __nv_bfloat16* act;
+  float* partials0;  // stream-K partial tiles, alternating between consecutive phases
+  float* partials1;
+  int* counters;     // [7 kinds][max_tiles]
+  float* ssp;        // [d/128][kMaxRows] per-tile partial sums of squares of h
+  unsigned long long* hflag;    // [d/128]
+  unsigned long long* qkvflag;  // [3d/128]
+  unsigned long long* attflag;  // [max_batch][H]
+  unsigned long long* guflag;   // [Ft]
+  float* amax_val;
+  int* amax_idx;
+  float* attn_po;
+  float* attn_pml;
+  int* attn_cnt;
+  const float* g_attn;
+  const float* g_mlp;
+  const float* g_final;
+  const float* rope_cos;
+  const float* rope_sin;
+  int* status;
+  int* abort_word;
+};
+struct MkTensorMaps {
+  CUtensorMap qkv, o, gu, down, lm, xo, xact;
+};
+size_t mk_smem_bytes(int n_pad, int stages, int head_dim);
+cudaError_t mk_prepare();
+int mk_max_blocks_per_sm(int head_dim, size_t smem);
+cudaError_t launch_verify_mk(const MkTensorMaps& tm, const MkParams& p, int grid, size_t smem, cudaStream_t s);
 
 // Records the message tss_last_error() returns on the calling thread.
 void set_last_error(const std::string& msg);

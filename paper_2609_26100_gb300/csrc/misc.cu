@@ -11,9 +11,7 @@ namespace tss {
 // that at least one request runs (the only layers that get launches) and, per layer, the
 // compacted list of rows of the requests that run it.
 // ------------------------------------------------------------------------------------------
-__global__ void controller_kernel(const MiscParams p) {
-  griddep_wait();
-  griddep_launch();
+__device__ void controller_body(const MiscParams& p) {
   const StepDesc* st = p.step;
   PlanDev* pl = p.plan;
   __shared__ unsigned long long smask[kMaxBatch];
@@ -59,6 +57,12 @@ __global__ void controller_kernel(const MiscParams p) {
     }
     pl->slot_M[slot] = crow;
   }
+}
+
+__global__ void controller_kernel(const MiscParams p) {
+  griddep_wait();
+  griddep_launch();
+  controller_body(p);
 }
 
 // h[m] = E[token[m]] (fp32 residual stream).
@@ -128,12 +132,8 @@ __device__ void write_result(const MiscParams& p, int b, int a, int bonus, const
   for (int i = 0; i <= a; ++i) p.plan->res_path[b][i] = path[i];
 }
 
-__global__ void accept_greedy_kernel(const MiscParams p) {
-  griddep_wait();
-  griddep_launch();
+__device__ void accept_greedy_body(const MiscParams& p, int b) {
   const StepDesc* st = p.step;
-  const int b = blockIdx.x;
-  if (b >= st->B) return;
   __shared__ int am[kMaxNodes];
   __shared__ int path[kMaxNodes];
   const int N = st->req_nodes[b], off = st->req_rowoff[b];
@@ -179,6 +179,13 @@ __global__ void accept_greedy_kernel(const MiscParams p) {
     }
     write_result(p, b, a, am[cur], path);
   }
+}
+
+__global__ void accept_greedy_kernel(const MiscParams p) {
+  griddep_wait();
+  griddep_launch();
+  if (blockIdx.x >= p.step->B) return;
+  accept_greedy_body(p, blockIdx.x);
 }
 
 // Philox4x32-10 (Salmon et al., SC'11): 10 rounds of the 4x32 Philox round with key bumps.
@@ -280,12 +287,8 @@ __device__ int inverse_cdf_block(int V, double u, WFn w, double* scan) {
 // as its base methods): p_i = softmax(logits_i / T); accept draft x_i iff r_i * q_i(x_i) <
 // p_{i-1}(x_i); at the first rejection draw the bonus from normalise(max(0, p_{i-1} - q_i));
 // if every draft is accepted draw it from p_k.  Uniform slots: r_i at i-1, u_i at k+i-1.
-__global__ void accept_sample_kernel(const MiscParams p) {
-  griddep_wait();
-  griddep_launch();
+__device__ void accept_sample_body(const MiscParams& p, int b) {
   const StepDesc* st = p.step;
-  const int b = blockIdx.x;
-  if (b >= st->B) return;
   __shared__ double scan[1025];
   __shared__ double redd[32];
   __shared__ int path[kMaxNodes];
@@ -332,6 +335,99 @@ __global__ void accept_sample_kernel(const MiscParams p) {
   if (threadIdx.x == 0) write_result(p, b, a, bonus, path);
 }
 
+__global__ void accept_sample_kernel(const MiscParams p) {
+  griddep_wait();
+  griddep_launch();
+  if (blockIdx.x >= p.step->B) return;
+  accept_sample_body(p, blockIdx.x);
+}
+
+// ------------------------------------------------------------------------------------------
+// Step prologue for the persistent verify kernel: block 0 runs the skip controller; block
+// 1 + m embeds row m and writes, per 128-feature tile t, the partial sum of squares
+// ssp[t][m] that the RMSNorm of the first active layer needs.
+// ------------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float* ssp, int* zero_ints, int n_zero) {
+  griddep_wait();
+  griddep_launch();
+  if (blockIdx.x == 0) {
+    // counters and the abort word of the persistent kernel start every step at zero, even after
+    // a step that gave up on a timeout
+    for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero_ints[i] = 0;
+    controller_body(p);
+    return;
+  }
+  const StepDesc* st = p.step;
+  const int m = blockIdx.x - 1;
+  if (m >= st->M) return;
+  int tok = st->tokens[m];
+  if (tok < 0 || tok >= p.vocab) {
+    if (threadIdx.x == 0) report(p.status, kStatusCheck);
+    tok = 0;
+  }
+  __shared__ float red[8];
+  const __nv_bfloat16* e = p.embed + static_cast<size_t>(tok) * p.d_model;
+  float* h = p.h + static_cast<size_t>(m) * p.d_model;
+  const int half = threadIdx.x >> 7, r = threadIdx.x & 127;
+  const int n_t = p.d_model / 128;
+  for (int t0 = 0; t0 < n_t; t0 += 2) {
+    const int t = t0 + half;
+    float sq = 0.f;
+    if (t < n_t) {
+      const float x = __bfloat162float(e[t * 128 + r]);
+      h[t * 128 + r] = x;
+      sq = x * x;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sq;
+    __syncthreads();
+    if (r == 0 && t < n_t)
+      ssp[static_cast<size_t>(t) * kMaxRows + m] =
+          (red[half * 4] + red[half * 4 + 1]) + (red[half * 4 + 2] + red[half * 4 + 3]);
+    __syncthreads();
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// Step finish: acceptance of request b (greedy walk or speculative sampling), then the KV
+// compaction of its accepted path in every layer it ran (one 1024-thread block per request).
+// ------------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(1024) finish_kernel(const MiscParams p) {
+  griddep_wait();
+  griddep_launch();
+  const StepDesc* st = p.step;
+  const PlanDev* pl = p.plan;
+  const int b = blockIdx.x;
+  if (b >= st->B) return;
+  if (st->mode == TSS_MODE_SAMPLE) {
+    accept_sample_body(p, b);
+  } else {
+    accept_greedy_body(p, b);
+  }
+  __syncthreads();
+  const int a = pl->res_accept[b];
+  if (a <= 0) return;
+  const int D = p.head_dim, H = p.n_heads;
+  const size_t cap = static_cast<size_t>(st->kv_cap);
+  const size_t ctx = static_cast<size_t>(st->req_ctx[b]);
+  for (int j = 0; j < pl->n_act; ++j) {
+    if (pl->slot_crow[j][b] < 0) continue;
+    __nv_bfloat16* base = st->kv_layer[pl->act_layer[j]] + static_cast<size_t>(st->req_slot[b]) * 2 * H * cap * D;
+    // Element e = (kind, head, dim) stays with one thread across the path steps, and a later
+    // step never reads a row an earlier step wrote, so the in-order copy needs no barrier.
+    for (int jj = 1; jj <= a; ++jj) {
+      const int src = pl->res_path[b][jj];
+      if (src == jj) continue;
+      for (int e = threadIdx.x; e < 2 * H * D; e += blockDim.x) {
+        const int kind_head = e / D, dd = e - kind_head * D;
+        __nv_bfloat16* row = base + static_cast<size_t>(kind_head) * cap * D;
+        row[(ctx + jj) * D + dd] = row[(ctx + src) * D + dd];
+      }
+    }
+  }
+}
+
 // ------------------------------------------------------------------------------------------
 // KV compaction: for every layer the request ran, cache rows ctx + path[j] move to ctx + j,
 // j = 1..a (the root's row stays).  path[j] > j - 1 and increasing, so copying j in increasing
@@ -373,9 +469,18 @@ cudaError_t misc_prepare() {
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(controller_kernel, a, c)) || (e = cudaFuncSetAttribute(embed_kernel, a, c)) ||
       (e = cudaFuncSetAttribute(rmsnorm_kernel, a, c)) || (e = cudaFuncSetAttribute(accept_greedy_kernel, a, c)) ||
-      (e = cudaFuncSetAttribute(accept_sample_kernel, a, c)) || (e = cudaFuncSetAttribute(compact_kernel, a, c)))
+      (e = cudaFuncSetAttribute(accept_sample_kernel, a, c)) || (e = cudaFuncSetAttribute(compact_kernel, a, c)) ||
+      (e = cudaFuncSetAttribute(prologue_kernel, a, c)) || (e = cudaFuncSetAttribute(finish_kernel, a, c)))
     return e;
   return cudaSuccess;
+}
+
+cudaError_t launch_prologue(const MiscParams& p, float* ssp, int* zero_ints, int n_zero, int M, cudaStream_t s,
+                            bool pdl) {
+  return launch_k(prologue_kernel, dim3(M + 1), dim3(256), 0, s, pdl, p, ssp, zero_ints, n_zero);
+}
+cudaError_t launch_finish(const MiscParams& p, int B, cudaStream_t s, bool pdl) {
+  return launch_k(finish_kernel, dim3(B), dim3(1024), 0, s, pdl, p);
 }
 
 cudaError_t launch_controller(const MiscParams& p, cudaStream_t s, bool pdl) {

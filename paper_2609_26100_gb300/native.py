@@ -57,11 +57,11 @@ class TssKvCache(ctypes.Structure):
 
 
 KERNEL_KINDS = ("controller+embed+norms", "qkv_gemm", "attention", "o_gemm", "gate_up_gemm", "down_gemm",
-                "lm_head_gemm", "accept+compact")
+                "lm_head_gemm", "accept+compact", "verify_persistent")
 
 
 class TssKernelTimes(ctypes.Structure):
-    _fields_ = [("ms", ctypes.c_float * 8), ("launches", ctypes.c_int * 8)]
+    _fields_ = [("ms", ctypes.c_float * 9), ("launches", ctypes.c_int * 9)]
 
 
 class TssVerifyResult(ctypes.Structure):

@@ -25,9 +25,17 @@ def weights():
     return w, oracle_weights(w), to_device_weights(w)
 
 
-def make_runner(wg, n_slots=4, cap=512, **kw):
+PATHS = ["persistent", "multi"]
+
+
+def make_runner(wg, n_slots=4, cap=512, path="persistent", **kw):
+    """path: "persistent" (one cooperative kernel for all layers) or "multi" (kernel per op)."""
     from paper_2609_26100_gb300.runner import TssRunner
-    return TssRunner(ARCH, wg, n_slots=n_slots, kv_cap=cap, max_batch=8, **kw)
+    os.environ["TSS_PATH"] = path
+    try:
+        return TssRunner(ARCH, wg, n_slots=n_slots, kv_cap=cap, max_batch=8, **kw)
+    finally:
+        os.environ.pop("TSS_PATH", None)
 
 
 def upload_context(run, kv, slot):
@@ -56,8 +64,9 @@ def run_step(run, reqs, **kw):
     return res, st
 
 
+@pytest.mark.parametrize("path", PATHS)
 @pytest.mark.parametrize("mask_layers", [(2,), ()])
-def test_chain_greedy_16_steps_lockstep(weights, mask_layers):
+def test_chain_greedy_16_steps_lockstep(weights, mask_layers, path):
     """Tiny config: 128-token context (oracle prefill under the mask), chain k=4 = oracle greedy
     continuation with the token at a seeded position replaced, 16 verify steps."""
     w, wo, wg = weights
@@ -65,7 +74,7 @@ def test_chain_greedy_16_steps_lockstep(weights, mask_layers):
     skip = O.mask_to_set(wl.phi[0])
     ctx = synth.uniform_ints(128, ARCH.vocab, SEED, "tiny.ctx").tolist()
     kv = O.prefill(wo, ARCH, skip, ctx)
-    run = make_runner(wg, n_slots=1, cap=256)
+    run = make_runner(wg, n_slots=1, cap=256, path=path)
     run.set_phi(wl.phi)
     upload_context(run, kv, 0)
     C, k = len(ctx), 4
@@ -111,14 +120,15 @@ def test_chain_greedy_16_steps_lockstep(weights, mask_layers):
     run.close()
 
 
-def test_tree_greedy_and_compaction(weights):
+@pytest.mark.parametrize("path", PATHS)
+def test_tree_greedy_and_compaction(weights, path):
     """60-node draft tree (branching 4,3,2,2,1,1) with a planted greedy path: per-node logits,
     longest matching root path, and the KV compacted to that path."""
     w, wo, wg = weights
     skip = frozenset({1})
     ctx = synth.uniform_ints(96, ARCH.vocab, SEED, "tree.ctx").tolist()
     kv = O.prefill(wo, ARCH, skip, ctx)
-    run = make_runner(wg, n_slots=2, cap=256)
+    run = make_runner(wg, n_slots=2, cap=256, path=path)
     run.set_phi({3: O.set_to_mask(skip)})
     upload_context(run, kv, 1)
     parents = synth.eagle_tree(60, (4, 3, 2, 2, 1, 1))
@@ -161,7 +171,8 @@ def test_tree_greedy_and_compaction(weights):
     run.close()
 
 
-def test_mixed_domain_batch_and_untouched_skipped_kv(weights):
+@pytest.mark.parametrize("path", PATHS)
+def test_mixed_domain_batch_and_untouched_skipped_kv(weights, path):
     """Four requests with different skip sets (one domain never configured = dense), different
     context lengths and draft lengths in one batch; skipped layers' KV keeps a sentinel."""
     w, wo, wg = weights
@@ -169,7 +180,7 @@ def test_mixed_domain_batch_and_untouched_skipped_kv(weights):
     doms = [0, 1, 2, 7]
     ctxs = [128, 77, 200, 5]
     ks = [4, 2, 0, 3]
-    run = make_runner(wg, n_slots=4, cap=256)
+    run = make_runner(wg, n_slots=4, cap=256, path=path)
     run.set_phi(phi)
     sentinel = 7.0
     for t in run.kv:
@@ -206,9 +217,10 @@ def test_mixed_domain_batch_and_untouched_skipped_kv(weights):
     run.close()
 
 
-def test_all_layers_skipped_is_embedding_norm_lm_head(weights):
+@pytest.mark.parametrize("path", PATHS)
+def test_all_layers_skipped_is_embedding_norm_lm_head(weights, path):
     w, wo, wg = weights
-    run = make_runner(wg, n_slots=1, cap=64)
+    run = make_runner(wg, n_slots=1, cap=64, path=path)
     run.set_phi({0: (1 << ARCH.n_layers) - 1})
     parents = synth.chain_parents(3)
     toks = [5, 17, 2047, 0]
@@ -238,10 +250,11 @@ def test_root_only_and_empty_context(weights):
     run.close()
 
 
-def test_speculative_sampling_chain(weights):
+@pytest.mark.parametrize("path", PATHS)
+def test_speculative_sampling_chain(weights, path):
     """B=3 chains (k=4, 1, 3) at temperature 1 with Philox uniforms and with caller uniforms."""
     w, wo, wg = weights
-    run = make_runner(wg, n_slots=3, cap=256)
+    run = make_runner(wg, n_slots=3, cap=256, path=path)
     run.set_phi({0: O.set_to_mask({1}), 1: 0})
     ks, ctxs, doms = [4, 1, 3], [64, 33, 90], [0, 1, 0]
     reqs, kvs, skips, qs = [], [], [], []
@@ -288,6 +301,25 @@ def test_speculative_sampling_chain(weights):
     run.close()
 
 
+def test_persistent_path_is_deterministic_and_close_to_multi_kernel_path(weights):
+    w, wo, wg = weights
+    reqs = [synth.Request(40, synth.chain_parents(4), [3, 1, 4, 1, 5], 0),
+            synth.Request(17, [-1, 0, 0, 1], [7, 8, 9, 10], 1)]
+    outs = {}
+    for path in PATHS:
+        run = make_runner(wg, n_slots=2, cap=64, path=path)
+        run.set_phi({0: O.set_to_mask({3}), 1: O.set_to_mask({0})})
+        for l in range(4):
+            run.kv[l].copy_(synth.normal_bf16(run.kv[l].shape, SEED, f"pm{l}", 0.5).cuda())
+        r1, s1 = run_step(run, reqs)
+        r2, s2 = run_step(run, reqs)
+        assert s1 == s2 == native.TSS_OK
+        assert torch.equal(r1["logits"], r2["logits"])
+        outs[path] = r1["logits"].cpu().numpy()
+        run.close()
+    assert np.abs(outs["persistent"] - outs["multi"]).max() < 2e-2
+
+
 def test_graph_and_eager_paths_agree_bitwise(weights):
     w, wo, wg = weights
     reqs = [synth.Request(40, synth.chain_parents(4), [3, 1, 4, 1, 5], 0)]
@@ -295,7 +327,7 @@ def test_graph_and_eager_paths_agree_bitwise(weights):
     for eager in (False, True):
         os.environ["TSS_NO_GRAPH"] = "1" if eager else "0"
         try:
-            run = make_runner(wg, n_slots=1, cap=64)
+            run = make_runner(wg, n_slots=1, cap=64, path="multi")
         finally:
             os.environ.pop("TSS_NO_GRAPH", None)
         run.set_phi({0: O.set_to_mask({3})})
