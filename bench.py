@@ -134,11 +134,14 @@ class ClockSampler:
 
 
 def kernel_bytes(w):
-    """Algorithmic bytes per launch of each kernel kind (weights + activations in and out + KV)."""
+    """Algorithmic bytes per launch of each kernel kind (weights + activations in and out + KV).
+    The persistent verify kernel streams every active layer and the LM head in one launch."""
+    from paper_2609_26100_gb300 import synth
     a = w.arch
     d, f, V, M = a.d_model, a.d_mlp, a.vocab, w.n_rows
     kv_read = sum(r.ctx_len for r in w.requests) * a.kv_bytes_per_token  # per layer, all requests
     return {
+        "verify_persistent": synth.algorithmic_bytes(w)["total"],
         "qkv_gemm": 3 * d * d * 2 + M * d * 2 + M * d * 2 + M * 2 * d * 2,
         "attention": kv_read + M * d * 2 * 2 + M * 2 * d * 2,
         "o_gemm": d * d * 2 + M * d * 2 + M * d * 4 * 2,
@@ -349,6 +352,7 @@ def run_tss(args):
         total_ms = float(t.item())
     ms = total_ms / args.steps
     value = world * w.n_rows * args.steps / (total_ms / 1e3)
+    print(f"[bench] {w.name}: {ms * 1e3:.1f} us/step, {value:.1f} tokens/s", file=sys.stderr)
 
     # ---------------- e2e: host buffers through the C ABI, one sync per step ----------------
     e2e = None

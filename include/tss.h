@@ -235,6 +235,15 @@ tss_status tss_verify_profiled(tss_ctx* ctx, const tss_verify_batch* batch, cons
  * Asynchronous on `stream`; no device status word is reported. */
 tss_status tss_linear_static(const void* x, const void* w, float* y, int m_rows, int k_dim, int n_out, void* stream);
 
+/* Diagnostic timeline of the last persistent-path step, recorded when the environment variable
+ * TSS_TRACE=1 was set at tss_create: globaltimer nanoseconds, per CTA (row of
+ * n_out / #SMs values), per phase pi (QKV, O, gate/up, down of each active layer in order, then
+ * the LM head) at [pi*8 + 2*role + {0 first, 1 last}] for roles 0 weight TMA, 1 B operand,
+ * 2 MMA, 3 epilogue, and the attention of layer slot j at [(4*64+1)*8 + 2j + {0,1}]; 0 = no
+ * activity.  With host == NULL only *n_out (values per device) is returned.  Synchronises the
+ * device. */
+tss_status tss_read_trace(tss_ctx* ctx, unsigned long long* host, size_t capacity, size_t* n_out);
+
 const char* tss_status_string(tss_status s);
 /* Message of the last error reported to the calling thread ("" if none). */
 const char* tss_last_error(void);

@@ -114,7 +114,6 @@ struct tss_ctx {
   float* io_unif = nullptr;
   int* io_res = nullptr;  // accept[kMaxBatch] bonus[kMaxBatch] new_ctx[kMaxBatch] path[kMaxBatch*kMaxPathStride]
   // tensor maps
-  CUtensorMap tm_wqkv, tm_wo, tm_wgu, tm_wdown, tm_lm;
   std::map<int, CUtensorMap> tm_xn, tm_o, tm_act;
   // graphs
   std::map<GraphKey, cudaGraphExec_t> graphs;
@@ -123,6 +122,8 @@ struct tss_ctx {
   int gemm_ctas_per_sm = 2;
   // persistent verify kernel
   bool use_mk = true;
+  int l2_ahead = 0;
+  unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
   unsigned long long epoch = 0;
   float* ssp = nullptr;
   unsigned long long* flags = nullptr;  // hflag | qkvflag | guflag | attflag
@@ -259,12 +260,16 @@ struct Prof {
   std::vector<cudaEvent_t> ev;
   std::vector<int> kind;
   cudaStream_t s = nullptr;
+  bool capturing = false;  // under stream capture an event record must be an external node
+  cudaError_t record(cudaEvent_t e) {
+    return capturing ? cudaEventRecordWithFlags(e, s, cudaEventRecordExternal) : cudaEventRecord(e, s);
+  }
   tss_status begin(int k) {
     cudaEvent_t e;
     TSS_CU(cudaEventCreate(&e));
     ev.push_back(e);
     kind.push_back(k);
-    TSS_CU(cudaEventRecordWithFlags(e, s, cudaEventRecordExternal));  // a record node under capture
+    TSS_CU(record(e));
     return TSS_OK;
   }
   tss_status end() {
@@ -272,7 +277,7 @@ struct Prof {
     TSS_CU(cudaEventCreate(&e));
     ev.push_back(e);
     kind.push_back(-1);
-    TSS_CU(cudaEventRecordWithFlags(e, s, cudaEventRecordExternal));  // a record node under capture
+    TSS_CU(record(e));
     return TSS_OK;
   }
 };
@@ -316,20 +321,31 @@ tss_status enqueue_step(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* pr
     TSS_K(0, TSS_CU(launch_rmsnorm(mp, j, 0, sp.M, s, pdl)));
     GemmParams g = gemm_base(c, n_pad);
     g.slot = j;
-    TSS_K(1, TSS_TRY(run_gemm(c, kEpiQkv, c->tm_wqkv, *txn, g, 3 * c->d / 128, kbd, s, pdl)));
+    const size_t dd = static_cast<size_t>(c->d) * c->d;
+    g.w_tiled = c->wqkv;
+    g.w_layer_elems = static_cast<long long>(3 * dd);
+    TSS_K(1, TSS_TRY(run_gemm(c, kEpiQkv, *txn, *txn, g, 3 * c->d / 128, kbd, s, pdl)));
     ap.slot = j;
     TSS_K(2, TSS_CU(launch_attention(ap, sp.B, s, pdl)));
-    TSS_K(3, TSS_TRY(run_gemm(c, kEpiResid, c->tm_wo, *to, g, c->d / 128, kbd, s, pdl)));
+    g.w_tiled = c->wo;
+    g.w_layer_elems = static_cast<long long>(dd);
+    TSS_K(3, TSS_TRY(run_gemm(c, kEpiResid, *to, *to, g, c->d / 128, kbd, s, pdl)));
     // feed-forward sub-block
     TSS_K(0, TSS_CU(launch_rmsnorm(mp, j, 1, sp.M, s, pdl)));
-    TSS_K(4, TSS_TRY(run_gemm(c, kEpiSwiglu, c->tm_wgu, *txn, g, c->Ft, kbd, s, pdl)));
-    TSS_K(5, TSS_TRY(run_gemm(c, kEpiResid, c->tm_wdown, *tact, g, c->d / 128, c->F_pad / 64, s, pdl)));
+    g.w_tiled = c->wgu;
+    g.w_layer_elems = static_cast<long long>(c->Ft) * 128 * c->d;
+    TSS_K(4, TSS_TRY(run_gemm(c, kEpiSwiglu, *txn, *txn, g, c->Ft, kbd, s, pdl)));
+    g.w_tiled = c->wdown;
+    g.w_layer_elems = static_cast<long long>(c->d) * c->F_pad;
+    TSS_K(5, TSS_TRY(run_gemm(c, kEpiResid, *tact, *tact, g, c->d / 128, c->F_pad / 64, s, pdl)));
   }
   TSS_K(0, TSS_CU(launch_rmsnorm(mp, kFinalSlot, 2, sp.M, s, pdl)));
   GemmParams g = gemm_base(c, n_pad);
   g.slot = kFinalSlot;
   g.layer_fixed = 0;
-  TSS_K(6, TSS_TRY(run_gemm(c, kEpiLmHead, c->tm_lm, *txn, g, c->V_pad / 128, kbd, s, pdl)));
+  g.w_tiled = c->lm;
+  g.w_layer_elems = 0;
+  TSS_K(6, TSS_TRY(run_gemm(c, kEpiLmHead, *txn, *txn, g, c->V_pad / 128, kbd, s, pdl)));
   if (sp.mode == TSS_MODE_SAMPLE) {
     TSS_K(7, TSS_CU(launch_accept_sample(mp, sp.B, s, pdl)));
   } else {
@@ -353,9 +369,10 @@ int mk_stages(const tss_ctx* c, int n_pad) {
 tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* prof) {
   MiscParams mp = misc_params(c);
   const int n_pad = sp.n_pad;
-  const CUtensorMap *to, *tact;
+  const CUtensorMap *to, *tact, *txn;
   TSS_TRY(get_xmap(c, c->tm_o, c->obuf, c->d, n_pad, &to));
   TSS_TRY(get_xmap(c, c->tm_act, c->act, c->F_pad, n_pad, &tact));
+  TSS_TRY(get_xmap(c, c->tm_xn, c->xn, c->d, n_pad, &txn));
   const int stages = mk_stages(c, n_pad);
   const size_t smem = mk_smem_bytes(n_pad, stages, c->D);
   const int nt = c->d / 128;
@@ -370,18 +387,33 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.V_pad = c->V_pad;
   p.n_pad = n_pad;
   p.stages = stages;
-  p.attn_splits = sp.splits;
+  // about one attention item per CTA: items = B * H * splits
+  {
+    const int per = sp.B * c->H;
+    int sl = c->num_sms / per;
+    if (sl < 1) sl = 1;
+    if (sl > c->max_splits) sl = c->max_splits;
+    p.attn_splits = sl;
+  }
   p.B = sp.B;
   p.max_tiles = c->mk_max_tiles;
+  p.l2_ahead = c->l2_ahead;
+  p.trace = c->trace;
   p.eps = c->a.rms_eps;
   p.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->D)));
   p.seq_base = ++c->epoch * 1024ull;
   p.step = c->d_step;
   p.plan = c->d_plan;
+  p.w_qkv = c->wqkv;
+  p.w_o = c->wo;
+  p.w_gu = c->wgu;
+  p.w_down = c->wdown;
+  p.w_lm = c->lm;
   p.h = c->h;
   p.qbuf = c->qbuf;
   p.obuf = c->obuf;
   p.act = c->act;
+  p.xn = c->xn;
   p.partials0 = c->mk_part0;
   p.partials1 = c->mk_part1;
   p.counters = c->mk_zero;
@@ -403,13 +435,9 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.rope_sin = c->rope_sin;
   p.status = c->d_status;
   MkTensorMaps tm;
-  tm.qkv = c->tm_wqkv;
-  tm.o = c->tm_wo;
-  tm.gu = c->tm_wgu;
-  tm.down = c->tm_wdown;
-  tm.lm = c->tm_lm;
   tm.xo = *to;
   tm.xact = *tact;
+  tm.xn = *txn;
 #define TSS_MK(kind, expr)                 \
   do {                                     \
     if (prof) TSS_TRY(prof->begin(kind));  \
@@ -460,9 +488,10 @@ tss_status build_weights(tss_ctx* c, const tss_weights* w) {
         !w->w_up[l] || !w->w_down[l])
       return fail(TSS_ERR_INVALID_ARG, "weights of layer " + std::to_string(l) + " incomplete");
   const size_t dd = static_cast<size_t>(d) * d;
+  const size_t gu_rows = static_cast<size_t>(c->Ft) * 128;
   TSS_TRY(c->alloc(&c->wqkv, static_cast<size_t>(L) * 3 * dd));
   TSS_TRY(c->alloc(&c->wo, static_cast<size_t>(L) * dd));
-  TSS_TRY(c->alloc(&c->wgu, static_cast<size_t>(L) * c->Ft * 128 * d));
+  TSS_TRY(c->alloc(&c->wgu, static_cast<size_t>(L) * gu_rows * d));
   TSS_TRY(c->alloc(&c->wdown, static_cast<size_t>(L) * d * c->F_pad));
   TSS_TRY(c->alloc(&c->embed, static_cast<size_t>(V) * d));
   TSS_TRY(c->alloc(&c->lm, static_cast<size_t>(c->V_pad) * d));
@@ -470,39 +499,48 @@ tss_status build_weights(tss_ctx* c, const tss_weights* w) {
   TSS_TRY(c->alloc(&c->g_mlp, static_cast<size_t>(L) * d));
   TSS_TRY(c->alloc(&c->g_final, d));
   const size_t b2 = sizeof(__nv_bfloat16);
-  TSS_CU(cudaMemset(c->wgu, 0, static_cast<size_t>(L) * c->Ft * 128 * d * b2));
-  TSS_CU(cudaMemset(c->wdown, 0, static_cast<size_t>(L) * d * c->F_pad * b2));
-  TSS_CU(cudaMemset(c->lm, 0, static_cast<size_t>(c->V_pad) * d * b2));
+  // Row-major staging of one matrix at a time, then tiling into the library's pre-tiled layout.
+  size_t tmp_elems = std::max(std::max(3 * dd, gu_rows * d), std::max(static_cast<size_t>(d) * c->F_pad,
+                                                                        static_cast<size_t>(c->V_pad) * d));
+  __nv_bfloat16* tmp = nullptr;
+  if (cudaMalloc(&tmp, tmp_elems * b2) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(TSS_ERR_OUT_OF_MEMORY, "weight staging allocation failed");
+  }
+  struct Free {
+    void* p;
+    ~Free() { cudaFree(p); }
+  } free_tmp{tmp};
   TSS_CU(cudaMemcpy(c->embed, w->embed, static_cast<size_t>(V) * d * b2, cudaMemcpyDeviceToDevice));
-  TSS_CU(cudaMemcpy(c->lm, w->lm_head, static_cast<size_t>(V) * d * b2, cudaMemcpyDeviceToDevice));
+  TSS_CU(cudaMemset(tmp, 0, static_cast<size_t>(c->V_pad) * d * b2));
+  TSS_CU(cudaMemcpy(tmp, w->lm_head, static_cast<size_t>(V) * d * b2, cudaMemcpyDeviceToDevice));
+  TSS_CU(launch_tile_weights(tmp, c->lm, c->V_pad, d, 0));
   TSS_CU(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(w->final_norm), c->g_final, d, 0));
   for (int l = 0; l < L; ++l) {
-    __nv_bfloat16* q = c->wqkv + static_cast<size_t>(l) * 3 * dd;
-    TSS_CU(cudaMemcpy(q, w->wq[l], dd * b2, cudaMemcpyDeviceToDevice));
-    TSS_CU(cudaMemcpy(q + dd, w->wk[l], dd * b2, cudaMemcpyDeviceToDevice));
-    TSS_CU(cudaMemcpy(q + 2 * dd, w->wv[l], dd * b2, cudaMemcpyDeviceToDevice));
-    TSS_CU(cudaMemcpy(c->wo + static_cast<size_t>(l) * dd, w->wo[l], dd * b2, cudaMemcpyDeviceToDevice));
+    TSS_CU(cudaMemcpy(tmp, w->wq[l], dd * b2, cudaMemcpyDeviceToDevice));
+    TSS_CU(cudaMemcpy(tmp + dd, w->wk[l], dd * b2, cudaMemcpyDeviceToDevice));
+    TSS_CU(cudaMemcpy(tmp + 2 * dd, w->wv[l], dd * b2, cudaMemcpyDeviceToDevice));
+    TSS_CU(launch_tile_weights(tmp, c->wqkv + static_cast<size_t>(l) * 3 * dd, 3 * d, d, 0));
+    TSS_CU(launch_tile_weights(static_cast<const __nv_bfloat16*>(w->wo[l]), c->wo + static_cast<size_t>(l) * dd, d, d, 0));
     // gate/up interleaved per 64 features: tile t = [gate rows 64t..64t+63 ; up rows 64t..64t+63]
-    __nv_bfloat16* gu = c->wgu + static_cast<size_t>(l) * c->Ft * 128 * d;
+    TSS_CU(cudaMemset(tmp, 0, gu_rows * d * b2));
     for (int t = 0; t < c->Ft; ++t) {
       const int rows = F - 64 * t < 64 ? F - 64 * t : 64;
       const size_t src_off = static_cast<size_t>(64) * t * d;
-      TSS_CU(cudaMemcpy(gu + static_cast<size_t>(t) * 128 * d, static_cast<const __nv_bfloat16*>(w->w_gate[l]) + src_off,
+      TSS_CU(cudaMemcpy(tmp + static_cast<size_t>(t) * 128 * d, static_cast<const __nv_bfloat16*>(w->w_gate[l]) + src_off,
                         static_cast<size_t>(rows) * d * b2, cudaMemcpyDeviceToDevice));
-      TSS_CU(cudaMemcpy(gu + (static_cast<size_t>(t) * 128 + 64) * d,
-                        static_cast<const __nv_bfloat16*>(w->w_up[l]) + src_off, static_cast<size_t>(rows) * d * b2,
-                        cudaMemcpyDeviceToDevice));
+      TSS_CU(cudaMemcpy(tmp + (static_cast<size_t>(t) * 128 + 64) * d, static_cast<const __nv_bfloat16*>(w->w_up[l]) + src_off,
+                        static_cast<size_t>(rows) * d * b2, cudaMemcpyDeviceToDevice));
     }
-    TSS_CU(cudaMemcpy2D(c->wdown + static_cast<size_t>(l) * d * c->F_pad, static_cast<size_t>(c->F_pad) * b2, w->w_down[l],
-                        static_cast<size_t>(F) * b2, static_cast<size_t>(F) * b2, d, cudaMemcpyDeviceToDevice));
+    TSS_CU(launch_tile_weights(tmp, c->wgu + static_cast<size_t>(l) * gu_rows * d, static_cast<int>(gu_rows), d, 0));
+    TSS_CU(cudaMemset(tmp, 0, static_cast<size_t>(d) * c->F_pad * b2));
+    TSS_CU(cudaMemcpy2D(tmp, static_cast<size_t>(c->F_pad) * b2, w->w_down[l], static_cast<size_t>(F) * b2,
+                        static_cast<size_t>(F) * b2, d, cudaMemcpyDeviceToDevice));
+    TSS_CU(launch_tile_weights(tmp, c->wdown + static_cast<size_t>(l) * d * c->F_pad, d, c->F_pad, 0));
     TSS_CU(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(w->attn_norm[l]), c->g_attn + static_cast<size_t>(l) * d, d, 0));
     TSS_CU(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(w->mlp_norm[l]), c->g_mlp + static_cast<size_t>(l) * d, d, 0));
+    TSS_CU(cudaDeviceSynchronize());  // the staging buffer is reused by the next layer
   }
-  TSS_CU(cudaDeviceSynchronize());
-  if (!make_tmap(&c->tm_wqkv, c->wqkv, d, 3 * d, L, 128) || !make_tmap(&c->tm_wo, c->wo, d, d, L, 128) ||
-      !make_tmap(&c->tm_wgu, c->wgu, d, static_cast<uint64_t>(c->Ft) * 128, L, 128) ||
-      !make_tmap(&c->tm_wdown, c->wdown, c->F_pad, d, L, 128) || !make_tmap(&c->tm_lm, c->lm, d, c->V_pad, 1, 128))
-    return fail(TSS_ERR_CUDA, "cuTensorMapEncodeTiled failed for a weight tensor");
   return TSS_OK;
 }
 
@@ -759,8 +797,15 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_NO_GRAPH")) c->use_graphs = std::atoi(e) == 0;
   if (const char* e = std::getenv("TSS_GEMM_CTAS_PER_SM")) c->gemm_ctas_per_sm = std::max(1, std::min(2, std::atoi(e)));
   if (const char* e = std::getenv("TSS_PATH")) c->use_mk = std::string(e) != "multi";
+  if (const char* e = std::getenv("TSS_L2_AHEAD")) c->l2_ahead = std::max(0, std::atoi(e));
+  const char* trace_env = std::getenv("TSS_TRACE");
   tss_status s = build_workspaces(c);
   if (s == TSS_OK) s = build_weights(c, weights);
+  if (s == TSS_OK && trace_env && std::atoi(trace_env) != 0) {
+    s = c->alloc(&c->trace, static_cast<size_t>(c->num_sms) * mk_trace_slots());
+    if (s == TSS_OK && cudaMemset(c->trace, 0, static_cast<size_t>(c->num_sms) * mk_trace_slots() * 8) != cudaSuccess)
+      s = fail(TSS_ERR_CUDA, "cudaMemset of the trace buffer failed");
+  }
   if (s != TSS_OK) {
     const std::string msg = g_err;
     destroy_ctx(c);
@@ -880,6 +925,7 @@ tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cach
     // Launches bracketed by events, captured into a graph so that the device runs them back to
     // back: the events then time device work only, not host launch latency.
     prof->s = c->cap_stream;
+    prof->capturing = true;
     cudaGraph_t graph = nullptr;
     TSS_CU(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal));
     tss_status st = enqueue_step(c, sp, c->cap_stream, prof);
@@ -975,6 +1021,17 @@ tss_status tss_sync_status(tss_ctx* c, void* stream) {
   TSS_CU(cudaStreamSynchronize(s));
   const int v = *c->h_status;
   if (v != 0) return fail(v, std::string("device status: ") + tss_status_string(v));
+  return TSS_OK;
+}
+
+tss_status tss_read_trace(tss_ctx* c, unsigned long long* host, size_t capacity, size_t* n_out) {
+  if (!c || !n_out) return fail(TSS_ERR_INVALID_ARG, "NULL argument");
+  const size_t n = c->trace ? static_cast<size_t>(c->num_sms) * mk_trace_slots() : 0;
+  *n_out = n;
+  if (!host || n == 0) return TSS_OK;
+  if (capacity < n) return fail(TSS_ERR_INVALID_ARG, "trace buffer too small");
+  TSS_CU(cudaDeviceSynchronize());
+  TSS_CU(cudaMemcpy(host, c->trace, n * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
   return TSS_OK;
 }
 

@@ -164,6 +164,25 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* m, uin
       : "memory");
 }
 
+// Linear bulk copy global -> shared of `bytes` (multiple of 16, both addresses 16-byte aligned).
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)), "r"(bytes)
+               : "memory");
+}
+
+// Weights are stored pre-tiled: for each 128-row x 64-column block (16 KiB) the exact byte image
+// that a 128-byte-swizzled TMA box of it would leave in shared memory, blocks ordered
+// [layer][row tile][k-block].  One linear bulk copy then fills a pipeline stage.
+constexpr uint32_t kTileBytes = 128 * 64 * 2;
+constexpr size_t kTileElems = 128 * 64;
+
 // ------------------------------------------------------------------------------------------
 // tcgen05: tensor memory and the 5th-generation MMA
 // ------------------------------------------------------------------------------------------

@@ -266,7 +266,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const long long it = it0 + i;
         const int t = static_cast<int>(it / p.kb), kk = static_cast<int>(it % p.kb);
         mbar_arrive_expect_tx(&full[i], kWTileBytes + x_bytes);
-        tma_load_3d(sW + static_cast<size_t>(i) * kWTileBytes, &tmW, &full[i], kk * 64, t * 128, layer);
+        if (p.w_tiled)
+          bulk_load(sW + static_cast<size_t>(i) * kWTileBytes,
+                    p.w_tiled + layer * p.w_layer_elems + (static_cast<size_t>(t) * p.kb + kk) * kTileElems, kWTileBytes,
+                    &full[i]);
+        else
+          tma_load_3d(sW + static_cast<size_t>(i) * kWTileBytes, &tmW, &full[i], kk * 64, t * 128, layer);
       }
       griddep_wait();
       griddep_launch();
@@ -281,7 +286,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const long long it = it0 + i;
         const int t = static_cast<int>(it / p.kb), kk = static_cast<int>(it % p.kb);
         mbar_arrive_expect_tx(&full[s], kWTileBytes + x_bytes);
-        tma_load_3d(sW + static_cast<size_t>(s) * kWTileBytes, &tmW, &full[s], kk * 64, t * 128, layer);
+        if (p.w_tiled)
+          bulk_load(sW + static_cast<size_t>(s) * kWTileBytes,
+                    p.w_tiled + layer * p.w_layer_elems + (static_cast<size_t>(t) * p.kb + kk) * kTileElems, kWTileBytes,
+                    &full[s]);
+        else
+          tma_load_3d(sW + static_cast<size_t>(s) * kWTileBytes, &tmW, &full[s], kk * 64, t * 128, layer);
         tma_load_2d(sX + static_cast<size_t>(s) * x_bytes, &tmX, &full[s], kk * 64, 0);
       }
     }

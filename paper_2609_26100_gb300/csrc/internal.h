@@ -26,6 +26,8 @@ struct GemmParams {
   int slot;         // plan slot whose compacted rows feed the GEMM; -1: plain rows [0, m_raw)
   int m_raw;
   int layer_fixed;  // >= 0: TMA layer coordinate; -1: plan->act_layer[slot]
+  const __nv_bfloat16* w_tiled;  // pre-tiled weights (bulk copies); nullptr: tensor-map TMA
+  long long w_layer_elems;       // elements per layer in w_tiled
   const PlanDev* plan;
   const StepDesc* step;
   float* partials;  // stream-K partial tiles [(grid + n_tiles) * 128 * n_pad]
@@ -103,18 +105,28 @@ cudaError_t launch_accept_greedy(const MiscParams& p, int B, cudaStream_t s, boo
 cudaError_t launch_accept_sample(const MiscParams& p, int B, cudaStream_t s, bool pdl);
 cudaError_t launch_compact(const MiscParams& p, int B, int n_act, cudaStream_t s, bool pdl);
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* src, float* dst, size_t n, cudaStream_t s);
+// Row-major [rows][cols] bf16 (rows % 128 == 0, cols % 64 == 0) -> pre-tiled, pre-swizzled blocks.
+cudaError_t launch_tile_weights(const __nv_bfloat16* src, __nv_bfloat16* dst, int rows, int cols, cudaStream_t s);
 
 // Persistent verify kernel (verify_mk.cu).
 struct MkParams {
   int n_act, d, H, D, F_pad, Ft, V, V_pad, n_pad, stages, attn_splits, B, max_tiles;
+  int l2_ahead;  // weight tiles per CTA prefetched into L2 ahead of the smem ring (0: off)
+  unsigned long long* trace;  // optional timeline [grid][mk_trace_slots()], nullptr when off
   float eps, scale_log2;
   unsigned long long seq_base;  // epoch * 1024: flag values grow over steps, never reset
   const StepDesc* step;
   const PlanDev* plan;
+  const __nv_bfloat16* w_qkv;  // pre-tiled weights [L][tiles][k-blocks][16 KiB]
+  const __nv_bfloat16* w_o;
+  const __nv_bfloat16* w_gu;
+  const __nv_bfloat16* w_down;
+  const __nv_bfloat16* w_lm;
   float* h;
   __nv_bfloat16* qbuf;
   __nv_bfloat16* obuf;
   __nv_bfloat16* act;
+  __nv_bfloat16* xn;  // [kMaxRows][d] bf16(h * g) of the next norm phase, compacted rows
   float* partials0;  // stream-K partial tiles, alternating between consecutive phases
   float* partials1;
   int* counters;     // [7 kinds][max_tiles]
@@ -137,9 +149,10 @@ struct MkParams {
   int* abort_word;
 };
 struct MkTensorMaps {
-  CUtensorMap qkv, o, gu, down, lm, xo, xact;
+  CUtensorMap xo, xact, xn;
 };
 size_t mk_smem_bytes(int n_pad, int stages, int head_dim);
+size_t mk_trace_slots();
 cudaError_t mk_prepare();
 int mk_max_blocks_per_sm(int head_dim, size_t smem);
 cudaError_t launch_verify_mk(const MkTensorMaps& tm, const MkParams& p, int grid, size_t smem, cudaStream_t s);

@@ -366,6 +366,38 @@ __global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float
     tok = 0;
   }
   __shared__ float red[8];
+  __shared__ unsigned long long smask[kMaxBatch];
+  __shared__ int s_l0, s_crow;
+  // The first norm phase is the QKV of the union's first layer (or the LM head when every layer
+  // is skipped); find this row's compacted position in it, as the controller does.
+  for (int b = threadIdx.x; b < st->B; b += blockDim.x) {
+    const int dom = st->req_domain[b];
+    smask[b] = (dom >= 0 && dom < p.max_domains && p.phi_valid[dom]) ? p.phi_mask[dom] : 0ull;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int l0 = -1;
+    for (int l = 0; l < p.n_layers && l0 < 0; ++l)
+      for (int b = 0; b < st->B; ++b)
+        if (!((smask[b] >> l) & 1ull)) {
+          l0 = l;
+          break;
+        }
+    const int rb = st->row_req[m];
+    int crow = -1;
+    if (l0 < 0) {
+      crow = m;
+    } else if (!((smask[rb] >> l0) & 1ull)) {
+      crow = m - st->req_rowoff[rb];
+      for (int b = 0; b < rb; ++b)
+        if (!((smask[b] >> l0) & 1ull)) crow += st->req_nodes[b];
+    }
+    s_l0 = l0;
+    s_crow = crow;
+  }
+  __syncthreads();
+  const float* gain = s_l0 >= 0 ? p.g_attn + static_cast<size_t>(s_l0) * p.d_model : p.g_final;
+  __nv_bfloat16* xn = s_crow >= 0 ? p.xn + static_cast<size_t>(s_crow) * p.d_model : nullptr;
   const __nv_bfloat16* e = p.embed + static_cast<size_t>(tok) * p.d_model;
   float* h = p.h + static_cast<size_t>(m) * p.d_model;
   const int half = threadIdx.x >> 7, r = threadIdx.x & 127;
@@ -376,6 +408,7 @@ __global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float
     if (t < n_t) {
       const float x = __bfloat162float(e[t * 128 + r]);
       h[t * 128 + r] = x;
+      if (xn) xn[t * 128 + r] = __float2bfloat16_rn(x * gain[t * 128 + r]);
       sq = x * x;
     }
 #pragma unroll
@@ -502,6 +535,28 @@ cudaError_t launch_compact(const MiscParams& p, int B, int n_act, cudaStream_t s
   if (n_act <= 0) n_act = 1;
   return launch_k(compact_kernel, dim3(p.n_heads, B, n_act), dim3(128), 0, s, pdl, p);
 }
+// One thread per 16-byte chunk (8 columns) of the source.
+__global__ void tile_weights_kernel(const __nv_bfloat16* src, __nv_bfloat16* dst, int rows, int cols) {
+  const size_t n_chunks = static_cast<size_t>(rows) * (cols / 8);
+  const int kbs = cols / 64;
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n_chunks;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const int row = static_cast<int>(i / (cols / 8));
+    const int col = static_cast<int>(i % (cols / 8)) * 8;
+    const int t = row >> 7, r = row & 127, kb = col >> 6, c8 = (col & 63) >> 3;
+    const size_t blk = static_cast<size_t>(t) * kbs + kb;
+    uint8_t* d = reinterpret_cast<uint8_t*>(dst + blk * kTileElems) + r * 128 + ((c8 ^ (r & 7)) << 4);
+    *reinterpret_cast<uint4*>(d) = *reinterpret_cast<const uint4*>(src + static_cast<size_t>(row) * cols + col);
+  }
+}
+
+cudaError_t launch_tile_weights(const __nv_bfloat16* src, __nv_bfloat16* dst, int rows, int cols, cudaStream_t s) {
+  const size_t n = static_cast<size_t>(rows) * (cols / 8);
+  const int blocks = static_cast<int>(n / 256 + 1 < 16384 ? n / 256 + 1 : 16384);
+  tile_weights_kernel<<<blocks, 256, 0, s>>>(src, dst, rows, cols);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* src, float* dst, size_t n, cudaStream_t s) {
   const int blocks = static_cast<int>((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
   bf16_to_f32_kernel<<<blocks > 0 ? blocks : 1, 256, 0, s>>>(src, dst, n);

@@ -10,9 +10,9 @@
 //               bounded only by the shared-memory ring).
 //   warp 1      tcgen05.mma issuer (accumulators in TMEM, double-buffered).
 //   warp 2      B-operand producer: for every k-block it waits until the activations it needs
-//               are final, then writes the N x 64 bf16 tile (128-byte swizzle) -- from h times the
-//               RMSNorm gain for QKV / gate-up / LM head, by TMA from the attention output or the
-//               SwiGLU activations for O / down.
+//               are final (flags polled 32 at a time), then loads the N x 64 bf16 tile by TMA --
+//               bf16(h * g) for QKV / gate-up / LM head, the attention output for O, the SwiGLU
+//               activations for down.
 //   warps 4-7   epilogues (TMEM -> registers, stream-K fixup, fused op) and the attention items.
 //
 // Phases hand data over through global memory and per-tile flags stamped with a sequence
@@ -20,9 +20,10 @@
 // + kind), so flags are never reset.  A consumer waits only for the producer tiles it reads:
 // a k-block of QKV / gate-up / LM head needs one 128-feature tile of h; an O k-block needs the
 // attention output of one head for every request; a down k-block needs one gate/up tile.
-// The RMSNorm is split accordingly: the B operand is bf16(h * g), and the per-row factor
+// The RMSNorm is split accordingly: the B operand is bf16(h * g) -- written, for the next norm
+// phase, by the epilogue that finalises each 128-feature tile of h -- and the per-row factor
 // 1/sqrt(mean(h^2) + eps) is applied to the accumulator in the epilogue, from per-tile partial
-// sums of squares written by the residual epilogues.
+// sums of squares written by the same residual epilogues.
 //
 // Every wait is bounded (2 s); on expiry the kernel records TIMEOUT, raises a grid-wide abort
 // word and all roles leave their loops.
@@ -31,6 +32,14 @@
 namespace tss {
 
 constexpr int kMkThreads = 256;
+constexpr int kMkMaxAcc = 8;  // TMEM accumulator buffers (fewer when N is large)
+
+// Accumulator buffers for an MMA width: a power of two, at most 8, within 512 TMEM columns.
+__host__ __device__ inline int mk_acc_bufs(int n_pad) {
+  int nb = kMkMaxAcc;
+  while (nb > 1 && nb * n_pad > 512) nb >>= 1;
+  return nb;
+}
 constexpr uint32_t kMkWBytes = 128 * 64 * 2;
 
 enum MkKind : int { kMkQkv = 1, kMkAtt = 2, kMkO = 3, kMkGu = 4, kMkDown = 5, kMkLm = 6 };
@@ -126,6 +135,15 @@ struct MkPhase {
   int kind, slot, layer, n_tiles, kb;
 };
 
+// Optional timeline (TSS_TRACE): per CTA, per phase, the first and last activity of each role.
+// trace[cta][pi * 8 + 2 * role + {0: first, 1: last}], roles 0 weight TMA, 1 B operand, 2 MMA,
+// 3 epilogue; the attention of slot j at [kMkTracePhases * 8 + 2j + {0,1}].
+constexpr int kMkTracePhases = 4 * kMaxLayers + 1;
+constexpr int kMkTraceSlots = kMkTracePhases * 8 + 2 * kMaxLayers;
+__device__ __forceinline__ void mk_trace(const MkParams& p, int idx) {
+  if (p.trace) p.trace[static_cast<size_t>(blockIdx.x) * kMkTraceSlots + idx] = globaltimer_ns();
+}
+
 __device__ __forceinline__ MkPhase mk_phase(const MkParams& p, const PlanDev* pl, int pi) {
   MkPhase ph;
   if (pi < 4 * p.n_act) {
@@ -145,6 +163,17 @@ __device__ __forceinline__ MkPhase mk_phase(const MkParams& p, const PlanDev* pl
     ph.kb = p.d / 64;
   }
   return ph;
+}
+
+// Pre-tiled weights of a phase's layer (blocks [tile][k-block] of 16 KiB).
+__device__ __forceinline__ const __nv_bfloat16* mk_weights(const MkParams& p, const MkPhase& ph) {
+  const size_t blocks = static_cast<size_t>(ph.n_tiles) * ph.kb;
+  const __nv_bfloat16* base = ph.kind == kMkQkv ? p.w_qkv
+                              : ph.kind == kMkO ? p.w_o
+                              : ph.kind == kMkGu ? p.w_gu
+                              : ph.kind == kMkDown ? p.w_down
+                                                   : p.w_lm;
+  return base + static_cast<size_t>(ph.layer) * blocks * kTileElems;
 }
 
 // CTA c's stream-K range of a phase over geff = min(grid, iterations) CTAs.
@@ -187,17 +216,25 @@ __device__ __forceinline__ unsigned long long mk_h_dep(const MkParams& p, const 
 
 struct MkEpi {
   int M;
-  const int* rows;
+  const int* rows;  // shared-memory copy of the phase's compacted row list
+  int* pos;         // [kMaxRows] RoPE position of each compacted row (QKV)
+  int* kvslot;      // [kMaxRows] KV-cache slot and row of each compacted row (QKV)
+  int* kvrow;
+  int nM;           // rows of the next norm phase (residual phases) and their list
+  const int* nrows;
   float* xch;    // [16][128]
   float* redv;   // [4][16]
   int* redi;     // [4][16]
-  float* rs;     // [kMaxRows] per-row RMSNorm factors of the current tile
+  float* rs;     // [kMaxRows] per-row RMSNorm factors of the current phase
   int q, lane, et;
 };
 
 // Wait until every 128-feature tile of h has reached `dep`, then compute the RMSNorm factors of
 // the phase's rows from the partial sums of squares (fixed order, deterministic).
-__device__ bool mk_prepare_rs(const MkParams& p, const MkEpi& e, unsigned long long dep, const MkShared& sh) {
+__device__ bool mk_prepare_rs(const MkParams& p, const MkEpi& e, unsigned long long dep, const MkShared& sh,
+                              bool& ready) {
+  if (ready) return true;  // once per phase
+  ready = true;
   const int nt = p.d / 128;
   bool ok = true;
   for (int t = e.et; dep != 0ull && t < nt && ok; t += 128) ok = mk_wait_flag(&p.hflag[t], dep, sh);
@@ -205,6 +242,7 @@ __device__ bool mk_prepare_rs(const MkParams& p, const MkEpi& e, unsigned long l
   for (int j = e.et; j < e.M; j += 128) {
     const int m = e.rows[j];
     float ss = 0.f;
+#pragma unroll 8
     for (int t = 0; t < nt; ++t) ss += __ldcg(&p.ssp[static_cast<size_t>(t) * kMaxRows + m]);
     e.rs[j] = rsqrtf(ss / static_cast<float>(p.d) + p.eps);
   }
@@ -237,7 +275,7 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
       for (int jj = 0; jj < 16; ++jj) {
         rot[jj] = 0.f;
         if (j0 + jj < e.M) {
-          const int pos = st->row_pos[e.rows[j0 + jj]];
+          const int pos = e.pos[j0 + jj];
           const float c = p.rope_cos[static_cast<size_t>(pos) * half + i];
           const float s = p.rope_sin[static_cast<size_t>(pos) * half + i];
           const float pv = e.xch[jj * 128 + pr];
@@ -255,11 +293,9 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
       if (sec == 0) {
         p.qbuf[static_cast<size_t>(j) * d + f] = __float2bfloat16_rn(val[jj]);
       } else {
-        const int m = e.rows[j];
-        const int b = st->row_req[m];
-        const int crow = st->req_ctx[b] + (m - st->req_rowoff[b]);
-        const size_t off =
-            ((static_cast<size_t>(st->req_slot[b]) * 2 + (sec - 1)) * p.H + head) * static_cast<size_t>(st->kv_cap) + crow;
+        const size_t off = ((static_cast<size_t>(e.kvslot[j]) * 2 + (sec - 1)) * p.H + head) *
+                               static_cast<size_t>(st->kv_cap) +
+                           e.kvrow[j];
         st->kv_layer[ph.layer][off * D + dim] = __float2bfloat16_rn(val[jj]);
       }
     }
@@ -360,6 +396,35 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
   }
 }
 
+// After a residual phase finalised tile t of h: write the next norm phase's B operand
+// bf16(h * g_next) for features [128t, 128t+128) of every row that phase runs, in its compacted
+// order (O -> gate/up of the same layer; down -> QKV of the next layer, or the LM head).
+__device__ __forceinline__ int mk_next_slot(const MkParams& p, const MkPhase& ph) {
+  if (ph.kind == kMkO) return ph.slot;
+  return ph.slot + 1 < p.n_act ? ph.slot + 1 : kFinalSlot;
+}
+
+__device__ void mk_write_next_xn(const MkParams& p, const PlanDev* pl, const MkPhase& ph, const MkEpi& e, int t,
+                                 int r) {
+  const int nslot = mk_next_slot(p, ph);
+  const float* g = ph.kind == kMkO ? p.g_mlp + static_cast<size_t>(ph.layer) * p.d
+                   : nslot != kFinalSlot ? p.g_attn + static_cast<size_t>(pl->act_layer[nslot]) * p.d
+                                         : p.g_final;
+  const int M = e.nM;
+  const int* rows = e.nrows;
+  const int f = t * 128 + r;
+  const float gf = g[f];
+  for (int n0 = 0; n0 < M; n0 += 8) {
+    float hv[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      hv[u] = n0 + u < M ? __ldcg(&p.h[static_cast<size_t>(rows[n0 + u]) * p.d + f]) : 0.f;
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (n0 + u < M) p.xn[static_cast<size_t>(n0 + u) * p.d + f] = __float2bfloat16_rn(hv[u] * gf);
+  }
+}
+
 __device__ __forceinline__ unsigned long long* mk_tile_flag(const MkParams& p, int kind, int t) {
   switch (kind) {
     case kMkQkv: return p.qkvflag + t;
@@ -372,10 +437,8 @@ __device__ __forceinline__ unsigned long long* mk_tile_flag(const MkParams& p, i
 
 template <int D>
 __global__ void __launch_bounds__(kMkThreads, 1)
-    verify_mk_kernel(const __grid_constant__ CUtensorMap tm_qkv, const __grid_constant__ CUtensorMap tm_o,
-                     const __grid_constant__ CUtensorMap tm_gu, const __grid_constant__ CUtensorMap tm_down,
-                     const __grid_constant__ CUtensorMap tm_lm, const __grid_constant__ CUtensorMap tm_xo,
-                     const __grid_constant__ CUtensorMap tm_xact, const MkParams p) {
+    verify_mk_kernel(const __grid_constant__ CUtensorMap tm_xo, const __grid_constant__ CUtensorMap tm_xact,
+                     const __grid_constant__ CUtensorMap tm_xn, const MkParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = p.stages, n_pad = p.n_pad;
@@ -386,18 +449,25 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   uint64_t* full = reinterpret_cast<uint64_t*>(s_attn + attn_smem_bytes_impl(D));
   uint64_t* empty = full + S;
   uint64_t* accf = empty + S;
-  uint64_t* acce = accf + 2;
-  int* misc = reinterpret_cast<int*>(acce + 2);  // [0] tmem addr, [1] abort, [2..4] bcast, [5] s_last
+  uint64_t* acce = accf + kMkMaxAcc;
+  int* misc = reinterpret_cast<int*>(acce + kMkMaxAcc);  // [0] tmem addr, [1] abort, [2..4] bcast, [5] s_last, [8] w_pos
   float* xch = reinterpret_cast<float*>(misc + 16);
   float* redv = xch + 16 * 128;
   int* redi = reinterpret_cast<int*>(redv + 64);
   float* rs = reinterpret_cast<float*>(redi + 64);
   float (*sM)[16] = reinterpret_cast<float (*)[16]>(rs + kMaxRows);
   float (*sL)[16] = reinterpret_cast<float (*)[16]>(rs + kMaxRows + 64);
+  int* s_rows = reinterpret_cast<int*>(rs + kMaxRows + 128);  // [kMaxRows] x 5: rows, pos, kv slot, kv row, next rows
+  int* s_pos = s_rows + kMaxRows;
+  int* s_kvslot = s_pos + kMaxRows;
+  int* s_kvrow = s_kvslot + kMaxRows;
+  int* s_nrows = s_kvrow + kMaxRows;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t ncols = gemm_tmem_cols(n_pad, 2);
+  const int NB = mk_acc_bufs(n_pad);
+  const uint32_t ncols = gemm_tmem_cols(n_pad, NB);
   const PlanDev* pl = p.plan;
+  volatile int* w_pos = misc + 8;  // weight tiles the TMA producer has issued
   MkShared sh;
   sh.abort_s = reinterpret_cast<volatile int*>(misc + 1);
   sh.abort_g = p.abort_word;
@@ -408,19 +478,16 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       mbar_init(&full[i], 2);  // weight TMA arrival + B-operand arrival
       mbar_init(&empty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kMkMaxAcc; ++i) {
       mbar_init(&accf[i], 1);
       mbar_init(&acce[i], 128);
     }
     *sh.abort_s = 0;
+    misc[8] = 0;
     fence_mbar_init();
-    prefetch_tmap(&tm_qkv);
-    prefetch_tmap(&tm_o);
-    prefetch_tmap(&tm_gu);
-    prefetch_tmap(&tm_down);
-    prefetch_tmap(&tm_lm);
     prefetch_tmap(&tm_xo);
     prefetch_tmap(&tm_xact);
+    prefetch_tmap(&tm_xn);
   }
   if (warp == 1) {
     tmem_alloc(reinterpret_cast<uint32_t*>(misc), ncols);
@@ -446,22 +513,23 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         long long it0, it1;
         int geff;
         mk_range(ph, c, G, it0, it1, geff);
-        const CUtensorMap* tm = ph.kind == kMkQkv ? &tm_qkv
-                                : ph.kind == kMkO ? &tm_o
-                                : ph.kind == kMkGu ? &tm_gu
-                                : ph.kind == kMkDown ? &tm_down
-                                                     : &tm_lm;
+        const __nv_bfloat16* wl = mk_weights(p, ph);
         for (long long it = it0; it < it1; ++it, ++i) {
           const int s = static_cast<int>(i % S);
           if (!mk_wait_bar(&empty[s], static_cast<uint32_t>((i / S) & 1) ^ 1u, sh)) {
             ok = false;
             break;
           }
+          if (it == it0) mk_trace(p, pi * 8 + 0);
+          if (it + 1 == it1) mk_trace(p, pi * 8 + 1);
           const int t = static_cast<int>(it / ph.kb), kk = static_cast<int>(it % ph.kb);
           mbar_arrive_expect_tx(&full[s], kMkWBytes);
-          tma_load_3d(sW + static_cast<size_t>(s) * kMkWBytes, tm, &full[s], kk * 64, t * 128, ph.layer);
+          bulk_load(sW + static_cast<size_t>(s) * kMkWBytes, wl + (static_cast<size_t>(t) * ph.kb + kk) * kTileElems,
+                    kMkWBytes, &full[s]);
+          *w_pos = static_cast<int>(i + 1);
         }
       }
+      *w_pos = 0x7fffffff;  // the prefetch warp may run to the end
       if (!ok) {  // let weight tiles already in flight land before the CTA can exit
         const uint64_t t0 = globaltimer_ns();
         while (globaltimer_ns() - t0 < 50000) {
@@ -483,8 +551,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         long long it = it0;
         int t, k0, k1;
         while (ok && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
-          const int buf = use & 1;
-          if (!mk_wait_bar(&acce[buf], static_cast<uint32_t>((use >> 1) & 1) ^ 1u, sh)) {
+          const int buf = use % NB;
+          if (!mk_wait_bar(&acce[buf], static_cast<uint32_t>((use / NB) & 1) ^ 1u, sh)) {
             ok = false;
             break;
           }
@@ -497,6 +565,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
               break;
             }
             tc_fence_after();
+            if (kk == k0 && static_cast<long long>(t) * ph.kb + k0 == it0) mk_trace(p, pi * 8 + 4);
             const uint32_t a0 = smem_u32(sW + static_cast<size_t>(s) * kMkWBytes);
             const uint32_t b0 = smem_u32(sX + static_cast<size_t>(s) * x_bytes);
 #pragma unroll
@@ -507,12 +576,13 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           }
           if (!ok) break;
           umma_commit(&accf[buf]);
+          if (it >= it1) mk_trace(p, pi * 8 + 5);
           ++use;
         }
       }
     }
   } else if (warp == 2) {
-    // ---------------- B-operand producer ----------------
+    // ---------------- B-operand producer: TMA after the producing tiles are flagged ----------------
     long long i = 0;
     bool ok = true;
     for (int pi = 0; ok && pi < n_phases; ++pi) {
@@ -521,74 +591,105 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       int geff;
       mk_range(ph, c, G, it0, it1, geff);
       if (it0 >= it1) continue;
-      const int rslot = mk_row_slot(ph);
-      const int M = pl->slot_M[rslot];
-      const int* rows = pl->slot_rows[rslot];
-      const unsigned long long hdep = (ph.kind == kMkO || ph.kind == kMkDown) ? 0ull : mk_h_dep(p, ph);
-      const float* gain = ph.kind == kMkQkv  ? p.g_attn + static_cast<size_t>(ph.layer) * p.d
-                          : ph.kind == kMkGu ? p.g_mlp + static_cast<size_t>(ph.layer) * p.d
-                                             : p.g_final;
-      int ready_dep = -1;  // last dependency index already seen complete
+      // dependency index space of this phase: h tiles, heads, or gate/up tiles
+      const unsigned long long* flags;
+      unsigned long long want;
+      int n_dep;
+      if (ph.kind == kMkO) {
+        flags = p.attflag;
+        want = mk_seq(p.seq_base, ph.slot, kMkAtt);
+        n_dep = p.H;
+      } else if (ph.kind == kMkDown) {
+        flags = p.guflag;
+        want = mk_seq(p.seq_base, ph.slot, kMkGu);
+        n_dep = p.Ft;
+      } else {
+        flags = p.hflag;
+        want = mk_h_dep(p, ph);
+        n_dep = p.d / 128;
+      }
+      const CUtensorMap* tmx = ph.kind == kMkO ? &tm_xo : ph.kind == kMkDown ? &tm_xact : &tm_xn;
+      uint32_t ready[8] = {0, 0, 0, 0, 0, 0, 0, 0};  // known-complete dependency indices (<= 256)
+      // one flag index is complete when every request that runs the slot has it (attention) or
+      // the single flag reached `want`
+      auto poll = [&](int x) -> bool {
+        if (ph.kind != kMkO) return ld_acquire_u64(&flags[x]) >= want;
+        for (int b = 0; b < p.B; ++b)
+          if (pl->slot_crow[ph.slot][b] >= 0 && ld_acquire_u64(&flags[b * p.H + x]) < want) return false;
+        return true;
+      };
       for (long long it = it0; ok && it < it1; ++it, ++i) {
         const int s = static_cast<int>(i % S);
         const int kk = static_cast<int>(it % ph.kb);
         if (lane == 0) ok = mk_wait_bar(&empty[s], static_cast<uint32_t>((i / S) & 1) ^ 1u, sh);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) break;
-        // dependency of this k-block
-        if (ph.kind == kMkO) {
-          const int head = kk * 64 / p.D;
-          if (head != ready_dep) {
-            const unsigned long long want = mk_seq(p.seq_base, ph.slot, kMkAtt);
-            bool good = true;
-            for (int b = lane; b < p.B; b += 32)
-              if (pl->slot_crow[ph.slot][b] >= 0) good = good && mk_wait_flag(&p.attflag[b * p.H + head], want, sh);
-            ok = __all_sync(0xffffffffu, good);
-            ready_dep = head;
-          }
-        } else if (ph.kind == kMkDown) {
-          if (kk != ready_dep) {
-            if (lane == 0) ok = mk_wait_flag(&p.guflag[kk], mk_seq(p.seq_base, ph.slot, kMkGu), sh);
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            ready_dep = kk;
-          }
-        } else if (hdep != 0ull) {
-          const int ht = kk >> 1;  // 128-feature tile of h holding this k-block
-          if (ht != ready_dep) {
-            if (lane == 0) ok = mk_wait_flag(&p.hflag[ht], hdep, sh);
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            ready_dep = ht;
+        const int x = want == 0ull ? -1 : (ph.kind == kMkO ? kk * 64 / p.D : ph.kind == kMkDown ? kk : (kk >> 1));
+        if (x >= 0 && !((ready[x >> 5] >> (x & 31)) & 1u)) {
+          // poll x .. x+31 at once; then wait (bounded) for x itself if it is not there yet
+          const int y = x + lane;
+          const bool rdy = y < n_dep && poll(y);
+          const uint32_t bal = __ballot_sync(0xffffffffu, rdy);
+          for (int l = 0; l < 32; ++l)
+            if ((bal >> l) & 1u) ready[(x + l) >> 5] |= 1u << ((x + l) & 31);
+          if (!(bal & 1u)) {
+            bool got = true;
+            if (lane == 0) {
+              const uint64_t t0 = globaltimer_ns();
+              while (!poll(x)) {
+                if (mk_aborted(sh)) {
+                  got = false;
+                  break;
+                }
+                if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                  mk_fail(sh);
+                  got = false;
+                  break;
+                }
+                __nanosleep(64);
+              }
+            }
+            ok = __shfl_sync(0xffffffffu, got, 0);
+            if (!ok) break;
+            ready[x >> 5] |= 1u << (x & 31);
           }
         }
-        if (!ok) break;
-        if (ph.kind == kMkO || ph.kind == kMkDown) {
-          if (lane == 0) {
-            fence_proxy_async_global();
-            mbar_arrive_expect_tx(&full[s], x_bytes);
-            tma_load_2d(sX + static_cast<size_t>(s) * x_bytes, ph.kind == kMkO ? &tm_xo : &tm_xact, &full[s], kk * 64, 0);
-          }
-        } else {
-          uint8_t* xs = sX + static_cast<size_t>(s) * x_bytes;
-          for (int idx = lane; idx < n_pad * 8; idx += 32) {
-            const int row = idx >> 3, c8 = idx & 7;
-            uint4 out = make_uint4(0, 0, 0, 0);
-            if (row < M) {
-              const float* hp = p.h + static_cast<size_t>(rows[row]) * p.d + kk * 64 + c8 * 8;
-              const float* gp = gain + kk * 64 + c8 * 8;
-              const float4 a = __ldcg(reinterpret_cast<const float4*>(hp));
-              const float4 b = __ldcg(reinterpret_cast<const float4*>(hp + 4));
-              const float4 ga = *reinterpret_cast<const float4*>(gp);
-              const float4 gb = *reinterpret_cast<const float4*>(gp + 4);
-              out.x = pack_bf16(a.x * ga.x, a.y * ga.y);
-              out.y = pack_bf16(a.z * ga.z, a.w * ga.w);
-              out.z = pack_bf16(b.x * gb.x, b.y * gb.y);
-              out.w = pack_bf16(b.z * gb.z, b.w * gb.w);
+        if (lane == 0) {
+          if (it == it0) mk_trace(p, pi * 8 + 2);
+          if (it + 1 == it1) mk_trace(p, pi * 8 + 3);
+          fence_proxy_async_global();
+          mbar_arrive_expect_tx(&full[s], x_bytes);
+          tma_load_2d(sX + static_cast<size_t>(s) * x_bytes, tmx, &full[s], kk * 64, 0);
+        }
+      }
+    }
+  } else if (warp == 3) {
+    if (lane == 0 && p.l2_ahead > 0) {
+      // ---------------- L2 prefetch of weight tiles ahead of the ring ----------------
+      // Keeps HBM streaming while the ring waits at a phase boundary for activations: the ring's
+      // TMA loads then hit in L2.  Stays at most l2_ahead tiles ahead of the TMA producer.
+      long long j = 0;
+      bool go = true;
+      for (int pi = 0; go && pi < n_phases; ++pi) {
+        const MkPhase ph = mk_phase(p, pl, pi);
+        long long it0, it1;
+        int geff;
+        mk_range(ph, c, G, it0, it1, geff);
+        const __nv_bfloat16* wl = mk_weights(p, ph);
+        for (long long it = it0; go && it < it1; ++it, ++j) {
+          if (j >= static_cast<long long>(*w_pos) + p.l2_ahead) {
+            const uint64_t t0 = globaltimer_ns();
+            while (j >= static_cast<long long>(*w_pos) + p.l2_ahead) {
+              if (*sh.abort_s || globaltimer_ns() - t0 > kWaitLimitNs) {
+                go = false;  // the other roles handle a timeout; prefetching is only a hint
+                break;
+              }
+              __nanosleep(128);
             }
-            *reinterpret_cast<uint4*>(xs + row * 128 + ((c8 ^ (row & 7)) << 4)) = out;
+            if (!go) break;
           }
-          fence_proxy_async_shared();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&full[s]);
+          const int t = static_cast<int>(it / ph.kb), kk = static_cast<int>(it % ph.kb);
+          bulk_prefetch_l2(wl + (static_cast<size_t>(t) * ph.kb + kk) * kTileElems, kMkWBytes);
         }
       }
     }
@@ -625,9 +726,33 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       long long it0, it1;
       int geff;
       mk_range(ph, c, G, it0, it1, geff);
+      if (it0 >= it1 && ph.kind != kMkQkv) continue;
+      // per-phase row metadata in shared memory (loaded while the first accumulator is pending)
       const int rslot = mk_row_slot(ph);
       e.M = pl->slot_M[rslot];
-      e.rows = pl->slot_rows[rslot];
+      named_bar_sync(1, 128);  // previous phase's readers of the caches are done
+      for (int j = e.et; j < e.M; j += 128) {
+        const int m = pl->slot_rows[rslot][j];
+        s_rows[j] = m;
+        if (ph.kind == kMkQkv) {
+          const int b = p.step->row_req[m];
+          s_pos[j] = p.step->row_pos[m];
+          s_kvslot[j] = p.step->req_slot[b];
+          s_kvrow[j] = p.step->req_ctx[b] + (m - p.step->req_rowoff[b]);
+        }
+      }
+      if (ph.kind == kMkO || ph.kind == kMkDown) {
+        const int ns = mk_next_slot(p, ph);
+        e.nM = pl->slot_M[ns];
+        for (int j = e.et; j < e.nM; j += 128) s_nrows[j] = pl->slot_rows[ns][j];
+      }
+      named_bar_sync(1, 128);
+      e.rows = s_rows;
+      e.pos = s_pos;
+      e.kvslot = s_kvslot;
+      e.kvrow = s_kvrow;
+      e.nrows = s_nrows;
+      bool rs_ready = false;
       const long long T = static_cast<long long>(ph.n_tiles) * ph.kb;
       float* partials = (pi & 1) ? p.partials1 : p.partials0;
       int* counters = p.counters + static_cast<size_t>(ph.kind) * p.max_tiles;
@@ -636,19 +761,20 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       long long it = it0;
       int t, k0, k1;
       while (ok && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
-        const int buf = use & 1;
-        const bool got = e.et == 0 ? mk_wait_bar(&accf[buf], static_cast<uint32_t>((use >> 1) & 1), sh) : true;
+        const int buf = use % NB;
+        const bool got = e.et == 0 ? mk_wait_bar(&accf[buf], static_cast<uint32_t>((use / NB) & 1), sh) : true;
         if (!bar_and(1, 128, got)) {
           ok = false;
           break;
         }
+        if (e.et == 0 && static_cast<long long>(t) * ph.kb + k0 == it0) mk_trace(p, pi * 8 + 6);
         tc_fence_after();
         const uint32_t tb = tmem_base + (static_cast<uint32_t>(e.q * 32) << 16) + static_cast<uint32_t>(buf * n_pad);
         const int n_ch = n_pad >> 4;
         bool finalize = false;
         int cf = 0, cl = 0;
         if (k0 == 0 && k1 == ph.kb) {
-          if (needs_rs && !mk_prepare_rs(p, e, hdep, sh)) {
+          if (needs_rs && !mk_prepare_rs(p, e, hdep, sh, rs_ready)) {
             ok = false;
             break;
           }
@@ -689,7 +815,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           named_bar_sync(1, 128);
           if (finalize) {
             __threadfence();
-            if (needs_rs && !mk_prepare_rs(p, e, hdep, sh)) {
+            if (needs_rs && !mk_prepare_rs(p, e, hdep, sh, rs_ready)) {
               ok = false;
               break;
             }
@@ -708,10 +834,15 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         }
         if (finalize) {
           unsigned long long* flag = mk_tile_flag(p, ph.kind, t);
+          if (ph.kind == kMkO || ph.kind == kMkDown) {
+            named_bar_sync(1, 128);  // h of this tile is final for every row of the phase
+            mk_write_next_xn(p, pl, ph, e, t, r);
+          }
           __threadfence();
           named_bar_sync(1, 128);
           if (flag && e.et == 0) st_release_u64(flag, mk_seq(p.seq_base, ph.slot, ph.kind));
         }
+        if (e.et == 0 && it >= it1) mk_trace(p, pi * 8 + 7);
         ++use;
       }
       if (!ok) break;
@@ -721,6 +852,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         const int per_req = p.H * p.attn_splits;
         const int n_items = p.B * per_req;
         const unsigned long long want = mk_seq(p.seq_base, ph.slot, kMkQkv);
+        if (e.et == 0) mk_trace(p, kMkTracePhases * 8 + 2 * ph.slot);
         for (int item = c; ok && item < n_items; item += G) {
           const int b = item / per_req;
           const int head = (item - b * per_req) / p.attn_splits;
@@ -743,6 +875,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           }
           named_bar_sync(1, 128);
         }
+        if (e.et == 0) mk_trace(p, kMkTracePhases * 8 + 2 * ph.slot + 1);
       }
     }
   }
@@ -756,10 +889,12 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   }
 }
 
+size_t mk_trace_slots() { return kMkTraceSlots; }
+
 size_t mk_smem_bytes(int n_pad, int stages, int head_dim) {
   return 1024 + static_cast<size_t>(stages) * (kMkWBytes + static_cast<size_t>(n_pad) * 128) +
-         attn_smem_bytes_impl(head_dim) + static_cast<size_t>(2 * stages + 4) * 8 + 64 + 16 * 128 * 4 + 64 * 4 * 2 +
-         kMaxRows * 4 + 128 * 4 + 64;
+         attn_smem_bytes_impl(head_dim) + static_cast<size_t>(2 * stages + 2 * kMkMaxAcc) * 8 + 64 + 16 * 128 * 4 +
+         64 * 4 * 2 + kMaxRows * 4 + 128 * 4 + 5 * kMaxRows * 4 + 64;
 }
 
 cudaError_t mk_prepare() {
@@ -781,9 +916,9 @@ cudaError_t launch_verify_mk(const MkTensorMaps& tm, const MkParams& p, int grid
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   if (p.D == 64)
-    return cudaLaunchKernelEx(&cfg, verify_mk_kernel<64>, tm.qkv, tm.o, tm.gu, tm.down, tm.lm, tm.xo, tm.xact, p);
+    return cudaLaunchKernelEx(&cfg, verify_mk_kernel<64>, tm.xo, tm.xact, tm.xn, p);
   if (p.D == 128)
-    return cudaLaunchKernelEx(&cfg, verify_mk_kernel<128>, tm.qkv, tm.o, tm.gu, tm.down, tm.lm, tm.xo, tm.xact, p);
+    return cudaLaunchKernelEx(&cfg, verify_mk_kernel<128>, tm.xo, tm.xact, tm.xn, p);
   return cudaErrorInvalidValue;
 }
 

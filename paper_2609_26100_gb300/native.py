@@ -26,7 +26,7 @@ TSS_MODE_SAMPLE = 1
 EXPORTS = (
     "tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_sync_status", "tss_destroy", "tss_linear",
-    "tss_linear_static", "tss_status_string", "tss_last_error",
+    "tss_linear_static", "tss_read_trace", "tss_status_string", "tss_last_error",
 )
 
 _P = ctypes.c_void_p
@@ -93,13 +93,14 @@ def lib() -> ctypes.CDLL:
         L.tss_destroy.restype = None
         L.tss_linear.argtypes = [_P, _P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P]
         L.tss_linear_static.argtypes = [_P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P]
+        L.tss_read_trace.argtypes = [_P, _P, ctypes.c_size_t, ctypes.POINTER(ctypes.c_size_t)]
         L.tss_status_string.argtypes = [ctypes.c_int]
         L.tss_status_string.restype = ctypes.c_char_p
         L.tss_last_error.argtypes = []
         L.tss_last_error.restype = ctypes.c_char_p
         for name in ("tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
                      "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_sync_status", "tss_linear",
-                     "tss_linear_static"):
+                     "tss_linear_static", "tss_read_trace"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -229,6 +230,18 @@ class Verifier:
     def verify_profiled(self, batch, kv, result, times: "TssKernelTimes", stream=None) -> None:
         check(lib().tss_verify_profiled(self.ctx, ctypes.byref(batch), ctypes.byref(kv), ctypes.byref(result), stream,
                                         ctypes.byref(times)), "tss_verify_profiled")
+
+    def read_trace(self):
+        """Persistent-kernel timeline of the last step (see tss_read_trace), as a numpy array
+        [n_sms, slots] of globaltimer ns, or None when tracing is off."""
+        import numpy as np
+        n = ctypes.c_size_t()
+        check(lib().tss_read_trace(self.ctx, None, 0, ctypes.byref(n)), "tss_read_trace")
+        if n.value == 0:
+            return None
+        buf = np.zeros(n.value, dtype=np.uint64)
+        check(lib().tss_read_trace(self.ctx, buf.ctypes.data, n.value, ctypes.byref(n)), "tss_read_trace")
+        return buf
 
     def active_layer_count(self, batch) -> int:
         out = ctypes.c_int()
