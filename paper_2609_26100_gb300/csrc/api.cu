@@ -123,6 +123,11 @@ struct tss_ctx {
   // persistent verify kernel
   bool use_mk = true;
   int l2_ahead = 0;
+  int mk_kps = 4;  // weight k-blocks per ring stage of the persistent kernel
+  int l2_pace = 0;       // cycles between paced L2 weight prefetches of 16 KiB (0: unpaced)
+  int w_evict_first = 1;
+  int pf_attn = 0, pf_next = 0;
+  int mk_max_stages = 12;
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
   unsigned long long epoch = 0;
   float* ssp = nullptr;
@@ -253,6 +258,7 @@ tss_status run_gemm(tss_ctx* c, int epi, const CUtensorMap& tmW, const CUtensorM
 
 struct StepPlan {
   int B, M, n_act, mode, splits, n_pad;
+  int tiles;  // 64-key tiles of the longest request (context + block)
 };
 
 // Optional per-launch event timing (tss_verify_profiled).
@@ -356,11 +362,50 @@ tss_status enqueue_step(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* pr
   return TSS_OK;
 }
 
-// Stages of the persistent kernel's ring that fit next to its attention buffers; 0 if none.
-int mk_stages(const tss_ctx* c, int n_pad) {
-  int s = 0;
-  while (s < 12 && mk_smem_bytes(n_pad, s + 1, c->D) <= 232448) ++s;
-  return s >= 2 ? s : 0;
+// Shared-memory plan of the persistent kernel: the ring (stages x kps weight blocks with their
+// B-operand blocks) and, behind it, attention-only space so that the attention, which borrows
+// the ring, keeps all key tiles of a split resident (or as many as fit, in rounds).
+struct MkConfig {
+  int kps = 0, stages = 0, attn_splits = 1;
+  size_t attn_extra = 0, smem = 0;
+};
+
+int mk_attn_splits(const tss_ctx* c, int B) {
+  // about one attention item per CTA: items = B * H * splits
+  int sl = c->num_sms / (B * c->H);
+  if (sl < 1) sl = 1;
+  if (sl > c->max_splits) sl = c->max_splits;
+  return sl;
+}
+
+bool mk_config(const tss_ctx* c, const StepPlan& sp, MkConfig* out) {
+  constexpr size_t kLimit = 232448;  // per-block shared-memory maximum of sm_103 (227 KiB)
+  const size_t q = static_cast<size_t>(kMaxNodes) * (c->D + 8) * 2;
+  const size_t tile = static_cast<size_t>(2) * 64 * (c->D + 8) * 2;
+  const int splits = mk_attn_splits(c, sp.B);
+  const int per = std::max(1, (std::max(sp.tiles, 1) + splits - 1) / splits);
+  for (int kps = c->mk_kps; kps >= 1; --kps) {
+    const size_t stage = static_cast<size_t>(kps) * (16384 + static_cast<size_t>(sp.n_pad) * 128);
+    for (int S = c->mk_max_stages; S >= 2; --S) {
+      const size_t ring = S * stage;
+      const size_t base = mk_smem_bytes(sp.n_pad, S, c->D, kps, 0);
+      if (base > kLimit) continue;
+      const size_t avail = kLimit - base;
+      const size_t need_min = ring >= q + tile ? 0 : q + tile - ring;
+      if (need_min > avail) continue;
+      const size_t want = q + per * tile > ring ? q + per * tile - ring : 0;
+      size_t extra = std::max(need_min, std::min(want, avail));
+      extra = (extra + 15) & ~size_t(15);
+      if (base + extra > kLimit) extra = need_min;
+      out->kps = kps;
+      out->stages = S;
+      out->attn_splits = splits;
+      out->attn_extra = extra;
+      out->smem = base + extra;
+      return true;
+    }
+  }
+  return false;
 }
 
 // One verification step on the persistent path: prologue (controller, embedding, sums of
@@ -369,12 +414,11 @@ int mk_stages(const tss_ctx* c, int n_pad) {
 tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* prof) {
   MiscParams mp = misc_params(c);
   const int n_pad = sp.n_pad;
-  const CUtensorMap *to, *tact, *txn;
-  TSS_TRY(get_xmap(c, c->tm_o, c->obuf, c->d, n_pad, &to));
-  TSS_TRY(get_xmap(c, c->tm_act, c->act, c->F_pad, n_pad, &tact));
-  TSS_TRY(get_xmap(c, c->tm_xn, c->xn, c->d, n_pad, &txn));
-  const int stages = mk_stages(c, n_pad);
-  const size_t smem = mk_smem_bytes(n_pad, stages, c->D);
+  mp.xt_npad = n_pad;  // the persistent kernel takes its B operands in the k-block tiled layout
+  MkConfig cfg;
+  if (!mk_config(c, sp, &cfg)) return fail(TSS_ERR_UNSUPPORTED_ARCH, "persistent kernel: no shared-memory plan");
+  const int kps = cfg.kps, stages = cfg.stages;
+  const size_t smem = cfg.smem;
   const int nt = c->d / 128;
   MkParams p{};
   p.n_act = sp.n_act;
@@ -387,14 +431,13 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.V_pad = c->V_pad;
   p.n_pad = n_pad;
   p.stages = stages;
-  // about one attention item per CTA: items = B * H * splits
-  {
-    const int per = sp.B * c->H;
-    int sl = c->num_sms / per;
-    if (sl < 1) sl = 1;
-    if (sl > c->max_splits) sl = c->max_splits;
-    p.attn_splits = sl;
-  }
+  p.kps = kps;
+  p.attn_extra = static_cast<int>(cfg.attn_extra);
+  p.l2_pace = c->l2_pace;
+  p.w_evict_first = c->w_evict_first;
+  p.pf_attn = c->pf_attn;
+  p.pf_next = c->pf_next;
+  p.attn_splits = cfg.attn_splits;
   p.B = sp.B;
   p.max_tiles = c->mk_max_tiles;
   p.l2_ahead = c->l2_ahead;
@@ -434,10 +477,6 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.rope_cos = c->rope_cos;
   p.rope_sin = c->rope_sin;
   p.status = c->d_status;
-  MkTensorMaps tm;
-  tm.xo = *to;
-  tm.xact = *tact;
-  tm.xn = *txn;
 #define TSS_MK(kind, expr)                 \
   do {                                     \
     if (prof) TSS_TRY(prof->begin(kind));  \
@@ -445,7 +484,7 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
     if (prof) TSS_TRY(prof->end());        \
   } while (0)
   TSS_MK(0, TSS_CU(launch_prologue(mp, c->ssp, c->mk_zero, c->mk_n_zero, sp.M, s, false)));
-  TSS_MK(8, TSS_CU(launch_verify_mk(tm, p, c->num_sms, smem, s)));
+  TSS_MK(8, TSS_CU(launch_verify_mk(p, c->num_sms, smem, s)));
   TSS_MK(7, TSS_CU(launch_finish(mp, sp.B, s, false)));
 #undef TSS_MK
   return TSS_OK;
@@ -453,9 +492,9 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
 
 bool mk_supported(const tss_ctx* c, const StepPlan& sp) {
   if (!c->use_mk) return false;
-  const int stages = mk_stages(c, sp.n_pad);
-  if (stages < 2) return false;
-  return mk_max_blocks_per_sm(c->D, mk_smem_bytes(sp.n_pad, stages, c->D)) >= 1;
+  MkConfig cfg;
+  if (!mk_config(c, sp, &cfg)) return false;
+  return mk_max_blocks_per_sm(c->D, cfg.smem) >= 1;
 }
 
 tss_status validate_arch(const tss_arch* a) {
@@ -746,6 +785,7 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
   sp->mode = bt->mode;
   sp->splits = splits;
   sp->n_pad = pad_to(M, 16);
+  sp->tiles = tiles;
   return TSS_OK;
 }
 
@@ -798,6 +838,12 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_GEMM_CTAS_PER_SM")) c->gemm_ctas_per_sm = std::max(1, std::min(2, std::atoi(e)));
   if (const char* e = std::getenv("TSS_PATH")) c->use_mk = std::string(e) != "multi";
   if (const char* e = std::getenv("TSS_L2_AHEAD")) c->l2_ahead = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("TSS_MK_KPS")) c->mk_kps = std::min(8, std::max(1, std::atoi(e)));
+  if (const char* e = std::getenv("TSS_L2_PACE")) c->l2_pace = std::min(100000, std::max(0, std::atoi(e)));
+  if (const char* e = std::getenv("TSS_EVICT_FIRST")) c->w_evict_first = std::atoi(e) != 0;
+  if (const char* e = std::getenv("TSS_PF_ATTN")) c->pf_attn = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("TSS_PF_NEXT")) c->pf_next = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
   const char* trace_env = std::getenv("TSS_TRACE");
   tss_status s = build_workspaces(c);
   if (s == TSS_OK) s = build_weights(c, weights);

@@ -19,199 +19,264 @@ __host__ __device__ inline size_t attn_smem_bytes_impl(int head_dim) {
   return static_cast<size_t>(kMaxNodes + 4 * kKeyTile) * ld * 2;  // Q + double-buffered K and V
 }
 
-// One work item (split, head, request) run by 128 threads (tid 0..127) that synchronise with
-// named barrier BAR.  smem: attn_smem_bytes(D) bytes, 16-byte aligned.  Returns true on the
-// call that wrote the final output rows of (request, head) (the only split, or the last split to
-// finish, which merges the others in split order).
-template <int D, int BAR>
-__device__ bool attention_item(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
-                               float (*sM)[16], float (*sL)[16], int* s_last) {
-  constexpr int LD = attn_ld<D>();
-  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [kMaxNodes][LD]
-  __nv_bfloat16* sK = sQ + kMaxNodes * LD;                       // [2][kKeyTile][LD]
-  __nv_bfloat16* sV = sK + 2 * kKeyTile * LD;                    // [2][kKeyTile][LD]
+// Keys [k0, k1) that split `split` of n_splits covers in a block of T keys (whole 64-key tiles,
+// the last split possibly shorter or empty).
+__host__ __device__ inline void attn_split_keys(int T, int n_splits, int split, int& k0, int& k1) {
+  const int n_tiles = (T + kKeyTile - 1) / kKeyTile;
+  const int per = (n_tiles + n_splits - 1) / n_splits;
+  const int t0 = split * per;
+  const int t1 = t0 + per < n_tiles ? t0 + per : n_tiles;
+  k0 = t0 * kKeyTile;
+  k1 = t1 * kKeyTile < T ? t1 * kKeyTile : T;
+}
+
+// Per-item geometry shared by the two item variants below.
+template <int D>
+struct AttnItem {
+  const __nv_bfloat16* Kg;  // this (request, head)'s keys / values in the cache: [cap][D]
+  const __nv_bfloat16* Vg;
+  int crow, N, ctx, T, t0, t1, mt, wm, wk, kpw, g, tq, warp, lane;
+  unsigned long long anc0, anc1;
+};
+
+// Fills `it`; false when the request does not run this layer or the item is out of range.
+template <int D>
+__device__ __forceinline__ bool attn_item_setup(const AttnParams& p, int split, int head, int b, int tid,
+                                                AttnItem<D>& it) {
   const StepDesc* st = p.step;
   const PlanDev* pl = p.plan;
   if (b >= st->B || p.slot >= pl->n_act) return false;
-  const int crow = pl->slot_crow[p.slot][b];
-  if (crow < 0) return false;  // request skips this layer: no KV read, no output
+  it.crow = pl->slot_crow[p.slot][b];
+  if (it.crow < 0) return false;  // request skips this layer: no KV read, no output
   const int layer = pl->act_layer[p.slot];
-  const int H = p.n_heads, d = p.d_model;
-  const int N = st->req_nodes[b], ctx = st->req_ctx[b], T = ctx + N;
+  const int H = p.n_heads;
+  it.N = st->req_nodes[b];
+  it.ctx = st->req_ctx[b];
+  it.T = it.ctx + it.N;
   const int row0 = st->req_rowoff[b];
   const size_t cap = static_cast<size_t>(st->kv_cap);
-  const int n_tiles = (T + kKeyTile - 1) / kKeyTile;
+  const int n_tiles = (it.T + kKeyTile - 1) / kKeyTile;
   const int per = (n_tiles + p.n_splits - 1) / p.n_splits;
-  const int t0 = split * per;
-  const int t1 = min(n_tiles, t0 + per);
-  const __nv_bfloat16* Kg =
-      st->kv_layer[layer] + ((static_cast<size_t>(st->req_slot[b]) * 2 + 0) * H + head) * cap * D;
-  const __nv_bfloat16* Vg = Kg + static_cast<size_t>(H) * cap * D;
+  it.t0 = split * per;
+  it.t1 = min(n_tiles, it.t0 + per);
+  it.Kg = st->kv_layer[layer] + ((static_cast<size_t>(st->req_slot[b]) * 2 + 0) * H + head) * cap * D;
+  it.Vg = it.Kg + static_cast<size_t>(H) * cap * D;
+  it.warp = tid >> 5;
+  it.lane = tid & 31;
+  it.mt = it.N <= 16 ? 1 : (it.N <= 32 ? 2 : 4);  // 16-row query tiles
+  const int ksplit = 4 / it.mt;                    // warps sharing one query tile
+  it.wm = it.warp % it.mt;
+  it.wk = it.warp / it.mt;
+  it.kpw = kKeyTile / ksplit;  // keys of each tile this warp scores
+  it.g = it.lane >> 2;
+  it.tq = it.lane & 3;
+  const int qr0 = it.wm * 16 + it.g, qr1 = qr0 + 8;
+  it.anc0 = qr0 < it.N ? st->row_anc[row0 + qr0] : 0ull;
+  it.anc1 = qr1 < it.N ? st->row_anc[row0 + qr1] : 0ull;
+  return true;
+}
 
-  const int warp = tid >> 5, lane = tid & 31;
-  const int mt = N <= 16 ? 1 : (N <= 32 ? 2 : 4);  // 16-row query tiles
-  const int ksplit = 4 / mt;                        // warps sharing one query tile
-  const int wm = warp % mt, wk = warp / mt;
-  const int kpw = kKeyTile / ksplit;  // keys of each tile this warp scores
-  const int g = lane >> 2, tq = lane & 3;
-  const int qr0 = wm * 16 + g, qr1 = qr0 + 8;
-  const unsigned long long anc0 = qr0 < N ? st->row_anc[row0 + qr0] : 0ull;
-  const unsigned long long anc1 = qr1 < N ? st->row_anc[row0 + qr1] : 0ull;
-
-  // Q rows of the request (rows >= N are zero).
-  constexpr int C8 = D / 8;
-  for (int idx = tid; idx < 16 * mt * C8; idx += kAttnThreads) {
+// Q rows of the request into sQ [16 * mt][LD] (rows >= N are zero); cp.async, not committed.
+template <int D>
+__device__ __forceinline__ void attn_load_q(const AttnParams& p, const AttnItem<D>& it, int head, int tid,
+                                            __nv_bfloat16* sQ) {
+  constexpr int LD = attn_ld<D>(), C8 = D / 8;
+  for (int idx = tid; idx < 16 * it.mt * C8; idx += kAttnThreads) {
     const int row = idx / C8, c8 = idx - row * C8;
     __nv_bfloat16* dst = sQ + row * LD + c8 * 8;
-    if (row < N) {
-      cp_async16(dst, p.q + static_cast<size_t>(crow + row) * d + head * D + c8 * 8, 16);
+    if (row < it.N) {
+      cp_async16(dst, p.q + static_cast<size_t>(it.crow + row) * p.d_model + head * D + c8 * 8, 16);
     } else {
       *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
     }
   }
-  auto load_tile = [&](int tile, int buf) {
-    for (int idx = tid; idx < kKeyTile * C8; idx += kAttnThreads) {
-      const int kr = idx / C8, c8 = idx - kr * C8;
-      const int key = tile * kKeyTile + kr;
-      const int bytes = key < T ? 16 : 0;  // keys past the block are zero-filled
-      const size_t src = static_cast<size_t>(key < T ? key : 0) * D + c8 * 8;
-      cp_async16(sK + (buf * kKeyTile + kr) * LD + c8 * 8, Kg + src, bytes);
-      cp_async16(sV + (buf * kKeyTile + kr) * LD + c8 * 8, Vg + src, bytes);
-    }
-  };
-  if (t0 < t1) load_tile(t0, 0);
-  cp_async_commit();
+}
 
+// Keys and values of one 64-key tile into sK / sV [kKeyTile][LD]; keys past the block are
+// zero-filled.  cp.async, not committed.
+template <int D>
+__device__ __forceinline__ void attn_load_tile(const AttnItem<D>& it, int tile, int tid, __nv_bfloat16* sK,
+                                               __nv_bfloat16* sV) {
+  constexpr int LD = attn_ld<D>(), C8 = D / 8;
+  for (int idx = tid; idx < kKeyTile * C8; idx += kAttnThreads) {
+    const int kr = idx / C8, c8 = idx - kr * C8;
+    const int key = tile * kKeyTile + kr;
+    const int bytes = key < it.T ? 16 : 0;
+    const size_t src = static_cast<size_t>(key < it.T ? key : 0) * D + c8 * 8;
+    cp_async16(sK + kr * LD + c8 * 8, it.Kg + src, bytes);
+    cp_async16(sV + kr * LD + c8 * 8, it.Vg + src, bytes);
+  }
+}
+
+// Online-softmax state of one warp: O accumulators of its two query rows (per lane fragment),
+// running max and sum in log2 units, and the Q fragments.
+template <int D>
+struct AttnAcc {
   float o[D / 8][4];
-#pragma unroll
-  for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+  float m0, m1, l0, l1;
   uint32_t qf[D / 16][4];
+};
 
-  for (int tile = t0; tile < t1; ++tile) {
-    const int buf = (tile - t0) & 1;
-    if (tile + 1 < t1) load_tile(tile + 1, buf ^ 1);
-    cp_async_commit();
-    cp_async_wait<1>();
-    named_bar_sync(BAR, kAttnThreads);
-    if (tile == t0) {
+template <int D>
+__device__ __forceinline__ void attn_acc_init(AttnAcc<D>& a) {
 #pragma unroll
-      for (int ks = 0; ks < D / 16; ++ks)
-        ldmatrix_x4(qf[ks], sQ + (wm * 16 + (lane & 15)) * LD + ks * 16 + (lane >> 4) * 8);
-    }
-    const int kbase = wk * kpw;
-    const __nv_bfloat16* tK = sK + (buf * kKeyTile + kbase) * LD;
-    const __nv_bfloat16* tV = sV + (buf * kKeyTile + kbase) * LD;
-    float s[8][4];
+  for (int i = 0; i < D / 8; ++i) a.o[i][0] = a.o[i][1] = a.o[i][2] = a.o[i][3] = 0.f;
+  a.m0 = a.m1 = -INFINITY;
+  a.l0 = a.l1 = 0.f;
+}
+
+template <int D>
+__device__ __forceinline__ void attn_load_qfrag(const AttnItem<D>& it, const __nv_bfloat16* sQ, AttnAcc<D>& a) {
+  constexpr int LD = attn_ld<D>();
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-    const int npairs = kpw / 16;
+  for (int ks = 0; ks < D / 16; ++ks)
+    ldmatrix_x4(a.qf[ks], sQ + (it.wm * 16 + (it.lane & 15)) * LD + ks * 16 + (it.lane >> 4) * 8);
+}
+
+// One online-softmax update over up to four 16-key blocks of this warp (kp / vp: their first K
+// and V rows in shared memory, key0: the key index of their first row): scores, context /
+// ancestor mask, rescale, P.V.  The blocks' score MMAs are independent, so a group of blocks
+// from several resident tiles keeps the tensor pipe busier than one block at a time.
+template <int D>
+__device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __nv_bfloat16* const (&kp)[4],
+                                                 const __nv_bfloat16* const (&vp)[4], const int (&key0)[4], int n,
+                                                 float scale_log2, AttnAcc<D>& a) {
+  constexpr int LD = attn_ld<D>();
+  const int lane = it.lane;
+  float s[8][4];
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+#pragma unroll
+  for (int ks = 0; ks < D / 16; ++ks) {
 #pragma unroll
     for (int np = 0; np < 4; ++np) {
-      if (np < npairs) {
-#pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          uint32_t kb4[4];
-          ldmatrix_x4(kb4, tK + (np * 16 + (lane & 7) + ((lane >> 4) << 3)) * LD + ks * 16 + ((lane >> 3) & 1) * 8);
-          mma_bf16_16816(s[2 * np], qf[ks], kb4);
-          mma_bf16_16816(s[2 * np + 1], qf[ks], kb4 + 2);
-        }
+      if (np < n) {
+        uint32_t kb4[4];
+        ldmatrix_x4(kb4, kp[np] + ((lane & 7) + ((lane >> 4) << 3)) * LD + ks * 16 + ((lane >> 3) & 1) * 8);
+        mma_bf16_16816(s[2 * np], a.qf[ks], kb4);
+        mma_bf16_16816(s[2 * np + 1], a.qf[ks], kb4 + 2);
       }
     }
-    // scale to log2 units and apply the context / ancestor mask
-    const int key0 = tile * kKeyTile + kbase;
-    const bool need_mask = tile * kKeyTile + kKeyTile > ctx;
-    float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-      if (nt < 2 * npairs) {
-#pragma unroll
-        for (int e2 = 0; e2 < 4; ++e2) {
-          float val = s[nt][e2] * p.scale_log2;
-          if (need_mask) {
-            const int key = key0 + nt * 8 + tq * 2 + (e2 & 1);
-            const unsigned long long anc = e2 < 2 ? anc0 : anc1;
-            if (key >= T || (key >= ctx && !((anc >> (key - ctx)) & 1ull))) val = -INFINITY;
-          }
-          s[nt][e2] = val;
-        }
-        mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
-        mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
-      }
-    }
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-    const float base0 = mn0 == -INFINITY ? 0.f : mn0;
-    const float base1 = mn1 == -INFINITY ? 0.f : mn1;
-    const float al0 = exp2f(m0 - base0), al1 = exp2f(m1 - base1);
-    m0 = mn0;
-    m1 = mn1;
-    float rs0 = 0.f, rs1 = 0.f;
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-      if (nt < 2 * npairs) {
-        s[nt][0] = exp2f(s[nt][0] - base0);
-        s[nt][1] = exp2f(s[nt][1] - base0);
-        s[nt][2] = exp2f(s[nt][2] - base1);
-        s[nt][3] = exp2f(s[nt][3] - base1);
-        rs0 += s[nt][0] + s[nt][1];
-        rs1 += s[nt][2] + s[nt][3];
-      }
-    }
-    l0 = l0 * al0 + rs0;
-    l1 = l1 * al1 + rs1;
-#pragma unroll
-    for (int dt = 0; dt < D / 8; ++dt) {
-      o[dt][0] *= al0;
-      o[dt][1] *= al0;
-      o[dt][2] *= al1;
-      o[dt][3] *= al1;
-    }
-#pragma unroll
-    for (int kc = 0; kc < 4; ++kc) {
-      if (kc < npairs) {
-        uint32_t a[4];
-        a[0] = pack_bf16(s[2 * kc][0], s[2 * kc][1]);
-        a[1] = pack_bf16(s[2 * kc][2], s[2 * kc][3]);
-        a[2] = pack_bf16(s[2 * kc + 1][0], s[2 * kc + 1][1]);
-        a[3] = pack_bf16(s[2 * kc + 1][2], s[2 * kc + 1][3]);
-#pragma unroll
-        for (int dp = 0; dp < D / 16; ++dp) {
-          uint32_t vb[4];
-          ldmatrix_x4_trans(vb, tV + (kc * 16 + (lane & 7) + (((lane >> 3) & 1) << 3)) * LD + dp * 16 + (lane >> 4) * 8);
-          mma_bf16_16816(o[2 * dp], a, vb);
-          mma_bf16_16816(o[2 * dp + 1], a, vb + 2);
-        }
-      }
-    }
-    named_bar_sync(BAR, kAttnThreads);
   }
-  cp_async_wait<0>();
+  // scale to log2 units and apply the context / ancestor mask
+  float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt) {
+    if (nt < 2 * n) {
+      const int kb0 = key0[nt >> 1] + (nt & 1) * 8;
+      const bool need_mask = key0[nt >> 1] + 16 > it.ctx;
+#pragma unroll
+      for (int e2 = 0; e2 < 4; ++e2) {
+        float val = s[nt][e2] * scale_log2;
+        if (need_mask) {
+          const int key = kb0 + it.tq * 2 + (e2 & 1);
+          const unsigned long long anc = e2 < 2 ? it.anc0 : it.anc1;
+          if (key >= it.T || (key >= it.ctx && !((anc >> (key - it.ctx)) & 1ull))) val = -INFINITY;
+        }
+        s[nt][e2] = val;
+      }
+      mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
+      mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
+    }
+  }
+  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+  const float mn0 = fmaxf(a.m0, mx0), mn1 = fmaxf(a.m1, mx1);
+  const float base0 = mn0 == -INFINITY ? 0.f : mn0;
+  const float base1 = mn1 == -INFINITY ? 0.f : mn1;
+  const float al0 = exp2f(a.m0 - base0), al1 = exp2f(a.m1 - base1);
+  a.m0 = mn0;
+  a.m1 = mn1;
+  float rs0 = 0.f, rs1 = 0.f;
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt) {
+    if (nt < 2 * n) {
+      s[nt][0] = exp2f(s[nt][0] - base0);
+      s[nt][1] = exp2f(s[nt][1] - base0);
+      s[nt][2] = exp2f(s[nt][2] - base1);
+      s[nt][3] = exp2f(s[nt][3] - base1);
+      rs0 += s[nt][0] + s[nt][1];
+      rs1 += s[nt][2] + s[nt][3];
+    }
+  }
+  a.l0 = a.l0 * al0 + rs0;
+  a.l1 = a.l1 * al1 + rs1;
+#pragma unroll
+  for (int dt = 0; dt < D / 8; ++dt) {
+    a.o[dt][0] *= al0;
+    a.o[dt][1] *= al0;
+    a.o[dt][2] *= al1;
+    a.o[dt][3] *= al1;
+  }
+#pragma unroll
+  for (int kc = 0; kc < 4; ++kc) {
+    if (kc < n) {
+      uint32_t pa[4];
+      pa[0] = pack_bf16(s[2 * kc][0], s[2 * kc][1]);
+      pa[1] = pack_bf16(s[2 * kc][2], s[2 * kc][3]);
+      pa[2] = pack_bf16(s[2 * kc + 1][0], s[2 * kc + 1][1]);
+      pa[3] = pack_bf16(s[2 * kc + 1][2], s[2 * kc + 1][3]);
+#pragma unroll
+      for (int dp = 0; dp < D / 16; ++dp) {
+        uint32_t vb[4];
+        ldmatrix_x4_trans(vb, vp[kc] + ((lane & 7) + (((lane >> 3) & 1) << 3)) * LD + dp * 16 + (lane >> 4) * 8);
+        mma_bf16_16816(a.o[2 * dp], pa, vb);
+        mma_bf16_16816(a.o[2 * dp + 1], pa, vb + 2);
+      }
+    }
+  }
+}
 
-  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+// This warp's keys of one resident 64-key tile (K / V buffers sK, sV).
+template <int D>
+__device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, const __nv_bfloat16* sK,
+                                               const __nv_bfloat16* sV, float scale_log2, AttnAcc<D>& a) {
+  constexpr int LD = attn_ld<D>();
+  const int kbase = it.wk * it.kpw;
+  const __nv_bfloat16* kp[4];
+  const __nv_bfloat16* vp[4];
+  int key0[4];
+#pragma unroll
+  for (int np = 0; np < 4; ++np) {
+    kp[np] = sK + (kbase + np * 16) * LD;
+    vp[np] = sV + (kbase + np * 16) * LD;
+    key0[np] = tile * kKeyTile + kbase + np * 16;
+  }
+  attn_blocks_step<D>(it, kp, vp, key0, it.kpw / 16, scale_log2, a);
+}
 
-  // Merge the warps that share a query tile (different key subsets) through shared memory.
+// Merge the warps that share a query tile through shared memory (sO: [4][16][D] floats, any
+// free 16-byte-aligned buffer of 32 KiB for D = 128), then write this split's result: the
+// normalised output when there is one split, else the partial, and the last split of
+// (request, head) merges all partials in split order.  Returns true on the call that wrote the
+// final output rows.  `stamp(k)` records diagnostics (k = 2, 3, 4).
+template <int D, int BAR, typename Stamp>
+__device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<D>& it, AttnAcc<D>& a, int split,
+                                            int head, int b, int tid, float* sO, float (*sM)[16], float (*sL)[16],
+                                            int* s_last, Stamp stamp) {
+  const int H = p.n_heads, d = p.d_model;
+  const int N = it.N, crow = it.crow, mt = it.mt, warp = it.warp, g = it.g, tq = it.tq;
+  a.l0 += __shfl_xor_sync(0xffffffffu, a.l0, 1);
+  a.l0 += __shfl_xor_sync(0xffffffffu, a.l0, 2);
+  a.l1 += __shfl_xor_sync(0xffffffffu, a.l1, 1);
+  a.l1 += __shfl_xor_sync(0xffffffffu, a.l1, 2);
+
   named_bar_sync(BAR, kAttnThreads);
-  float* sO = reinterpret_cast<float*>(sK);  // [4][16][D] (K/V buffers are free now)
 #pragma unroll
   for (int dt = 0; dt < D / 8; ++dt) {
     const int col = dt * 8 + tq * 2;
-    sO[(warp * 16 + g) * D + col] = o[dt][0];
-    sO[(warp * 16 + g) * D + col + 1] = o[dt][1];
-    sO[(warp * 16 + g + 8) * D + col] = o[dt][2];
-    sO[(warp * 16 + g + 8) * D + col + 1] = o[dt][3];
+    sO[(warp * 16 + g) * D + col] = a.o[dt][0];
+    sO[(warp * 16 + g) * D + col + 1] = a.o[dt][1];
+    sO[(warp * 16 + g + 8) * D + col] = a.o[dt][2];
+    sO[(warp * 16 + g + 8) * D + col + 1] = a.o[dt][3];
   }
   if (tq == 0) {
-    sM[warp][g] = m0;
-    sM[warp][g + 8] = m1;
-    sL[warp][g] = l0;
-    sL[warp][g + 8] = l1;
+    sM[warp][g] = a.m0;
+    sM[warp][g + 8] = a.m1;
+    sL[warp][g] = a.l0;
+    sL[warp][g + 8] = a.l1;
   }
   named_bar_sync(BAR, kAttnThreads);
 
@@ -231,7 +296,8 @@ __device__ bool attention_item(const AttnParams& p, int split, int head, int b, 
     if (p.n_splits == 1) {
       if (!(L > 0.f)) report(p.status, kStatusCheck);
       const float val = L > 0.f ? O / L : 0.f;
-      p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
+      p.o[p.o_tiled_npad ? xt_index(crow + i, head * D + dd, p.o_tiled_npad)
+                         : static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
     } else {
       const size_t pi = (ph + split) * kMaxNodes + i;
       __stcg(&p.part_o[pi * D + dd], O);
@@ -242,6 +308,7 @@ __device__ bool attention_item(const AttnParams& p, int split, int head, int b, 
     }
   }
   if (p.n_splits == 1) return true;
+  stamp(2);
 
   // Last CTA of (request, head) merges the splits in order.
   __threadfence();
@@ -253,24 +320,176 @@ __device__ bool attention_item(const AttnParams& p, int split, int head, int b, 
     if (*s_last) atomicExch(cnt, 0);
   }
   named_bar_sync(BAR, kAttnThreads);
+  stamp(3);
   if (!*s_last) return false;
   __threadfence();
+  constexpr int kMergeRegs = 8;  // splits whose partials are loaded at once
   for (int idx = tid; idx < N * D; idx += kAttnThreads) {
     const int i = idx / D, dd = idx - i * D;
-    float M = -INFINITY;
-    for (int sp = 0; sp < p.n_splits; ++sp) M = fmaxf(M, __ldcg(&p.part_ml[((ph + sp) * kMaxNodes + i) * 2]));
-    const float base = M == -INFINITY ? 0.f : M;
-    float L = 0.f, O = 0.f;
-    for (int sp = 0; sp < p.n_splits; ++sp) {
-      const size_t pi = (ph + sp) * kMaxNodes + i;
-      const float f = exp2f(__ldcg(&p.part_ml[pi * 2]) - base);
-      L += f * __ldcg(&p.part_ml[pi * 2 + 1]);
-      O += f * __ldcg(&p.part_o[pi * D + dd]);
+    float M = -INFINITY, L = 0.f, O = 0.f;
+    if (p.n_splits <= kMergeRegs) {
+      // every split's (max, sum, O) in one round of loads, then the same fixed-order merge
+      float pm[kMergeRegs], pl[kMergeRegs], po[kMergeRegs];
+#pragma unroll
+      for (int sp = 0; sp < kMergeRegs; ++sp) {
+        if (sp < p.n_splits) {
+          const size_t pi = (ph + sp) * kMaxNodes + i;
+          pm[sp] = __ldcg(&p.part_ml[pi * 2]);
+          pl[sp] = __ldcg(&p.part_ml[pi * 2 + 1]);
+          po[sp] = __ldcg(&p.part_o[pi * D + dd]);
+        }
+      }
+#pragma unroll
+      for (int sp = 0; sp < kMergeRegs; ++sp)
+        if (sp < p.n_splits) M = fmaxf(M, pm[sp]);
+      const float base = M == -INFINITY ? 0.f : M;
+#pragma unroll
+      for (int sp = 0; sp < kMergeRegs; ++sp) {
+        if (sp < p.n_splits) {
+          const float f = exp2f(pm[sp] - base);
+          L += f * pl[sp];
+          O += f * po[sp];
+        }
+      }
+    } else {
+      for (int sp = 0; sp < p.n_splits; ++sp) M = fmaxf(M, __ldcg(&p.part_ml[((ph + sp) * kMaxNodes + i) * 2]));
+      const float base = M == -INFINITY ? 0.f : M;
+      for (int sp = 0; sp < p.n_splits; ++sp) {
+        const size_t pi = (ph + sp) * kMaxNodes + i;
+        const float f = exp2f(__ldcg(&p.part_ml[pi * 2]) - base);
+        L += f * __ldcg(&p.part_ml[pi * 2 + 1]);
+        O += f * __ldcg(&p.part_o[pi * D + dd]);
+      }
     }
     if (!(L > 0.f)) report(p.status, kStatusCheck);
-    p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(L > 0.f ? O / L : 0.f);
+    p.o[p.o_tiled_npad ? xt_index(crow + i, head * D + dd, p.o_tiled_npad)
+                       : static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(L > 0.f ? O / L : 0.f);
   }
+  stamp(4);
   return true;
+}
+
+// One work item (split, head, request) run by 128 threads (tid 0..127) that synchronise with
+// named barrier BAR, streaming its key tiles through a double buffer.  smem: attn_smem_bytes(D)
+// bytes, 16-byte aligned.  Returns true on the call that wrote the final output rows of
+// (request, head) (the only split, or the last split to finish, which merges the others in
+// split order).
+template <int D, int BAR>
+__device__ bool attention_item(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
+                               float (*sM)[16], float (*sL)[16], int* s_last) {
+  constexpr int LD = attn_ld<D>();
+  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [kMaxNodes][LD]
+  __nv_bfloat16* sK = sQ + kMaxNodes * LD;                       // [2][kKeyTile][LD]
+  __nv_bfloat16* sV = sK + 2 * kKeyTile * LD;                    // [2][kKeyTile][LD]
+  AttnItem<D> it;
+  if (!attn_item_setup<D>(p, split, head, b, tid, it)) return false;
+  attn_load_q<D>(p, it, head, tid, sQ);
+  if (it.t0 < it.t1) attn_load_tile<D>(it, it.t0, tid, sK, sV);
+  cp_async_commit();
+  AttnAcc<D> a;
+  attn_acc_init<D>(a);
+  for (int tile = it.t0; tile < it.t1; ++tile) {
+    const int buf = (tile - it.t0) & 1;
+    if (tile + 1 < it.t1)
+      attn_load_tile<D>(it, tile + 1, tid, sK + (buf ^ 1) * kKeyTile * LD, sV + (buf ^ 1) * kKeyTile * LD);
+    cp_async_commit();
+    cp_async_wait<1>();
+    named_bar_sync(BAR, kAttnThreads);
+    if (tile == it.t0) attn_load_qfrag<D>(it, sQ, a);
+    attn_tile_step<D>(it, tile, sK + buf * kKeyTile * LD, sV + buf * kKeyTile * LD, p.scale_log2, a);
+    named_bar_sync(BAR, kAttnThreads);
+  }
+  cp_async_wait<0>();
+  return attn_finish<D, BAR>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sK), sM, sL, s_last,
+                             [](int) {});
+}
+
+// Tiles of K and V that attention_item_resident keeps resident in `smem_bytes` of shared memory.
+__host__ __device__ inline int attn_resident_tiles(int head_dim, size_t smem_bytes) {
+  const size_t ld = head_dim + 8, q = static_cast<size_t>(kMaxNodes) * ld * 2, tile = 2ull * kKeyTile * ld * 2;
+  return smem_bytes > q ? static_cast<int>((smem_bytes - q) / tile) : 0;
+}
+
+// The same work item with all of the split's key tiles resident at once (in rounds of
+// attn_resident_tiles(D, smem_bytes) tiles when they do not all fit): loads of tiles that hold
+// only context keys (which this step does not write) are issued first, then `wait_inputs()`
+// waits for the step's own Q/K/V rows, then Q and the remaining tiles are loaded.  One memory
+// round trip per round instead of one per tile.  Needs smem_bytes >= the Q buffer + 1 tile and
+// the 32 KiB merge buffer (D = 128) to fit behind Q.  If wait_inputs() fails, drains its copies
+// and returns false without output.
+template <int D, int BAR, typename Wait>
+__device__ bool attention_item_resident(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
+                                        size_t smem_bytes, float (*sM)[16], float (*sL)[16], int* s_last,
+                                        unsigned long long* trace, Wait wait_inputs, bool& failed) {
+  constexpr int LD = attn_ld<D>();
+  auto stamp = [&](int k) {
+    if (trace && tid == 0) trace[k] = globaltimer_ns();
+  };
+  failed = false;
+  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [kMaxNodes][LD]
+  __nv_bfloat16* sKV = sQ + kMaxNodes * LD;                      // per tile: K [kKeyTile][LD], V [kKeyTile][LD]
+  const int R = attn_resident_tiles(D, smem_bytes);
+  AttnItem<D> it;
+  const bool run = attn_item_setup<D>(p, split, head, b, tid, it);
+  if (!run || R < 1) {
+    failed = !wait_inputs();
+    return false;
+  }
+  AttnAcc<D> a;
+  attn_acc_init<D>(a);
+  for (int r0 = it.t0; r0 < it.t1 || r0 == it.t0; r0 += R) {
+    const int r1 = min(it.t1, r0 + R);
+    const bool first = r0 == it.t0;
+    // context-only tiles do not depend on this step
+    for (int tile = r0; tile < r1; ++tile)
+      if (!first || (tile + 1) * kKeyTile <= it.ctx)
+        attn_load_tile<D>(it, tile, tid, sKV + (tile - r0) * 2 * kKeyTile * LD,
+                          sKV + ((tile - r0) * 2 + 1) * kKeyTile * LD);
+    cp_async_commit();
+    if (first) {
+      if (!wait_inputs()) {
+        cp_async_wait<0>();
+        failed = true;
+        return false;
+      }
+      attn_load_q<D>(p, it, head, tid, sQ);
+      for (int tile = r0; tile < r1; ++tile)
+        if ((tile + 1) * kKeyTile > it.ctx)
+          attn_load_tile<D>(it, tile, tid, sKV + (tile - r0) * 2 * kKeyTile * LD,
+                            sKV + ((tile - r0) * 2 + 1) * kKeyTile * LD);
+      cp_async_commit();
+    }
+    cp_async_wait<0>();
+    named_bar_sync(BAR, kAttnThreads);
+    if (first) {
+      stamp(0);
+      attn_load_qfrag<D>(it, sQ, a);
+    }
+    {
+      // this warp's 16-key blocks of the round, four per softmax update
+      const int npairs = it.kpw / 16, kbase = it.wk * it.kpw;
+      const int nb = (r1 - r0) * npairs;
+      for (int q0 = 0; q0 < nb; q0 += 4) {
+        const __nv_bfloat16* kp[4];
+        const __nv_bfloat16* vp[4];
+        int key0[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int q = min(q0 + j, nb - 1);
+          const int tl = q / npairs, np = q - tl * npairs;
+          kp[j] = sKV + (tl * 2 * kKeyTile + kbase + np * 16) * LD;
+          vp[j] = sKV + ((tl * 2 + 1) * kKeyTile + kbase + np * 16) * LD;
+          key0[j] = (r0 + tl) * kKeyTile + kbase + np * 16;
+        }
+        attn_blocks_step<D>(it, kp, vp, key0, min(4, nb - q0), p.scale_log2, a);
+      }
+    }
+    named_bar_sync(BAR, kAttnThreads);  // the next round overwrites the tiles
+    if (r1 >= it.t1) break;
+  }
+  stamp(1);
+  if (trace && it.lane == 0) trace[5 + it.warp] = globaltimer_ns();
+  return attn_finish<D, BAR>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sKV), sM, sL, s_last, stamp);
 }
 
 }  // namespace tss

@@ -165,6 +165,20 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* m, uin
 }
 
 // Linear bulk copy global -> shared of `bytes` (multiple of 16, both addresses 16-byte aligned).
+// L2 policy for data read exactly once (streamed weights): evicted before anything else.
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ void bulk_load_hint(void* dst, const void* src, uint32_t bytes, uint64_t* bar,
+                                               uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
 __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                    smem_u32(dst)),
@@ -182,6 +196,15 @@ __device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes
 // [layer][row tile][k-block].  One linear bulk copy then fills a pipeline stage.
 constexpr uint32_t kTileBytes = 128 * 64 * 2;
 constexpr size_t kTileElems = 128 * 64;
+
+// Activation operands of the persistent kernel use the same idea: per 64-column k-block a
+// contiguous [n_pad rows][64] bf16 block in 128-byte-swizzled order, blocks by k-block, so the
+// operand of consecutive k-blocks is one linear bulk copy.  Element index of (row n, column k):
+__host__ __device__ __forceinline__ size_t xt_index(int n, int k, int n_pad) {
+  const int kb = k >> 6, kc = k & 63;
+  return static_cast<size_t>(kb) * n_pad * 64 + static_cast<size_t>(n) * 64 +
+         static_cast<size_t>((((kc >> 3) ^ (n & 7)) << 3) | (kc & 7));
+}
 
 // ------------------------------------------------------------------------------------------
 // tcgen05: tensor memory and the 5th-generation MMA

@@ -70,6 +70,7 @@ struct AttnParams {
   float* part_ml;          // [B][H][n_splits][kMaxNodes][2]
   int* counters;           // [B][H], self-resetting
   int* status;
+  int o_tiled_npad;        // 0: o row-major [row][d]; > 0: k-block tiled for this MMA width
 };
 size_t attn_smem_bytes(int head_dim);
 cudaError_t attn_prepare();
@@ -92,6 +93,7 @@ struct MiscParams {
   const int* amax_idx;
   int n_vtiles;
   int* status;
+  int xt_npad;  // persistent path: MMA width of the k-block tiled activation operands
 };
 
 cudaError_t misc_prepare();
@@ -111,6 +113,12 @@ cudaError_t launch_tile_weights(const __nv_bfloat16* src, __nv_bfloat16* dst, in
 // Persistent verify kernel (verify_mk.cu).
 struct MkParams {
   int n_act, d, H, D, F_pad, Ft, V, V_pad, n_pad, stages, attn_splits, B, max_tiles;
+  int kps;  // k-blocks (16 KiB of weights each) per pipeline stage
+  int l2_pace;  // SM clock cycles between L2 prefetches of 16 KiB (0: unpaced)
+  int w_evict_first;  // stream weights with the evict-first L2 policy
+  int pf_attn;  // 16 KiB weight blocks of the O phase warmed into L2 while the attention runs
+  int pf_next;  // blocks of the next phase (beyond the ring) warmed into L2 when a phase ends
+  int attn_extra;  // shared memory behind the ring that only the attention uses (bytes)
   int l2_ahead;  // weight tiles per CTA prefetched into L2 ahead of the smem ring (0: off)
   unsigned long long* trace;  // optional timeline [grid][mk_trace_slots()], nullptr when off
   float eps, scale_log2;
@@ -148,14 +156,11 @@ struct MkParams {
   int* status;
   int* abort_word;
 };
-struct MkTensorMaps {
-  CUtensorMap xo, xact, xn;
-};
-size_t mk_smem_bytes(int n_pad, int stages, int head_dim);
+size_t mk_smem_bytes(int n_pad, int stages, int head_dim, int kps, size_t attn_extra);
 size_t mk_trace_slots();
 cudaError_t mk_prepare();
 int mk_max_blocks_per_sm(int head_dim, size_t smem);
-cudaError_t launch_verify_mk(const MkTensorMaps& tm, const MkParams& p, int grid, size_t smem, cudaStream_t s);
+cudaError_t launch_verify_mk(const MkParams& p, int grid, size_t smem, cudaStream_t s);
 
 // Records the message tss_last_error() returns on the calling thread.
 void set_last_error(const std::string& msg);

@@ -397,7 +397,7 @@ __global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float
   }
   __syncthreads();
   const float* gain = s_l0 >= 0 ? p.g_attn + static_cast<size_t>(s_l0) * p.d_model : p.g_final;
-  __nv_bfloat16* xn = s_crow >= 0 ? p.xn + static_cast<size_t>(s_crow) * p.d_model : nullptr;
+  const int xrow = s_crow;
   const __nv_bfloat16* e = p.embed + static_cast<size_t>(tok) * p.d_model;
   float* h = p.h + static_cast<size_t>(m) * p.d_model;
   const int half = threadIdx.x >> 7, r = threadIdx.x & 127;
@@ -408,7 +408,9 @@ __global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float
     if (t < n_t) {
       const float x = __bfloat162float(e[t * 128 + r]);
       h[t * 128 + r] = x;
-      if (xn) xn[t * 128 + r] = __float2bfloat16_rn(x * gain[t * 128 + r]);
+      if (xrow >= 0)
+        p.xn[p.xt_npad ? xt_index(xrow, t * 128 + r, p.xt_npad) : static_cast<size_t>(xrow) * p.d_model + t * 128 + r] =
+            __float2bfloat16_rn(x * gain[t * 128 + r]);
       sq = x * x;
     }
 #pragma unroll

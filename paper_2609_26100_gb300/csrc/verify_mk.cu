@@ -115,6 +115,23 @@ __device__ bool mk_wait_flag(const unsigned long long* f, unsigned long long tar
   }
 }
 
+// Bounded wait until this CTA's attention of QKV slot `slot` has released the ring.
+__device__ bool mk_wait_gate(const volatile int* gate, int slot, const MkShared& sh) {
+  if (*gate > slot) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (*gate > slot) return true;
+    if ((i & 255) == 0) {
+      if (mk_aborted(sh)) return false;
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        mk_fail(sh);
+        return false;
+      }
+    }
+    __nanosleep(32);
+  }
+}
+
 // Bounded mbarrier wait that also leaves when another CTA aborted.
 __device__ bool mk_wait_bar(uint64_t* bar, uint32_t parity, const MkShared& sh) {
   if (mbar_try_wait(bar, parity)) return true;
@@ -139,7 +156,9 @@ struct MkPhase {
 // trace[cta][pi * 8 + 2 * role + {0: first, 1: last}], roles 0 weight TMA, 1 B operand, 2 MMA,
 // 3 epilogue; the attention of slot j at [kMkTracePhases * 8 + 2j + {0,1}].
 constexpr int kMkTracePhases = 4 * kMaxLayers + 1;
-constexpr int kMkTraceSlots = kMkTracePhases * 8 + 2 * kMaxLayers;
+constexpr int kMkTraceSub = kMkTracePhases * 8 + 2 * kMaxLayers;  // epilogue sub-steps of a phase's last segment
+constexpr int kMkTraceAttn = kMkTraceSub + kMkTracePhases * 8;  // sub-steps of the slot-1 attention item
+constexpr int kMkTraceSlots = kMkTraceAttn + 16;
 __device__ __forceinline__ void mk_trace(const MkParams& p, int idx) {
   if (p.trace) p.trace[static_cast<size_t>(blockIdx.x) * kMkTraceSlots + idx] = globaltimer_ns();
 }
@@ -174,6 +193,24 @@ __device__ __forceinline__ const __nv_bfloat16* mk_weights(const MkParams& p, co
                               : ph.kind == kMkDown ? p.w_down
                                                    : p.w_lm;
   return base + static_cast<size_t>(ph.layer) * blocks * kTileElems;
+}
+
+// CTA c's stream-K range of a phase over geff = min(grid, iterations) CTAs.
+__device__ __forceinline__ void mk_range(const MkPhase& ph, int c, int G, long long& it0, long long& it1, int& geff);
+
+// Warm L2 with blocks [skip, skip + count) of CTA c's range of phase pi: the range is one
+// contiguous run of pre-tiled weight blocks, so this is one bulk prefetch.
+__device__ void mk_prefetch_phase(const MkParams& p, const PlanDev* pl, int pi, int n_phases, int c, int G,
+                                  long long skip, long long count) {
+  if (pi >= n_phases || count <= 0) return;
+  const MkPhase ph = mk_phase(p, pl, pi);
+  long long it0, it1;
+  int geff;
+  mk_range(ph, c, G, it0, it1, geff);
+  const long long a = it0 + skip;
+  const long long b = a + count < it1 ? a + count : it1;
+  if (b <= a) return;
+  bulk_prefetch_l2(mk_weights(p, ph) + static_cast<size_t>(a) * kTileElems, static_cast<uint32_t>(b - a) * kMkWBytes);
 }
 
 // CTA c's stream-K range of a phase over geff = min(grid, iterations) CTAs.
@@ -226,6 +263,11 @@ struct MkEpi {
   float* redv;   // [4][16]
   int* redi;     // [4][16]
   float* rs;     // [kMaxRows] per-row RMSNorm factors of the current phase
+  const float* rcos;  // [16][D/2] RoPE cos / sin of the first 16 rows (QKV), staged at phase start
+  const float* rsin;
+  const float* gnext;  // residual phases: RMSNorm gain of the next norm phase
+  bool direct_xn;      // residual phases: the next norm phase runs the same rows in the same order,
+                       // so the epilogue writes its B operand straight from the updated h
   int q, lane, et;
 };
 
@@ -276,8 +318,8 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
         rot[jj] = 0.f;
         if (j0 + jj < e.M) {
           const int pos = e.pos[j0 + jj];
-          const float c = p.rope_cos[static_cast<size_t>(pos) * half + i];
-          const float s = p.rope_sin[static_cast<size_t>(pos) * half + i];
+          const float c = j0 == 0 ? e.rcos[jj * half + i] : p.rope_cos[static_cast<size_t>(pos) * half + i];
+          const float s = j0 == 0 ? e.rsin[jj * half + i] : p.rope_sin[static_cast<size_t>(pos) * half + i];
           const float pv = e.xch[jj * 128 + pr];
           rot[jj] = dim < half ? val[jj] * c - pv * s : val[jj] * c + pv * s;
         }
@@ -302,6 +344,7 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
   } else if (ph.kind == kMkO || ph.kind == kMkDown) {
     // residual add, then this tile's partial sum of squares of the updated rows
     const int o = t * 128 + r;
+    const float gn = e.direct_xn ? e.gnext[o] : 0.f;
     float sq[16];
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) {
@@ -312,6 +355,7 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
         const float nv = __ldcg(hp) + v[jj];
         *hp = nv;
         sq[jj] = nv * nv;
+        if (e.direct_xn) p.xn[xt_index(j, o, p.n_pad)] = __float2bfloat16_rn(nv * gn);
       }
     }
 #pragma unroll
@@ -342,7 +386,7 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
         if (j < e.M) {
           const float g = v[jj] * e.rs[j];
           const float u = e.xch[jj * 128 + r + 64] * e.rs[j];
-          p.act[static_cast<size_t>(j) * p.F_pad + fcol] = __float2bfloat16_rn(g / (1.f + expf(-g)) * u);
+          p.act[xt_index(j, fcol, p.n_pad)] = __float2bfloat16_rn(g / (1.f + expf(-g)) * u);
         }
       }
     }
@@ -421,7 +465,7 @@ __device__ void mk_write_next_xn(const MkParams& p, const PlanDev* pl, const MkP
       hv[u] = n0 + u < M ? __ldcg(&p.h[static_cast<size_t>(rows[n0 + u]) * p.d + f]) : 0.f;
 #pragma unroll
     for (int u = 0; u < 8; ++u)
-      if (n0 + u < M) p.xn[static_cast<size_t>(n0 + u) * p.d + f] = __float2bfloat16_rn(hv[u] * gf);
+      if (n0 + u < M) p.xn[xt_index(n0 + u, f, p.n_pad)] = __float2bfloat16_rn(hv[u] * gf);
   }
 }
 
@@ -437,16 +481,16 @@ __device__ __forceinline__ unsigned long long* mk_tile_flag(const MkParams& p, i
 
 template <int D>
 __global__ void __launch_bounds__(kMkThreads, 1)
-    verify_mk_kernel(const __grid_constant__ CUtensorMap tm_xo, const __grid_constant__ CUtensorMap tm_xact,
-                     const __grid_constant__ CUtensorMap tm_xn, const MkParams p) {
+    verify_mk_kernel(const MkParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const int S = p.stages, n_pad = p.n_pad;
-  const uint32_t x_bytes = static_cast<uint32_t>(n_pad) * 128u;
+  const int S = p.stages, n_pad = p.n_pad, KPS = p.kps;
+  const uint32_t x_bytes = static_cast<uint32_t>(n_pad) * 128u;  // one k-block of the B operand
+  const uint32_t sw_bytes = KPS * kMkWBytes, sx_bytes = KPS * x_bytes;
   uint8_t* sW = base;
-  uint8_t* sX = sW + static_cast<size_t>(S) * kMkWBytes;
-  uint8_t* s_attn = sX + static_cast<size_t>(S) * x_bytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(s_attn + attn_smem_bytes_impl(D));
+  uint8_t* sX = sW + static_cast<size_t>(S) * sw_bytes;
+  uint8_t* s_attn = sX + static_cast<size_t>(S) * sx_bytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(s_attn + p.attn_extra);
   uint64_t* empty = full + S;
   uint64_t* accf = empty + S;
   uint64_t* acce = accf + kMkMaxAcc;
@@ -462,12 +506,15 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   int* s_kvslot = s_pos + kMaxRows;
   int* s_kvrow = s_kvslot + kMaxRows;
   int* s_nrows = s_kvrow + kMaxRows;
+  float* s_rope = reinterpret_cast<float*>(s_nrows + kMaxRows);  // [2][16][64]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int NB = mk_acc_bufs(n_pad);
   const uint32_t ncols = gemm_tmem_cols(n_pad, NB);
   const PlanDev* pl = p.plan;
   volatile int* w_pos = misc + 8;  // weight tiles the TMA producer has issued
+  volatile int* attn_gate = misc + 9;  // QKV slots whose attention in this CTA is done (ring free)
+  const size_t ring_attn_bytes = static_cast<size_t>(s_attn - base) + p.attn_extra;
   MkShared sh;
   sh.abort_s = reinterpret_cast<volatile int*>(misc + 1);
   sh.abort_g = p.abort_word;
@@ -484,10 +531,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     }
     *sh.abort_s = 0;
     misc[8] = 0;
+    misc[9] = 0;
     fence_mbar_init();
-    prefetch_tmap(&tm_xo);
-    prefetch_tmap(&tm_xact);
-    prefetch_tmap(&tm_xn);
   }
   if (warp == 1) {
     tmem_alloc(reinterpret_cast<uint32_t*>(misc), ncols);
@@ -506,6 +551,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- weight TMA producer: never waits for activations ----------------
+      // (only for the ring to come back from the attention that borrows it before each O phase)
+      const uint64_t wpol = l2_policy_evict_first();
       long long i = 0;
       bool ok = true;
       for (int pi = 0; ok && pi < n_phases; ++pi) {
@@ -513,20 +560,32 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         long long it0, it1;
         int geff;
         mk_range(ph, c, G, it0, it1, geff);
+        if (ph.kind == kMkO && !mk_wait_gate(attn_gate, ph.slot, sh)) {
+          ok = false;
+          break;
+        }
         const __nv_bfloat16* wl = mk_weights(p, ph);
-        for (long long it = it0; it < it1; ++it, ++i) {
-          const int s = static_cast<int>(i % S);
-          if (!mk_wait_bar(&empty[s], static_cast<uint32_t>((i / S) & 1) ^ 1u, sh)) {
-            ok = false;
-            break;
+        long long it = it0;
+        int t, k0, k1;
+        while (ok && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
+          for (int kc = k0; kc < k1; kc += KPS, ++i) {
+            const int nk = min(KPS, k1 - kc);
+            const int s = static_cast<int>(i % S);
+            if (!mk_wait_bar(&empty[s], static_cast<uint32_t>((i / S) & 1) ^ 1u, sh)) {
+              ok = false;
+              break;
+            }
+            if (static_cast<long long>(t) * ph.kb + kc == it0) mk_trace(p, pi * 8 + 0);
+            if (static_cast<long long>(t) * ph.kb + kc + nk == it1) mk_trace(p, pi * 8 + 1);
+            mbar_arrive_expect_tx(&full[s], nk * kMkWBytes);
+            if (p.w_evict_first)
+              bulk_load_hint(sW + static_cast<size_t>(s) * sw_bytes,
+                             wl + (static_cast<size_t>(t) * ph.kb + kc) * kTileElems, nk * kMkWBytes, &full[s], wpol);
+            else
+              bulk_load(sW + static_cast<size_t>(s) * sw_bytes,
+                        wl + (static_cast<size_t>(t) * ph.kb + kc) * kTileElems, nk * kMkWBytes, &full[s]);
+            *w_pos = static_cast<int>(i + 1);
           }
-          if (it == it0) mk_trace(p, pi * 8 + 0);
-          if (it + 1 == it1) mk_trace(p, pi * 8 + 1);
-          const int t = static_cast<int>(it / ph.kb), kk = static_cast<int>(it % ph.kb);
-          mbar_arrive_expect_tx(&full[s], kMkWBytes);
-          bulk_load(sW + static_cast<size_t>(s) * kMkWBytes, wl + (static_cast<size_t>(t) * ph.kb + kk) * kTileElems,
-                    kMkWBytes, &full[s]);
-          *w_pos = static_cast<int>(i + 1);
         }
       }
       *w_pos = 0x7fffffff;  // the prefetch warp may run to the end
@@ -558,20 +617,23 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           }
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * n_pad);
-          for (int kk = k0; kk < k1; ++kk, ++i) {
+          for (int kc = k0; kc < k1; kc += KPS, ++i) {
+            const int nk = min(KPS, k1 - kc);
             const int s = static_cast<int>(i % S);
             if (!mk_wait_bar(&full[s], static_cast<uint32_t>((i / S) & 1), sh)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            if (kk == k0 && static_cast<long long>(t) * ph.kb + k0 == it0) mk_trace(p, pi * 8 + 4);
-            const uint32_t a0 = smem_u32(sW + static_cast<size_t>(s) * kMkWBytes);
-            const uint32_t b0 = smem_u32(sX + static_cast<size_t>(s) * x_bytes);
+            if (kc == k0 && static_cast<long long>(t) * ph.kb + k0 == it0) mk_trace(p, pi * 8 + 4);
+            for (int j = 0; j < nk; ++j) {
+              const uint32_t a0 = smem_u32(sW + static_cast<size_t>(s) * sw_bytes + j * kMkWBytes);
+              const uint32_t b0 = smem_u32(sX + static_cast<size_t>(s) * sx_bytes + j * x_bytes);
 #pragma unroll
-            for (int k16 = 0; k16 < 4; ++k16)
-              umma_bf16(d_tmem, sdesc_sw128(a0 + k16 * 32), sdesc_sw128(b0 + k16 * 32), idesc,
-                        (kk > k0 || k16 > 0) ? 1u : 0u);
+              for (int k16 = 0; k16 < 4; ++k16)
+                umma_bf16(d_tmem, sdesc_sw128(a0 + k16 * 32), sdesc_sw128(b0 + k16 * 32), idesc,
+                          (kc + j > k0 || k16 > 0) ? 1u : 0u);
+            }
             umma_commit(&empty[s]);
           }
           if (!ok) break;
@@ -591,6 +653,14 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       int geff;
       mk_range(ph, c, G, it0, it1, geff);
       if (it0 >= it1) continue;
+      if (ph.kind == kMkO) {
+        bool free = true;
+        if (lane == 0) free = mk_wait_gate(attn_gate, ph.slot, sh);
+        if (!__shfl_sync(0xffffffffu, free, 0)) {
+          ok = false;
+          break;
+        }
+      }
       // dependency index space of this phase: h tiles, heads, or gate/up tiles
       const unsigned long long* flags;
       unsigned long long want;
@@ -608,7 +678,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         want = mk_h_dep(p, ph);
         n_dep = p.d / 128;
       }
-      const CUtensorMap* tmx = ph.kind == kMkO ? &tm_xo : ph.kind == kMkDown ? &tm_xact : &tm_xn;
+      const __nv_bfloat16* xsrc = ph.kind == kMkO ? p.obuf : ph.kind == kMkDown ? p.act : p.xn;
       uint32_t ready[8] = {0, 0, 0, 0, 0, 0, 0, 0};  // known-complete dependency indices (<= 256)
       // one flag index is complete when every request that runs the slot has it (attention) or
       // the single flag reached `want`
@@ -618,12 +688,16 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           if (pl->slot_crow[ph.slot][b] >= 0 && ld_acquire_u64(&flags[b * p.H + x]) < want) return false;
         return true;
       };
-      for (long long it = it0; ok && it < it1; ++it, ++i) {
+      long long it = it0;
+      int t, k0, k1;
+      while (ok && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
+       for (int kc = k0; ok && kc < k1; kc += KPS, ++i) {
+        const int nk = min(KPS, k1 - kc);
         const int s = static_cast<int>(i % S);
-        const int kk = static_cast<int>(it % ph.kb);
         if (lane == 0) ok = mk_wait_bar(&empty[s], static_cast<uint32_t>((i / S) & 1) ^ 1u, sh);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) break;
+        for (int kk = kc; kk < kc + nk; ++kk) {
         const int x = want == 0ull ? -1 : (ph.kind == kMkO ? kk * 64 / p.D : ph.kind == kMkDown ? kk : (kk >> 1));
         if (x >= 0 && !((ready[x >> 5] >> (x & 31)) & 1u)) {
           // poll x .. x+31 at once; then wait (bounded) for x itself if it is not there yet
@@ -654,13 +728,18 @@ __global__ void __launch_bounds__(kMkThreads, 1)
             ready[x >> 5] |= 1u << (x & 31);
           }
         }
-        if (lane == 0) {
-          if (it == it0) mk_trace(p, pi * 8 + 2);
-          if (it + 1 == it1) mk_trace(p, pi * 8 + 3);
-          fence_proxy_async_global();
-          mbar_arrive_expect_tx(&full[s], x_bytes);
-          tma_load_2d(sX + static_cast<size_t>(s) * x_bytes, tmx, &full[s], kk * 64, 0);
         }
+        if (!ok) break;
+        if (lane == 0) {
+          const long long g0 = static_cast<long long>(t) * ph.kb + kc;
+          if (g0 == it0) mk_trace(p, pi * 8 + 2);
+          if (g0 + nk == it1) mk_trace(p, pi * 8 + 3);
+          fence_proxy_async_global();
+          mbar_arrive_expect_tx(&full[s], nk * x_bytes);
+          bulk_load(sX + static_cast<size_t>(s) * sx_bytes, xsrc + static_cast<size_t>(kc) * n_pad * 64, nk * x_bytes,
+                    &full[s]);
+        }
+       }
       }
     }
   } else if (warp == 3) {
@@ -670,13 +749,19 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       // TMA loads then hit in L2.  Stays at most l2_ahead tiles ahead of the TMA producer.
       long long j = 0;
       bool go = true;
+      long long next_pf = clock64();
       for (int pi = 0; go && pi < n_phases; ++pi) {
         const MkPhase ph = mk_phase(p, pl, pi);
         long long it0, it1;
         int geff;
         mk_range(ph, c, G, it0, it1, geff);
         const __nv_bfloat16* wl = mk_weights(p, ph);
-        for (long long it = it0; go && it < it1; ++it, ++j) {
+        long long it = it0;
+        int t, k0, k1;
+        while (go && mk_next_segment(it, it1, ph.kb, t, k0, k1))
+        for (int kc = k0; go && kc < k1; kc += KPS, ++j) {
+          const int nk = min(KPS, k1 - kc);
+          if (j < static_cast<long long>(*w_pos) + S) continue;  // the ring is about to load it itself
           if (j >= static_cast<long long>(*w_pos) + p.l2_ahead) {
             const uint64_t t0 = globaltimer_ns();
             while (j >= static_cast<long long>(*w_pos) + p.l2_ahead) {
@@ -688,8 +773,18 @@ __global__ void __launch_bounds__(kMkThreads, 1)
             }
             if (!go) break;
           }
-          const int t = static_cast<int>(it / ph.kb), kk = static_cast<int>(it % ph.kb);
-          bulk_prefetch_l2(wl + (static_cast<size_t>(t) * ph.kb + kk) * kTileElems, kMkWBytes);
+          if (p.l2_pace > 0) {
+            // pace to about this SM's share of HBM bandwidth so that prefetches do not pile up in
+            // the memory queues ahead of the latency-critical loads
+            long long now = clock64();
+            if (now > next_pf) next_pf = now;
+            while (now < next_pf) {
+              __nanosleep(32);
+              now = clock64();
+            }
+            next_pf += static_cast<long long>(p.l2_pace) * nk;
+          }
+          bulk_prefetch_l2(wl + (static_cast<size_t>(t) * ph.kb + kc) * kTileElems, nk * kMkWBytes);
         }
       }
     }
@@ -703,6 +798,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     e.redv = redv;
     e.redi = redi;
     e.rs = rs;
+    e.rcos = s_rope;
+    e.rsin = s_rope + 16 * 64;
     const int r = e.q * 32 + lane;
     int* bcast = misc + 2;
     int use = 0;
@@ -717,6 +814,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     ap.step = p.step;
     ap.q = p.qbuf;
     ap.o = p.obuf;
+    ap.o_tiled_npad = p.n_pad;
     ap.part_o = p.attn_po;
     ap.part_ml = p.attn_pml;
     ap.counters = p.attn_cnt;
@@ -741,10 +839,20 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           s_kvrow[j] = p.step->req_ctx[b] + (m - p.step->req_rowoff[b]);
         }
       }
+      e.direct_xn = false;
       if (ph.kind == kMkO || ph.kind == kMkDown) {
         const int ns = mk_next_slot(p, ph);
         e.nM = pl->slot_M[ns];
-        for (int j = e.et; j < e.nM; j += 128) s_nrows[j] = pl->slot_rows[ns][j];
+        bool same = e.nM == e.M;
+        for (int j = e.et; j < e.nM; j += 128) {
+          const int m = pl->slot_rows[ns][j];
+          s_nrows[j] = m;
+          same = same && j < e.M && pl->slot_rows[rslot][j] == m;
+        }
+        e.direct_xn = bar_and(1, 128, same);
+        e.gnext = ph.kind == kMkO ? p.g_mlp + static_cast<size_t>(ph.layer) * p.d
+                  : ns != kFinalSlot ? p.g_attn + static_cast<size_t>(pl->act_layer[ns]) * p.d
+                                     : p.g_final;
       }
       named_bar_sync(1, 128);
       e.rows = s_rows;
@@ -752,12 +860,49 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       e.kvslot = s_kvslot;
       e.kvrow = s_kvrow;
       e.nrows = s_nrows;
+      if (ph.kind == kMkQkv) {
+        // stage the RoPE factors of the first 16 rows; warm L2 with the context keys and values
+        // this CTA's attention items will read (they do not depend on this step)
+        const int half = D / 2, m16 = e.M < 16 ? e.M : 16;
+        for (int x = e.et; x < m16 * half; x += 128) {
+          const int j = x / half, i = x - j * half;
+          s_rope[j * half + i] = p.rope_cos[static_cast<size_t>(s_pos[j]) * half + i];
+          s_rope[16 * 64 + j * half + i] = p.rope_sin[static_cast<size_t>(s_pos[j]) * half + i];
+        }
+        if (e.et == 0) {
+          const int per_req = p.H * p.attn_splits;
+          const StepDesc* st = p.step;
+          for (int item = c; item < p.B * per_req; item += G) {
+            const int b = item / per_req;
+            const int head = (item - b * per_req) / p.attn_splits;
+            const int split = item - b * per_req - head * p.attn_splits;
+            if (pl->slot_crow[ph.slot][b] < 0) continue;
+            const int ctx = st->req_ctx[b];
+            int k0, k1;
+            attn_split_keys(ctx + st->req_nodes[b], p.attn_splits, split, k0, k1);
+            k1 = k1 < ctx ? k1 : ctx;
+            if (k1 <= k0) continue;
+            const size_t cap = static_cast<size_t>(st->kv_cap);
+            const __nv_bfloat16* kg =
+                st->kv_layer[ph.layer] + ((static_cast<size_t>(st->req_slot[b]) * 2) * p.H + head) * cap * D;
+            const uint32_t bytes = static_cast<uint32_t>(k1 - k0) * D * 2;
+            bulk_prefetch_l2(kg + static_cast<size_t>(k0) * D, bytes);
+            bulk_prefetch_l2(kg + static_cast<size_t>(p.H) * cap * D + static_cast<size_t>(k0) * D, bytes);
+          }
+        }
+        named_bar_sync(1, 128);
+      }
       bool rs_ready = false;
       const long long T = static_cast<long long>(ph.n_tiles) * ph.kb;
       float* partials = (pi & 1) ? p.partials1 : p.partials0;
       int* counters = p.counters + static_cast<size_t>(ph.kind) * p.max_tiles;
       const bool needs_rs = ph.kind == kMkQkv || ph.kind == kMkGu || ph.kind == kMkLm;
       const unsigned long long hdep = needs_rs ? mk_h_dep(p, ph) : 0ull;
+      // the norm factors need only h, which is final before this phase's first accumulator
+      if (needs_rs && !mk_prepare_rs(p, e, hdep, sh, rs_ready)) {
+        ok = false;
+        break;
+      }
       long long it = it0;
       int t, k0, k1;
       while (ok && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
@@ -771,6 +916,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         tc_fence_after();
         const uint32_t tb = tmem_base + (static_cast<uint32_t>(e.q * 32) << 16) + static_cast<uint32_t>(buf * n_pad);
         const int n_ch = n_pad >> 4;
+        const bool tr_last = e.et == 0 && it >= it1;
+        if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 0);
         bool finalize = false;
         int cf = 0, cl = 0;
         if (k0 == 0 && k1 == ph.kb) {
@@ -792,12 +939,14 @@ __global__ void __launch_bounds__(kMkThreads, 1)
             float v[16];
             tmem_ld16(tb + ch * 16, v);
 #pragma unroll
-            for (int jj = 0; jj < 16; ++jj) __stcg(&part[(ch * 16 + jj) * 128 + r], v[jj]);
+            for (int jj = 0; jj < 16; ++jj)
+              if (ch * 16 + jj < e.M) __stcg(&part[(ch * 16 + jj) * 128 + r], v[jj]);
           }
           tc_fence_before();
           mbar_arrive(&acce[buf]);
           __threadfence();
           named_bar_sync(1, 128);
+          if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 1);
           if (e.et == 0) {
             const int f = mk_cta_of(static_cast<long long>(t) * ph.kb, T, geff);
             const int l = mk_cta_of(static_cast<long long>(t + 1) * ph.kb - 1, T, geff);
@@ -813,39 +962,62 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           cf = bcast[1];
           cl = bcast[2];
           named_bar_sync(1, 128);
+          if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 2);
           if (finalize) {
             __threadfence();
             if (needs_rs && !mk_prepare_rs(p, e, hdep, sh, rs_ready)) {
               ok = false;
               break;
             }
+            if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 3);
             for (int ch = 0; ch < n_ch; ++ch) {
               float v[16];
 #pragma unroll
               for (int jj = 0; jj < 16; ++jj) v[jj] = 0.f;
-              for (int cc = cf; cc <= cl; ++cc) {
-                const float* pp = partials + static_cast<size_t>(cc + t) * 128 * n_pad;
+              // contributors in order (deterministic sum), two at a time in flight
+              int cc = cf;
+              for (; cc + 1 <= cl; cc += 2) {
+                const float* pa = partials + static_cast<size_t>(cc + t) * 128 * n_pad;
+                const float* pb = pa + static_cast<size_t>(128) * n_pad;
+                float a[16], bq[16];
 #pragma unroll
-                for (int jj = 0; jj < 16; ++jj) v[jj] += __ldcg(&pp[(ch * 16 + jj) * 128 + r]);
+                for (int jj = 0; jj < 16; ++jj) {
+                  const bool in = ch * 16 + jj < e.M;
+                  a[jj] = in ? __ldcg(&pa[(ch * 16 + jj) * 128 + r]) : 0.f;
+                  bq[jj] = in ? __ldcg(&pb[(ch * 16 + jj) * 128 + r]) : 0.f;
+                }
+#pragma unroll
+                for (int jj = 0; jj < 16; ++jj) v[jj] = (v[jj] + a[jj]) + bq[jj];
+              }
+              if (cc <= cl) {
+                const float* pa = partials + static_cast<size_t>(cc + t) * 128 * n_pad;
+#pragma unroll
+                for (int jj = 0; jj < 16; ++jj)
+                  if (ch * 16 + jj < e.M) v[jj] += __ldcg(&pa[(ch * 16 + jj) * 128 + r]);
               }
               mk_epilogue_chunk(p, ph, e, t, r, ch, v);
             }
+            if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 4);
           }
         }
         if (finalize) {
           unsigned long long* flag = mk_tile_flag(p, ph.kind, t);
-          if (ph.kind == kMkO || ph.kind == kMkDown) {
+          if ((ph.kind == kMkO || ph.kind == kMkDown) && !e.direct_xn) {
             named_bar_sync(1, 128);  // h of this tile is final for every row of the phase
             mk_write_next_xn(p, pl, ph, e, t, r);
           }
+          if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 5);
           __threadfence();
           named_bar_sync(1, 128);
+          if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 6);
           if (flag && e.et == 0) st_release_u64(flag, mk_seq(p.seq_base, ph.slot, ph.kind));
         }
         if (e.et == 0 && it >= it1) mk_trace(p, pi * 8 + 7);
         ++use;
       }
       if (!ok) break;
+      if (ph.kind != kMkQkv && e.et == 0)
+        mk_prefetch_phase(p, pl, pi + 1, n_phases, c, G, static_cast<long long>(S) * KPS, p.pf_next);
       if (ph.kind == kMkQkv) {
         // attention items of this layer: (request, head, split) round-robin over the grid
         ap.slot = ph.slot;
@@ -853,21 +1025,33 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         const int n_items = p.B * per_req;
         const unsigned long long want = mk_seq(p.seq_base, ph.slot, kMkQkv);
         if (e.et == 0) mk_trace(p, kMkTracePhases * 8 + 2 * ph.slot);
+        if (e.et == 0) mk_prefetch_phase(p, pl, pi + 1, n_phases, c, G, 0, p.pf_attn);
+        // The attention borrows the weight/activation ring and its own buffer: this CTA's QKV
+        // MMAs have all completed, and the producers start the O phase only after the gate.
+        fence_proxy_async_shared();
         for (int item = c; ok && item < n_items; item += G) {
           const int b = item / per_req;
           const int head = (item - b * per_req) / p.attn_splits;
           const int split = item - b * per_req - head * p.attn_splits;
           if (pl->slot_crow[ph.slot][b] < 0) continue;
-          bool good = true;
-          if (e.et < 3) {
-            const int tile = (e.et * p.d + head * D) / 128;
-            good = mk_wait_flag(&p.qkvflag[tile], want, sh);
-          }
-          if (!bar_and(1, 128, good)) {
+          // the Q, K and V tiles of this head (written by the QKV epilogues of this step)
+          auto wait_inputs = [&]() -> bool {
+            bool good = true;
+            if (e.et < 3) {
+              const int tile = (e.et * p.d + head * D) / 128;
+              good = mk_wait_flag(&p.qkvflag[tile], want, sh);
+            }
+            return bar_and(1, 128, good);
+          };
+          unsigned long long* atr =
+              p.trace && ph.slot == 1 ? p.trace + static_cast<size_t>(blockIdx.x) * kMkTraceSlots + kMkTraceAttn : nullptr;
+          bool failed = false;
+          const bool wrote = attention_item_resident<D, 1>(ap, split, head, b, e.et, base, ring_attn_bytes, sM, sL,
+                                                           misc + 5, atr, wait_inputs, failed);
+          if (failed) {
             ok = false;
             break;
           }
-          const bool wrote = attention_item<D, 1>(ap, split, head, b, e.et, s_attn, sM, sL, misc + 5);
           if (wrote) {
             __threadfence();
             named_bar_sync(1, 128);
@@ -876,6 +1060,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           named_bar_sync(1, 128);
         }
         if (e.et == 0) mk_trace(p, kMkTracePhases * 8 + 2 * ph.slot + 1);
+        fence_proxy_async_shared();  // generic-proxy use of the ring ends before the next TMA writes
+        named_bar_sync(1, 128);
+        if (e.et == 0) *attn_gate = ph.slot + 1;
       }
     }
   }
@@ -891,10 +1078,10 @@ __global__ void __launch_bounds__(kMkThreads, 1)
 
 size_t mk_trace_slots() { return kMkTraceSlots; }
 
-size_t mk_smem_bytes(int n_pad, int stages, int head_dim) {
-  return 1024 + static_cast<size_t>(stages) * (kMkWBytes + static_cast<size_t>(n_pad) * 128) +
-         attn_smem_bytes_impl(head_dim) + static_cast<size_t>(2 * stages + 2 * kMkMaxAcc) * 8 + 64 + 16 * 128 * 4 +
-         64 * 4 * 2 + kMaxRows * 4 + 128 * 4 + 5 * kMaxRows * 4 + 64;
+size_t mk_smem_bytes(int n_pad, int stages, int head_dim, int kps, size_t attn_extra) {
+  return 1024 + static_cast<size_t>(stages) * kps * (kMkWBytes + static_cast<size_t>(n_pad) * 128) +
+         attn_extra + static_cast<size_t>(2 * stages + 2 * kMkMaxAcc) * 8 + 64 + 16 * 128 * 4 +
+         64 * 4 * 2 + kMaxRows * 4 + 128 * 4 + 5 * kMaxRows * 4 + 2 * 16 * 64 * 4 + 64;
 }
 
 cudaError_t mk_prepare() {
@@ -904,7 +1091,7 @@ cudaError_t mk_prepare() {
   return e;
 }
 
-cudaError_t launch_verify_mk(const MkTensorMaps& tm, const MkParams& p, int grid, size_t smem, cudaStream_t s) {
+cudaError_t launch_verify_mk(const MkParams& p, int grid, size_t smem, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kMkThreads);
@@ -916,9 +1103,9 @@ cudaError_t launch_verify_mk(const MkTensorMaps& tm, const MkParams& p, int grid
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   if (p.D == 64)
-    return cudaLaunchKernelEx(&cfg, verify_mk_kernel<64>, tm.xo, tm.xact, tm.xn, p);
+    return cudaLaunchKernelEx(&cfg, verify_mk_kernel<64>, p);
   if (p.D == 128)
-    return cudaLaunchKernelEx(&cfg, verify_mk_kernel<128>, tm.xo, tm.xact, tm.xn, p);
+    return cudaLaunchKernelEx(&cfg, verify_mk_kernel<128>, p);
   return cudaErrorInvalidValue;
 }
 
