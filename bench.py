@@ -41,6 +41,8 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-profile", action="store_true")
+    p.add_argument("--traffic", default=os.path.join(ROOT, "profiles", "verify_persistent_7b_chain_traffic.txt"),
+                   help="JSON summary of an ncu DRAM-traffic capture of the dominant kernel")
     return p.parse_args()
 
 
@@ -131,6 +133,17 @@ class ClockSampler:
                 "sm_max_mhz": float(rows[0][2]) if rows[0][2].replace(".", "").isdigit() else None,
                 "reasons": reasons, "samples": len(rows),
                 "power_w_max": max(float(r[3]) for r in rows if r[3].replace(".", "").isdigit())}
+
+
+def kernel_sources_hash():
+    """sha256 over the sources of the persistent verify kernel (an ncu traffic figure is only
+    valid for the kernel it was taken on)."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("verify_mk.cu", "attn_body.cuh", "common.cuh", "internal.h"):
+        with open(os.path.join(ROOT, "paper_2609_26100_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
 
 
 def kernel_bytes(w):
@@ -380,9 +393,11 @@ def run_tss(args):
     roofline = None
     kernels = None
     peak, peak_kind = measured_peak()
-    if not args.no_profile:
+    launches_per_step = None
+    if True:
+        # with --no-profile one profiled step still counts the launches of a step
         times = native.TssKernelTimes()
-        n_prof = max(5, min(args.steps, 20))
+        n_prof = 1 if args.no_profile else max(5, min(args.steps, 20))
         for i in range(n_prof):
             run.v.verify_profiled(batches[i % n_var], run.kv_struct, res["_struct"], times, stream.cuda_stream)
         kb = kernel_bytes(w)
@@ -394,6 +409,7 @@ def run_tss(args):
                                  "avg_launch_us": avg * 1e3}
                 if name in kb:
                     kernels[name]["gbs"] = kb[name] / (avg * 1e-3) / 1e9
+        launches_per_step = sum(v["launches_per_step"] for v in kernels.values())
         tot = sum(v["ms_per_step"] for v in kernels.values())
         for v in kernels.values():
             v["share"] = v["ms_per_step"] / tot
@@ -401,11 +417,23 @@ def run_tss(args):
         ach = kernels[dom]["gbs"]
         roofline = {"kernel": dom, "bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
                     "frac": ach / peak, "peak_source": f"{peak_kind} copy bandwidth",
+                    "frac_of_nominal_8TBs": ach / NOMINAL_HBM_GBS,
                     "bytes_per_launch": kb[dom], "traffic": None}
+        if args.traffic and os.path.exists(args.traffic):
+            # DRAM bytes per launch of this kernel from an ncu capture (a summary with "kernel",
+            # "workload", "traffic_bytes" and the hash of the kernel sources it was taken on);
+            # used only for the same workload and unchanged kernel sources
+            with open(args.traffic) as f:
+                tr = json.load(f)
+            if tr.get("kernel") == dom and tr.get("workload") == w.name and tr.get("sources_sha256") == kernel_sources_hash():
+                roofline["traffic"] = tr["traffic_bytes"]
+                roofline["traffic_source"] = tr.get("source")
+        if args.no_profile:
+            kernels = None
+            roofline = None
 
     ab = synth.algorithmic_bytes(w)
     step_gbs = ab["total"] / (ms * 1e-3) / 1e9
-    launches_per_step = 6 + 7 * len(union)
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -418,7 +446,8 @@ def run_tss(args):
                           "achieved_gbs": step_gbs, "frac_of_measured": step_gbs / peak,
                           "frac_of_nominal_8TBs": step_gbs / NOMINAL_HBM_GBS},
         "roofline": roofline, "kernels": kernels, "e2e": e2e,
-        "gpu_launches": launches_per_step * args.steps,
+        "gpu_launches": int(round(launches_per_step * args.steps)),
+        "gpu_launches_per_step": launches_per_step,
         "clocks": clk.summary(),
     }
     mean_acc = statistics.mean(accepts) if accepts else 0.0
