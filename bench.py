@@ -272,25 +272,13 @@ def run_tss(args):
         w.phi = {d: m & ((1 << args.layers) - 1) for d, m in w.phi.items()}
     a = w.arch
     union = w.active_union()
-    max_ctx = max(r.ctx_len for r in w.requests)
-    max_n = max(len(r.parents) for r in w.requests)
 
     # cpu baseline sample needs host copies of a few layers; take them before the GPU run
     sample = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         sample = OracleSample(w, "cuda")
 
-    weights = synth.make_weights(a, w.seed, device="cuda", layers=union)
-    for l in range(a.n_layers):  # layers no request runs still need (unused) tensors for the ABI
-        if weights["layers"][l] is None:
-            weights["layers"][l] = {k: torch.zeros(s, dtype=torch.bfloat16, device="cuda")
-                                    for k, s in synth.layer_shapes(a).items()}
-    run = TssRunner(a, weights, n_slots=len(w.requests), kv_cap=max_ctx + max_n + 8, max_batch=len(w.requests),
-                    max_rows=max(16, w.n_rows), max_nodes=max_n, kv_layers=union)
-    del weights
-    torch.cuda.empty_cache()
-    run.set_phi(w.phi)
-    run.fill_synthetic(w)
+    run = TssRunner.for_workload(w)
     stream = torch.cuda.current_stream()
 
     # Per-step drafts.  7B chain: 20% of steps carry a greedy prefix of length 0-5, built from the

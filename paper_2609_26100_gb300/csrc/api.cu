@@ -128,6 +128,8 @@ struct tss_ctx {
   int w_evict_first = 1;
   int pf_attn = 0, pf_next = 0;
   int mk_max_stages = 12;
+  int attn_early_conv = 1;
+  int attn_plo = 1;
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
   unsigned long long epoch = 0;
   float* ssp = nullptr;
@@ -385,10 +387,11 @@ bool mk_config(const tss_ctx* c, const StepPlan& sp, MkConfig* out) {
   const int splits = mk_attn_splits(c, sp.B);
   const int per = std::max(1, (std::max(sp.tiles, 1) + splits - 1) / splits);
   for (int kps = c->mk_kps; kps >= 1; --kps) {
-    const size_t stage = static_cast<size_t>(kps) * (16384 + static_cast<size_t>(sp.n_pad) * 128);
+    const XsLayout xs = xs_layout(sp.M);
+    const size_t stage = static_cast<size_t>(kps) * (16384 + static_cast<size_t>(xs.rows) * xs.parts * 128);
     for (int S = c->mk_max_stages; S >= 2; --S) {
       const size_t ring = S * stage;
-      const size_t base = mk_smem_bytes(sp.n_pad, S, c->D, kps, 0);
+      const size_t base = mk_smem_bytes(xs.rows, xs.parts, S, c->D, kps, 0);
       if (base > kLimit) continue;
       const size_t avail = kLimit - base;
       const size_t need_min = ring >= q + tile ? 0 : q + tile - ring;
@@ -413,8 +416,10 @@ bool mk_config(const tss_ctx* c, const StepPlan& sp, MkConfig* out) {
 // compaction).
 tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* prof) {
   MiscParams mp = misc_params(c);
-  const int n_pad = sp.n_pad;
-  mp.xt_npad = n_pad;  // the persistent kernel takes its B operands in the k-block tiled layout
+  // the persistent kernel takes its B operands split into hi/lo parts in the k-block tiled layout
+  const XsLayout xs = xs_layout(sp.M);
+  const int n_pad = xs.rows;
+  mp.xs = xs;
   MkConfig cfg;
   if (!mk_config(c, sp, &cfg)) return fail(TSS_ERR_UNSUPPORTED_ARCH, "persistent kernel: no shared-memory plan");
   const int kps = cfg.kps, stages = cfg.stages;
@@ -432,6 +437,9 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.n_pad = n_pad;
   p.stages = stages;
   p.kps = kps;
+  p.xs = xs;
+  p.attn_early_conv = c->attn_early_conv;
+  p.attn_plo = c->attn_plo;
   p.attn_extra = static_cast<int>(cfg.attn_extra);
   p.l2_pace = c->l2_pace;
   p.w_evict_first = c->w_evict_first;
@@ -587,14 +595,14 @@ tss_status build_workspaces(tss_ctx* c) {
   const int d = c->d;
   const size_t R = kMaxRows;
   TSS_TRY(c->alloc(&c->h, R * d));
-  TSS_TRY(c->alloc(&c->xn, R * d));
+  TSS_TRY(c->alloc(&c->xn, 2 * R * d));  // persistent path: hi and lo parts
   TSS_TRY(c->alloc(&c->qbuf, R * d));
-  TSS_TRY(c->alloc(&c->obuf, R * d));
-  TSS_TRY(c->alloc(&c->act, R * c->F_pad));
+  TSS_TRY(c->alloc(&c->obuf, 2 * R * d));
+  TSS_TRY(c->alloc(&c->act, 2 * R * c->F_pad));
   TSS_TRY(c->alloc(&c->logits_ws, static_cast<size_t>(c->a.max_rows) * c->V));
-  TSS_CU(cudaMemset(c->xn, 0, R * d * 2));
-  TSS_CU(cudaMemset(c->obuf, 0, R * d * 2));
-  TSS_CU(cudaMemset(c->act, 0, R * c->F_pad * 2));
+  TSS_CU(cudaMemset(c->xn, 0, 2 * R * d * 2));
+  TSS_CU(cudaMemset(c->obuf, 0, 2 * R * d * 2));
+  TSS_CU(cudaMemset(c->act, 0, 2 * R * c->F_pad * 2));
   const int max_tiles = std::max(std::max(3 * d / 128, c->Ft), c->V_pad / 128);
   const size_t max_grid = static_cast<size_t>(c->num_sms) * 2;
   c->partials_floats = (max_grid + max_tiles) * 128 * static_cast<size_t>(pad_to(c->a.max_rows, 16));
@@ -661,7 +669,10 @@ tss_status build_workspaces(tss_ctx* c) {
     c->mk_n_zero = 7 * max_tiles + 1;
     TSS_TRY(c->alloc(&c->mk_zero, static_cast<size_t>(c->mk_n_zero)));
     TSS_CU(cudaMemset(c->mk_zero, 0, static_cast<size_t>(c->mk_n_zero) * sizeof(int)));
-    c->mk_part_floats = (static_cast<size_t>(c->num_sms) + max_tiles) * 128 * static_cast<size_t>(pad_to(c->a.max_rows, 16));
+    // partial tiles are strided by the MMA width of the split B operand (up to 256 rows)
+    int xs_rows_max = 16;
+    for (int m = 1; m <= c->a.max_rows; ++m) xs_rows_max = std::max(xs_rows_max, xs_layout(m).rows);
+    c->mk_part_floats = (static_cast<size_t>(c->num_sms) + max_tiles) * 128 * static_cast<size_t>(xs_rows_max);
     TSS_TRY(c->alloc(&c->mk_part0, c->mk_part_floats));
     TSS_TRY(c->alloc(&c->mk_part1, c->mk_part_floats));
   }
@@ -843,6 +854,8 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_EVICT_FIRST")) c->w_evict_first = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_PF_ATTN")) c->pf_attn = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_PF_NEXT")) c->pf_next = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("TSS_ATTN_EARLY_CONV")) c->attn_early_conv = std::atoi(e) != 0;
+  if (const char* e = std::getenv("TSS_ATTN_PLO")) c->attn_plo = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
   const char* trace_env = std::getenv("TSS_TRACE");
   tss_status s = build_workspaces(c);

@@ -137,7 +137,9 @@ __device__ __forceinline__ void attn_load_qfrag(const AttnItem<D>& it, const __n
 // and V rows in shared memory, key0: the key index of their first row): scores, context /
 // ancestor mask, rescale, P.V.  The blocks' score MMAs are independent, so a group of blocks
 // from several resident tiles keeps the tensor pipe busier than one block at a time.
-template <int D>
+// QK16: q and k in fp16 for the score MMAs (else bf16).  PLO: P.V with P as two bf16 parts,
+// hi = bf16(p) and lo = bf16(p - hi), both multiplied by the bf16 values (else P in bf16).
+template <int D, bool QK16 = false, bool PLO = false>
 __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __nv_bfloat16* const (&kp)[4],
                                                  const __nv_bfloat16* const (&vp)[4], const int (&key0)[4], int n,
                                                  float scale_log2, AttnAcc<D>& a) {
@@ -153,8 +155,13 @@ __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __
       if (np < n) {
         uint32_t kb4[4];
         ldmatrix_x4(kb4, kp[np] + ((lane & 7) + ((lane >> 4) << 3)) * LD + ks * 16 + ((lane >> 3) & 1) * 8);
-        mma_bf16_16816(s[2 * np], a.qf[ks], kb4);
-        mma_bf16_16816(s[2 * np + 1], a.qf[ks], kb4 + 2);
+        if (QK16) {
+          mma_f16_16816(s[2 * np], a.qf[ks], kb4);
+          mma_f16_16816(s[2 * np + 1], a.qf[ks], kb4 + 2);
+        } else {
+          mma_bf16_16816(s[2 * np], a.qf[ks], kb4);
+          mma_bf16_16816(s[2 * np + 1], a.qf[ks], kb4 + 2);
+        }
       }
     }
   }
@@ -213,17 +220,31 @@ __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __
 #pragma unroll
   for (int kc = 0; kc < 4; ++kc) {
     if (kc < n) {
-      uint32_t pa[4];
+      uint32_t pa[4], pl[4];
       pa[0] = pack_bf16(s[2 * kc][0], s[2 * kc][1]);
       pa[1] = pack_bf16(s[2 * kc][2], s[2 * kc][3]);
       pa[2] = pack_bf16(s[2 * kc + 1][0], s[2 * kc + 1][1]);
       pa[3] = pack_bf16(s[2 * kc + 1][2], s[2 * kc + 1][3]);
+      if (PLO) {
+        // residuals of the rounding: p - float(bf16(p)), packed the same way
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float x0 = (i < 2 ? s[2 * kc][2 * (i & 1)] : s[2 * kc + 1][2 * (i & 1)]);
+          const float x1 = (i < 2 ? s[2 * kc][2 * (i & 1) + 1] : s[2 * kc + 1][2 * (i & 1) + 1]);
+          const float h0 = __uint_as_float(pa[i] << 16), h1 = __uint_as_float(pa[i] & 0xffff0000u);
+          pl[i] = pack_bf16(x0 - h0, x1 - h1);
+        }
+      }
 #pragma unroll
       for (int dp = 0; dp < D / 16; ++dp) {
         uint32_t vb[4];
         ldmatrix_x4_trans(vb, vp[kc] + ((lane & 7) + (((lane >> 3) & 1) << 3)) * LD + dp * 16 + (lane >> 4) * 8);
         mma_bf16_16816(a.o[2 * dp], pa, vb);
         mma_bf16_16816(a.o[2 * dp + 1], pa, vb + 2);
+        if (PLO) {
+          mma_bf16_16816(a.o[2 * dp], pl, vb);
+          mma_bf16_16816(a.o[2 * dp + 1], pl, vb + 2);
+        }
       }
     }
   }
@@ -296,8 +317,10 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
     if (p.n_splits == 1) {
       if (!(L > 0.f)) report(p.status, kStatusCheck);
       const float val = L > 0.f ? O / L : 0.f;
-      p.o[p.o_tiled_npad ? xt_index(crow + i, head * D + dd, p.o_tiled_npad)
-                         : static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
+      if (p.o_xs.rows)
+        store_split(p.o, p.o_xs, crow + i, head * D + dd, val);
+      else
+        p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
     } else {
       const size_t pi = (ph + split) * kMaxNodes + i;
       __stcg(&p.part_o[pi * D + dd], O);
@@ -362,8 +385,11 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
       }
     }
     if (!(L > 0.f)) report(p.status, kStatusCheck);
-    p.o[p.o_tiled_npad ? xt_index(crow + i, head * D + dd, p.o_tiled_npad)
-                       : static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(L > 0.f ? O / L : 0.f);
+    const float val = L > 0.f ? O / L : 0.f;
+    if (p.o_xs.rows)
+      store_split(p.o, p.o_xs, crow + i, head * D + dd, val);
+    else
+      p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
   }
   stamp(4);
   return true;
@@ -404,6 +430,27 @@ __device__ bool attention_item(const AttnParams& p, int split, int head, int b, 
                              [](int) {});
 }
 
+// bf16 -> fp16 in place for the K rows of `tiles` resident tiles (each tile: K [kKeyTile][LD],
+// then V); the bf16 cache values are exact in fp16 within its range (|x| < 65504; below 6.1e-5
+// fp16 is subnormal).
+template <int D>
+__device__ __forceinline__ void attn_k_to_f16(__nv_bfloat16* tiles0, int tiles, int tid) {
+  constexpr int LD = attn_ld<D>(), C8 = D / 8;
+  for (int idx = tid; idx < tiles * kKeyTile * C8; idx += kAttnThreads) {
+    const int row = idx / C8, c8 = idx - row * C8;  // row over the tiles' K rows
+    const int tl = row / kKeyTile, kr = row - tl * kKeyTile;
+    uint4* ptr = reinterpret_cast<uint4*>(tiles0 + (tl * 2 * kKeyTile + kr) * LD + c8 * 8);
+    uint4 v = *ptr;
+    uint32_t* w = reinterpret_cast<uint32_t*>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float lo = __uint_as_float(w[i] << 16), hi = __uint_as_float(w[i] & 0xffff0000u);
+      w[i] = pack_f16(lo, hi);
+    }
+    *ptr = v;
+  }
+}
+
 // Tiles of K and V that attention_item_resident keeps resident in `smem_bytes` of shared memory.
 __host__ __device__ inline int attn_resident_tiles(int head_dim, size_t smem_bytes) {
   const size_t ld = head_dim + 8, q = static_cast<size_t>(kMaxNodes) * ld * 2, tile = 2ull * kKeyTile * ld * 2;
@@ -420,7 +467,8 @@ __host__ __device__ inline int attn_resident_tiles(int head_dim, size_t smem_byt
 template <int D, int BAR, typename Wait>
 __device__ bool attention_item_resident(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
                                         size_t smem_bytes, float (*sM)[16], float (*sL)[16], int* s_last,
-                                        unsigned long long* trace, Wait wait_inputs, bool& failed) {
+                                        unsigned long long* trace, Wait wait_inputs, bool& failed,
+                                        bool early_convert = true, bool plo = true) {
   constexpr int LD = attn_ld<D>();
   auto stamp = [&](int k) {
     if (trace && tid == 0) trace[k] = globaltimer_ns();
@@ -446,6 +494,23 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
         attn_load_tile<D>(it, tile, tid, sKV + (tile - r0) * 2 * kKeyTile * LD,
                           sKV + ((tile - r0) * 2 + 1) * kKeyTile * LD);
     cp_async_commit();
+    // the score MMAs run in fp16 (q is written in fp16): convert the keys in place as they
+    // land, the context tiles of the first round while the step's own rows are still produced
+    int ready = r0;  // tiles [r0, ready) are converted
+    if (early_convert) {
+      cp_async_wait<0>();
+      named_bar_sync(BAR, kAttnThreads);
+      for (int tile = r0; tile < r1; ++tile) {
+        if (first && (tile + 1) * kKeyTile > it.ctx) break;
+        ready = tile + 1;
+      }
+      attn_k_to_f16<D>(sKV, ready - r0, tid);
+    } else if (!first) {
+      cp_async_wait<0>();
+      named_bar_sync(BAR, kAttnThreads);
+      ready = r1;
+      attn_k_to_f16<D>(sKV, r1 - r0, tid);
+    }
     if (first) {
       if (!wait_inputs()) {
         cp_async_wait<0>();
@@ -458,8 +523,10 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
           attn_load_tile<D>(it, tile, tid, sKV + (tile - r0) * 2 * kKeyTile * LD,
                             sKV + ((tile - r0) * 2 + 1) * kKeyTile * LD);
       cp_async_commit();
+      cp_async_wait<0>();
+      named_bar_sync(BAR, kAttnThreads);
+      attn_k_to_f16<D>(sKV + (ready - r0) * 2 * kKeyTile * LD, r1 - ready, tid);
     }
-    cp_async_wait<0>();
     named_bar_sync(BAR, kAttnThreads);
     if (first) {
       stamp(0);
@@ -481,7 +548,10 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
           vp[j] = sKV + ((tl * 2 + 1) * kKeyTile + kbase + np * 16) * LD;
           key0[j] = (r0 + tl) * kKeyTile + kbase + np * 16;
         }
-        attn_blocks_step<D>(it, kp, vp, key0, min(4, nb - q0), p.scale_log2, a);
+        if (plo)
+          attn_blocks_step<D, true, true>(it, kp, vp, key0, min(4, nb - q0), p.scale_log2, a);
+        else
+          attn_blocks_step<D, true, false>(it, kp, vp, key0, min(4, nb - q0), p.scale_log2, a);
       }
     }
     named_bar_sync(BAR, kAttnThreads);  // the next round overwrites the tiles

@@ -8,6 +8,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -197,13 +198,37 @@ __device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes
 constexpr uint32_t kTileBytes = 128 * 64 * 2;
 constexpr size_t kTileElems = 128 * 64;
 
-// Activation operands of the persistent kernel use the same idea: per 64-column k-block a
-// contiguous [n_pad rows][64] bf16 block in 128-byte-swizzled order, blocks by k-block, so the
-// operand of consecutive k-blocks is one linear bulk copy.  Element index of (row n, column k):
-__host__ __device__ __forceinline__ size_t xt_index(int n, int k, int n_pad) {
-  const int kb = k >> 6, kc = k & 63;
-  return static_cast<size_t>(kb) * n_pad * 64 + static_cast<size_t>(n) * 64 +
-         static_cast<size_t>((((kc >> 3) ^ (n & 7)) << 3) | (kc & 7));
+// Activation (B) operands of the persistent kernel use the same idea: per 64-column k-block,
+// contiguous [rows][64] bf16 blocks in 128-byte-swizzled order, so the operand of consecutive
+// k-blocks is one linear bulk copy.  Each activation x is kept as two bf16 parts, hi = bf16(x)
+// and lo = bf16(x - hi); the GEMM multiplies both by the weights, so the activation keeps about
+// 16 significant bits while the tensor cores see bf16 only.  For up to 128 token rows M both
+// parts share one block: hi in row j, lo in row half + j (half = xs_half(M)), one MMA of width
+// rows = pad16(half + M) yields W.hi and W.lo in separate accumulator columns, and the epilogue
+// adds them in fp32.  Beyond that (parts = 2) hi and lo are consecutive blocks of pad16(M) rows
+// and two MMAs accumulate into the same columns.
+struct XsLayout {
+  int rows;   // rows of one block (the MMA width N); 0: plain row-major [row][K] bf16
+  int parts;  // 1: hi and lo in one block; 2: a hi block then a lo block per k-block
+  int half;   // parts == 1: row offset of the lo part
+};
+__host__ __device__ inline int xs_half(int M) { return M <= 8 ? 8 : (M + 15) & ~15; }
+__host__ __device__ inline XsLayout xs_layout(int M) {
+  const int half = xs_half(M);
+  if (half + M <= 256) return XsLayout{(half + M + 15) & ~15, 1, half};
+  return XsLayout{(M + 15) & ~15, 2, 0};
+}
+// (32-bit index arithmetic: an operand holds at most 2 x 256 rows x 32768 columns)
+__host__ __device__ __forceinline__ uint32_t xs_elem(const XsLayout& L, int j, int k, int lo) {
+  const uint32_t kb = static_cast<uint32_t>(k) >> 6, kc = static_cast<uint32_t>(k) & 63u;
+  const uint32_t part = L.parts == 2 ? static_cast<uint32_t>(lo) : 0u;
+  const uint32_t row = static_cast<uint32_t>(L.parts == 1 && lo ? L.half + j : j);
+  return ((kb * L.parts + part) * L.rows + row) * 64u + ((((kc >> 3) ^ (row & 7u)) << 3) | (kc & 7u));
+}
+__device__ __forceinline__ void store_split(__nv_bfloat16* buf, const XsLayout& L, int j, int k, float x) {
+  const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+  buf[xs_elem(L, j, k, 0)] = hi;
+  buf[xs_elem(L, j, k, 1)] = __float2bfloat16_rn(x - __bfloat162float(hi));
 }
 
 // ------------------------------------------------------------------------------------------
@@ -282,6 +307,18 @@ __device__ __forceinline__ void mma_bf16_16816(float* d, const uint32_t* a, cons
       "{%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+__device__ __forceinline__ void mma_f16_16816(float* d, const uint32_t* a, const uint32_t* b) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
 }
 
 __device__ __forceinline__ void ldmatrix_x4(uint32_t* r, const void* p) {

@@ -70,7 +70,7 @@ struct AttnParams {
   float* part_ml;          // [B][H][n_splits][kMaxNodes][2]
   int* counters;           // [B][H], self-resetting
   int* status;
-  int o_tiled_npad;        // 0: o row-major [row][d]; > 0: k-block tiled for this MMA width
+  XsLayout o_xs;           // o_xs.rows == 0: o row-major [row][d]; else split k-block tiled
 };
 size_t attn_smem_bytes(int head_dim);
 cudaError_t attn_prepare();
@@ -93,7 +93,7 @@ struct MiscParams {
   const int* amax_idx;
   int n_vtiles;
   int* status;
-  int xt_npad;  // persistent path: MMA width of the k-block tiled activation operands
+  XsLayout xs;  // xs.rows == 0: xn row-major; else the persistent kernel's split tiled operand
 };
 
 cudaError_t misc_prepare();
@@ -114,6 +114,9 @@ cudaError_t launch_tile_weights(const __nv_bfloat16* src, __nv_bfloat16* dst, in
 struct MkParams {
   int n_act, d, H, D, F_pad, Ft, V, V_pad, n_pad, stages, attn_splits, B, max_tiles;
   int kps;  // k-blocks (16 KiB of weights each) per pipeline stage
+  XsLayout xs;  // B-operand layout (n_pad == xs.rows)
+  int attn_early_conv;  // convert context keys to fp16 before waiting for the step's own rows
+  int attn_plo;         // attention P.V with P split into hi/lo bf16 parts
   int l2_pace;  // SM clock cycles between L2 prefetches of 16 KiB (0: unpaced)
   int w_evict_first;  // stream weights with the evict-first L2 policy
   int pf_attn;  // 16 KiB weight blocks of the O phase warmed into L2 while the attention runs
@@ -156,7 +159,7 @@ struct MkParams {
   int* status;
   int* abort_word;
 };
-size_t mk_smem_bytes(int n_pad, int stages, int head_dim, int kps, size_t attn_extra);
+size_t mk_smem_bytes(int n_pad, int parts, int stages, int head_dim, int kps, size_t attn_extra);
 size_t mk_trace_slots();
 cudaError_t mk_prepare();
 int mk_max_blocks_per_sm(int head_dim, size_t smem);

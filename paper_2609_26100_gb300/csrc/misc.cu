@@ -409,8 +409,13 @@ __global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float
       const float x = __bfloat162float(e[t * 128 + r]);
       h[t * 128 + r] = x;
       if (xrow >= 0)
-        p.xn[p.xt_npad ? xt_index(xrow, t * 128 + r, p.xt_npad) : static_cast<size_t>(xrow) * p.d_model + t * 128 + r] =
-            __float2bfloat16_rn(x * gain[t * 128 + r]);
+      {
+        const float xv = x * gain[t * 128 + r];
+        if (p.xs.rows)
+          store_split(p.xn, p.xs, xrow, t * 128 + r, xv);
+        else
+          p.xn[static_cast<size_t>(xrow) * p.d_model + t * 128 + r] = __float2bfloat16_rn(xv);
+      }
       sq = x * x;
     }
 #pragma unroll

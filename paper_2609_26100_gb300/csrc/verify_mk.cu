@@ -251,6 +251,28 @@ __device__ __forceinline__ unsigned long long mk_h_dep(const MkParams& p, const 
   return p.n_act == 0 ? 0ull : mk_seq(p.seq_base, p.n_act - 1, kMkDown);  // LM head
 }
 
+// Accumulator values of tokens [16 ch, 16 ch + 16) of this thread's output row: W.hi + W.lo
+// (the two parts are separate columns of one MMA when xs.parts == 1, already summed otherwise).
+__device__ __forceinline__ void mk_acc_tokens(uint32_t tb, int ch, const XsLayout& xs, float* v) {
+  if (xs.parts == 2) {
+    tmem_ld16(tb + ch * 16, v);
+  } else if (xs.half == 8) {  // up to 8 tokens: hi in columns 0..7, lo in 8..15
+    float r[16];
+    tmem_ld16(tb, r);
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj) {
+      v[jj] = r[jj] + r[8 + jj];
+      v[8 + jj] = 0.f;
+    }
+  } else {
+    float lo[16];
+    tmem_ld16(tb + ch * 16, v);
+    tmem_ld16(tb + xs.half + ch * 16, lo);
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) v[jj] += lo[jj];
+  }
+}
+
 struct MkEpi {
   int M;
   const int* rows;  // shared-memory copy of the phase's compacted row list
@@ -333,7 +355,8 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
       const int j = j0 + jj;
       if (j >= e.M) continue;
       if (sec == 0) {
-        p.qbuf[static_cast<size_t>(j) * d + f] = __float2bfloat16_rn(val[jj]);
+        // q in fp16 (11 significant bits): the attention of this kernel runs its MMAs in fp16
+        reinterpret_cast<__half*>(p.qbuf)[static_cast<size_t>(j) * d + f] = __float2half_rn(val[jj]);
       } else {
         const size_t off = ((static_cast<size_t>(e.kvslot[j]) * 2 + (sec - 1)) * p.H + head) *
                                static_cast<size_t>(st->kv_cap) +
@@ -355,7 +378,7 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
         const float nv = __ldcg(hp) + v[jj];
         *hp = nv;
         sq[jj] = nv * nv;
-        if (e.direct_xn) p.xn[xt_index(j, o, p.n_pad)] = __float2bfloat16_rn(nv * gn);
+        if (e.direct_xn) store_split(p.xn, p.xs, j, o, nv * gn);
       }
     }
 #pragma unroll
@@ -386,7 +409,7 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
         if (j < e.M) {
           const float g = v[jj] * e.rs[j];
           const float u = e.xch[jj * 128 + r + 64] * e.rs[j];
-          p.act[xt_index(j, fcol, p.n_pad)] = __float2bfloat16_rn(g / (1.f + expf(-g)) * u);
+          store_split(p.act, p.xs, j, fcol, g / (1.f + expf(-g)) * u);
         }
       }
     }
@@ -465,7 +488,7 @@ __device__ void mk_write_next_xn(const MkParams& p, const PlanDev* pl, const MkP
       hv[u] = n0 + u < M ? __ldcg(&p.h[static_cast<size_t>(rows[n0 + u]) * p.d + f]) : 0.f;
 #pragma unroll
     for (int u = 0; u < 8; ++u)
-      if (n0 + u < M) p.xn[xt_index(n0 + u, f, p.n_pad)] = __float2bfloat16_rn(hv[u] * gf);
+      if (n0 + u < M) store_split(p.xn, p.xs, n0 + u, f, hv[u] * gf);
   }
 }
 
@@ -485,8 +508,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = p.stages, n_pad = p.n_pad, KPS = p.kps;
-  const uint32_t x_bytes = static_cast<uint32_t>(n_pad) * 128u;  // one k-block of the B operand
-  const uint32_t sw_bytes = KPS * kMkWBytes, sx_bytes = KPS * x_bytes;
+  const int XP = p.xs.parts;
+  const uint32_t x_bytes = static_cast<uint32_t>(n_pad) * 128u;  // one block of one k-block of the B operand
+  const uint32_t sw_bytes = KPS * kMkWBytes, sx_bytes = KPS * XP * x_bytes;
   uint8_t* sW = base;
   uint8_t* sX = sW + static_cast<size_t>(S) * sw_bytes;
   uint8_t* s_attn = sX + static_cast<size_t>(S) * sx_bytes;
@@ -628,11 +652,22 @@ __global__ void __launch_bounds__(kMkThreads, 1)
             if (kc == k0 && static_cast<long long>(t) * ph.kb + k0 == it0) mk_trace(p, pi * 8 + 4);
             for (int j = 0; j < nk; ++j) {
               const uint32_t a0 = smem_u32(sW + static_cast<size_t>(s) * sw_bytes + j * kMkWBytes);
-              const uint32_t b0 = smem_u32(sX + static_cast<size_t>(s) * sx_bytes + j * x_bytes);
+              const uint32_t b0 = smem_u32(sX + static_cast<size_t>(s) * sx_bytes + j * XP * x_bytes);
+              // (branch outside the issue loops: a conditional MMA inside them was measured to
+              // slow every stage down)
+              if (XP == 1) {
 #pragma unroll
-              for (int k16 = 0; k16 < 4; ++k16)
-                umma_bf16(d_tmem, sdesc_sw128(a0 + k16 * 32), sdesc_sw128(b0 + k16 * 32), idesc,
-                          (kc + j > k0 || k16 > 0) ? 1u : 0u);
+                for (int k16 = 0; k16 < 4; ++k16)
+                  umma_bf16(d_tmem, sdesc_sw128(a0 + k16 * 32), sdesc_sw128(b0 + k16 * 32), idesc,
+                            (kc + j > k0 || k16 > 0) ? 1u : 0u);
+              } else {  // the lo block accumulates into the same columns
+#pragma unroll
+                for (int k16 = 0; k16 < 4; ++k16) {
+                  umma_bf16(d_tmem, sdesc_sw128(a0 + k16 * 32), sdesc_sw128(b0 + k16 * 32), idesc,
+                            (kc + j > k0 || k16 > 0) ? 1u : 0u);
+                  umma_bf16(d_tmem, sdesc_sw128(a0 + k16 * 32), sdesc_sw128(b0 + x_bytes + k16 * 32), idesc, 1u);
+                }
+              }
             }
             umma_commit(&empty[s]);
           }
@@ -735,8 +770,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           if (g0 == it0) mk_trace(p, pi * 8 + 2);
           if (g0 + nk == it1) mk_trace(p, pi * 8 + 3);
           fence_proxy_async_global();
-          mbar_arrive_expect_tx(&full[s], nk * x_bytes);
-          bulk_load(sX + static_cast<size_t>(s) * sx_bytes, xsrc + static_cast<size_t>(kc) * n_pad * 64, nk * x_bytes,
+          mbar_arrive_expect_tx(&full[s], nk * XP * x_bytes);
+          bulk_load(sX + static_cast<size_t>(s) * sx_bytes, xsrc + static_cast<size_t>(kc) * XP * n_pad * 64, nk * XP * x_bytes,
                     &full[s]);
         }
        }
@@ -814,7 +849,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     ap.step = p.step;
     ap.q = p.qbuf;
     ap.o = p.obuf;
-    ap.o_tiled_npad = p.n_pad;
+    ap.o_xs = p.xs;
     ap.part_o = p.attn_po;
     ap.part_ml = p.attn_pml;
     ap.counters = p.attn_cnt;
@@ -915,7 +950,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         if (e.et == 0 && static_cast<long long>(t) * ph.kb + k0 == it0) mk_trace(p, pi * 8 + 6);
         tc_fence_after();
         const uint32_t tb = tmem_base + (static_cast<uint32_t>(e.q * 32) << 16) + static_cast<uint32_t>(buf * n_pad);
-        const int n_ch = n_pad >> 4;
+        const int n_ch = (e.M + 15) >> 4;  // 16-token chunks of the accumulator
         const bool tr_last = e.et == 0 && it >= it1;
         if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 0);
         bool finalize = false;
@@ -927,7 +962,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           }
           for (int ch = 0; ch < n_ch; ++ch) {
             float v[16];
-            tmem_ld16(tb + ch * 16, v);
+            mk_acc_tokens(tb, ch, p.xs, v);
             mk_epilogue_chunk(p, ph, e, t, r, ch, v);
           }
           tc_fence_before();
@@ -937,7 +972,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           float* part = partials + static_cast<size_t>(c + t) * 128 * n_pad;
           for (int ch = 0; ch < n_ch; ++ch) {
             float v[16];
-            tmem_ld16(tb + ch * 16, v);
+            mk_acc_tokens(tb, ch, p.xs, v);
 #pragma unroll
             for (int jj = 0; jj < 16; ++jj)
               if (ch * 16 + jj < e.M) __stcg(&part[(ch * 16 + jj) * 128 + r], v[jj]);
@@ -1047,7 +1082,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
               p.trace && ph.slot == 1 ? p.trace + static_cast<size_t>(blockIdx.x) * kMkTraceSlots + kMkTraceAttn : nullptr;
           bool failed = false;
           const bool wrote = attention_item_resident<D, 1>(ap, split, head, b, e.et, base, ring_attn_bytes, sM, sL,
-                                                           misc + 5, atr, wait_inputs, failed);
+                                                           misc + 5, atr, wait_inputs, failed, p.attn_early_conv != 0,
+                                                           p.attn_plo != 0);
           if (failed) {
             ok = false;
             break;
@@ -1078,8 +1114,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
 
 size_t mk_trace_slots() { return kMkTraceSlots; }
 
-size_t mk_smem_bytes(int n_pad, int stages, int head_dim, int kps, size_t attn_extra) {
-  return 1024 + static_cast<size_t>(stages) * kps * (kMkWBytes + static_cast<size_t>(n_pad) * 128) +
+size_t mk_smem_bytes(int n_pad, int parts, int stages, int head_dim, int kps, size_t attn_extra) {
+  return 1024 + static_cast<size_t>(stages) * kps * (kMkWBytes + static_cast<size_t>(n_pad) * parts * 128) +
          attn_extra + static_cast<size_t>(2 * stages + 2 * kMkMaxAcc) * 8 + 64 + 16 * 128 * 4 +
          64 * 4 * 2 + kMaxRows * 4 + 128 * 4 + 5 * kMaxRows * 4 + 2 * 16 * 64 * 4 + 64;
 }

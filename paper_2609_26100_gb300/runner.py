@@ -28,6 +28,29 @@ class TssRunner:
             self.kv[l] = torch.zeros((n_slots, 2, H, kv_cap, D), dtype=torch.bfloat16, device=device)
         self.kv_struct = self.v.make_kv([t.data_ptr() if t is not None else None for t in self.kv], n_slots, kv_cap)
 
+    @classmethod
+    def for_workload(cls, w: synth.Workload, device: str = "cuda") -> "TssRunner":
+        """The configuration bench.py times for workload w: seeded weights of the layers some
+        request runs (generated on the device), one KV slot per request sized to its context plus
+        the draft block, synthetic context KV, and the workload's skip configurations."""
+        a = w.arch
+        union = w.active_union()
+        max_ctx = max(r.ctx_len for r in w.requests)
+        max_n = max(len(r.parents) for r in w.requests)
+        weights = synth.make_weights(a, w.seed, device=device, layers=union)
+        for l in range(a.n_layers):  # layers no request runs still need (unused) tensors for the ABI
+            if weights["layers"][l] is None:
+                weights["layers"][l] = {k: torch.zeros(s, dtype=torch.bfloat16, device=device)
+                                        for k, s in synth.layer_shapes(a).items()}
+        run = cls(a, weights, n_slots=len(w.requests), kv_cap=max_ctx + max_n + 8, max_batch=len(w.requests),
+                  max_rows=max(16, w.n_rows), max_nodes=max_n, kv_layers=union, device=device)
+        del weights
+        if device != "cpu":
+            torch.cuda.empty_cache()
+        run.set_phi(w.phi)
+        run.fill_synthetic(w)
+        return run
+
     def close(self):
         self.v.close()
 

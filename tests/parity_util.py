@@ -17,6 +17,7 @@ def logits_close(gpu: np.ndarray, ref: np.ndarray):
 
 def assert_logits(gpu, ref, what=""):
     mx, rel = logits_close(gpu, ref)
+    print(f"[parity] {what}: logits max-abs {mx:.3e}, rel-L2 {rel:.3e}")
     assert mx <= LOGIT_MAX_ABS and rel <= LOGIT_REL_L2, f"{what}: logits max-abs {mx:.3e}, rel-L2 {rel:.3e}"
     return mx, rel
 
