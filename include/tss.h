@@ -17,7 +17,11 @@
  *     method's, unchanged (greedy at temperature 0; speculative sampling otherwise).
  *
  * f_l is a LLaMA block (App. "Models"): RMSNorm, rotary multi-head attention (rotate-half
- * pairing), SwiGLU MLP.  Weights are bf16; residual and accumulation are fp32.
+ * pairing), SwiGLU MLP.  Weights are bf16; residual and accumulation are fp32.  On the default
+ * (persistent) path every GEMM activation keeps about 16 significant bits (it is fed to the bf16
+ * tensor cores as two parts, bf16(x) and bf16(x - bf16(x))), attention scores use fp16 q and k,
+ * and the attention probabilities enter P.V as two bf16 parts; the new K/V rows are stored in
+ * bf16.
  *
  * Conventions for every entry point:
  *   - Pointers are plain addresses.  "device" means CUDA device memory of the current device,
@@ -178,7 +182,12 @@ tss_status tss_active_layer_count(const tss_ctx* ctx, const tss_verify_batch* ba
  * O projection, RMSNorm+SwiGLU MLP -> final norm + LM head with fused argmax -> acceptance
  * (greedy walk or speculative sampling) -> KV compaction of the accepted path.  A skipped layer
  * gets no launch, reads no weight byte and no KV row.  Asynchronous; steps on one context must
- * not overlap on different streams (they share workspaces). */
+ * not overlap on different streams (they share workspaces).
+ * Default path: three launches -- a prologue (controller, embedding), one persistent cooperative
+ * kernel for every active layer and the LM head, and a finish kernel (acceptance, compaction).
+ * With the environment variable TSS_PATH=multi at tss_create, or when a step's rows do not fit the
+ * persistent kernel's shared-memory plan, one kernel per operation runs instead (bf16 GEMM
+ * activations, 6 + 7 x active layers launches). */
 tss_status tss_verify(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
                       const tss_verify_result* result, void* stream);
 
@@ -239,9 +248,10 @@ tss_status tss_linear_static(const void* x, const void* w, float* y, int m_rows,
  * TSS_TRACE=1 was set at tss_create: globaltimer nanoseconds, per CTA (row of
  * n_out / #SMs values), per phase pi (QKV, O, gate/up, down of each active layer in order, then
  * the LM head) at [pi*8 + 2*role + {0 first, 1 last}] for roles 0 weight TMA, 1 B operand,
- * 2 MMA, 3 epilogue, and the attention of layer slot j at [(4*64+1)*8 + 2j + {0,1}]; 0 = no
- * activity.  With host == NULL only *n_out (values per device) is returned.  Synchronises the
- * device. */
+ * 2 MMA, 3 epilogue, and the attention of layer slot j at [(4*64+1)*8 + 2j + {0,1}]; further
+ * diagnostic slots follow (epilogue sub-steps of each phase's last segment, attention sub-steps
+ * of layer slot 1).  0 = no activity.  With host == NULL only *n_out (values per device) is
+ * returned.  Synchronises the device. */
 tss_status tss_read_trace(tss_ctx* ctx, unsigned long long* host, size_t capacity, size_t* n_out);
 
 const char* tss_status_string(tss_status s);
