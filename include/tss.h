@@ -60,7 +60,8 @@ typedef int tss_status;
 typedef struct tss_ctx tss_ctx; /* opaque; owns repacked weights and all workspaces */
 
 /* Model shape and capacity limits.
- *   n_layers <= 64; head_dim 64 or 128; d_model = n_heads * head_dim and a multiple of 128.
+ *   n_layers <= 64; head_dim 64 or 128; d_model = n_heads * head_dim, a multiple of 128 and at
+ *   most 8192.
  *   max_batch: requests per verify (<= 64).  max_rows: total draft-block rows per verify
  *   (<= 256).  max_nodes: rows per request, root included (<= 64).  max_domains: size of the
  *   domain table Phi.  max_positions: RoPE positions must be < max_positions. */

@@ -128,7 +128,6 @@ struct tss_ctx {
   int w_evict_first = 1;
   int pf_attn = 0, pf_next = 0;
   int mk_max_stages = 12;
-  int attn_early_conv = 1;
   int attn_plo = 1;
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
   unsigned long long epoch = 0;
@@ -372,19 +371,30 @@ struct MkConfig {
   size_t attn_extra = 0, smem = 0;
 };
 
-int mk_attn_splits(const tss_ctx* c, int B) {
-  // about one attention item per CTA: items = B * H * splits
-  int sl = c->num_sms / (B * c->H);
-  if (sl < 1) sl = 1;
-  if (sl > c->max_splits) sl = c->max_splits;
-  return sl;
+// Key splits per (request, head) for the persistent kernel's attention: the fewest waves of
+// items over the grid times the tiles an item scores, plus a fixed per-item cost (flags, merge)
+// of about three tiles.  Short contexts get about one item per CTA.
+int mk_attn_splits(const tss_ctx* c, int B, int tiles) {
+  const int pairs = B * c->H;
+  int best = 1;
+  long long best_cost = -1;
+  for (int sl = 1; sl <= c->max_splits; ++sl) {
+    if (sl > 1 && sl > tiles) break;
+    const long long waves = (static_cast<long long>(pairs) * sl + c->num_sms - 1) / c->num_sms;
+    const long long cost = waves * ((tiles + sl - 1) / sl + 3);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = sl;
+    }
+  }
+  return best;
 }
 
 bool mk_config(const tss_ctx* c, const StepPlan& sp, MkConfig* out) {
   constexpr size_t kLimit = 232448;  // per-block shared-memory maximum of sm_103 (227 KiB)
   const size_t q = static_cast<size_t>(kMaxNodes) * (c->D + 8) * 2;
   const size_t tile = static_cast<size_t>(2) * 64 * (c->D + 8) * 2;
-  const int splits = mk_attn_splits(c, sp.B);
+  const int splits = mk_attn_splits(c, sp.B, std::max(sp.tiles, 1));
   const int per = std::max(1, (std::max(sp.tiles, 1) + splits - 1) / splits);
   for (int kps = c->mk_kps; kps >= 1; --kps) {
     const XsLayout xs = xs_layout(sp.M);
@@ -438,7 +448,6 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.stages = stages;
   p.kps = kps;
   p.xs = xs;
-  p.attn_early_conv = c->attn_early_conv;
   p.attn_plo = c->attn_plo;
   p.attn_extra = static_cast<int>(cfg.attn_extra);
   p.l2_pace = c->l2_pace;
@@ -512,6 +521,7 @@ tss_status validate_arch(const tss_arch* a) {
   if (a->n_heads < 1 || a->d_model != a->n_heads * a->head_dim)
     return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_model must equal n_heads * head_dim");
   if (a->d_model % 128 != 0) return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_model must be a multiple of 128");
+  if (a->d_model > 8192) return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_model must be at most 8192");
   if (a->d_mlp < 1 || a->vocab < 1) return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_mlp and vocab must be positive");
   if (a->d_mlp % 8 != 0) return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_mlp must be a multiple of 8");
   if (a->max_batch < 1 || a->max_batch > kMaxBatch) return fail(TSS_ERR_INVALID_ARG, "max_batch must be in [1, 64]");
@@ -854,7 +864,6 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_EVICT_FIRST")) c->w_evict_first = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_PF_ATTN")) c->pf_attn = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_PF_NEXT")) c->pf_next = std::max(0, std::atoi(e));
-  if (const char* e = std::getenv("TSS_ATTN_EARLY_CONV")) c->attn_early_conv = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ATTN_PLO")) c->attn_plo = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
   const char* trace_env = std::getenv("TSS_TRACE");

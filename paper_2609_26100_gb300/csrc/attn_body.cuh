@@ -272,7 +272,7 @@ __device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, 
 // free 16-byte-aligned buffer of 32 KiB for D = 128), then write this split's result: the
 // normalised output when there is one split, else the partial, and the last split of
 // (request, head) merges all partials in split order.  Returns true on the call that wrote the
-// final output rows.  `stamp(k)` records diagnostics (k = 2, 3, 4).
+// final output rows.  `stamp(k)` records diagnostics (k = 9, 2, 3, 4 in that order).
 template <int D, int BAR, typename Stamp>
 __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<D>& it, AttnAcc<D>& a, int split,
                                             int head, int b, int tid, float* sO, float (*sM)[16], float (*sL)[16],
@@ -300,6 +300,7 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
     sL[warp][g + 8] = a.l1;
   }
   named_bar_sync(BAR, kAttnThreads);
+  stamp(9);
 
   const size_t ph = (static_cast<size_t>(b) * H + head) * p.n_splits;
   for (int idx = tid; idx < N * D; idx += kAttnThreads) {
@@ -467,15 +468,14 @@ __host__ __device__ inline int attn_resident_tiles(int head_dim, size_t smem_byt
 template <int D, int BAR, typename Wait>
 __device__ bool attention_item_resident(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
                                         size_t smem_bytes, float (*sM)[16], float (*sL)[16], int* s_last,
-                                        unsigned long long* trace, Wait wait_inputs, bool& failed,
-                                        bool early_convert = true, bool plo = true) {
+                                        unsigned long long* trace, Wait wait_inputs, bool& failed, bool plo = true) {
   constexpr int LD = attn_ld<D>();
   auto stamp = [&](int k) {
     if (trace && tid == 0) trace[k] = globaltimer_ns();
   };
   failed = false;
   __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [kMaxNodes][LD]
-  __nv_bfloat16* sKV = sQ + kMaxNodes * LD;                      // per tile: K [kKeyTile][LD], V [kKeyTile][LD]
+  __nv_bfloat16* sKV = sQ + kMaxNodes * LD;                      // per tile slot: K [kKeyTile][LD], V [kKeyTile][LD]
   const int R = attn_resident_tiles(D, smem_bytes);
   AttnItem<D> it;
   const bool run = attn_item_setup<D>(p, split, head, b, tid, it);
@@ -483,79 +483,101 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
     failed = !wait_inputs();
     return false;
   }
+  auto tile_k = [&](int slot) { return sKV + slot * 2 * kKeyTile * LD; };
+  auto tile_v = [&](int slot) { return sKV + (slot * 2 + 1) * kKeyTile * LD; };
+  auto load_round = [&](int r0, int r1, int slot0, bool ctx_only) {
+    for (int tile = r0; tile < r1; ++tile)
+      if (!ctx_only || (tile + 1) * kKeyTile <= it.ctx)
+        attn_load_tile<D>(it, tile, tid, tile_k(slot0 + tile - r0), tile_v(slot0 + tile - r0));
+  };
   AttnAcc<D> a;
   attn_acc_init<D>(a);
-  for (int r0 = it.t0; r0 < it.t1 || r0 == it.t0; r0 += R) {
-    const int r1 = min(it.t1, r0 + R);
-    const bool first = r0 == it.t0;
-    // context-only tiles do not depend on this step
-    for (int tile = r0; tile < r1; ++tile)
-      if (!first || (tile + 1) * kKeyTile <= it.ctx)
-        attn_load_tile<D>(it, tile, tid, sKV + (tile - r0) * 2 * kKeyTile * LD,
-                          sKV + ((tile - r0) * 2 + 1) * kKeyTile * LD);
-    cp_async_commit();
-    // the score MMAs run in fp16 (q is written in fp16): convert the keys in place as they
-    // land, the context tiles of the first round while the step's own rows are still produced
-    int ready = r0;  // tiles [r0, ready) are converted
-    if (early_convert) {
-      cp_async_wait<0>();
-      named_bar_sync(BAR, kAttnThreads);
-      for (int tile = r0; tile < r1; ++tile) {
-        if (first && (tile + 1) * kKeyTile > it.ctx) break;
-        ready = tile + 1;
-      }
-      attn_k_to_f16<D>(sKV, ready - r0, tid);
-    } else if (!first) {
-      cp_async_wait<0>();
-      named_bar_sync(BAR, kAttnThreads);
-      ready = r1;
-      attn_k_to_f16<D>(sKV, r1 - r0, tid);
-    }
-    if (first) {
-      if (!wait_inputs()) {
-        cp_async_wait<0>();
-        failed = true;
-        return false;
-      }
-      attn_load_q<D>(p, it, head, tid, sQ);
-      for (int tile = r0; tile < r1; ++tile)
-        if ((tile + 1) * kKeyTile > it.ctx)
-          attn_load_tile<D>(it, tile, tid, sKV + (tile - r0) * 2 * kKeyTile * LD,
-                            sKV + ((tile - r0) * 2 + 1) * kKeyTile * LD);
-      cp_async_commit();
-      cp_async_wait<0>();
-      named_bar_sync(BAR, kAttnThreads);
-      attn_k_to_f16<D>(sKV + (ready - r0) * 2 * kKeyTile * LD, r1 - ready, tid);
-    }
-    named_bar_sync(BAR, kAttnThreads);
-    if (first) {
-      stamp(0);
-      attn_load_qfrag<D>(it, sQ, a);
-    }
-    {
-      // this warp's 16-key blocks of the round, four per softmax update
-      const int npairs = it.kpw / 16, kbase = it.wk * it.kpw;
-      const int nb = (r1 - r0) * npairs;
-      for (int q0 = 0; q0 < nb; q0 += 4) {
-        const __nv_bfloat16* kp[4];
-        const __nv_bfloat16* vp[4];
-        int key0[4];
+  // this warp's 16-key blocks of tiles [r0, r1) held from slot0 on, four per softmax update
+  auto score_round = [&](int r0, int r1, int slot0) {
+    const int npairs = it.kpw / 16, kbase = it.wk * it.kpw;
+    const int nb = (r1 - r0) * npairs;
+    for (int q0 = 0; q0 < nb; q0 += 4) {
+      const __nv_bfloat16* kp[4];
+      const __nv_bfloat16* vp[4];
+      int key0[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int q = min(q0 + j, nb - 1);
-          const int tl = q / npairs, np = q - tl * npairs;
-          kp[j] = sKV + (tl * 2 * kKeyTile + kbase + np * 16) * LD;
-          vp[j] = sKV + ((tl * 2 + 1) * kKeyTile + kbase + np * 16) * LD;
-          key0[j] = (r0 + tl) * kKeyTile + kbase + np * 16;
-        }
-        if (plo)
-          attn_blocks_step<D, true, true>(it, kp, vp, key0, min(4, nb - q0), p.scale_log2, a);
-        else
-          attn_blocks_step<D, true, false>(it, kp, vp, key0, min(4, nb - q0), p.scale_log2, a);
+      for (int j = 0; j < 4; ++j) {
+        const int q = min(q0 + j, nb - 1);
+        const int tl = q / npairs, np = q - tl * npairs;
+        kp[j] = tile_k(slot0 + tl) + (kbase + np * 16) * LD;
+        vp[j] = tile_v(slot0 + tl) + (kbase + np * 16) * LD;
+        key0[j] = (r0 + tl) * kKeyTile + kbase + np * 16;
       }
+      if (plo)
+        attn_blocks_step<D, true, true>(it, kp, vp, key0, min(4, nb - q0), p.scale_log2, a);
+      else
+        attn_blocks_step<D, true, false>(it, kp, vp, key0, min(4, nb - q0), p.scale_log2, a);
     }
-    named_bar_sync(BAR, kAttnThreads);  // the next round overwrites the tiles
-    if (r1 >= it.t1) break;
+  };
+  const int nt = it.t1 - it.t0;
+  if (nt <= R) {
+    // one round: the context tiles (which this step does not write) are requested first, the
+    // Q rows and the block's own tiles once the step's QKV flags are set
+    load_round(it.t0, it.t1, 0, true);
+    cp_async_commit();
+    if (!wait_inputs()) {
+      cp_async_wait<0>();
+      failed = true;
+      return false;
+    }
+    attn_load_q<D>(p, it, head, tid, sQ);
+    for (int tile = it.t0; tile < it.t1; ++tile)
+      if ((tile + 1) * kKeyTile > it.ctx) attn_load_tile<D>(it, tile, tid, tile_k(tile - it.t0), tile_v(tile - it.t0));
+    cp_async_commit();
+    cp_async_wait<0>();
+    named_bar_sync(BAR, kAttnThreads);
+    attn_k_to_f16<D>(sKV, nt, tid);  // the score MMAs run in fp16 (q is written in fp16)
+    named_bar_sync(BAR, kAttnThreads);
+    stamp(0);
+    attn_load_qfrag<D>(it, sQ, a);
+    score_round(it.t0, it.t1, 0);
+    named_bar_sync(BAR, kAttnThreads);
+  } else {
+    // Rounds of H tiles through two halves of the resident space: the next round's copies are in
+    // flight while this round is scored.  Round 0 holds only context tiles (the block's own keys
+    // are in the last two tiles at most, and nt > R >= 2H).
+    const int nbuf = R >= 2 ? 2 : 1;
+    const int H = R / nbuf;
+    const int nr = (nt + H - 1) / H;
+    load_round(it.t0, min(it.t1, it.t0 + H), 0, false);
+    cp_async_commit();
+    if (!wait_inputs()) {
+      cp_async_wait<0>();
+      failed = true;
+      return false;
+    }
+    attn_load_q<D>(p, it, head, tid, sQ);
+    cp_async_commit();
+    for (int r = 0; r < nr; ++r) {
+      const int r0 = it.t0 + r * H, r1 = min(it.t1, r0 + H);
+      const int slot0 = (r % nbuf) * H;
+      if (nbuf == 1 && r > 0) {
+        load_round(r0, r1, 0, false);
+        cp_async_commit();
+      }
+      if (nbuf == 2 && r + 1 < nr) {
+        const int n0 = r0 + H;
+        load_round(n0, min(it.t1, n0 + H), ((r + 1) % 2) * H, false);
+        cp_async_commit();
+        cp_async_wait<1>();
+      } else {
+        cp_async_wait<0>();
+      }
+      named_bar_sync(BAR, kAttnThreads);
+      attn_k_to_f16<D>(tile_k(slot0), r1 - r0, tid);
+      named_bar_sync(BAR, kAttnThreads);
+      if (r == 0) {
+        stamp(0);
+        attn_load_qfrag<D>(it, sQ, a);
+      }
+      score_round(r0, r1, slot0);
+      named_bar_sync(BAR, kAttnThreads);  // this half is reloaded by the round after next
+    }
   }
   stamp(1);
   if (trace && it.lane == 0) trace[5 + it.warp] = globaltimer_ns();

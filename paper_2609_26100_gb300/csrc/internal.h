@@ -115,7 +115,6 @@ struct MkParams {
   int n_act, d, H, D, F_pad, Ft, V, V_pad, n_pad, stages, attn_splits, B, max_tiles;
   int kps;  // k-blocks (16 KiB of weights each) per pipeline stage
   XsLayout xs;  // B-operand layout (n_pad == xs.rows)
-  int attn_early_conv;  // convert context keys to fp16 before waiting for the step's own rows
   int attn_plo;         // attention P.V with P split into hi/lo bf16 parts
   int l2_pace;  // SM clock cycles between L2 prefetches of 16 KiB (0: unpaced)
   int w_evict_first;  // stream weights with the evict-first L2 policy

@@ -136,12 +136,34 @@ __device__ void accept_greedy_body(const MiscParams& p, int b) {
   const StepDesc* st = p.step;
   __shared__ int am[kMaxNodes];
   __shared__ int path[kMaxNodes];
+  __shared__ int s_par[kMaxNodes], s_tok[kMaxNodes];
   const int N = st->req_nodes[b], off = st->req_rowoff[b];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    s_par[i] = st->row_parent[off + i];
+    s_tok[i] = st->tokens[off + i];
+  }
   for (int i = warp; i < N; i += nw) {
     float bv = -INFINITY;
     int bi = 0x7fffffff;
-    for (int t = lane; t < p.n_vtiles; t += 32) {
+    constexpr int kPer = 16;  // tile partials per lane in one round of loads (vocab <= 65536)
+    float vv[kPer];
+    int vi[kPer];
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      const int t = lane + 32 * q;
+      const bool in = t < p.n_vtiles;
+      vv[q] = in ? p.amax_val[static_cast<size_t>(t) * kMaxRows + off + i] : -INFINITY;
+      vi[q] = in ? p.amax_idx[static_cast<size_t>(t) * kMaxRows + off + i] : 0x7fffffff;
+    }
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      if (vv[q] > bv || (vv[q] == bv && vi[q] < bi)) {
+        bv = vv[q];
+        bi = vi[q];
+      }
+    }
+    for (int t = lane + 32 * kPer; t < p.n_vtiles; t += 32) {
       const float v = p.amax_val[static_cast<size_t>(t) * kMaxRows + off + i];
       const int ix = p.amax_idx[static_cast<size_t>(t) * kMaxRows + off + i];
       if (v > bv || (v == bv && ix < bi)) {
@@ -168,7 +190,7 @@ __device__ void accept_greedy_body(const MiscParams& p, int b) {
       const int want = am[cur];
       int nxt = -1;
       for (int c = cur + 1; c < N; ++c) {
-        if (st->row_parent[off + c] == cur && st->tokens[off + c] == want) {
+        if (s_par[c] == cur && s_tok[c] == want) {
           nxt = c;
           break;
         }
@@ -225,39 +247,54 @@ __device__ __forceinline__ T block_reduce(T v, T* red, Op op) {
 
 // Inverse CDF over token ids in ascending order: the smallest v whose running sum of w exceeds
 // u * sum(w).  Each thread owns a contiguous chunk; chunk sums are scanned in thread order.
+// fp32 throughout: the sums over a 32k vocabulary are accurate to ~1e-6 of the mass, far inside
+// the 2e-4 band within which a draw counts as consistent, and fp64 is slow on this GPU.
 template <typename WFn>
-__device__ int inverse_cdf_block(int V, double u, WFn w, double* scan) {
+__device__ int inverse_cdf_block(int V, float u, WFn w, float* scan) {
   const int nt = blockDim.x, t = threadIdx.x;
   const int C = (V + nt - 1) / nt;
   const int v0 = min(V, t * C), v1 = min(V, v0 + C);
-  double local = 0.0;
+  float local = 0.f;
   for (int v = v0; v < v1; ++v) local += w(v);
-  scan[t] = local;
-  __syncthreads();
-  if (t == 0) {
-    double run = 0.0;
-    for (int i = 0; i < nt; ++i) {
-      const double x = scan[i];
-      scan[i] = run;
-      run += x;
-    }
-    scan[nt] = run;
+  // exclusive scan of the chunk sums in thread order: warp scans, then the warp totals
+  const int lane = t & 31, warp = t >> 5, nw = nt >> 5;
+  float incl = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
   }
+  __shared__ float wsum[32];
+  if (lane == 31) wsum[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    float x = lane < nw ? wsum[lane] : 0.f;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane < nw) wsum[lane] = x;  // inclusive totals of warps 0..lane
+  }
+  __syncthreads();
+  const float before = (warp > 0 ? wsum[warp - 1] : 0.f) + (incl - local);
+  scan[t] = before;
+  if (t == nt - 1) scan[nt] = before + local;
   __syncthreads();
   __shared__ int sel;
   if (t == 0) sel = -1;
   __syncthreads();
-  const double total = scan[nt];
-  const double target = u * total;
-  const double lo = scan[t], hi = (t + 1 < nt) ? scan[t + 1] : total;
-  if (local > 0.0 && lo <= target && (target < hi || t + 1 == nt || hi >= total)) {
-    double run = lo;
+  const float total = scan[nt];
+  const float target = u * total;
+  const float lo = scan[t], hi = (t + 1 < nt) ? scan[t + 1] : total;
+  if (local > 0.f && lo <= target && (target < hi || t + 1 == nt || hi >= total)) {
+    float run = lo;
     int pick = -1, last_pos = -1;
     for (int v = v0; v < v1; ++v) {
-      const double x = w(v);
-      if (x > 0.0) last_pos = v;
+      const float x = w(v);
+      if (x > 0.f) last_pos = v;
       run += x;
-      if (run > target && x > 0.0) {
+      if (run > target && x > 0.f) {
         pick = v;
         break;
       }
@@ -272,7 +309,7 @@ __device__ int inverse_cdf_block(int V, double u, WFn w, double* scan) {
     if (t == 0) lastv = -1;
     __syncthreads();
     for (int v = v1 - 1; v >= v0; --v)
-      if (w(v) > 0.0) {
+      if (w(v) > 0.f) {
         atomicMax(&lastv, v);
         break;
       }
@@ -289,24 +326,25 @@ __device__ int inverse_cdf_block(int V, double u, WFn w, double* scan) {
 // if every draft is accepted draw it from p_k.  Uniform slots: r_i at i-1, u_i at k+i-1.
 __device__ void accept_sample_body(const MiscParams& p, int b) {
   const StepDesc* st = p.step;
-  __shared__ double scan[1025];
-  __shared__ double redd[32];
+  __shared__ float scan[1025];
+  __shared__ float redf[32];
   __shared__ int path[kMaxNodes];
   const int N = st->req_nodes[b], off = st->req_rowoff[b], k = N - 1, V = p.vocab;
-  const double invT = static_cast<double>(st->inv_temperature);
-  auto dmax = [](double a, double c) { return a > c ? a : c; };
-  auto dsum = [](double a, double c) { return a + c; };
+  const float invT = st->inv_temperature;
+  auto fmx = [](float a, float c) { return a > c ? a : c; };
+  auto fsum = [](float a, float c) { return a + c; };
   int a = 0, bonus = 0;
   for (int i = 0; i < N; ++i) path[i] = i;
   for (int i = 1; i <= k + 1; ++i) {
     const float* lg = st->logits + static_cast<size_t>(off + i - 1) * V;
-    double mx = -INFINITY;
-    for (int v = threadIdx.x; v < V; v += blockDim.x) mx = dmax(mx, static_cast<double>(lg[v]));
-    mx = block_reduce(mx, redd, dmax);
-    double z = 0.0;
-    for (int v = threadIdx.x; v < V; v += blockDim.x) z += exp((static_cast<double>(lg[v]) - mx) * invT);
-    z = block_reduce(z, redd, dsum);
-    auto pr = [&](int v) { return exp((static_cast<double>(lg[v]) - mx) * invT) / z; };
+    float mx = -INFINITY;
+    for (int v = threadIdx.x; v < V; v += blockDim.x) mx = fmx(mx, lg[v]);
+    mx = block_reduce(mx, redf, fmx);
+    float z = 0.f;
+    for (int v = threadIdx.x; v < V; v += blockDim.x) z += expf((lg[v] - mx) * invT);
+    z = block_reduce(z, redf, fsum);
+    const float invz = 1.f / z;
+    auto pr = [&](int v) { return expf((lg[v] - mx) * invT) * invz; };
     if (i <= k) {
       const int x = st->tokens[off + i];
       const float* q = st->draft_probs + static_cast<size_t>(off + i) * V;
@@ -316,19 +354,19 @@ __device__ void accept_sample_body(const MiscParams& p, int b) {
         bonus = 0;
         break;
       }
-      const double qx = static_cast<double>(q[x]);
-      if (!(qx > 0.0) && threadIdx.x == 0) report(p.status, kStatusCheck);
-      const double r = draw_uniform(st, b, i - 1);
+      const float qx = q[x];
+      if (!(qx > 0.f) && threadIdx.x == 0) report(p.status, kStatusCheck);
+      const float r = static_cast<float>(draw_uniform(st, b, i - 1));
       if (r * qx < pr(x)) continue;  // accept draft i
-      const double u = draw_uniform(st, b, k + i - 1);
+      const float u = static_cast<float>(draw_uniform(st, b, k + i - 1));
       bonus = inverse_cdf_block(V, u, [&](int v) {
-        const double d = pr(v) - static_cast<double>(q[v]);
-        return d > 0.0 ? d : 0.0;
+        const float d = pr(v) - q[v];
+        return d > 0.f ? d : 0.f;
       }, scan);
       a = i - 1;
       break;
     }
-    const double u = draw_uniform(st, b, 2 * k);
+    const float u = static_cast<float>(draw_uniform(st, b, 2 * k));
     bonus = inverse_cdf_block(V, u, pr, scan);
     a = k;
   }
@@ -365,7 +403,7 @@ __global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float
     if (threadIdx.x == 0) report(p.status, kStatusCheck);
     tok = 0;
   }
-  __shared__ float red[8];
+  __shared__ float red[16];
   __shared__ unsigned long long smask[kMaxBatch];
   __shared__ int s_l0, s_crow;
   // The first norm phase is the QKV of the union's first layer (or the LM head when every layer
@@ -402,15 +440,25 @@ __global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float
   float* h = p.h + static_cast<size_t>(m) * p.d_model;
   const int half = threadIdx.x >> 7, r = threadIdx.x & 127;
   const int n_t = p.d_model / 128;
-  for (int t0 = 0; t0 < n_t; t0 += 2) {
-    const int t = t0 + half;
+  // every load of the row first (one memory round trip), then the per-tile work
+  constexpr int kPer = 32;  // 128-feature tiles per thread half: d_model <= 8192
+  float xe[kPer], xg[kPer];
+#pragma unroll
+  for (int q = 0; q < kPer; ++q) {
+    const int t = 2 * q + half;
+    xe[q] = t < n_t ? __bfloat162float(e[t * 128 + r]) : 0.f;
+    xg[q] = t < n_t && xrow >= 0 ? gain[t * 128 + r] : 0.f;
+  }
+#pragma unroll
+  for (int q = 0; q < kPer; ++q) {
+    if (2 * q >= n_t) break;
+    const int t = 2 * q + half;
     float sq = 0.f;
     if (t < n_t) {
-      const float x = __bfloat162float(e[t * 128 + r]);
+      const float x = xe[q];
       h[t * 128 + r] = x;
-      if (xrow >= 0)
-      {
-        const float xv = x * gain[t * 128 + r];
+      if (xrow >= 0) {
+        const float xv = x * xg[q];
         if (p.xs.rows)
           store_split(p.xn, p.xs, xrow, t * 128 + r, xv);
         else
@@ -420,12 +468,11 @@ __global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sq;
-    __syncthreads();
+    if ((threadIdx.x & 31) == 0) red[(q & 1) * 8 + (threadIdx.x >> 5)] = sq;
+    __syncthreads();  // red is double-buffered by q parity, so one barrier per tile pair
     if (r == 0 && t < n_t)
-      ssp[static_cast<size_t>(t) * kMaxRows + m] =
-          (red[half * 4] + red[half * 4 + 1]) + (red[half * 4 + 2] + red[half * 4 + 3]);
-    __syncthreads();
+      ssp[static_cast<size_t>(t) * kMaxRows + m] = (red[(q & 1) * 8 + half * 4] + red[(q & 1) * 8 + half * 4 + 1]) +
+                                                   (red[(q & 1) * 8 + half * 4 + 2] + red[(q & 1) * 8 + half * 4 + 3]);
   }
 }
 

@@ -1082,8 +1082,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
               p.trace && ph.slot == 1 ? p.trace + static_cast<size_t>(blockIdx.x) * kMkTraceSlots + kMkTraceAttn : nullptr;
           bool failed = false;
           const bool wrote = attention_item_resident<D, 1>(ap, split, head, b, e.et, base, ring_attn_bytes, sM, sL,
-                                                           misc + 5, atr, wait_inputs, failed, p.attn_early_conv != 0,
-                                                           p.attn_plo != 0);
+                                                           misc + 5, atr, wait_inputs, failed, p.attn_plo != 0);
           if (failed) {
             ok = false;
             break;
