@@ -41,6 +41,9 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-profile", action="store_true")
+    p.add_argument("--sweep", default=None,
+                   help="7b_long: comma-separated skipped-layer counts (e.g. 0,2,4,...,12); one process, one "
+                        "weight and KV set, latency vs active layers with a least-squares line")
     p.add_argument("--traffic", default=os.path.join(ROOT, "profiles", "verify_persistent_7b_chain_traffic.txt"),
                    help="JSON summary of an ncu DRAM-traffic capture of the dominant kernel")
     return p.parse_args()
@@ -453,10 +456,70 @@ def run_tss(args):
         dist.destroy_process_group()
 
 
+def run_sweep(args):
+    """Verify latency of the KV-bound 7B workload (B=16, ctx 16384, k=8) against the number of
+    active layers: the skip sets are nested prefixes of one seeded permutation, the weights and
+    the context KV of every layer are generated once, and each point is timed with CUDA events.
+    Prints one JSON line: the points, the least-squares line (slope, intercept, R^2) and each
+    point's bytes against the measured and nominal HBM peaks."""
+    import torch
+    from paper_2609_26100_gb300 import build as _build
+    from paper_2609_26100_gb300 import native, synth
+    from paper_2609_26100_gb300.runner import TssRunner
+    torch.cuda.set_device(0)
+    _build.build()
+    counts = [int(x) for x in args.sweep.split(",")]
+    dense = synth.workload_7b_long(n_skip=0)
+    run = TssRunner.for_workload(dense)
+    stream = torch.cuda.current_stream()
+    peak, _ = measured_peak()
+    points = []
+    for n in counts:
+        w = synth.workload_7b_long(n_skip=n)
+        run.set_phi(w.phi)
+        res = run.alloc_results(len(w.requests), w.n_rows, logits=False)
+        b = run.batch(w.requests)
+        for _ in range(max(2, args.warmup)):
+            run.verify(b, res)
+        if run.sync_status() != native.TSS_OK:
+            raise RuntimeError(f"device status error at {n} skipped layers")
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+        torch.cuda.synchronize()
+        ev[0].record(stream)
+        for i in range(args.steps):
+            run.verify(b, res)
+            ev[i + 1].record(stream)
+        torch.cuda.synchronize()
+        ms = ev[0].elapsed_time(ev[-1]) / args.steps
+        ab = synth.algorithmic_bytes(w)
+        gbs = ab["total"] / (ms * 1e-3) / 1e9
+        points.append({"skipped": n, "active_layers": ab["active_union"], "us_per_step": ms * 1e3,
+                       "bytes_per_step": ab["total"], "achieved_gbs": gbs, "frac_of_measured": gbs / peak,
+                       "frac_of_nominal_8TBs": gbs / NOMINAL_HBM_GBS})
+        print(f"[sweep] skipped {n:2d}: {ms * 1e3:9.1f} us/step, {gbs:7.1f} GB/s", file=sys.stderr)
+    run.close()
+    xs = [p_["active_layers"] for p_ in points]
+    ys = [p_["us_per_step"] for p_ in points]
+    n = len(xs)
+    mx, my = sum(xs) / n, sum(ys) / n
+    sxx = sum((x - mx) ** 2 for x in xs)
+    slope = sum((x - mx) * (y - my) for x, y in zip(xs, ys)) / sxx if sxx > 0 else 0.0
+    icpt = my - slope * mx
+    ss_tot = sum((y - my) ** 2 for y in ys)
+    ss_res = sum((y - (icpt + slope * x)) ** 2 for x, y in zip(xs, ys))
+    r2 = 1.0 - ss_res / ss_tot if ss_tot > 0 else 1.0
+    print(json.dumps({"metric": "7B KV-bound verify latency vs active layers (B=16, ctx 16384, k=8)",
+                      "unit": "us/step", "higher_is_better": False, "steps": args.steps, "points": points,
+                      "fit": {"slope_us_per_layer": slope, "intercept_us": icpt, "r2": r2},
+                      "data": "synthetic (seeded random-init weights, synthetic KV)"}))
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.sweep:
+        run_sweep(args)
     else:
         run_tss(args)
 
