@@ -124,6 +124,7 @@ struct tss_ctx {
   bool use_mk = true;
   int l2_ahead = 0;
   int mk_kps = 4;  // weight k-blocks per ring stage of the persistent kernel
+  int attn_mode = 0;  // 0 auto, 1 attention inside the persistent kernel, 2 separate attention kernels
   int l2_pace = 0;       // cycles between paced L2 weight prefetches of 16 KiB (0: unpaced)
   int w_evict_first = 1;
   int pf_attn = 0, pf_next = 0;
@@ -259,7 +260,8 @@ tss_status run_gemm(tss_ctx* c, int epi, const CUtensorMap& tmW, const CUtensorM
 
 struct StepPlan {
   int B, M, n_act, mode, splits, n_pad;
-  int tiles;  // 64-key tiles of the longest request (context + block)
+  int tiles;          // 64-key tiles of the longest request (context + block)
+  long long ctx_sum;  // context tokens over the batch
 };
 
 // Optional per-launch event timing (tss_verify_profiled).
@@ -500,8 +502,47 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
     expr;                                  \
     if (prof) TSS_TRY(prof->end());        \
   } while (0)
+  // Long contexts: the KV stream outweighs the weights, and the attention wants more warps per
+  // SM than the persistent kernel has; each layer's attention is then a separate kernel between
+  // launches of the persistent kernel over the GEMM phases in between.
+  const double layer_bytes = (4.0 * c->d * c->d + 3.0 * c->d * c->a.d_mlp) * 2.0;
+  const double kv_bytes = static_cast<double>(sp.ctx_sum) * 4.0 * c->d;
+  const bool ext = c->attn_mode == 2 || (c->attn_mode == 0 && kv_bytes >= 0.5 * layer_bytes);
+  p.attn_external = ext ? 1 : 0;
   TSS_MK(0, TSS_CU(launch_prologue(mp, c->ssp, c->mk_zero, c->mk_n_zero, sp.M, s, false)));
-  TSS_MK(8, TSS_CU(launch_verify_mk(p, c->num_sms, smem, s)));
+  if (!ext) {
+    p.ph_begin = 0;
+    p.ph_end = 1 << 30;
+    TSS_MK(8, TSS_CU(launch_verify_mk(p, c->num_sms, smem, s)));
+  } else {
+    AttnParams ap{};
+    ap.n_splits = sp.splits;
+    ap.n_heads = c->H;
+    ap.d_model = c->d;
+    ap.head_dim = c->D;
+    ap.scale_log2 = p.scale_log2;
+    ap.plan = c->d_plan;
+    ap.step = c->d_step;
+    ap.q = c->qbuf;
+    ap.o = c->obuf;
+    ap.o_xs = xs;  // fp16 q, hi/lo output: the persistent kernel's operands
+    ap.part_o = c->attn_po;
+    ap.part_ml = c->attn_pml;
+    ap.counters = c->attn_cnt;
+    ap.status = c->d_status;
+    int pb = 0;
+    for (int j = 0; j < sp.n_act; ++j) {
+      p.ph_begin = pb;  // phases 4j .. 4j+3 are QKV, O, gate/up, down of slot j; 4 n_act the LM head
+      p.ph_end = 4 * j + 1;
+      TSS_MK(8, TSS_CU(launch_verify_mk(p, c->num_sms, smem, s)));
+      ap.slot = j;
+      TSS_MK(2, TSS_CU(launch_attention(ap, sp.B, s, false)));
+      pb = 4 * j + 1;
+    }
+    p.ph_begin = pb;
+    p.ph_end = 1 << 30;
+    TSS_MK(8, TSS_CU(launch_verify_mk(p, c->num_sms, smem, s)));
+  }
   TSS_MK(7, TSS_CU(launch_finish(mp, sp.B, s, false)));
 #undef TSS_MK
   return TSS_OK;
@@ -807,6 +848,8 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
   sp->splits = splits;
   sp->n_pad = pad_to(M, 16);
   sp->tiles = tiles;
+  sp->ctx_sum = 0;
+  for (int b = 0; b < B; ++b) sp->ctx_sum += bt->ctx_len[b];
   return TSS_OK;
 }
 
@@ -859,6 +902,10 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_GEMM_CTAS_PER_SM")) c->gemm_ctas_per_sm = std::max(1, std::min(2, std::atoi(e)));
   if (const char* e = std::getenv("TSS_PATH")) c->use_mk = std::string(e) != "multi";
   if (const char* e = std::getenv("TSS_L2_AHEAD")) c->l2_ahead = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("TSS_ATTN")) {
+    const std::string v(e);
+    c->attn_mode = v == "internal" ? 1 : v == "external" ? 2 : 0;
+  }
   if (const char* e = std::getenv("TSS_MK_KPS")) c->mk_kps = std::min(8, std::max(1, std::atoi(e)));
   if (const char* e = std::getenv("TSS_L2_PACE")) c->l2_pace = std::min(100000, std::max(0, std::atoi(e)));
   if (const char* e = std::getenv("TSS_EVICT_FIRST")) c->w_evict_first = std::atoi(e) != 0;

@@ -18,34 +18,42 @@ namespace tss {
 
 size_t attn_smem_bytes(int head_dim) { return attn_smem_bytes_impl(head_dim); }
 
-template <int D>
+template <int D, bool P16>
 __global__ void __launch_bounds__(kAttnThreads) attn_kernel(const AttnParams p) {
   extern __shared__ __align__(16) uint8_t smem_raw[];
   __shared__ float sM[4][16], sL[4][16];
   __shared__ int s_last;
   griddep_wait();
   griddep_launch();
-  attention_item<D, 0>(p, blockIdx.x, blockIdx.y, blockIdx.z, threadIdx.x, smem_raw, sM, sL, &s_last);
+  attention_item<D, 0, P16>(p, blockIdx.x, blockIdx.y, blockIdx.z, threadIdx.x, smem_raw, sM, sL, &s_last);
+}
+
+template <int D, bool P16>
+static cudaError_t attn_prepare_one() {
+  cudaError_t e = cudaFuncSetAttribute(attn_kernel<D, P16>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                       cudaSharedmemCarveoutMaxShared);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attn_kernel<D, P16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(attn_smem_bytes(D)));
 }
 
 cudaError_t attn_prepare() {
-  cudaError_t e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                       cudaSharedmemCarveoutMaxShared);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                             cudaSharedmemCarveoutMaxShared);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(attn_smem_bytes(64)));
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(attn_smem_bytes(128)));
+  cudaError_t e = attn_prepare_one<64, false>();
+  if (e == cudaSuccess) e = attn_prepare_one<128, false>();
+  if (e == cudaSuccess) e = attn_prepare_one<64, true>();
+  if (e == cudaSuccess) e = attn_prepare_one<128, true>();
+  return e;
 }
 
 cudaError_t launch_attention(const AttnParams& p, int B, cudaStream_t s, bool pdl) {
   const dim3 grid(p.n_splits, p.n_heads, B), block(kAttnThreads);
-  if (p.head_dim == 64) return launch_k(attn_kernel<64>, grid, block, attn_smem_bytes(64), s, pdl, p);
-  if (p.head_dim == 128) return launch_k(attn_kernel<128>, grid, block, attn_smem_bytes(128), s, pdl, p);
+  const bool p16 = p.o_xs.rows != 0;  // the persistent path's operands and precision
+  if (p.head_dim == 64)
+    return p16 ? launch_k(attn_kernel<64, true>, grid, block, attn_smem_bytes(64), s, pdl, p)
+               : launch_k(attn_kernel<64, false>, grid, block, attn_smem_bytes(64), s, pdl, p);
+  if (p.head_dim == 128)
+    return p16 ? launch_k(attn_kernel<128, true>, grid, block, attn_smem_bytes(128), s, pdl, p)
+               : launch_k(attn_kernel<128, false>, grid, block, attn_smem_bytes(128), s, pdl, p);
   return cudaErrorInvalidValue;
 }
 

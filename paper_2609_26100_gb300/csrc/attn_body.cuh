@@ -251,7 +251,7 @@ __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __
 }
 
 // This warp's keys of one resident 64-key tile (K / V buffers sK, sV).
-template <int D>
+template <int D, bool QK16 = false, bool PLO = false>
 __device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, const __nv_bfloat16* sK,
                                                const __nv_bfloat16* sV, float scale_log2, AttnAcc<D>& a) {
   constexpr int LD = attn_ld<D>();
@@ -265,7 +265,7 @@ __device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, 
     vp[np] = sV + (kbase + np * 16) * LD;
     key0[np] = tile * kKeyTile + kbase + np * 16;
   }
-  attn_blocks_step<D>(it, kp, vp, key0, it.kpw / 16, scale_log2, a);
+  attn_blocks_step<D, QK16, PLO>(it, kp, vp, key0, it.kpw / 16, scale_log2, a);
 }
 
 // Merge the warps that share a query tile through shared memory (sO: [4][16][D] floats, any
@@ -396,12 +396,34 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
   return true;
 }
 
+// bf16 -> fp16 in place for the K rows of `tiles` resident tiles (each tile: K [kKeyTile][LD],
+// then V); the bf16 cache values are exact in fp16 within its range (|x| < 65504; below 6.1e-5
+// fp16 is subnormal).
+template <int D>
+__device__ __forceinline__ void attn_k_to_f16(__nv_bfloat16* tiles0, int tiles, int tid) {
+  constexpr int LD = attn_ld<D>(), C8 = D / 8;
+  for (int idx = tid; idx < tiles * kKeyTile * C8; idx += kAttnThreads) {
+    const int row = idx / C8, c8 = idx - row * C8;  // row over the tiles' K rows
+    const int tl = row / kKeyTile, kr = row - tl * kKeyTile;
+    uint4* ptr = reinterpret_cast<uint4*>(tiles0 + (tl * 2 * kKeyTile + kr) * LD + c8 * 8);
+    uint4 v = *ptr;
+    uint32_t* w = reinterpret_cast<uint32_t*>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float lo = __uint_as_float(w[i] << 16), hi = __uint_as_float(w[i] & 0xffff0000u);
+      w[i] = pack_f16(lo, hi);
+    }
+    *ptr = v;
+  }
+}
+
 // One work item (split, head, request) run by 128 threads (tid 0..127) that synchronise with
 // named barrier BAR, streaming its key tiles through a double buffer.  smem: attn_smem_bytes(D)
 // bytes, 16-byte aligned.  Returns true on the call that wrote the final output rows of
 // (request, head) (the only split, or the last split to finish, which merges the others in
-// split order).
-template <int D, int BAR>
+// split order).  P16: the persistent path's precision (q in fp16, keys converted to fp16 for the
+// score MMAs, P as hi/lo bf16 parts in P.V); else all bf16.
+template <int D, int BAR, bool P16 = false>
 __device__ bool attention_item(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
                                float (*sM)[16], float (*sL)[16], int* s_last) {
   constexpr int LD = attn_ld<D>();
@@ -422,34 +444,17 @@ __device__ bool attention_item(const AttnParams& p, int split, int head, int b, 
     cp_async_commit();
     cp_async_wait<1>();
     named_bar_sync(BAR, kAttnThreads);
+    if (P16) {
+      attn_k_to_f16<D>(sK + buf * kKeyTile * LD, 1, tid);
+      named_bar_sync(BAR, kAttnThreads);
+    }
     if (tile == it.t0) attn_load_qfrag<D>(it, sQ, a);
-    attn_tile_step<D>(it, tile, sK + buf * kKeyTile * LD, sV + buf * kKeyTile * LD, p.scale_log2, a);
+    attn_tile_step<D, P16, P16>(it, tile, sK + buf * kKeyTile * LD, sV + buf * kKeyTile * LD, p.scale_log2, a);
     named_bar_sync(BAR, kAttnThreads);
   }
   cp_async_wait<0>();
   return attn_finish<D, BAR>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sK), sM, sL, s_last,
                              [](int) {});
-}
-
-// bf16 -> fp16 in place for the K rows of `tiles` resident tiles (each tile: K [kKeyTile][LD],
-// then V); the bf16 cache values are exact in fp16 within its range (|x| < 65504; below 6.1e-5
-// fp16 is subnormal).
-template <int D>
-__device__ __forceinline__ void attn_k_to_f16(__nv_bfloat16* tiles0, int tiles, int tid) {
-  constexpr int LD = attn_ld<D>(), C8 = D / 8;
-  for (int idx = tid; idx < tiles * kKeyTile * C8; idx += kAttnThreads) {
-    const int row = idx / C8, c8 = idx - row * C8;  // row over the tiles' K rows
-    const int tl = row / kKeyTile, kr = row - tl * kKeyTile;
-    uint4* ptr = reinterpret_cast<uint4*>(tiles0 + (tl * 2 * kKeyTile + kr) * LD + c8 * 8);
-    uint4 v = *ptr;
-    uint32_t* w = reinterpret_cast<uint32_t*>(&v);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float lo = __uint_as_float(w[i] << 16), hi = __uint_as_float(w[i] & 0xffff0000u);
-      w[i] = pack_f16(lo, hi);
-    }
-    *ptr = v;
-  }
 }
 
 // Tiles of K and V that attention_item_resident keeps resident in `smem_bytes` of shared memory.

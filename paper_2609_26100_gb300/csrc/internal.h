@@ -121,6 +121,10 @@ struct MkParams {
   int pf_attn;  // 16 KiB weight blocks of the O phase warmed into L2 while the attention runs
   int pf_next;  // blocks of the next phase (beyond the ring) warmed into L2 when a phase ends
   int attn_extra;  // shared memory behind the ring that only the attention uses (bytes)
+  // Phases [ph_begin, ph_end) run in this launch.  attn_external: the attention of each layer is a
+  // separate kernel launched between the launches (long contexts), so none runs in here and an
+  // O phase needs no flag from it.
+  int ph_begin, ph_end, attn_external;
   int l2_ahead;  // weight tiles per CTA prefetched into L2 ahead of the smem ring (0: off)
   unsigned long long* trace;  // optional timeline [grid][mk_trace_slots()], nullptr when off
   float eps, scale_log2;

@@ -570,7 +570,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
 
   const int G = gridDim.x, c = blockIdx.x;
   // A host/device disagreement on the layer union (reported by the controller) runs nothing.
-  const int n_phases = pl->n_act == p.n_act ? 4 * p.n_act + 1 : 0;
+  const int n_phases = pl->n_act == p.n_act ? min(4 * p.n_act + 1, p.ph_end) : 0;
+  const int ph0 = p.ph_begin;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -579,12 +580,12 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       const uint64_t wpol = l2_policy_evict_first();
       long long i = 0;
       bool ok = true;
-      for (int pi = 0; ok && pi < n_phases; ++pi) {
+      for (int pi = ph0; ok && pi < n_phases; ++pi) {
         const MkPhase ph = mk_phase(p, pl, pi);
         long long it0, it1;
         int geff;
         mk_range(ph, c, G, it0, it1, geff);
-        if (ph.kind == kMkO && !mk_wait_gate(attn_gate, ph.slot, sh)) {
+        if (ph.kind == kMkO && !p.attn_external && !mk_wait_gate(attn_gate, ph.slot, sh)) {
           ok = false;
           break;
         }
@@ -626,7 +627,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       long long i = 0;
       int use = 0;
       bool ok = true;
-      for (int pi = 0; ok && pi < n_phases; ++pi) {
+      for (int pi = ph0; ok && pi < n_phases; ++pi) {
         const MkPhase ph = mk_phase(p, pl, pi);
         long long it0, it1;
         int geff;
@@ -682,13 +683,13 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     // ---------------- B-operand producer: TMA after the producing tiles are flagged ----------------
     long long i = 0;
     bool ok = true;
-    for (int pi = 0; ok && pi < n_phases; ++pi) {
+    for (int pi = ph0; ok && pi < n_phases; ++pi) {
       const MkPhase ph = mk_phase(p, pl, pi);
       long long it0, it1;
       int geff;
       mk_range(ph, c, G, it0, it1, geff);
       if (it0 >= it1) continue;
-      if (ph.kind == kMkO) {
+      if (ph.kind == kMkO && !p.attn_external) {
         bool free = true;
         if (lane == 0) free = mk_wait_gate(attn_gate, ph.slot, sh);
         if (!__shfl_sync(0xffffffffu, free, 0)) {
@@ -702,7 +703,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       int n_dep;
       if (ph.kind == kMkO) {
         flags = p.attflag;
-        want = mk_seq(p.seq_base, ph.slot, kMkAtt);
+        want = p.attn_external ? 0ull : mk_seq(p.seq_base, ph.slot, kMkAtt);  // else: an earlier launch
         n_dep = p.H;
       } else if (ph.kind == kMkDown) {
         flags = p.guflag;
@@ -785,7 +786,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       long long j = 0;
       bool go = true;
       long long next_pf = clock64();
-      for (int pi = 0; go && pi < n_phases; ++pi) {
+      for (int pi = ph0; go && pi < n_phases; ++pi) {
         const MkPhase ph = mk_phase(p, pl, pi);
         long long it0, it1;
         int geff;
@@ -854,7 +855,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     ap.part_ml = p.attn_pml;
     ap.counters = p.attn_cnt;
     ap.status = p.status;
-    for (int pi = 0; ok && pi < n_phases; ++pi) {
+    for (int pi = ph0; ok && pi < n_phases; ++pi) {
       const MkPhase ph = mk_phase(p, pl, pi);
       long long it0, it1;
       int geff;
@@ -904,7 +905,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           s_rope[j * half + i] = p.rope_cos[static_cast<size_t>(s_pos[j]) * half + i];
           s_rope[16 * 64 + j * half + i] = p.rope_sin[static_cast<size_t>(s_pos[j]) * half + i];
         }
-        if (e.et == 0) {
+        if (e.et == 0 && !p.attn_external) {
           const int per_req = p.H * p.attn_splits;
           const StepDesc* st = p.step;
           for (int item = c; item < p.B * per_req; item += G) {
@@ -1053,7 +1054,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       if (!ok) break;
       if (ph.kind != kMkQkv && e.et == 0)
         mk_prefetch_phase(p, pl, pi + 1, n_phases, c, G, static_cast<long long>(S) * KPS, p.pf_next);
-      if (ph.kind == kMkQkv) {
+      if (ph.kind == kMkQkv && !p.attn_external) {
         // attention items of this layer: (request, head, split) round-robin over the grid
         ap.slot = ph.slot;
         const int per_req = p.H * p.attn_splits;
