@@ -149,15 +149,26 @@ def kernel_sources_hash():
     return h.hexdigest()
 
 
-def kernel_bytes(w):
-    """Algorithmic bytes per launch of each kernel kind (weights + activations in and out + KV).
-    The persistent verify kernel streams every active layer and the LM head in one launch."""
+def kernel_bytes(w, kinds):
+    """Algorithmic bytes per STEP of each kernel kind present (weights + activations + KV).
+    Persistent path: the persistent kernel streams every active layer's weights and the LM head
+    (and the KV too when the attention runs inside it); with separate attention launches (long
+    contexts) the attention kind carries the KV reads.  Kernel-per-op path: the per-layer
+    formulas times the launches."""
     from paper_2609_26100_gb300 import synth
     a = w.arch
     d, f, V, M = a.d_model, a.d_mlp, a.vocab, w.n_rows
+    ab = synth.algorithmic_bytes(w)
     kv_read = sum(r.ctx_len for r in w.requests) * a.kv_bytes_per_token  # per layer, all requests
-    return {
-        "verify_persistent": synth.algorithmic_bytes(w)["total"],
+    out = {}
+    if "verify_persistent" in kinds:
+        if "attention" in kinds:
+            out["verify_persistent"] = ab["total"] - ab["kv_read"]
+            out["attention"] = ab["kv_read"]
+        else:
+            out["verify_persistent"] = ab["total"]
+        return out
+    per_launch = {
         "qkv_gemm": 3 * d * d * 2 + M * d * 2 + M * d * 2 + M * 2 * d * 2,
         "attention": kv_read + M * d * 2 * 2 + M * 2 * d * 2,
         "o_gemm": d * d * 2 + M * d * 2 + M * d * 4 * 2,
@@ -165,6 +176,10 @@ def kernel_bytes(w):
         "down_gemm": d * f * 2 + M * f * 2 + M * d * 4 * 2,
         "lm_head_gemm": V * d * 2 + M * d * 2 + M * V * 4,
     }
+    for k, v in kinds.items():
+        if k in per_launch:
+            out[k] = per_launch[k] * v
+    return out
 
 
 # ----------------------------------------------------------------------------------------------
@@ -360,10 +375,14 @@ def run_tss(args):
 
     # ---------------- e2e: host buffers through the C ABI, one sync per step ----------------
     e2e = None
-    if not args.no_e2e and not sample_mode:
+    if not args.no_e2e:
         hres = run.alloc_results(len(w.requests), w.n_rows, logits=False, host=True)
         htoks = [torch.tensor(token_sets[v], dtype=torch.int32).pin_memory() for v in range(n_var)]
-        hb = [run.batch(w.requests, tokens=htoks[v], io_host=True) for v in range(n_var)]
+        hprobs = probs.cpu().pin_memory() if sample_mode else None
+        hb = [run.batch(w.requests, tokens=htoks[v], io_host=True,
+                        mode=native.TSS_MODE_SAMPLE if sample_mode else native.TSS_MODE_GREEDY,
+                        temperature=w.temperature, draft_probs=hprobs, philox_seed=w.seed, philox_offset=v)
+              for v in range(n_var)]
         for i in range(3):
             run.verify(hb[i % n_var], hres)
         torch.cuda.synchronize()
@@ -376,7 +395,7 @@ def run_tss(args):
             acc_sum += int(hres["accept_len"].sum())
         e2e_s = time.perf_counter() - t0
         e2e = {"value": world * w.n_rows * n_e2e / e2e_s, "unit": "tokens/s",
-               "h2d_bytes_per_step": 4 * w.n_rows,
+               "h2d_bytes_per_step": 4 * w.n_rows + (hprobs.numel() * 4 if sample_mode else 0),
                "d2h_bytes_per_step": 4 * (3 * len(w.requests) + hres["path"].numel()),
                "ms_per_step": e2e_s / n_e2e * 1e3, "steps": n_e2e}
 
@@ -391,15 +410,17 @@ def run_tss(args):
         n_prof = 1 if args.no_profile else max(5, min(args.steps, 20))
         for i in range(n_prof):
             run.v.verify_profiled(batches[i % n_var], run.kv_struct, res["_struct"], times, stream.cuda_stream)
-        kb = kernel_bytes(w)
         kernels = {}
         for k, name in enumerate(native.KERNEL_KINDS):
             if times.launches[k]:
                 avg = times.ms[k] / times.launches[k]
                 kernels[name] = {"launches_per_step": times.launches[k] / n_prof, "ms_per_step": times.ms[k] / n_prof,
                                  "avg_launch_us": avg * 1e3}
-                if name in kb:
-                    kernels[name]["gbs"] = kb[name] / (avg * 1e-3) / 1e9
+        kb = kernel_bytes(w, {n: v["launches_per_step"] for n, v in kernels.items()})
+        for name, v in kernels.items():
+            if name in kb:
+                v["bytes_per_step"] = kb[name]
+                v["gbs"] = kb[name] / (v["ms_per_step"] * 1e-3) / 1e9
         launches_per_step = sum(v["launches_per_step"] for v in kernels.values())
         tot = sum(v["ms_per_step"] for v in kernels.values())
         for v in kernels.values():
@@ -409,7 +430,7 @@ def run_tss(args):
         roofline = {"kernel": dom, "bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
                     "frac": ach / peak, "peak_source": f"{peak_kind} copy bandwidth",
                     "frac_of_nominal_8TBs": ach / NOMINAL_HBM_GBS,
-                    "bytes_per_launch": kb[dom], "traffic": None}
+                    "bytes_per_launch": kb[dom] / kernels[dom]["launches_per_step"], "traffic": None}
         if args.traffic and os.path.exists(args.traffic):
             # DRAM bytes per launch of this kernel from an ncu capture (a summary with "kernel",
             # "workload", "traffic_bytes" and the hash of the kernel sources it was taken on);
