@@ -347,50 +347,56 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
   stamp(3);
   if (!*s_last) return false;
   __threadfence();
-  constexpr int kMergeRegs = 8;  // splits whose partials are loaded at once
-  for (int idx = tid; idx < N * D; idx += kAttnThreads) {
-    const int i = idx / D, dd = idx - i * D;
-    float M = -INFINITY, L = 0.f, O = 0.f;
-    if (p.n_splits <= kMergeRegs) {
-      // every split's (max, sum, O) in one round of loads, then the same fixed-order merge
-      float pm[kMergeRegs], pl[kMergeRegs], po[kMergeRegs];
-#pragma unroll
-      for (int sp = 0; sp < kMergeRegs; ++sp) {
-        if (sp < p.n_splits) {
-          const size_t pi = (ph + sp) * kMaxNodes + i;
-          pm[sp] = __ldcg(&p.part_ml[pi * 2]);
-          pl[sp] = __ldcg(&p.part_ml[pi * 2 + 1]);
-          po[sp] = __ldcg(&p.part_o[pi * D + dd]);
-        }
-      }
-#pragma unroll
-      for (int sp = 0; sp < kMergeRegs; ++sp)
-        if (sp < p.n_splits) M = fmaxf(M, pm[sp]);
-      const float base = M == -INFINITY ? 0.f : M;
-#pragma unroll
-      for (int sp = 0; sp < kMergeRegs; ++sp) {
-        if (sp < p.n_splits) {
-          const float f = exp2f(pm[sp] - base);
-          L += f * pl[sp];
-          O += f * po[sp];
-        }
-      }
-    } else {
-      for (int sp = 0; sp < p.n_splits; ++sp) M = fmaxf(M, __ldcg(&p.part_ml[((ph + sp) * kMaxNodes + i) * 2]));
-      const float base = M == -INFINITY ? 0.f : M;
-      for (int sp = 0; sp < p.n_splits; ++sp) {
-        const size_t pi = (ph + sp) * kMaxNodes + i;
-        const float f = exp2f(__ldcg(&p.part_ml[pi * 2]) - base);
-        L += f * __ldcg(&p.part_ml[pi * 2 + 1]);
-        O += f * __ldcg(&p.part_o[pi * D + dd]);
-      }
+  // Merge weights per (row, split) first -- w = 2^(m_s - M) / L with L = sum 2^(m_s - M) l_s, in
+  // split order -- into shared memory (sO is free again), then every output element is a
+  // weighted sum of the splits' O, several elements' loads in flight per thread.
+  float* wgt = sO;  // [N][n_splits]
+  const int ns = p.n_splits;
+  for (int i = tid; i < N; i += kAttnThreads) {
+    float M = -INFINITY;
+    for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, __ldcg(&p.part_ml[((ph + sp) * kMaxNodes + i) * 2]));
+    const float base = M == -INFINITY ? 0.f : M;
+    float L = 0.f;
+    for (int sp = 0; sp < ns; ++sp) {
+      const size_t pi = (ph + sp) * kMaxNodes + i;
+      const float f = exp2f(__ldcg(&p.part_ml[pi * 2]) - base);
+      L += f * __ldcg(&p.part_ml[pi * 2 + 1]);
+      wgt[i * ns + sp] = f;
     }
     if (!(L > 0.f)) report(p.status, kStatusCheck);
-    const float val = L > 0.f ? O / L : 0.f;
-    if (p.o_xs.rows)
-      store_split(p.o, p.o_xs, crow + i, head * D + dd, val);
-    else
-      p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    for (int sp = 0; sp < ns; ++sp) wgt[i * ns + sp] *= inv;
+  }
+  named_bar_sync(BAR, kAttnThreads);
+  constexpr int kU = 4;  // output elements per thread with their loads in flight together
+  for (int idx0 = tid; idx0 < N * D; idx0 += kU * kAttnThreads) {
+    float O[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) O[u] = 0.f;
+    for (int sp = 0; sp < ns; ++sp) {
+      float po[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int idx = idx0 + u * kAttnThreads;
+        const int i = idx / D, dd = idx - i * D;
+        po[u] = idx < N * D ? __ldcg(&p.part_o[((ph + sp) * kMaxNodes + i) * D + dd]) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int idx = idx0 + u * kAttnThreads;
+        if (idx < N * D) O[u] += wgt[(idx / D) * ns + sp] * po[u];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int idx = idx0 + u * kAttnThreads;
+      if (idx >= N * D) continue;
+      const int i = idx / D, dd = idx - i * D;
+      if (p.o_xs.rows)
+        store_split(p.o, p.o_xs, crow + i, head * D + dd, O[u]);
+      else
+        p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(O[u]);
+    }
   }
   stamp(4);
   return true;
