@@ -137,7 +137,7 @@ __device__ bool mk_wait_bar(uint64_t* bar, uint32_t parity, const MkShared& sh) 
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     if ((i & 255) == 0) {
       if (mk_aborted(sh)) return false;
       if (globaltimer_ns() - t0 > kWaitLimitNs) {
@@ -290,6 +290,12 @@ struct MkEpi {
   const float* gnext;  // residual phases: RMSNorm gain of the next norm phase
   bool direct_xn;      // residual phases: the next norm phase runs the same rows in the same order,
                        // so the epilogue writes its B operand straight from the updated h
+  int hpre_tile;       // residual phases: tile whose h rows were preloaded into xch (-1: none)
+  float gn_pre;        // ... and this thread's next-norm gain on that tile
+  // values the epilogue chunks would otherwise load from the step descriptor in global memory
+  __nv_bfloat16* kv_base;  // QKV: this layer's KV cache
+  size_t kv_cap;
+  float* logits;           // LM head: caller's logits or null
   int q, lane, et;
 };
 
@@ -359,15 +365,15 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
         reinterpret_cast<__half*>(p.qbuf)[static_cast<size_t>(j) * d + f] = __float2half_rn(val[jj]);
       } else {
         const size_t off = ((static_cast<size_t>(e.kvslot[j]) * 2 + (sec - 1)) * p.H + head) *
-                               static_cast<size_t>(st->kv_cap) +
+                               e.kv_cap +
                            e.kvrow[j];
-        st->kv_layer[ph.layer][off * D + dim] = __float2bfloat16_rn(val[jj]);
+        e.kv_base[off * D + dim] = __float2bfloat16_rn(val[jj]);
       }
     }
   } else if (ph.kind == kMkO || ph.kind == kMkDown) {
     // residual add, then this tile's partial sum of squares of the updated rows
     const int o = t * 128 + r;
-    const float gn = e.direct_xn ? e.gnext[o] : 0.f;
+    const float gn = e.direct_xn ? (t == e.hpre_tile ? e.gn_pre : e.gnext[o]) : 0.f;
     float sq[16];
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) {
@@ -375,7 +381,8 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
       sq[jj] = 0.f;
       if (j < e.M) {
         float* hp = p.h + static_cast<size_t>(e.rows[j]) * p.d + o;
-        const float nv = __ldcg(hp) + v[jj];
+        // h of the CTA's last tile was loaded at phase start (off the critical path)
+        const float nv = (t == e.hpre_tile ? e.xch[jj * 128 + r] : __ldcg(hp)) + v[jj];
         *hp = nv;
         sq[jj] = nv * nv;
         if (e.direct_xn) store_split(p.xn, p.xs, j, o, nv * gn);
@@ -417,7 +424,7 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
   } else {  // LM head: logits (optional) and per-tile argmax, lowest index on ties
     const int o = t * 128 + r;
     const bool valid = o < p.V;
-    float* logits = st->logits;
+    float* logits = e.logits;
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) {
       const int j = j0 + jj;
@@ -896,6 +903,27 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       e.kvslot = s_kvslot;
       e.kvrow = s_kvrow;
       e.nrows = s_nrows;
+      e.hpre_tile = -1;
+      if ((ph.kind == kMkO || ph.kind == kMkDown) && it1 > it0 && e.M <= 16) {
+        // h is final for this phase (only this phase's finaliser of a tile writes it): load the
+        // rows of the CTA's last tile now, one thread per feature, into xch (unused by residual
+        // epilogues), so that finalising that tile -- typically the phase's last -- skips a
+        // memory round trip
+        const int tl = static_cast<int>((it1 - 1) / ph.kb);
+        float hv[16];
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj)
+          hv[jj] = jj < e.M ? __ldcg(&p.h[static_cast<size_t>(s_rows[jj]) * p.d + tl * 128 + e.q * 32 + lane]) : 0.f;
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj) xch[jj * 128 + e.q * 32 + lane] = hv[jj];
+        e.hpre_tile = tl;
+        e.gn_pre = e.direct_xn ? e.gnext[tl * 128 + e.q * 32 + lane] : 0.f;
+      }
+      if (ph.kind == kMkQkv) {
+        e.kv_base = p.step->kv_layer[ph.layer];
+        e.kv_cap = static_cast<size_t>(p.step->kv_cap);
+      }
+      if (ph.kind == kMkLm) e.logits = p.step->logits;
       if (ph.kind == kMkQkv) {
         // stage the RoPE factors of the first 16 rows; warm L2 with the context keys and values
         // this CTA's attention items will read (they do not depend on this step)
@@ -1006,6 +1034,27 @@ __global__ void __launch_bounds__(kMkThreads, 1)
               break;
             }
             if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 3);
+            if (e.M <= 8 && cl - cf < 8) {
+              // up to 8 rows and 8 contributors: every partial in one round of loads, then the
+              // same sum in contributor order (an absent contributor adds an exact 0)
+              float pv[8][8];
+#pragma unroll
+              for (int q = 0; q < 8; ++q) {
+                const bool cin = cf + q <= cl;
+                const float* pa = partials + static_cast<size_t>(cf + q + t) * 128 * n_pad;
+#pragma unroll
+                for (int jj = 0; jj < 8; ++jj) pv[q][jj] = cin && jj < e.M ? __ldcg(&pa[jj * 128 + r]) : 0.f;
+              }
+              float v[16];
+#pragma unroll
+              for (int jj = 0; jj < 16; ++jj) v[jj] = 0.f;
+#pragma unroll
+              for (int q = 0; q < 8; ++q)
+#pragma unroll
+                for (int jj = 0; jj < 8; ++jj) v[jj] += pv[q][jj];
+              if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 7);
+              mk_epilogue_chunk(p, ph, e, t, r, 0, v);
+            } else
             for (int ch = 0; ch < n_ch; ++ch) {
               float v[16];
 #pragma unroll
