@@ -25,17 +25,21 @@ def weights():
     return w, oracle_weights(w), to_device_weights(w)
 
 
-PATHS = ["persistent", "multi"]
+PATHS = ["persistent", "hybrid", "multi"]
 
 
 def make_runner(wg, n_slots=4, cap=512, path="persistent", **kw):
-    """path: "persistent" (one cooperative kernel for all layers) or "multi" (kernel per op)."""
+    """path: "persistent" (one cooperative kernel for all layers), "hybrid" (persistent-kernel
+    launches over the GEMM phases with each layer's attention as its own kernel, the long-context
+    plan) or "multi" (kernel per op)."""
     from paper_2609_26100_gb300.runner import TssRunner
-    os.environ["TSS_PATH"] = path
+    os.environ["TSS_PATH"] = "persistent" if path == "hybrid" else path
+    os.environ["TSS_ATTN"] = "external" if path == "hybrid" else "internal"
     try:
         return TssRunner(ARCH, wg, n_slots=n_slots, kv_cap=cap, max_batch=8, **kw)
     finally:
         os.environ.pop("TSS_PATH", None)
+        os.environ.pop("TSS_ATTN", None)
 
 
 def upload_context(run, kv, slot):
@@ -318,6 +322,7 @@ def test_persistent_path_is_deterministic_and_close_to_multi_kernel_path(weights
         outs[path] = r1["logits"].cpu().numpy()
         run.close()
     assert np.abs(outs["persistent"] - outs["multi"]).max() < 2e-2
+    assert np.abs(outs["persistent"] - outs["hybrid"]).max() < 2e-2
 
 
 def test_graph_and_eager_paths_agree_bitwise(weights):
