@@ -122,12 +122,9 @@ struct tss_ctx {
   int gemm_ctas_per_sm = 2;
   // persistent verify kernel
   bool use_mk = true;
-  int l2_ahead = 0;
   int mk_kps = 4;  // weight k-blocks per ring stage of the persistent kernel
   int attn_mode = 0;  // 0 auto, 1 attention inside the persistent kernel, 2 separate attention kernels
-  int l2_pace = 0;       // cycles between paced L2 weight prefetches of 16 KiB (0: unpaced)
   int w_evict_first = 1;
-  int pf_attn = 0, pf_next = 0;
   int mk_max_stages = 12;
   int attn_plo = 1;
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
@@ -452,14 +449,10 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.xs = xs;
   p.attn_plo = c->attn_plo;
   p.attn_extra = static_cast<int>(cfg.attn_extra);
-  p.l2_pace = c->l2_pace;
   p.w_evict_first = c->w_evict_first;
-  p.pf_attn = c->pf_attn;
-  p.pf_next = c->pf_next;
   p.attn_splits = cfg.attn_splits;
   p.B = sp.B;
   p.max_tiles = c->mk_max_tiles;
-  p.l2_ahead = c->l2_ahead;
   p.trace = c->trace;
   p.eps = c->a.rms_eps;
   p.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c->D)));
@@ -901,16 +894,12 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_NO_GRAPH")) c->use_graphs = std::atoi(e) == 0;
   if (const char* e = std::getenv("TSS_GEMM_CTAS_PER_SM")) c->gemm_ctas_per_sm = std::max(1, std::min(2, std::atoi(e)));
   if (const char* e = std::getenv("TSS_PATH")) c->use_mk = std::string(e) != "multi";
-  if (const char* e = std::getenv("TSS_L2_AHEAD")) c->l2_ahead = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_ATTN")) {
     const std::string v(e);
     c->attn_mode = v == "internal" ? 1 : v == "external" ? 2 : 0;
   }
   if (const char* e = std::getenv("TSS_MK_KPS")) c->mk_kps = std::min(8, std::max(1, std::atoi(e)));
-  if (const char* e = std::getenv("TSS_L2_PACE")) c->l2_pace = std::min(100000, std::max(0, std::atoi(e)));
   if (const char* e = std::getenv("TSS_EVICT_FIRST")) c->w_evict_first = std::atoi(e) != 0;
-  if (const char* e = std::getenv("TSS_PF_ATTN")) c->pf_attn = std::max(0, std::atoi(e));
-  if (const char* e = std::getenv("TSS_PF_NEXT")) c->pf_next = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_ATTN_PLO")) c->attn_plo = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
   const char* trace_env = std::getenv("TSS_TRACE");

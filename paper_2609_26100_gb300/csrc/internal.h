@@ -116,16 +116,12 @@ struct MkParams {
   int kps;  // k-blocks (16 KiB of weights each) per pipeline stage
   XsLayout xs;  // B-operand layout (n_pad == xs.rows)
   int attn_plo;         // attention P.V with P split into hi/lo bf16 parts
-  int l2_pace;  // SM clock cycles between L2 prefetches of 16 KiB (0: unpaced)
   int w_evict_first;  // stream weights with the evict-first L2 policy
-  int pf_attn;  // 16 KiB weight blocks of the O phase warmed into L2 while the attention runs
-  int pf_next;  // blocks of the next phase (beyond the ring) warmed into L2 when a phase ends
   int attn_extra;  // shared memory behind the ring that only the attention uses (bytes)
   // Phases [ph_begin, ph_end) run in this launch.  attn_external: the attention of each layer is a
   // separate kernel launched between the launches (long contexts), so none runs in here and an
   // O phase needs no flag from it.
   int ph_begin, ph_end, attn_external;
-  int l2_ahead;  // weight tiles per CTA prefetched into L2 ahead of the smem ring (0: off)
   unsigned long long* trace;  // optional timeline [grid][mk_trace_slots()], nullptr when off
   float eps, scale_log2;
   unsigned long long seq_base;  // epoch * 1024: flag values grow over steps, never reset

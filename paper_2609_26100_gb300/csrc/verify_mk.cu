@@ -196,24 +196,6 @@ __device__ __forceinline__ const __nv_bfloat16* mk_weights(const MkParams& p, co
 }
 
 // CTA c's stream-K range of a phase over geff = min(grid, iterations) CTAs.
-__device__ __forceinline__ void mk_range(const MkPhase& ph, int c, int G, long long& it0, long long& it1, int& geff);
-
-// Warm L2 with blocks [skip, skip + count) of CTA c's range of phase pi: the range is one
-// contiguous run of pre-tiled weight blocks, so this is one bulk prefetch.
-__device__ void mk_prefetch_phase(const MkParams& p, const PlanDev* pl, int pi, int n_phases, int c, int G,
-                                  long long skip, long long count) {
-  if (pi >= n_phases || count <= 0) return;
-  const MkPhase ph = mk_phase(p, pl, pi);
-  long long it0, it1;
-  int geff;
-  mk_range(ph, c, G, it0, it1, geff);
-  const long long a = it0 + skip;
-  const long long b = a + count < it1 ? a + count : it1;
-  if (b <= a) return;
-  bulk_prefetch_l2(mk_weights(p, ph) + static_cast<size_t>(a) * kTileElems, static_cast<uint32_t>(b - a) * kMkWBytes);
-}
-
-// CTA c's stream-K range of a phase over geff = min(grid, iterations) CTAs.
 __device__ __forceinline__ void mk_range(const MkPhase& ph, int c, int G, long long& it0, long long& it1, int& geff) {
   const long long T = static_cast<long long>(ph.n_tiles) * ph.kb;
   geff = static_cast<int>(T < G ? T : G);
@@ -525,7 +507,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   uint64_t* empty = full + S;
   uint64_t* accf = empty + S;
   uint64_t* acce = accf + kMkMaxAcc;
-  int* misc = reinterpret_cast<int*>(acce + kMkMaxAcc);  // [0] tmem addr, [1] abort, [2..4] bcast, [5] s_last, [8] w_pos
+  int* misc = reinterpret_cast<int*>(acce + kMkMaxAcc);  // [0] tmem addr, [1] abort, [2..4] bcast, [5] s_last
   float* xch = reinterpret_cast<float*>(misc + 16);
   float* redv = xch + 16 * 128;
   int* redi = reinterpret_cast<int*>(redv + 64);
@@ -543,7 +525,6 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   const int NB = mk_acc_bufs(n_pad);
   const uint32_t ncols = gemm_tmem_cols(n_pad, NB);
   const PlanDev* pl = p.plan;
-  volatile int* w_pos = misc + 8;  // weight tiles the TMA producer has issued
   volatile int* attn_gate = misc + 9;  // QKV slots whose attention in this CTA is done (ring free)
   const size_t ring_attn_bytes = static_cast<size_t>(s_attn - base) + p.attn_extra;
   MkShared sh;
@@ -561,7 +542,6 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       mbar_init(&acce[i], 128);
     }
     *sh.abort_s = 0;
-    misc[8] = 0;
     misc[9] = 0;
     fence_mbar_init();
   }
@@ -616,11 +596,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
             else
               bulk_load(sW + static_cast<size_t>(s) * sw_bytes,
                         wl + (static_cast<size_t>(t) * ph.kb + kc) * kTileElems, nk * kMkWBytes, &full[s]);
-            *w_pos = static_cast<int>(i + 1);
           }
         }
       }
-      *w_pos = 0x7fffffff;  // the prefetch warp may run to the end
       if (!ok) {  // let weight tiles already in flight land before the CTA can exit
         const uint64_t t0 = globaltimer_ns();
         while (globaltimer_ns() - t0 < 50000) {
@@ -783,52 +761,6 @@ __global__ void __launch_bounds__(kMkThreads, 1)
                     &full[s]);
         }
        }
-      }
-    }
-  } else if (warp == 3) {
-    if (lane == 0 && p.l2_ahead > 0) {
-      // ---------------- L2 prefetch of weight tiles ahead of the ring ----------------
-      // Keeps HBM streaming while the ring waits at a phase boundary for activations: the ring's
-      // TMA loads then hit in L2.  Stays at most l2_ahead tiles ahead of the TMA producer.
-      long long j = 0;
-      bool go = true;
-      long long next_pf = clock64();
-      for (int pi = ph0; go && pi < n_phases; ++pi) {
-        const MkPhase ph = mk_phase(p, pl, pi);
-        long long it0, it1;
-        int geff;
-        mk_range(ph, c, G, it0, it1, geff);
-        const __nv_bfloat16* wl = mk_weights(p, ph);
-        long long it = it0;
-        int t, k0, k1;
-        while (go && mk_next_segment(it, it1, ph.kb, t, k0, k1))
-        for (int kc = k0; go && kc < k1; kc += KPS, ++j) {
-          const int nk = min(KPS, k1 - kc);
-          if (j < static_cast<long long>(*w_pos) + S) continue;  // the ring is about to load it itself
-          if (j >= static_cast<long long>(*w_pos) + p.l2_ahead) {
-            const uint64_t t0 = globaltimer_ns();
-            while (j >= static_cast<long long>(*w_pos) + p.l2_ahead) {
-              if (*sh.abort_s || globaltimer_ns() - t0 > kWaitLimitNs) {
-                go = false;  // the other roles handle a timeout; prefetching is only a hint
-                break;
-              }
-              __nanosleep(128);
-            }
-            if (!go) break;
-          }
-          if (p.l2_pace > 0) {
-            // pace to about this SM's share of HBM bandwidth so that prefetches do not pile up in
-            // the memory queues ahead of the latency-critical loads
-            long long now = clock64();
-            if (now > next_pf) next_pf = now;
-            while (now < next_pf) {
-              __nanosleep(32);
-              now = clock64();
-            }
-            next_pf += static_cast<long long>(p.l2_pace) * nk;
-          }
-          bulk_prefetch_l2(wl + (static_cast<size_t>(t) * ph.kb + kc) * kTileElems, nk * kMkWBytes);
-        }
       }
     }
   } else if (warp >= 4) {
@@ -1101,8 +1033,6 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         ++use;
       }
       if (!ok) break;
-      if (ph.kind != kMkQkv && e.et == 0)
-        mk_prefetch_phase(p, pl, pi + 1, n_phases, c, G, static_cast<long long>(S) * KPS, p.pf_next);
       if (ph.kind == kMkQkv && !p.attn_external) {
         // attention items of this layer: (request, head, split) round-robin over the grid
         ap.slot = ph.slot;
@@ -1110,7 +1040,6 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         const int n_items = p.B * per_req;
         const unsigned long long want = mk_seq(p.seq_base, ph.slot, kMkQkv);
         if (e.et == 0) mk_trace(p, kMkTracePhases * 8 + 2 * ph.slot);
-        if (e.et == 0) mk_prefetch_phase(p, pl, pi + 1, n_phases, c, G, 0, p.pf_attn);
         // The attention borrows the weight/activation ring and its own buffer: this CTA's QKV
         // MMAs have all completed, and the producers start the O phase only after the gate.
         fence_proxy_async_shared();
