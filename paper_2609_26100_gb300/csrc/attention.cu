@@ -34,7 +34,7 @@ static cudaError_t attn_prepare_one() {
                                        cudaSharedmemCarveoutMaxShared);
   if (e != cudaSuccess) return e;
   return cudaFuncSetAttribute(attn_kernel<D, P16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(attn_smem_bytes(D)));
+                              static_cast<int>(attn_smem_bytes(D) + (P16 ? attn_qlo_bytes(D) : 0)));
 }
 
 cudaError_t attn_prepare() {
@@ -49,10 +49,10 @@ cudaError_t launch_attention(const AttnParams& p, int B, cudaStream_t s, bool pd
   const dim3 grid(p.n_splits, p.n_heads, B), block(kAttnThreads);
   const bool p16 = p.o_xs.rows != 0;  // the persistent path's operands and precision
   if (p.head_dim == 64)
-    return p16 ? launch_k(attn_kernel<64, true>, grid, block, attn_smem_bytes(64), s, pdl, p)
+    return p16 ? launch_k(attn_kernel<64, true>, grid, block, attn_smem_bytes(64) + attn_qlo_bytes(64), s, pdl, p)
                : launch_k(attn_kernel<64, false>, grid, block, attn_smem_bytes(64), s, pdl, p);
   if (p.head_dim == 128)
-    return p16 ? launch_k(attn_kernel<128, true>, grid, block, attn_smem_bytes(128), s, pdl, p)
+    return p16 ? launch_k(attn_kernel<128, true>, grid, block, attn_smem_bytes(128) + attn_qlo_bytes(128), s, pdl, p)
                : launch_k(attn_kernel<128, false>, grid, block, attn_smem_bytes(128), s, pdl, p);
   return cudaErrorInvalidValue;
 }

@@ -14,6 +14,10 @@ constexpr int attn_ld() {
   return D + 8;  // padded smem row (bf16 elements): conflict-free ldmatrix
 }
 
+__host__ __device__ inline size_t attn_qlo_bytes(int head_dim) {
+  return static_cast<size_t>(kMaxNodes) * (head_dim + 8) * 2;  // lo parts of q
+}
+
 __host__ __device__ inline size_t attn_smem_bytes_impl(int head_dim) {
   const int ld = head_dim + 8;
   return static_cast<size_t>(kMaxNodes + 4 * kKeyTile) * ld * 2;  // Q + double-buffered K and V
@@ -115,6 +119,7 @@ struct AttnAcc {
   float o[D / 8][4];
   float m0, m1, l0, l1;
   uint32_t qf[D / 16][4];
+  uint32_t qlo[D / 16][4];  // lo parts of q (bf16) when the scores use q = hi + lo
 };
 
 template <int D>
@@ -139,7 +144,8 @@ __device__ __forceinline__ void attn_load_qfrag(const AttnItem<D>& it, const __n
 // from several resident tiles keeps the tensor pipe busier than one block at a time.
 // QK16: q and k in fp16 for the score MMAs (else bf16).  PLO: P.V with P as two bf16 parts,
 // hi = bf16(p) and lo = bf16(p - hi), both multiplied by the bf16 values (else P in bf16).
-template <int D, bool QK16 = false, bool PLO = false>
+// QLO: bf16 scores with q as two bf16 parts (a.qf hi, a.qlo lo), keys as stored.
+template <int D, bool QK16 = false, bool PLO = false, bool QLO = false>
 __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __nv_bfloat16* const (&kp)[4],
                                                  const __nv_bfloat16* const (&vp)[4], const int (&key0)[4], int n,
                                                  float scale_log2, AttnAcc<D>& a) {
@@ -158,6 +164,11 @@ __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __
         if (QK16) {
           mma_f16_16816(s[2 * np], a.qf[ks], kb4);
           mma_f16_16816(s[2 * np + 1], a.qf[ks], kb4 + 2);
+        } else if (QLO) {
+          mma_bf16_16816(s[2 * np], a.qf[ks], kb4);
+          mma_bf16_16816(s[2 * np + 1], a.qf[ks], kb4 + 2);
+          mma_bf16_16816(s[2 * np], a.qlo[ks], kb4);
+          mma_bf16_16816(s[2 * np + 1], a.qlo[ks], kb4 + 2);
         } else {
           mma_bf16_16816(s[2 * np], a.qf[ks], kb4);
           mma_bf16_16816(s[2 * np + 1], a.qf[ks], kb4 + 2);
@@ -251,7 +262,7 @@ __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __
 }
 
 // This warp's keys of one resident 64-key tile (K / V buffers sK, sV).
-template <int D, bool QK16 = false, bool PLO = false>
+template <int D, bool QK16 = false, bool PLO = false, bool QLO = false>
 __device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, const __nv_bfloat16* sK,
                                                const __nv_bfloat16* sV, float scale_log2, AttnAcc<D>& a) {
   constexpr int LD = attn_ld<D>();
@@ -265,7 +276,7 @@ __device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, 
     vp[np] = sV + (kbase + np * 16) * LD;
     key0[np] = tile * kKeyTile + kbase + np * 16;
   }
-  attn_blocks_step<D, QK16, PLO>(it, kp, vp, key0, it.kpw / 16, scale_log2, a);
+  attn_blocks_step<D, QK16, PLO, QLO>(it, kp, vp, key0, it.kpw / 16, scale_log2, a);
 }
 
 // Merge the warps that share a query tile through shared memory (sO: [4][16][D] floats, any
@@ -427,8 +438,10 @@ __device__ __forceinline__ void attn_k_to_f16(__nv_bfloat16* tiles0, int tiles, 
 // named barrier BAR, streaming its key tiles through a double buffer.  smem: attn_smem_bytes(D)
 // bytes, 16-byte aligned.  Returns true on the call that wrote the final output rows of
 // (request, head) (the only split, or the last split to finish, which merges the others in
-// split order).  P16: the persistent path's precision (q in fp16, keys converted to fp16 for the
-// score MMAs, P as hi/lo bf16 parts in P.V); else all bf16.
+// split order).  P16: the persistent path's operands and precision (q arrives in fp16 and is split
+// once into bf16 hi/lo parts for the score MMAs, so the bf16 keys need no conversion; P as hi/lo
+// bf16 parts in P.V; output split hi/lo); else all bf16.  With P16 the kernel needs
+// attn_smem_bytes(D) + attn_qlo_bytes(D) of shared memory.
 template <int D, int BAR, bool P16 = false>
 __device__ bool attention_item(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
                                float (*sM)[16], float (*sL)[16], int* s_last) {
@@ -450,12 +463,32 @@ __device__ bool attention_item(const AttnParams& p, int split, int head, int b, 
     cp_async_commit();
     cp_async_wait<1>();
     named_bar_sync(BAR, kAttnThreads);
-    if (P16) {
-      attn_k_to_f16<D>(sK + buf * kKeyTile * LD, 1, tid);
-      named_bar_sync(BAR, kAttnThreads);
+    if (tile == it.t0) {
+      if (P16) {
+        // q (fp16, 11 bits) = hi + lo exactly, both bf16
+        __nv_bfloat16* sQlo = sV + 2 * kKeyTile * LD;
+        constexpr int C2 = D / 2;
+        for (int idx = tid; idx < 16 * it.mt * C2; idx += kAttnThreads) {
+          const int row = idx / C2, c2 = idx - row * C2;
+          uint32_t* qw = reinterpret_cast<uint32_t*>(sQ + row * LD) + c2;
+          const __half2 hq = *reinterpret_cast<const __half2*>(qw);
+          const float2 f = __half22float2(hq);
+          const uint32_t hi = pack_bf16(f.x, f.y);
+          const float hx = __uint_as_float(hi << 16), hy = __uint_as_float(hi & 0xffff0000u);
+          *qw = hi;
+          reinterpret_cast<uint32_t*>(sQlo + row * LD)[c2] = pack_bf16(f.x - hx, f.y - hy);
+        }
+        named_bar_sync(BAR, kAttnThreads);
+        attn_load_qfrag<D>(it, sQ, a);
+        constexpr int LDq = attn_ld<D>();
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks)
+          ldmatrix_x4(a.qlo[ks], sQlo + (it.wm * 16 + (it.lane & 15)) * LDq + ks * 16 + (it.lane >> 4) * 8);
+      } else {
+        attn_load_qfrag<D>(it, sQ, a);
+      }
     }
-    if (tile == it.t0) attn_load_qfrag<D>(it, sQ, a);
-    attn_tile_step<D, P16, P16>(it, tile, sK + buf * kKeyTile * LD, sV + buf * kKeyTile * LD, p.scale_log2, a);
+    attn_tile_step<D, false, P16, P16>(it, tile, sK + buf * kKeyTile * LD, sV + buf * kKeyTile * LD, p.scale_log2, a);
     named_bar_sync(BAR, kAttnThreads);
   }
   cp_async_wait<0>();
