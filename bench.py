@@ -242,6 +242,24 @@ def cores():
 
 
 # ----------------------------------------------------------------------------------------------
+def max_over_ranks(ms, device):
+    """The job's time for a timed region: the slowest rank's (every rank gets it).  One process per
+    GPU, each timing its own replica; without an initialised process group this is `ms`."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return ms
+    t = torch.tensor([ms], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(rows_per_step, steps, world, max_ms):
+    """Whole-job throughput: every rank verified rows_per_step rows in each of `steps` steps, and
+    the job took the slowest rank's time (weak scaling: per-GPU work fixed)."""
+    return world * rows_per_step * steps / (max_ms / 1e3)
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -365,12 +383,9 @@ def run_tss(args):
     if status != native.TSS_OK:
         raise RuntimeError(f"device status {status} in the timed region")
     accepts.append(res["accept_len"].float().mean().item())
-    if world > 1:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, "cuda")
     ms = total_ms / args.steps
-    value = world * w.n_rows * args.steps / (total_ms / 1e3)
+    value = job_tokens_per_s(w.n_rows, args.steps, world, total_ms)
     print(f"[bench] {w.name}: {ms * 1e3:.1f} us/step, {value:.1f} tokens/s", file=sys.stderr)
 
     # ---------------- e2e: host buffers through the C ABI, one sync per step ----------------
