@@ -346,18 +346,16 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
   stamp(2);
 
   // Last CTA of (request, head) merges the splits in order.
-  __threadfence();
-  named_bar_sync(BAR, kAttnThreads);
+  named_bar_sync(BAR, kAttnThreads);  // every thread's partial stores precede the release below
   if (tid == 0) {
     int* cnt = p.counters + static_cast<size_t>(b) * H + head;
-    const int old = atomicAdd(cnt, 1);
+    const int old = atom_add_acq_rel_gpu(cnt, 1);
     *s_last = old == p.n_splits - 1;
     if (*s_last) atomicExch(cnt, 0);
   }
   named_bar_sync(BAR, kAttnThreads);
   stamp(3);
-  if (!*s_last) return false;
-  __threadfence();
+  if (!*s_last) return false;  // (the counter's acquire, then the barrier: the partials are visible)
   // Merge weights per (row, split) first -- w = 2^(m_s - M) / L with L = sum 2^(m_s - M) l_s, in
   // split order -- into shared memory (sO is free again), then every output element is a
   // weighted sum of the splits' O, several elements' loads in flight per thread.

@@ -82,6 +82,16 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s bound on every spin
 
+// Arrival on a cross-CTA counter with release and acquire semantics at GPU scope.  Issued by one
+// thread after a CTA barrier, its release covers the stores every thread of the CTA made before
+// that barrier, and its acquire (with a barrier after it) orders the CTA's later loads after
+// the other arrivals' stores: the fences around the counter are in the atomic itself.
+__device__ __forceinline__ int atom_add_acq_rel_gpu(int* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
 // ------------------------------------------------------------------------------------------
 // Programmatic dependent launch
 // ------------------------------------------------------------------------------------------

@@ -382,12 +382,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         tc_fence_before();
         mbar_arrive(&acce[buf]);
-        __threadfence();
-        named_bar_sync(1, 128);
+        named_bar_sync(1, 128);  // every thread's partial stores precede the release below
         if (e.et == 0) {
           const int cf = cta_of(static_cast<long long>(t) * p.kb, T, G);
           const int cl = cta_of(static_cast<long long>(t + 1) * p.kb - 1, T, G);
-          const int old = atomicAdd(&p.counters[t], 1);
+          const int old = atom_add_acq_rel_gpu(&p.counters[t], 1);
           const int last = old == cl - cf;
           if (last) atomicExch(&p.counters[t], 0);
           bcast[0] = last;
@@ -395,8 +394,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           bcast[2] = cl;
         }
         named_bar_sync(1, 128);
-        if (bcast[0]) {
-          __threadfence();
+        if (bcast[0]) {  // (the counter's acquire, then the barrier: the other partials are visible)
           const int cf = bcast[1], cl = bcast[2];
           for (int ch = 0; ch < n_ch; ++ch) {
             float v[16];

@@ -725,6 +725,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           const int y = x + lane;
           const bool rdy = y < n_dep && poll(y);
           const uint32_t bal = __ballot_sync(0xffffffffu, rdy);
+          __syncwarp();  // memory ordering: lane 0's copy follows the acquire loads of the others
           for (int l = 0; l < 32; ++l)
             if ((bal >> l) & 1u) ready[(x + l) >> 5] |= 1u << ((x + l) & 31);
           if (!(bal & 1u)) {
@@ -940,13 +941,12 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           }
           tc_fence_before();
           mbar_arrive(&acce[buf]);
-          __threadfence();
-          named_bar_sync(1, 128);
+          named_bar_sync(1, 128);  // every thread's partial stores precede the release below
           if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 1);
           if (e.et == 0) {
             const int f = mk_cta_of(static_cast<long long>(t) * ph.kb, T, geff);
             const int l = mk_cta_of(static_cast<long long>(t + 1) * ph.kb - 1, T, geff);
-            const int old = atomicAdd(&counters[t], 1);
+            const int old = atom_add_acq_rel_gpu(&counters[t], 1);
             const int last = old == l - f;
             if (last) atomicExch(&counters[t], 0);
             bcast[0] = last;
@@ -959,8 +959,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           cl = bcast[2];
           named_bar_sync(1, 128);
           if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 2);
-          if (finalize) {
-            __threadfence();
+          if (finalize) {  // (the counter's acquire, then the barrier: the other partials are visible)
             if (needs_rs && !mk_prepare_rs(p, e, hdep, sh, rs_ready)) {
               ok = false;
               break;
@@ -1024,8 +1023,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
             mk_write_next_xn(p, pl, ph, e, t, r);
           }
           if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 5);
-          __threadfence();
-          named_bar_sync(1, 128);
+          named_bar_sync(1, 128);  // the tile's outputs precede the flag's release
           if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 6);
           if (flag && e.et == 0) st_release_u64(flag, mk_seq(p.seq_base, ph.slot, ph.kind));
         }
@@ -1067,8 +1065,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
             break;
           }
           if (wrote) {
-            __threadfence();
-            named_bar_sync(1, 128);
+            named_bar_sync(1, 128);  // the head's output precedes the flag's release
             if (e.et == 0) st_release_u64(&p.attflag[b * p.H + head], mk_seq(p.seq_base, ph.slot, kMkAtt));
           }
           named_bar_sync(1, 128);
