@@ -95,7 +95,7 @@ struct tss_ctx {
   int* amax_idx = nullptr;
   float *attn_po = nullptr, *attn_pml = nullptr;
   int* attn_cnt = nullptr;
-  int max_splits = 16;
+  int max_splits = kMaxSplits;
   StepDesc* d_step = nullptr;
   StepDesc* h_ring[kRing] = {};
   cudaEvent_t ring_ev[kRing] = {};

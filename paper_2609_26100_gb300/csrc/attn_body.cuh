@@ -138,11 +138,39 @@ __device__ __forceinline__ void attn_load_qfrag(const AttnItem<D>& it, const __n
     ldmatrix_x4(a.qf[ks], sQ + (it.wm * 16 + (it.lane & 15)) * LD + ks * 16 + (it.lane >> 4) * 8);
 }
 
+// q arrives in fp16 (11 significant bits) and is split exactly into two bf16 parts: hi in place
+// of q, lo into sQlo (rows of the warps' query tiles).
+template <int D>
+__device__ __forceinline__ void attn_split_q(const AttnItem<D>& it, __nv_bfloat16* sQ, __nv_bfloat16* sQlo, int tid) {
+  constexpr int LD = attn_ld<D>(), C2 = D / 2;
+  for (int idx = tid; idx < 16 * it.mt * C2; idx += kAttnThreads) {
+    const int row = idx / C2, c2 = idx - row * C2;
+    uint32_t* qw = reinterpret_cast<uint32_t*>(sQ + row * LD) + c2;
+    const __half2 hq = *reinterpret_cast<const __half2*>(qw);
+    const float2 f = __half22float2(hq);
+    const uint32_t hi = pack_bf16(f.x, f.y);
+    const float hx = __uint_as_float(hi << 16), hy = __uint_as_float(hi & 0xffff0000u);
+    *qw = hi;
+    reinterpret_cast<uint32_t*>(sQlo + row * LD)[c2] = pack_bf16(f.x - hx, f.y - hy);
+  }
+}
+
+template <int D>
+__device__ __forceinline__ void attn_load_qfrag_hilo(const AttnItem<D>& it, const __nv_bfloat16* sQ,
+                                                     const __nv_bfloat16* sQlo, AttnAcc<D>& a) {
+  constexpr int LD = attn_ld<D>();
+  attn_load_qfrag<D>(it, sQ, a);
+#pragma unroll
+  for (int ks = 0; ks < D / 16; ++ks)
+    ldmatrix_x4(a.qlo[ks], sQlo + (it.wm * 16 + (it.lane & 15)) * LD + ks * 16 + (it.lane >> 4) * 8);
+}
+
 // One online-softmax update over up to four 16-key blocks of this warp (kp / vp: their first K
 // and V rows in shared memory, key0: the key index of their first row): scores, context /
 // ancestor mask, rescale, P.V.  The blocks' score MMAs are independent, so a group of blocks
 // from several resident tiles keeps the tensor pipe busier than one block at a time.
-// QK16: q and k in fp16 for the score MMAs (else bf16).  PLO: P.V with P as two bf16 parts,
+// QK16: fp16 score MMAs, q in fp16 (a.qf) and each bf16 key fragment converted to fp16 in
+// registers (exact for |k| in [6.1e-5, 65504]).  PLO: P.V with P as two bf16 parts,
 // hi = bf16(p) and lo = bf16(p - hi), both multiplied by the bf16 values (else P in bf16).
 // QLO: bf16 scores with q as two bf16 parts (a.qf hi, a.qlo lo), keys as stored.
 template <int D, bool QK16 = false, bool PLO = false, bool QLO = false>
@@ -162,6 +190,8 @@ __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __
         uint32_t kb4[4];
         ldmatrix_x4(kb4, kp[np] + ((lane & 7) + ((lane >> 4) << 3)) * LD + ks * 16 + ((lane >> 3) & 1) * 8);
         if (QK16) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) kb4[j] = bf16x2_to_f16x2(kb4[j]);
           mma_f16_16816(s[2 * np], a.qf[ks], kb4);
           mma_f16_16816(s[2 * np + 1], a.qf[ks], kb4 + 2);
         } else if (QLO) {
@@ -279,12 +309,49 @@ __device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, 
   attn_blocks_step<D, QK16, PLO, QLO>(it, kp, vp, key0, it.kpw / 16, scale_log2, a);
 }
 
+// Weighted sum over the splits of every output element of a (request, head): each thread takes
+// kU elements per round with the partial outputs of all (<= kS) splits loaded together; the first
+// round's loads are issued before `weights()` (which computes wgt) so that they overlap.
+template <int D, int kU, int kS, typename Weights, typename Put>
+__device__ __forceinline__ void attn_merge_rounds(const AttnParams& p, size_t ph, int N, int ns, int tid,
+                                                  const float* wgt, Weights weights, Put put) {
+  float po[kU][kS];
+  auto load = [&](int idx0) {
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int idx = idx0 + u * kAttnThreads;
+      const int i = idx / D, dd = idx - i * D;
+#pragma unroll
+      for (int sp = 0; sp < kS; ++sp)
+        po[u][sp] = idx < N * D && sp < ns ? __ldcg(&p.part_o[((ph + sp) * kMaxNodes + i) * D + dd]) : 0.f;
+    }
+  };
+  load(tid);
+  weights();
+  for (int idx0 = tid; idx0 < N * D; idx0 += kU * kAttnThreads) {
+    if (idx0 != tid) load(idx0);
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int idx = idx0 + u * kAttnThreads;
+      if (idx >= N * D) continue;
+      const float* w = wgt + (idx / D) * ns;
+      float o = 0.f;
+#pragma unroll
+      for (int sp = 0; sp < kS; ++sp)
+        if (sp < ns) o += w[sp] * po[u][sp];
+      put(idx, o);
+    }
+  }
+}
+
 // Merge the warps that share a query tile through shared memory (sO: [4][16][D] floats, any
 // free 16-byte-aligned buffer of 32 KiB for D = 128), then write this split's result: the
 // normalised output when there is one split, else the partial, and the last split of
 // (request, head) merges all partials in split order.  Returns true on the call that wrote the
 // final output rows.  `stamp(k)` records diagnostics (k = 9, 2, 3, 4 in that order).
-template <int D, int BAR, typename Stamp>
+// kFastMerge: the merge's loads in one round (attn_merge_rounds), used by the persistent
+// kernel; the standalone kernel keeps the plain loop, which measured faster there.
+template <int D, int BAR, bool kFastMerge, typename Stamp>
 __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<D>& it, AttnAcc<D>& a, int split,
                                             int head, int b, int tid, float* sO, float (*sM)[16], float (*sL)[16],
                                             int* s_last, Stamp stamp) {
@@ -356,80 +423,106 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
   named_bar_sync(BAR, kAttnThreads);
   stamp(3);
   if (!*s_last) return false;  // (the counter's acquire, then the barrier: the partials are visible)
-  // Merge weights per (row, split) first -- w = 2^(m_s - M) / L with L = sum 2^(m_s - M) l_s, in
-  // split order -- into shared memory (sO is free again), then every output element is a
-  // weighted sum of the splits' O, several elements' loads in flight per thread.
-  float* wgt = sO;  // [N][n_splits]
-  const int ns = p.n_splits;
-  for (int i = tid; i < N; i += kAttnThreads) {
-    float M = -INFINITY;
-    for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, __ldcg(&p.part_ml[((ph + sp) * kMaxNodes + i) * 2]));
-    const float base = M == -INFINITY ? 0.f : M;
-    float L = 0.f;
-    for (int sp = 0; sp < ns; ++sp) {
+  if (kFastMerge) {
+    // Merge weights per (row, split) -- w = 2^(m_s - M) / L with L = sum 2^(m_s - M) l_s, in split
+    // order -- and the weighted sum of the splits' O for every output element.  The (m, l) pairs go
+    // to shared memory (sO is free again) while the first elements' partial outputs are already in
+    // flight, so that the merge of a small block costs one round of loads.
+    const int ns = p.n_splits;
+    float* wgt = sO;                          // [N][ns]
+    float* sml = sO + kMaxNodes * kMaxSplits;  // [N][ns] x (m, l)
+    for (int x = tid; x < N * ns; x += kAttnThreads) {
+      const int i = x / ns, sp = x - i * ns;
       const size_t pi = (ph + sp) * kMaxNodes + i;
-      const float f = exp2f(__ldcg(&p.part_ml[pi * 2]) - base);
-      L += f * __ldcg(&p.part_ml[pi * 2 + 1]);
-      wgt[i * ns + sp] = f;
+      sml[2 * x] = __ldcg(&p.part_ml[pi * 2]);
+      sml[2 * x + 1] = __ldcg(&p.part_ml[pi * 2 + 1]);
     }
-    if (!(L > 0.f)) report(p.status, kStatusCheck);
-    const float inv = L > 0.f ? 1.f / L : 0.f;
-    for (int sp = 0; sp < ns; ++sp) wgt[i * ns + sp] *= inv;
-  }
-  named_bar_sync(BAR, kAttnThreads);
-  constexpr int kU = 4;  // output elements per thread with their loads in flight together
-  for (int idx0 = tid; idx0 < N * D; idx0 += kU * kAttnThreads) {
-    float O[kU];
-#pragma unroll
-    for (int u = 0; u < kU; ++u) O[u] = 0.f;
-    for (int sp = 0; sp < ns; ++sp) {
-      float po[kU];
-#pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const int idx = idx0 + u * kAttnThreads;
-        const int i = idx / D, dd = idx - i * D;
-        po[u] = idx < N * D ? __ldcg(&p.part_o[((ph + sp) * kMaxNodes + i) * D + dd]) : 0.f;
+    auto weights = [&]() {
+      named_bar_sync(BAR, kAttnThreads);
+      for (int i = tid; i < N; i += kAttnThreads) {
+        float M = -INFINITY;
+        for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, sml[2 * (i * ns + sp)]);
+        const float base = M == -INFINITY ? 0.f : M;
+        float L = 0.f;
+        for (int sp = 0; sp < ns; ++sp) {
+          const float f = exp2f(sml[2 * (i * ns + sp)] - base);
+          L += f * sml[2 * (i * ns + sp) + 1];
+          wgt[i * ns + sp] = f;
+        }
+        if (!(L > 0.f)) report(p.status, kStatusCheck);
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        for (int sp = 0; sp < ns; ++sp) wgt[i * ns + sp] *= inv;
       }
-#pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const int idx = idx0 + u * kAttnThreads;
-        if (idx < N * D) O[u] += wgt[(idx / D) * ns + sp] * po[u];
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      const int idx = idx0 + u * kAttnThreads;
-      if (idx >= N * D) continue;
+      named_bar_sync(BAR, kAttnThreads);
+    };
+    auto put = [&](int idx, float val) {
       const int i = idx / D, dd = idx - i * D;
       if (p.o_xs.rows)
-        store_split(p.o, p.o_xs, crow + i, head * D + dd, O[u]);
+        store_split(p.o, p.o_xs, crow + i, head * D + dd, val);
       else
-        p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(O[u]);
+        p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
+    };
+    if (ns <= 4)
+      attn_merge_rounds<D, 8, 4>(p, ph, N, ns, tid, wgt, weights, put);
+    else if (ns <= 8)
+      attn_merge_rounds<D, 4, 8>(p, ph, N, ns, tid, wgt, weights, put);
+    else
+      attn_merge_rounds<D, 2, 16>(p, ph, N, ns, tid, wgt, weights, put);
+  } else {
+    // Merge weights per (row, split) first -- w = 2^(m_s - M) / L with L = sum 2^(m_s - M) l_s, in
+    // split order -- into shared memory (sO is free again), then every output element is a
+    // weighted sum of the splits' O, several elements' loads in flight per thread.
+    float* wgt = sO;  // [N][n_splits]
+    const int ns = p.n_splits;
+    for (int i = tid; i < N; i += kAttnThreads) {
+      float M = -INFINITY;
+      for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, __ldcg(&p.part_ml[((ph + sp) * kMaxNodes + i) * 2]));
+      const float base = M == -INFINITY ? 0.f : M;
+      float L = 0.f;
+      for (int sp = 0; sp < ns; ++sp) {
+        const size_t pi = (ph + sp) * kMaxNodes + i;
+        const float f = exp2f(__ldcg(&p.part_ml[pi * 2]) - base);
+        L += f * __ldcg(&p.part_ml[pi * 2 + 1]);
+        wgt[i * ns + sp] = f;
+      }
+      if (!(L > 0.f)) report(p.status, kStatusCheck);
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+      for (int sp = 0; sp < ns; ++sp) wgt[i * ns + sp] *= inv;
+    }
+    named_bar_sync(BAR, kAttnThreads);
+    constexpr int kU = 4;  // output elements per thread with their loads in flight together
+    for (int idx0 = tid; idx0 < N * D; idx0 += kU * kAttnThreads) {
+      float O[kU];
+  #pragma unroll
+      for (int u = 0; u < kU; ++u) O[u] = 0.f;
+      for (int sp = 0; sp < ns; ++sp) {
+        float po[kU];
+  #pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          const int idx = idx0 + u * kAttnThreads;
+          const int i = idx / D, dd = idx - i * D;
+          po[u] = idx < N * D ? __ldcg(&p.part_o[((ph + sp) * kMaxNodes + i) * D + dd]) : 0.f;
+        }
+  #pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          const int idx = idx0 + u * kAttnThreads;
+          if (idx < N * D) O[u] += wgt[(idx / D) * ns + sp] * po[u];
+        }
+      }
+  #pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int idx = idx0 + u * kAttnThreads;
+        if (idx >= N * D) continue;
+        const int i = idx / D, dd = idx - i * D;
+        if (p.o_xs.rows)
+          store_split(p.o, p.o_xs, crow + i, head * D + dd, O[u]);
+        else
+          p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(O[u]);
+      }
     }
   }
   stamp(4);
   return true;
-}
-
-// bf16 -> fp16 in place for the K rows of `tiles` resident tiles (each tile: K [kKeyTile][LD],
-// then V); the bf16 cache values are exact in fp16 within its range (|x| < 65504; below 6.1e-5
-// fp16 is subnormal).
-template <int D>
-__device__ __forceinline__ void attn_k_to_f16(__nv_bfloat16* tiles0, int tiles, int tid) {
-  constexpr int LD = attn_ld<D>(), C8 = D / 8;
-  for (int idx = tid; idx < tiles * kKeyTile * C8; idx += kAttnThreads) {
-    const int row = idx / C8, c8 = idx - row * C8;  // row over the tiles' K rows
-    const int tl = row / kKeyTile, kr = row - tl * kKeyTile;
-    uint4* ptr = reinterpret_cast<uint4*>(tiles0 + (tl * 2 * kKeyTile + kr) * LD + c8 * 8);
-    uint4 v = *ptr;
-    uint32_t* w = reinterpret_cast<uint32_t*>(&v);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float lo = __uint_as_float(w[i] << 16), hi = __uint_as_float(w[i] & 0xffff0000u);
-      w[i] = pack_f16(lo, hi);
-    }
-    *ptr = v;
-  }
 }
 
 // One work item (split, head, request) run by 128 threads (tid 0..127) that synchronise with
@@ -463,25 +556,10 @@ __device__ bool attention_item(const AttnParams& p, int split, int head, int b, 
     named_bar_sync(BAR, kAttnThreads);
     if (tile == it.t0) {
       if (P16) {
-        // q (fp16, 11 bits) = hi + lo exactly, both bf16
         __nv_bfloat16* sQlo = sV + 2 * kKeyTile * LD;
-        constexpr int C2 = D / 2;
-        for (int idx = tid; idx < 16 * it.mt * C2; idx += kAttnThreads) {
-          const int row = idx / C2, c2 = idx - row * C2;
-          uint32_t* qw = reinterpret_cast<uint32_t*>(sQ + row * LD) + c2;
-          const __half2 hq = *reinterpret_cast<const __half2*>(qw);
-          const float2 f = __half22float2(hq);
-          const uint32_t hi = pack_bf16(f.x, f.y);
-          const float hx = __uint_as_float(hi << 16), hy = __uint_as_float(hi & 0xffff0000u);
-          *qw = hi;
-          reinterpret_cast<uint32_t*>(sQlo + row * LD)[c2] = pack_bf16(f.x - hx, f.y - hy);
-        }
+        attn_split_q<D>(it, sQ, sQlo, tid);
         named_bar_sync(BAR, kAttnThreads);
-        attn_load_qfrag<D>(it, sQ, a);
-        constexpr int LDq = attn_ld<D>();
-#pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks)
-          ldmatrix_x4(a.qlo[ks], sQlo + (it.wm * 16 + (it.lane & 15)) * LDq + ks * 16 + (it.lane >> 4) * 8);
+        attn_load_qfrag_hilo<D>(it, sQ, sQlo, a);
       } else {
         attn_load_qfrag<D>(it, sQ, a);
       }
@@ -490,7 +568,7 @@ __device__ bool attention_item(const AttnParams& p, int split, int head, int b, 
     named_bar_sync(BAR, kAttnThreads);
   }
   cp_async_wait<0>();
-  return attn_finish<D, BAR>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sK), sM, sL, s_last,
+  return attn_finish<D, BAR, false>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sK), sM, sL, s_last,
                              [](int) {});
 }
 
@@ -504,8 +582,9 @@ __host__ __device__ inline int attn_resident_tiles(int head_dim, size_t smem_byt
 // attn_resident_tiles(D, smem_bytes) tiles when they do not all fit): loads of tiles that hold
 // only context keys (which this step does not write) are issued first, then `wait_inputs()`
 // waits for the step's own Q/K/V rows, then Q and the remaining tiles are loaded.  One memory
-// round trip per round instead of one per tile.  Needs smem_bytes >= the Q buffer + 1 tile and
-// the 32 KiB merge buffer (D = 128) to fit behind Q.  If wait_inputs() fails, drains its copies
+// round trip per round instead of one per tile.  The scores are fp16 MMAs (q arrives in fp16, the
+// keys are converted in registers).  Needs smem_bytes >= the Q buffer + 1 tile and the 32 KiB
+// merge buffer (D = 128) to fit behind Q.  If wait_inputs() fails, drains its copies
 // and returns false without output.
 template <int D, int BAR, typename Wait>
 __device__ bool attention_item_resident(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
@@ -516,7 +595,7 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
     if (trace && tid == 0) trace[k] = globaltimer_ns();
   };
   failed = false;
-  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [kMaxNodes][LD]
+  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [kMaxNodes][LD] (q in fp16)
   __nv_bfloat16* sKV = sQ + kMaxNodes * LD;                      // per tile slot: K [kKeyTile][LD], V [kKeyTile][LD]
   const int R = attn_resident_tiles(D, smem_bytes);
   AttnItem<D> it;
@@ -573,8 +652,6 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
     cp_async_commit();
     cp_async_wait<0>();
     named_bar_sync(BAR, kAttnThreads);
-    attn_k_to_f16<D>(sKV, nt, tid);  // the score MMAs run in fp16 (q is written in fp16)
-    named_bar_sync(BAR, kAttnThreads);
     stamp(0);
     attn_load_qfrag<D>(it, sQ, a);
     score_round(it.t0, it.t1, 0);
@@ -611,8 +688,6 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
         cp_async_wait<0>();
       }
       named_bar_sync(BAR, kAttnThreads);
-      attn_k_to_f16<D>(tile_k(slot0), r1 - r0, tid);
-      named_bar_sync(BAR, kAttnThreads);
       if (r == 0) {
         stamp(0);
         attn_load_qfrag<D>(it, sQ, a);
@@ -623,7 +698,7 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
   }
   stamp(1);
   if (trace && it.lane == 0) trace[5 + it.warp] = globaltimer_ns();
-  return attn_finish<D, BAR>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sKV), sM, sL, s_last, stamp);
+  return attn_finish<D, BAR, true>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sKV), sM, sL, s_last, stamp);
 }
 
 }  // namespace tss

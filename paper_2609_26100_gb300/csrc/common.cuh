@@ -20,6 +20,7 @@ constexpr int kMaxLayers = 64;
 constexpr int kMaxBatch = 64;
 constexpr int kMaxRows = 256;
 constexpr int kMaxNodes = 64;
+constexpr int kMaxSplits = 16;  // key splits of one (request, head) in the attention
 constexpr int kFinalSlot = kMaxLayers;  // plan slot of the final norm + LM head (all rows)
 constexpr int kPathStride = kMaxNodes;  // internal copy of each request's accepted path
 
@@ -341,9 +342,13 @@ __device__ __forceinline__ void mma_f16_16816(float* d, const uint32_t* a, const
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
-__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
-  __half2 v = __floats2half2_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
+
+// Two bf16 values (low half first) to two fp16 values, round to nearest.
+__device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t v) {
+  const float lo = __uint_as_float(v << 16), hi = __uint_as_float(v & 0xffff0000u);
+  uint32_t r;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
 }
 
 __device__ __forceinline__ void ldmatrix_x4(uint32_t* r, const void* p) {

@@ -343,7 +343,7 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
       const int j = j0 + jj;
       if (j >= e.M) continue;
       if (sec == 0) {
-        // q in fp16 (11 significant bits): the attention of this kernel runs its MMAs in fp16
+        // q in fp16 (11 significant bits), split exactly into bf16 hi + lo by the attention
         reinterpret_cast<__half*>(p.qbuf)[static_cast<size_t>(j) * d + f] = __float2half_rn(val[jj]);
       } else {
         const size_t off = ((static_cast<size_t>(e.kvslot[j]) * 2 + (sec - 1)) * p.H + head) *
