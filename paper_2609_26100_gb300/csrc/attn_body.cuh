@@ -381,32 +381,45 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
   stamp(9);
 
   const size_t ph = (static_cast<size_t>(b) * H + head) * p.n_splits;
-  for (int idx = tid; idx < N * D; idx += kAttnThreads) {
-    const int i = idx / D, dd = idx - i * D;
+  // Per query row (one thread each): the warps' common max M, their weights 2^(m_w - M) (written
+  // over sM) and the merged sum L (over sL of the row's first warp); then every output element
+  // is a plain weighted sum of the warps' O, the loads of several elements in flight.
+  for (int i = tid; i < N; i += kAttnThreads) {
     const int wt = i >> 4, rr = i & 15;
     float M = -INFINITY;
     for (int w = wt; w < 4; w += mt) M = fmaxf(M, sM[w][rr]);
     const float base = M == -INFINITY ? 0.f : M;
-    float L = 0.f, O = 0.f;
+    float L = 0.f;
     for (int w = wt; w < 4; w += mt) {
       const float f = exp2f(sM[w][rr] - base);
       L += f * sL[w][rr];
-      O += f * sO[(w * 16 + rr) * D + dd];
+      sM[w][rr] = f;
     }
+    sL[wt][rr] = L;
     if (p.n_splits == 1) {
       if (!(L > 0.f)) report(p.status, kStatusCheck);
+    } else {
+      const size_t pi = (ph + split) * kMaxNodes + i;
+      __stcg(&p.part_ml[pi * 2 + 0], M);
+      __stcg(&p.part_ml[pi * 2 + 1], L);
+    }
+  }
+  named_bar_sync(BAR, kAttnThreads);
+#pragma unroll 4
+  for (int idx = tid; idx < N * D; idx += kAttnThreads) {
+    const int i = idx / D, dd = idx - i * D;
+    const int wt = i >> 4, rr = i & 15;
+    float O = 0.f;
+    for (int w = wt; w < 4; w += mt) O += sM[w][rr] * sO[(w * 16 + rr) * D + dd];
+    if (p.n_splits == 1) {
+      const float L = sL[wt][rr];
       const float val = L > 0.f ? O / L : 0.f;
       if (p.o_xs.rows)
         store_split(p.o, p.o_xs, crow + i, head * D + dd, val);
       else
         p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
     } else {
-      const size_t pi = (ph + split) * kMaxNodes + i;
-      __stcg(&p.part_o[pi * D + dd], O);
-      if (dd == 0) {
-        __stcg(&p.part_ml[pi * 2 + 0], M);
-        __stcg(&p.part_ml[pi * 2 + 1], L);
-      }
+      __stcg(&p.part_o[((ph + split) * kMaxNodes + i) * D + dd], O);
     }
   }
   if (p.n_splits == 1) return true;
