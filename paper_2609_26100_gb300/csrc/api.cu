@@ -403,7 +403,9 @@ bool mk_config(const tss_ctx* c, const StepPlan& sp, MkConfig* out) {
       const size_t base = mk_smem_bytes(xs.rows, xs.parts, S, c->D, kps, 0);
       if (base > kLimit) continue;
       const size_t avail = kLimit - base;
-      const size_t need_min = ring >= q + tile ? 0 : q + tile - ring;
+      // at least Q + one tile, and Q + the warps' merge buffer (8 warps x 16 rows x D floats)
+      const size_t first = q + std::max(tile, static_cast<size_t>(8) * 16 * c->D * 4);
+      const size_t need_min = ring >= first ? 0 : first - ring;
       if (need_min > avail) continue;
       const size_t want = q + per * tile > ring ? q + per * tile - ring : 0;
       size_t extra = std::max(need_min, std::min(want, avail));

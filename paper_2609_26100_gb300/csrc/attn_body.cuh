@@ -39,12 +39,13 @@ template <int D>
 struct AttnItem {
   const __nv_bfloat16* Kg;  // this (request, head)'s keys / values in the cache: [cap][D]
   const __nv_bfloat16* Vg;
-  int crow, N, ctx, T, t0, t1, mt, wm, wk, kpw, g, tq, warp, lane;
+  int crow, N, ctx, T, t0, t1, mt, wm, wk, ksplit, kpw, g, tq, warp, lane;
   unsigned long long anc0, anc1;
 };
 
-// Fills `it`; false when the request does not run this layer or the item is out of range.
-template <int D>
+// Fills `it` for thread `tid` of a team of NT threads; false when the request does not run this
+// layer or the item is out of range.
+template <int D, int NT = kAttnThreads>
 __device__ __forceinline__ bool attn_item_setup(const AttnParams& p, int split, int head, int b, int tid,
                                                 AttnItem<D>& it) {
   const StepDesc* st = p.step;
@@ -68,10 +69,10 @@ __device__ __forceinline__ bool attn_item_setup(const AttnParams& p, int split, 
   it.warp = tid >> 5;
   it.lane = tid & 31;
   it.mt = it.N <= 16 ? 1 : (it.N <= 32 ? 2 : 4);  // 16-row query tiles
-  const int ksplit = 4 / it.mt;                    // warps sharing one query tile
+  it.ksplit = NT / 32 / it.mt;  // warps sharing one query tile
   it.wm = it.warp % it.mt;
   it.wk = it.warp / it.mt;
-  it.kpw = kKeyTile / ksplit;  // keys of each tile this warp scores
+  it.kpw = kKeyTile / it.ksplit;  // keys of each tile this warp scores (tile-sliced variant)
   it.g = it.lane >> 2;
   it.tq = it.lane & 3;
   const int qr0 = it.wm * 16 + it.g, qr1 = qr0 + 8;
@@ -81,11 +82,11 @@ __device__ __forceinline__ bool attn_item_setup(const AttnParams& p, int split, 
 }
 
 // Q rows of the request into sQ [16 * mt][LD] (rows >= N are zero); cp.async, not committed.
-template <int D>
+template <int D, int NT = kAttnThreads>
 __device__ __forceinline__ void attn_load_q(const AttnParams& p, const AttnItem<D>& it, int head, int tid,
                                             __nv_bfloat16* sQ) {
   constexpr int LD = attn_ld<D>(), C8 = D / 8;
-  for (int idx = tid; idx < 16 * it.mt * C8; idx += kAttnThreads) {
+  for (int idx = tid; idx < 16 * it.mt * C8; idx += NT) {
     const int row = idx / C8, c8 = idx - row * C8;
     __nv_bfloat16* dst = sQ + row * LD + c8 * 8;
     if (row < it.N) {
@@ -98,11 +99,11 @@ __device__ __forceinline__ void attn_load_q(const AttnParams& p, const AttnItem<
 
 // Keys and values of one 64-key tile into sK / sV [kKeyTile][LD]; keys past the block are
 // zero-filled.  cp.async, not committed.
-template <int D>
+template <int D, int NT = kAttnThreads>
 __device__ __forceinline__ void attn_load_tile(const AttnItem<D>& it, int tile, int tid, __nv_bfloat16* sK,
                                                __nv_bfloat16* sV) {
   constexpr int LD = attn_ld<D>(), C8 = D / 8;
-  for (int idx = tid; idx < kKeyTile * C8; idx += kAttnThreads) {
+  for (int idx = tid; idx < kKeyTile * C8; idx += NT) {
     const int kr = idx / C8, c8 = idx - kr * C8;
     const int key = tile * kKeyTile + kr;
     const int bytes = key < it.T ? 16 : 0;
@@ -312,14 +313,14 @@ __device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, 
 // Weighted sum over the splits of every output element of a (request, head): each thread takes
 // kU elements per round with the partial outputs of all (<= kS) splits loaded together; the first
 // round's loads are issued before `weights()` (which computes wgt) so that they overlap.
-template <int D, int kU, int kS, typename Weights, typename Put>
+template <int D, int NT, int kU, int kS, typename Weights, typename Put>
 __device__ __forceinline__ void attn_merge_rounds(const AttnParams& p, size_t ph, int N, int ns, int tid,
                                                   const float* wgt, Weights weights, Put put) {
   float po[kU][kS];
   auto load = [&](int idx0) {
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
-      const int idx = idx0 + u * kAttnThreads;
+      const int idx = idx0 + u * NT;
       const int i = idx / D, dd = idx - i * D;
 #pragma unroll
       for (int sp = 0; sp < kS; ++sp)
@@ -328,11 +329,11 @@ __device__ __forceinline__ void attn_merge_rounds(const AttnParams& p, size_t ph
   };
   load(tid);
   weights();
-  for (int idx0 = tid; idx0 < N * D; idx0 += kU * kAttnThreads) {
+  for (int idx0 = tid; idx0 < N * D; idx0 += kU * NT) {
     if (idx0 != tid) load(idx0);
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
-      const int idx = idx0 + u * kAttnThreads;
+      const int idx = idx0 + u * NT;
       if (idx >= N * D) continue;
       const float* w = wgt + (idx / D) * ns;
       float o = 0.f;
@@ -344,25 +345,26 @@ __device__ __forceinline__ void attn_merge_rounds(const AttnParams& p, size_t ph
   }
 }
 
-// Merge the warps that share a query tile through shared memory (sO: [4][16][D] floats, any
-// free 16-byte-aligned buffer of 32 KiB for D = 128), then write this split's result: the
+// Merge the warps that share a query tile through shared memory (sO: [NT / 32][16][D] floats, any
+// free 16-byte-aligned buffer of NT / 4 KiB for D = 128; sM, sL: [NT / 32][16]), then write this split's result: the
 // normalised output when there is one split, else the partial, and the last split of
 // (request, head) merges all partials in split order.  Returns true on the call that wrote the
 // final output rows.  `stamp(k)` records diagnostics (k = 9, 2, 3, 4 in that order).
 // kFastMerge: the merge's loads in one round (attn_merge_rounds), used by the persistent
 // kernel; the standalone kernel keeps the plain loop, which measured faster there.
-template <int D, int BAR, bool kFastMerge, typename Stamp>
+template <int D, int BAR, int NT, bool kFastMerge, typename Stamp>
 __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<D>& it, AttnAcc<D>& a, int split,
                                             int head, int b, int tid, float* sO, float (*sM)[16], float (*sL)[16],
                                             int* s_last, Stamp stamp) {
   const int H = p.n_heads, d = p.d_model;
+  constexpr int NW = NT / 32;
   const int N = it.N, crow = it.crow, mt = it.mt, warp = it.warp, g = it.g, tq = it.tq;
   a.l0 += __shfl_xor_sync(0xffffffffu, a.l0, 1);
   a.l0 += __shfl_xor_sync(0xffffffffu, a.l0, 2);
   a.l1 += __shfl_xor_sync(0xffffffffu, a.l1, 1);
   a.l1 += __shfl_xor_sync(0xffffffffu, a.l1, 2);
 
-  named_bar_sync(BAR, kAttnThreads);
+  named_bar_sync(BAR, NT);
 #pragma unroll
   for (int dt = 0; dt < D / 8; ++dt) {
     const int col = dt * 8 + tq * 2;
@@ -377,20 +379,20 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
     sL[warp][g] = a.l0;
     sL[warp][g + 8] = a.l1;
   }
-  named_bar_sync(BAR, kAttnThreads);
+  named_bar_sync(BAR, NT);
   stamp(9);
 
   const size_t ph = (static_cast<size_t>(b) * H + head) * p.n_splits;
   // Per query row (one thread each): the warps' common max M, their weights 2^(m_w - M) (written
   // over sM) and the merged sum L (over sL of the row's first warp); then every output element
   // is a plain weighted sum of the warps' O, the loads of several elements in flight.
-  for (int i = tid; i < N; i += kAttnThreads) {
+  for (int i = tid; i < N; i += NT) {
     const int wt = i >> 4, rr = i & 15;
     float M = -INFINITY;
-    for (int w = wt; w < 4; w += mt) M = fmaxf(M, sM[w][rr]);
+    for (int w = wt; w < NW; w += mt) M = fmaxf(M, sM[w][rr]);
     const float base = M == -INFINITY ? 0.f : M;
     float L = 0.f;
-    for (int w = wt; w < 4; w += mt) {
+    for (int w = wt; w < NW; w += mt) {
       const float f = exp2f(sM[w][rr] - base);
       L += f * sL[w][rr];
       sM[w][rr] = f;
@@ -404,13 +406,13 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
       __stcg(&p.part_ml[pi * 2 + 1], L);
     }
   }
-  named_bar_sync(BAR, kAttnThreads);
+  named_bar_sync(BAR, NT);
 #pragma unroll 4
-  for (int idx = tid; idx < N * D; idx += kAttnThreads) {
+  for (int idx = tid; idx < N * D; idx += NT) {
     const int i = idx / D, dd = idx - i * D;
     const int wt = i >> 4, rr = i & 15;
     float O = 0.f;
-    for (int w = wt; w < 4; w += mt) O += sM[w][rr] * sO[(w * 16 + rr) * D + dd];
+    for (int w = wt; w < NW; w += mt) O += sM[w][rr] * sO[(w * 16 + rr) * D + dd];
     if (p.n_splits == 1) {
       const float L = sL[wt][rr];
       const float val = L > 0.f ? O / L : 0.f;
@@ -426,14 +428,14 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
   stamp(2);
 
   // Last CTA of (request, head) merges the splits in order.
-  named_bar_sync(BAR, kAttnThreads);  // every thread's partial stores precede the release below
+  named_bar_sync(BAR, NT);  // every thread's partial stores precede the release below
   if (tid == 0) {
     int* cnt = p.counters + static_cast<size_t>(b) * H + head;
     const int old = atom_add_acq_rel_gpu(cnt, 1);
     *s_last = old == p.n_splits - 1;
     if (*s_last) atomicExch(cnt, 0);
   }
-  named_bar_sync(BAR, kAttnThreads);
+  named_bar_sync(BAR, NT);
   stamp(3);
   if (!*s_last) return false;  // (the counter's acquire, then the barrier: the partials are visible)
   if (kFastMerge) {
@@ -444,15 +446,15 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
     const int ns = p.n_splits;
     float* wgt = sO;                          // [N][ns]
     float* sml = sO + kMaxNodes * kMaxSplits;  // [N][ns] x (m, l)
-    for (int x = tid; x < N * ns; x += kAttnThreads) {
+    for (int x = tid; x < N * ns; x += NT) {
       const int i = x / ns, sp = x - i * ns;
       const size_t pi = (ph + sp) * kMaxNodes + i;
       sml[2 * x] = __ldcg(&p.part_ml[pi * 2]);
       sml[2 * x + 1] = __ldcg(&p.part_ml[pi * 2 + 1]);
     }
     auto weights = [&]() {
-      named_bar_sync(BAR, kAttnThreads);
-      for (int i = tid; i < N; i += kAttnThreads) {
+      named_bar_sync(BAR, NT);
+      for (int i = tid; i < N; i += NT) {
         float M = -INFINITY;
         for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, sml[2 * (i * ns + sp)]);
         const float base = M == -INFINITY ? 0.f : M;
@@ -466,7 +468,7 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
         const float inv = L > 0.f ? 1.f / L : 0.f;
         for (int sp = 0; sp < ns; ++sp) wgt[i * ns + sp] *= inv;
       }
-      named_bar_sync(BAR, kAttnThreads);
+      named_bar_sync(BAR, NT);
     };
     auto put = [&](int idx, float val) {
       const int i = idx / D, dd = idx - i * D;
@@ -476,18 +478,18 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
         p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
     };
     if (ns <= 4)
-      attn_merge_rounds<D, 8, 4>(p, ph, N, ns, tid, wgt, weights, put);
+      attn_merge_rounds<D, NT, 8, 4>(p, ph, N, ns, tid, wgt, weights, put);
     else if (ns <= 8)
-      attn_merge_rounds<D, 4, 8>(p, ph, N, ns, tid, wgt, weights, put);
+      attn_merge_rounds<D, NT, 4, 8>(p, ph, N, ns, tid, wgt, weights, put);
     else
-      attn_merge_rounds<D, 2, 16>(p, ph, N, ns, tid, wgt, weights, put);
+      attn_merge_rounds<D, NT, 2, 16>(p, ph, N, ns, tid, wgt, weights, put);
   } else {
     // Merge weights per (row, split) first -- w = 2^(m_s - M) / L with L = sum 2^(m_s - M) l_s, in
     // split order -- into shared memory (sO is free again), then every output element is a
     // weighted sum of the splits' O, several elements' loads in flight per thread.
     float* wgt = sO;  // [N][n_splits]
     const int ns = p.n_splits;
-    for (int i = tid; i < N; i += kAttnThreads) {
+    for (int i = tid; i < N; i += NT) {
       float M = -INFINITY;
       for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, __ldcg(&p.part_ml[((ph + sp) * kMaxNodes + i) * 2]));
       const float base = M == -INFINITY ? 0.f : M;
@@ -502,9 +504,9 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
       const float inv = L > 0.f ? 1.f / L : 0.f;
       for (int sp = 0; sp < ns; ++sp) wgt[i * ns + sp] *= inv;
     }
-    named_bar_sync(BAR, kAttnThreads);
+    named_bar_sync(BAR, NT);
     constexpr int kU = 4;  // output elements per thread with their loads in flight together
-    for (int idx0 = tid; idx0 < N * D; idx0 += kU * kAttnThreads) {
+    for (int idx0 = tid; idx0 < N * D; idx0 += kU * NT) {
       float O[kU];
   #pragma unroll
       for (int u = 0; u < kU; ++u) O[u] = 0.f;
@@ -512,19 +514,19 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
         float po[kU];
   #pragma unroll
         for (int u = 0; u < kU; ++u) {
-          const int idx = idx0 + u * kAttnThreads;
+          const int idx = idx0 + u * NT;
           const int i = idx / D, dd = idx - i * D;
           po[u] = idx < N * D ? __ldcg(&p.part_o[((ph + sp) * kMaxNodes + i) * D + dd]) : 0.f;
         }
   #pragma unroll
         for (int u = 0; u < kU; ++u) {
-          const int idx = idx0 + u * kAttnThreads;
+          const int idx = idx0 + u * NT;
           if (idx < N * D) O[u] += wgt[(idx / D) * ns + sp] * po[u];
         }
       }
   #pragma unroll
       for (int u = 0; u < kU; ++u) {
-        const int idx = idx0 + u * kAttnThreads;
+        const int idx = idx0 + u * NT;
         if (idx >= N * D) continue;
         const int i = idx / D, dd = idx - i * D;
         if (p.o_xs.rows)
@@ -581,7 +583,7 @@ __device__ bool attention_item(const AttnParams& p, int split, int head, int b, 
     named_bar_sync(BAR, kAttnThreads);
   }
   cp_async_wait<0>();
-  return attn_finish<D, BAR, false>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sK), sM, sL, s_last,
+  return attn_finish<D, BAR, kAttnThreads, false>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sK), sM, sL, s_last,
                              [](int) {});
 }
 
@@ -596,10 +598,11 @@ __host__ __device__ inline int attn_resident_tiles(int head_dim, size_t smem_byt
 // only context keys (which this step does not write) are issued first, then `wait_inputs()`
 // waits for the step's own Q/K/V rows, then Q and the remaining tiles are loaded.  One memory
 // round trip per round instead of one per tile.  The scores are fp16 MMAs (q arrives in fp16, the
-// keys are converted in registers).  Needs smem_bytes >= the Q buffer + 1 tile and the 32 KiB
-// merge buffer (D = 128) to fit behind Q.  If wait_inputs() fails, drains its copies
-// and returns false without output.
-template <int D, int BAR, typename Wait>
+// keys are converted in registers).  Run by a team of NT threads (tid < NT); each warp scores
+// every (NT / 32 / query tiles)-th 16-key block of a round.  Needs smem_bytes >= the Q buffer +
+// 1 tile and the NT / 4 KiB merge buffer (D = 128) to fit behind Q.  If wait_inputs() fails,
+// drains its copies and returns false without output.
+template <int D, int BAR, int NT, typename Wait>
 __device__ bool attention_item_resident(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
                                         size_t smem_bytes, float (*sM)[16], float (*sL)[16], int* s_last,
                                         unsigned long long* trace, Wait wait_inputs, bool& failed, bool plo = true) {
@@ -612,7 +615,7 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
   __nv_bfloat16* sKV = sQ + kMaxNodes * LD;                      // per tile slot: K [kKeyTile][LD], V [kKeyTile][LD]
   const int R = attn_resident_tiles(D, smem_bytes);
   AttnItem<D> it;
-  const bool run = attn_item_setup<D>(p, split, head, b, tid, it);
+  const bool run = attn_item_setup<D, NT>(p, split, head, b, tid, it);
   if (!run || R < 1) {
     failed = !wait_inputs();
     return false;
@@ -622,25 +625,27 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
   auto load_round = [&](int r0, int r1, int slot0, bool ctx_only) {
     for (int tile = r0; tile < r1; ++tile)
       if (!ctx_only || (tile + 1) * kKeyTile <= it.ctx)
-        attn_load_tile<D>(it, tile, tid, tile_k(slot0 + tile - r0), tile_v(slot0 + tile - r0));
+        attn_load_tile<D, NT>(it, tile, tid, tile_k(slot0 + tile - r0), tile_v(slot0 + tile - r0));
   };
   AttnAcc<D> a;
   attn_acc_init<D>(a);
-  // this warp's 16-key blocks of tiles [r0, r1) held from slot0 on, four per softmax update
+  // this warp's 16-key blocks of tiles [r0, r1) held from slot0 on -- every ksplit-th block of
+  // the round, starting at wk -- four per softmax update
   auto score_round = [&](int r0, int r1, int slot0) {
-    const int npairs = it.kpw / 16, kbase = it.wk * it.kpw;
-    const int nb = (r1 - r0) * npairs;
+    constexpr int kBlocks = kKeyTile / 16;  // 16-key blocks per tile
+    const int nall = (r1 - r0) * kBlocks;
+    const int nb = nall > it.wk ? (nall - it.wk + it.ksplit - 1) / it.ksplit : 0;
     for (int q0 = 0; q0 < nb; q0 += 4) {
       const __nv_bfloat16* kp[4];
       const __nv_bfloat16* vp[4];
       int key0[4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const int q = min(q0 + j, nb - 1);
-        const int tl = q / npairs, np = q - tl * npairs;
-        kp[j] = tile_k(slot0 + tl) + (kbase + np * 16) * LD;
-        vp[j] = tile_v(slot0 + tl) + (kbase + np * 16) * LD;
-        key0[j] = (r0 + tl) * kKeyTile + kbase + np * 16;
+        const int gb = it.wk + min(q0 + j, nb - 1) * it.ksplit;
+        const int tl = gb / kBlocks, np = gb - tl * kBlocks;
+        kp[j] = tile_k(slot0 + tl) + np * 16 * LD;
+        vp[j] = tile_v(slot0 + tl) + np * 16 * LD;
+        key0[j] = (r0 + tl) * kKeyTile + np * 16;
       }
       if (plo)
         attn_blocks_step<D, true, true>(it, kp, vp, key0, min(4, nb - q0), p.scale_log2, a);
@@ -659,16 +664,16 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
       failed = true;
       return false;
     }
-    attn_load_q<D>(p, it, head, tid, sQ);
+    attn_load_q<D, NT>(p, it, head, tid, sQ);
     for (int tile = it.t0; tile < it.t1; ++tile)
-      if ((tile + 1) * kKeyTile > it.ctx) attn_load_tile<D>(it, tile, tid, tile_k(tile - it.t0), tile_v(tile - it.t0));
+      if ((tile + 1) * kKeyTile > it.ctx) attn_load_tile<D, NT>(it, tile, tid, tile_k(tile - it.t0), tile_v(tile - it.t0));
     cp_async_commit();
     cp_async_wait<0>();
-    named_bar_sync(BAR, kAttnThreads);
+    named_bar_sync(BAR, NT);
     stamp(0);
     attn_load_qfrag<D>(it, sQ, a);
     score_round(it.t0, it.t1, 0);
-    named_bar_sync(BAR, kAttnThreads);
+    named_bar_sync(BAR, NT);
   } else {
     // Rounds of H tiles through two halves of the resident space: the next round's copies are in
     // flight while this round is scored.  Round 0 holds only context tiles (the block's own keys
@@ -683,7 +688,7 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
       failed = true;
       return false;
     }
-    attn_load_q<D>(p, it, head, tid, sQ);
+    attn_load_q<D, NT>(p, it, head, tid, sQ);
     cp_async_commit();
     for (int r = 0; r < nr; ++r) {
       const int r0 = it.t0 + r * H, r1 = min(it.t1, r0 + H);
@@ -700,18 +705,18 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
       } else {
         cp_async_wait<0>();
       }
-      named_bar_sync(BAR, kAttnThreads);
+      named_bar_sync(BAR, NT);
       if (r == 0) {
         stamp(0);
         attn_load_qfrag<D>(it, sQ, a);
       }
       score_round(r0, r1, slot0);
-      named_bar_sync(BAR, kAttnThreads);  // this half is reloaded by the round after next
+      named_bar_sync(BAR, NT);  // this half is reloaded by the round after next
     }
   }
   stamp(1);
-  if (trace && it.lane == 0) trace[5 + it.warp] = globaltimer_ns();
-  return attn_finish<D, BAR, true>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sKV), sM, sL, s_last, stamp);
+  if (trace && it.lane == 0 && it.warp < 4) trace[5 + it.warp] = globaltimer_ns();
+  return attn_finish<D, BAR, NT, true>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sKV), sM, sL, s_last, stamp);
 }
 
 }  // namespace tss

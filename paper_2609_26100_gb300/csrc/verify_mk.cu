@@ -115,23 +115,6 @@ __device__ bool mk_wait_flag(const unsigned long long* f, unsigned long long tar
   }
 }
 
-// Bounded wait until this CTA's attention of QKV slot `slot` has released the ring.
-__device__ bool mk_wait_gate(const volatile int* gate, int slot, const MkShared& sh) {
-  if (*gate > slot) return true;
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t i = 1;; ++i) {
-    if (*gate > slot) return true;
-    if ((i & 255) == 0) {
-      if (mk_aborted(sh)) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
-        mk_fail(sh);
-        return false;
-      }
-    }
-    __nanosleep(32);
-  }
-}
-
 // Bounded mbarrier wait that also leaves when another CTA aborted.
 __device__ bool mk_wait_bar(uint64_t* bar, uint32_t parity, const MkShared& sh) {
   if (mbar_try_wait(bar, parity)) return true;
@@ -146,6 +129,15 @@ __device__ bool mk_wait_bar(uint64_t* bar, uint32_t parity, const MkShared& sh) 
       }
     }
   }
+}
+
+// Every thread of the CTA arrives on `bar` and waits (bounded) for all to arrive; n counts this
+// thread's syncs on it (phase parity).
+__device__ __forceinline__ bool mk_team_sync(uint64_t* bar, uint32_t& n, const MkShared& sh) {
+  mbar_arrive(bar);
+  const bool ok = mk_wait_bar(bar, n & 1u, sh);
+  ++n;
+  return ok;
 }
 
 struct MkPhase {
@@ -491,6 +483,59 @@ __device__ __forceinline__ unsigned long long* mk_tile_flag(const MkParams& p, i
   }
 }
 
+// The attention of QKV slot `slot` in this CTA: its (request, head, split) items round-robin over
+// the grid, each run by all 256 threads of the CTA (team thread ttid; the epilogue warps are
+// 0..127) in the weight / activation ring, which every role has stopped using when it enters:
+// the epilogue warps after the slot's QKV epilogues, the other warps before their O phase.
+// Returns false after a failed wait (the kernel is aborting).
+template <int D>
+__device__ __forceinline__ bool mk_team_attention(const MkParams& p, const AttnParams& ap0, int slot, int ttid,
+                                               uint8_t* ring, size_t ring_bytes, float (*sM)[16], float (*sL)[16],
+                                               int* s_last, uint64_t* team, uint32_t& team_n, const MkShared& sh) {
+  if (!mk_team_sync(team, team_n, sh)) return false;
+  const PlanDev* pl = p.plan;
+  AttnParams ap = ap0;
+  ap.slot = slot;
+  const int c = blockIdx.x, G = gridDim.x;
+  const int per_req = p.H * p.attn_splits, n_items = p.B * per_req;
+  const unsigned long long want = mk_seq(p.seq_base, slot, kMkQkv);
+  if (ttid == 0) mk_trace(p, kMkTracePhases * 8 + 2 * slot);
+  fence_proxy_async_shared();  // the ring's async-proxy (TMA / MMA) use ends before generic use
+  bool ok = true;
+  for (int item = c; ok && item < n_items; item += G) {
+    const int b = item / per_req;
+    const int head = (item - b * per_req) / p.attn_splits;
+    const int split = item - b * per_req - head * p.attn_splits;
+    if (pl->slot_crow[slot][b] < 0) continue;
+    // the Q, K and V tiles of this head (written by the QKV epilogues of this step)
+    auto wait_inputs = [&]() -> bool {
+      bool good = true;
+      if (ttid < 3) {
+        const int tile = (ttid * p.d + head * D) / 128;
+        good = mk_wait_flag(&p.qkvflag[tile], want, sh);
+      }
+      return bar_and(2, kMkThreads, good);
+    };
+    unsigned long long* atr =
+        p.trace && slot == 1 ? p.trace + static_cast<size_t>(blockIdx.x) * kMkTraceSlots + kMkTraceAttn : nullptr;
+    bool failed = false;
+    const bool wrote = attention_item_resident<D, 2, kMkThreads>(ap, split, head, b, ttid, ring, ring_bytes, sM, sL,
+                                                                  s_last, atr, wait_inputs, failed, p.attn_plo != 0);
+    if (failed) {
+      ok = false;
+      break;
+    }
+    if (wrote) {
+      named_bar_sync(2, kMkThreads);  // the head's output precedes the flag's release
+      if (ttid == 0) st_release_u64(&p.attflag[b * p.H + head], mk_seq(p.seq_base, slot, kMkAtt));
+    }
+    named_bar_sync(2, kMkThreads);
+  }
+  if (ttid == 0) mk_trace(p, kMkTracePhases * 8 + 2 * slot + 1);
+  fence_proxy_async_shared();  // generic-proxy use of the ring ends before the next TMA writes
+  return mk_team_sync(team, team_n, sh) && ok;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kMkThreads, 1)
     verify_mk_kernel(const MkParams p) {
@@ -507,14 +552,15 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   uint64_t* empty = full + S;
   uint64_t* accf = empty + S;
   uint64_t* acce = accf + kMkMaxAcc;
-  int* misc = reinterpret_cast<int*>(acce + kMkMaxAcc);  // [0] tmem addr, [1] abort, [2..4] bcast, [5] s_last
+  uint64_t* team = acce + kMkMaxAcc;  // all 256 threads: entry to / exit from a layer's attention
+  int* misc = reinterpret_cast<int*>(team + 1);  // [0] tmem addr, [1] abort, [2..4] bcast, [5] s_last
   float* xch = reinterpret_cast<float*>(misc + 16);
   float* redv = xch + 16 * 128;
   int* redi = reinterpret_cast<int*>(redv + 64);
   float* rs = reinterpret_cast<float*>(redi + 64);
-  float (*sM)[16] = reinterpret_cast<float (*)[16]>(rs + kMaxRows);
-  float (*sL)[16] = reinterpret_cast<float (*)[16]>(rs + kMaxRows + 64);
-  int* s_rows = reinterpret_cast<int*>(rs + kMaxRows + 128);  // [kMaxRows] x 5: rows, pos, kv slot, kv row, next rows
+  float (*sM)[16] = reinterpret_cast<float (*)[16]>(rs + kMaxRows);  // [8][16] per attention warp
+  float (*sL)[16] = reinterpret_cast<float (*)[16]>(rs + kMaxRows + 128);
+  int* s_rows = reinterpret_cast<int*>(rs + kMaxRows + 256);  // [kMaxRows] x 5: rows, pos, kv slot, kv row, next rows
   int* s_pos = s_rows + kMaxRows;
   int* s_kvslot = s_pos + kMaxRows;
   int* s_kvrow = s_kvslot + kMaxRows;
@@ -525,7 +571,6 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   const int NB = mk_acc_bufs(n_pad);
   const uint32_t ncols = gemm_tmem_cols(n_pad, NB);
   const PlanDev* pl = p.plan;
-  volatile int* attn_gate = misc + 9;  // QKV slots whose attention in this CTA is done (ring free)
   const size_t ring_attn_bytes = static_cast<size_t>(s_attn - base) + p.attn_extra;
   MkShared sh;
   sh.abort_s = reinterpret_cast<volatile int*>(misc + 1);
@@ -541,8 +586,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       mbar_init(&accf[i], 1);
       mbar_init(&acce[i], 128);
     }
+    mbar_init(team, kMkThreads);
     *sh.abort_s = 0;
-    misc[9] = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -560,22 +605,65 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   const int n_phases = pl->n_act == p.n_act ? min(4 * p.n_act + 1, p.ph_end) : 0;
   const int ph0 = p.ph_begin;
 
-  if (warp == 0) {
-    if (lane == 0) {
-      // ---------------- weight TMA producer: never waits for activations ----------------
-      // (only for the ring to come back from the attention that borrows it before each O phase)
-      const uint64_t wpol = l2_policy_evict_first();
-      long long i = 0;
-      bool ok = true;
-      for (int pi = ph0; ok && pi < n_phases; ++pi) {
-        const MkPhase ph = mk_phase(p, pl, pi);
+  // The attention inside this kernel (not with attn_external): every warp joins the team that runs
+  // a layer's attention items -- the epilogue warps after the layer's QKV phase, the others before
+  // its O phase.
+  AttnParams ap{};
+  ap.n_splits = p.attn_splits;
+  ap.n_heads = p.H;
+  ap.d_model = p.d;
+  ap.head_dim = D;
+  ap.scale_log2 = p.scale_log2;
+  ap.plan = pl;
+  ap.step = p.step;
+  ap.q = p.qbuf;
+  ap.o = p.obuf;
+  ap.o_xs = p.xs;
+  ap.part_o = p.attn_po;
+  ap.part_ml = p.attn_pml;
+  ap.counters = p.attn_cnt;
+  ap.status = p.status;
+  uint32_t team_n = 0;
+  auto team_attention = [&](int slot) -> bool {
+    return mk_team_attention<D>(p, ap, slot, static_cast<int>(threadIdx.x) ^ 128, base, ring_attn_bytes, sM, sL,
+                                misc + 5, team, team_n, sh);
+  };
+
+  // Roles, all in one loop over the phases: warp 0 lane 0 streams the weights, warp 1 lane 0
+  // issues the MMAs, warp 2 loads the B operands, warps 4-7 run the epilogues; at each O phase
+  // (inside this kernel's attention) all eight warps first run the layer's attention as one team.
+  const uint64_t wpol = l2_policy_evict_first();
+  const uint32_t idesc = idesc_bf16_m128(n_pad);
+  long long i = 0;  // this role's ring stage counter
+  int use = 0;      // this role's accumulator buffer counter
+  bool ok = true;
+  MkEpi e;
+  e.q = warp & 3;
+  e.lane = lane;
+  e.et = threadIdx.x - 128;
+  e.xch = xch;
+  e.redv = redv;
+  e.redi = redi;
+  e.rs = rs;
+  e.rcos = s_rope;
+  e.rsin = s_rope + 16 * 64;
+  const int r = e.q * 32 + lane;
+  int* bcast = misc + 2;
+  for (int pi = ph0; ok && pi < n_phases; ++pi) {
+    const MkPhase ph = mk_phase(p, pl, pi);
+    if (ph.kind == kMkO && !p.attn_external) {
+      // this layer's attention: the epilogue warps come after the QKV epilogues (every QKV MMA of
+      // this CTA has completed), the other warps before they start the O phase
+      const bool t = team_attention(ph.slot);
+      ok = warp >= 4 ? bar_and(1, 128, t) : __shfl_sync(0xffffffffu, t, 0);
+      if (!ok) break;
+    }
+    if (warp == 0) {
+      // ---------------- weight TMA producer (lane 0): never waits for activations ----------------
+      if (lane == 0) {
         long long it0, it1;
         int geff;
         mk_range(ph, c, G, it0, it1, geff);
-        if (ph.kind == kMkO && !p.attn_external && !mk_wait_gate(attn_gate, ph.slot, sh)) {
-          ok = false;
-          break;
-        }
         const __nv_bfloat16* wl = mk_weights(p, ph);
         long long it = it0;
         int t, k0, k1;
@@ -599,21 +687,10 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           }
         }
       }
-      if (!ok) {  // let weight tiles already in flight land before the CTA can exit
-        const uint64_t t0 = globaltimer_ns();
-        while (globaltimer_ns() - t0 < 50000) {
-        }
-      }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      // ---------------- MMA issuer ----------------
-      const uint32_t idesc = idesc_bf16_m128(n_pad);
-      long long i = 0;
-      int use = 0;
-      bool ok = true;
-      for (int pi = ph0; ok && pi < n_phases; ++pi) {
-        const MkPhase ph = mk_phase(p, pl, pi);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+    } else if (warp == 1) {
+      // ---------------- MMA issuer (lane 0) ----------------
+      if (lane == 0) {
         long long it0, it1;
         int geff;
         mk_range(ph, c, G, it0, it1, geff);
@@ -663,25 +740,13 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           ++use;
         }
       }
-    }
-  } else if (warp == 2) {
-    // ---------------- B-operand producer: TMA after the producing tiles are flagged ----------------
-    long long i = 0;
-    bool ok = true;
-    for (int pi = ph0; ok && pi < n_phases; ++pi) {
-      const MkPhase ph = mk_phase(p, pl, pi);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+    } else if (warp == 2) {
+      // ---------------- B-operand producer: TMA after the producing tiles are flagged ----------------
       long long it0, it1;
       int geff;
       mk_range(ph, c, G, it0, it1, geff);
       if (it0 >= it1) continue;
-      if (ph.kind == kMkO && !p.attn_external) {
-        bool free = true;
-        if (lane == 0) free = mk_wait_gate(attn_gate, ph.slot, sh);
-        if (!__shfl_sync(0xffffffffu, free, 0)) {
-          ok = false;
-          break;
-        }
-      }
       // dependency index space of this phase: h tiles, heads, or gate/up tiles
       const unsigned long long* flags;
       unsigned long long want;
@@ -763,40 +828,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         }
        }
       }
-    }
-  } else if (warp >= 4) {
-    // ---------------- epilogues and attention ----------------
-    MkEpi e;
-    e.q = warp & 3;
-    e.lane = lane;
-    e.et = threadIdx.x - 128;
-    e.xch = xch;
-    e.redv = redv;
-    e.redi = redi;
-    e.rs = rs;
-    e.rcos = s_rope;
-    e.rsin = s_rope + 16 * 64;
-    const int r = e.q * 32 + lane;
-    int* bcast = misc + 2;
-    int use = 0;
-    bool ok = true;
-    AttnParams ap{};
-    ap.n_splits = p.attn_splits;
-    ap.n_heads = p.H;
-    ap.d_model = p.d;
-    ap.head_dim = D;
-    ap.scale_log2 = p.scale_log2;
-    ap.plan = pl;
-    ap.step = p.step;
-    ap.q = p.qbuf;
-    ap.o = p.obuf;
-    ap.o_xs = p.xs;
-    ap.part_o = p.attn_po;
-    ap.part_ml = p.attn_pml;
-    ap.counters = p.attn_cnt;
-    ap.status = p.status;
-    for (int pi = ph0; ok && pi < n_phases; ++pi) {
-      const MkPhase ph = mk_phase(p, pl, pi);
+    } else if (warp >= 4) {
+      // ---------------- epilogues ----------------
       long long it0, it1;
       int geff;
       mk_range(ph, c, G, it0, it1, geff);
@@ -1030,51 +1063,11 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         if (e.et == 0 && it >= it1) mk_trace(p, pi * 8 + 7);
         ++use;
       }
-      if (!ok) break;
-      if (ph.kind == kMkQkv && !p.attn_external) {
-        // attention items of this layer: (request, head, split) round-robin over the grid
-        ap.slot = ph.slot;
-        const int per_req = p.H * p.attn_splits;
-        const int n_items = p.B * per_req;
-        const unsigned long long want = mk_seq(p.seq_base, ph.slot, kMkQkv);
-        if (e.et == 0) mk_trace(p, kMkTracePhases * 8 + 2 * ph.slot);
-        // The attention borrows the weight/activation ring and its own buffer: this CTA's QKV
-        // MMAs have all completed, and the producers start the O phase only after the gate.
-        fence_proxy_async_shared();
-        for (int item = c; ok && item < n_items; item += G) {
-          const int b = item / per_req;
-          const int head = (item - b * per_req) / p.attn_splits;
-          const int split = item - b * per_req - head * p.attn_splits;
-          if (pl->slot_crow[ph.slot][b] < 0) continue;
-          // the Q, K and V tiles of this head (written by the QKV epilogues of this step)
-          auto wait_inputs = [&]() -> bool {
-            bool good = true;
-            if (e.et < 3) {
-              const int tile = (e.et * p.d + head * D) / 128;
-              good = mk_wait_flag(&p.qkvflag[tile], want, sh);
-            }
-            return bar_and(1, 128, good);
-          };
-          unsigned long long* atr =
-              p.trace && ph.slot == 1 ? p.trace + static_cast<size_t>(blockIdx.x) * kMkTraceSlots + kMkTraceAttn : nullptr;
-          bool failed = false;
-          const bool wrote = attention_item_resident<D, 1>(ap, split, head, b, e.et, base, ring_attn_bytes, sM, sL,
-                                                           misc + 5, atr, wait_inputs, failed, p.attn_plo != 0);
-          if (failed) {
-            ok = false;
-            break;
-          }
-          if (wrote) {
-            named_bar_sync(1, 128);  // the head's output precedes the flag's release
-            if (e.et == 0) st_release_u64(&p.attflag[b * p.H + head], mk_seq(p.seq_base, ph.slot, kMkAtt));
-          }
-          named_bar_sync(1, 128);
-        }
-        if (e.et == 0) mk_trace(p, kMkTracePhases * 8 + 2 * ph.slot + 1);
-        fence_proxy_async_shared();  // generic-proxy use of the ring ends before the next TMA writes
-        named_bar_sync(1, 128);
-        if (e.et == 0) *attn_gate = ph.slot + 1;
-      }
+    }
+  }
+  if (warp == 0 && !ok && lane == 0) {  // let weight tiles already in flight land before the CTA can exit
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < 50000) {
     }
   }
 
@@ -1091,8 +1084,8 @@ size_t mk_trace_slots() { return kMkTraceSlots; }
 
 size_t mk_smem_bytes(int n_pad, int parts, int stages, int head_dim, int kps, size_t attn_extra) {
   return 1024 + static_cast<size_t>(stages) * kps * (kMkWBytes + static_cast<size_t>(n_pad) * parts * 128) +
-         attn_extra + static_cast<size_t>(2 * stages + 2 * kMkMaxAcc) * 8 + 64 + 16 * 128 * 4 +
-         64 * 4 * 2 + kMaxRows * 4 + 128 * 4 + 5 * kMaxRows * 4 + 2 * 16 * 64 * 4 + 64;
+         attn_extra + static_cast<size_t>(2 * stages + 2 * kMkMaxAcc + 1) * 8 + 64 + 16 * 128 * 4 +
+         64 * 4 * 2 + kMaxRows * 4 + 256 * 4 + 5 * kMaxRows * 4 + 2 * 16 * 64 * 4 + 64;
 }
 
 cudaError_t mk_prepare() {
