@@ -295,8 +295,10 @@ __device__ bool mk_prepare_rs(const MkParams& p, const MkEpi& e, unsigned long l
 }
 
 // Fused epilogue of one 16-token chunk (tokens ch*16 ..) of output row r of tile t.
+// hv (residual phases, optional): h of these 16 rows at this thread's feature, loaded by the caller
+// together with the partial sums.
 __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const MkEpi& e, int t, int r, int ch,
-                                  const float* v) {
+                                  const float* v, const float* hv = nullptr) {
   const StepDesc* st = p.step;
   const int j0 = ch * 16;
   if (ph.kind == kMkQkv) {
@@ -356,7 +358,7 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
       if (j < e.M) {
         float* hp = p.h + static_cast<size_t>(e.rows[j]) * p.d + o;
         // h of the CTA's last tile was loaded at phase start (off the critical path)
-        const float nv = (t == e.hpre_tile ? e.xch[jj * 128 + r] : __ldcg(hp)) + v[jj];
+        const float nv = (t == e.hpre_tile ? e.xch[jj * 128 + r] : hv ? hv[jj] : __ldcg(hp)) + v[jj];
         *hp = nv;
         sq[jj] = nv * nv;
         if (e.direct_xn) store_split(p.xn, p.xs, j, o, nv * gn);
@@ -1018,33 +1020,35 @@ __global__ void __launch_bounds__(kMkThreads, 1)
                 for (int jj = 0; jj < 8; ++jj) v[jj] += pv[q][jj];
               if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 7);
               mk_epilogue_chunk(p, ph, e, t, r, 0, v);
-            } else
-            for (int ch = 0; ch < n_ch; ++ch) {
-              float v[16];
-#pragma unroll
-              for (int jj = 0; jj < 16; ++jj) v[jj] = 0.f;
-              // contributors in order (deterministic sum), two at a time in flight
-              int cc = cf;
-              for (; cc + 1 <= cl; cc += 2) {
-                const float* pa = partials + static_cast<size_t>(cc + t) * 128 * n_pad;
-                const float* pb = pa + static_cast<size_t>(128) * n_pad;
-                float a[16], bq[16];
+            } else {
+              // contributors in order (deterministic sum), four partials' loads in flight at once
+              const bool pre_h = (ph.kind == kMkO || ph.kind == kMkDown) && t != e.hpre_tile;
+              for (int ch = 0; ch < n_ch; ++ch) {
+                float v[16], hv[16];
 #pragma unroll
                 for (int jj = 0; jj < 16; ++jj) {
-                  const bool in = ch * 16 + jj < e.M;
-                  a[jj] = in ? __ldcg(&pa[(ch * 16 + jj) * 128 + r]) : 0.f;
-                  bq[jj] = in ? __ldcg(&pb[(ch * 16 + jj) * 128 + r]) : 0.f;
+                  v[jj] = 0.f;
+                  hv[jj] = pre_h && ch * 16 + jj < e.M
+                               ? __ldcg(&p.h[static_cast<size_t>(e.rows[ch * 16 + jj]) * p.d + t * 128 + r])
+                               : 0.f;
                 }
+                for (int c0 = cf; c0 <= cl; c0 += 4) {
+                  float pv[4][16];
 #pragma unroll
-                for (int jj = 0; jj < 16; ++jj) v[jj] = (v[jj] + a[jj]) + bq[jj];
-              }
-              if (cc <= cl) {
-                const float* pa = partials + static_cast<size_t>(cc + t) * 128 * n_pad;
+                  for (int q = 0; q < 4; ++q) {
+                    const bool cin = c0 + q <= cl;
+                    const float* pa = partials + static_cast<size_t>(c0 + q + t) * 128 * n_pad;
 #pragma unroll
-                for (int jj = 0; jj < 16; ++jj)
-                  if (ch * 16 + jj < e.M) v[jj] += __ldcg(&pa[(ch * 16 + jj) * 128 + r]);
+                    for (int jj = 0; jj < 16; ++jj)
+                      pv[q][jj] = cin && ch * 16 + jj < e.M ? __ldcg(&pa[(ch * 16 + jj) * 128 + r]) : 0.f;
+                  }
+#pragma unroll
+                  for (int q = 0; q < 4; ++q)
+#pragma unroll
+                    for (int jj = 0; jj < 16; ++jj) v[jj] += pv[q][jj];
+                }
+                mk_epilogue_chunk(p, ph, e, t, r, ch, v, pre_h ? hv : nullptr);
               }
-              mk_epilogue_chunk(p, ph, e, t, r, ch, v);
             }
             if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 4);
           }
