@@ -311,22 +311,34 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) val[jj] = j0 + jj < e.M ? v[jj] * e.rs[j0 + jj] : 0.f;
     if (sec < 2) {
+      // rotation factors first (the first 16 rows staged in shared memory, later rows' loads in
+      // flight during the exchange of the partner elements)
+      const int i = dim & (half - 1);
+      float cs[16], sn[16];
+      if (j0 == 0) {
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj) {
+          cs[jj] = e.rcos[jj * half + i];
+          sn[jj] = e.rsin[jj * half + i];
+        }
+      } else {
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj) {
+          const bool in = j0 + jj < e.M;
+          const size_t pe = static_cast<size_t>(in ? e.pos[j0 + jj] : 0) * half + i;
+          cs[jj] = in ? __ldg(&p.rope_cos[pe]) : 0.f;
+          sn[jj] = in ? __ldg(&p.rope_sin[pe]) : 0.f;
+        }
+      }
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) e.xch[jj * 128 + r] = val[jj];
       named_bar_sync(1, 128);
       const int pr = r ^ half;
-      const int i = dim & (half - 1);
       float rot[16];
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) {
-        rot[jj] = 0.f;
-        if (j0 + jj < e.M) {
-          const int pos = e.pos[j0 + jj];
-          const float c = j0 == 0 ? e.rcos[jj * half + i] : p.rope_cos[static_cast<size_t>(pos) * half + i];
-          const float s = j0 == 0 ? e.rsin[jj * half + i] : p.rope_sin[static_cast<size_t>(pos) * half + i];
-          const float pv = e.xch[jj * 128 + pr];
-          rot[jj] = dim < half ? val[jj] * c - pv * s : val[jj] * c + pv * s;
-        }
+        const float pv = e.xch[jj * 128 + pr];
+        rot[jj] = j0 + jj < e.M ? (dim < half ? val[jj] * cs[jj] - pv * sn[jj] : val[jj] * cs[jj] + pv * sn[jj]) : 0.f;
       }
       named_bar_sync(1, 128);
 #pragma unroll
