@@ -222,6 +222,50 @@ def test_mixed_domain_batch_and_untouched_skipped_kv(weights, path):
 
 
 @pytest.mark.parametrize("path", PATHS)
+def test_maximum_block_rows(weights, path):
+    """Blocks at the size limits: a 64-node chain (the most nodes a request may have), a 63-node
+    draft tree and a 64-node chain of a second domain in one batch -- 192 rows, so the
+    activations take the two-block hi/lo layout and every fix-up runs twelve 16-row chunks."""
+    w, wo, wg = weights
+    phi = {0: O.set_to_mask({1}), 1: O.set_to_mask({0, 2})}
+    doms = [0, 1, 0]
+    ctxs = [40, 9, 0]
+    shapes = [synth.chain_parents(63), synth.eagle_tree(62, (4, 3, 2, 2, 1, 1)), synth.chain_parents(63)]
+    run = make_runner(wg, n_slots=3, cap=160, path=path, max_nodes=64)
+    run.set_phi(phi)
+    reqs, kvs, skips = [], [], []
+    for b in range(3):
+        skip = O.skip_set({d: O.mask_to_set(m) for d, m in phi.items()}, doms[b])
+        if ctxs[b]:
+            kv = O.prefill(wo, ARCH, skip, synth.uniform_ints(ctxs[b], ARCH.vocab, SEED, f"max.ctx{b}").tolist())
+            upload_context(run, kv, b)
+        else:
+            kv = [O.empty_kv(ARCH) for _ in range(ARCH.n_layers)]
+        parents = shapes[b]
+        toks = synth.draft_tokens(parents, ARCH.vocab, SEED, f"max.tok{b}")
+        reqs.append(synth.Request(ctxs[b], parents, toks, doms[b]))
+        kvs.append(kv)
+        skips.append(skip)
+    res, st = run_step(run, reqs)
+    assert st == native.TSS_OK
+    gl = res["logits"].cpu().numpy()
+    off = 0
+    for b, r in enumerate(reqs):
+        n = len(r.parents)
+        ref, nk = O.verify_request(wo, ARCH, skips[b], r.tokens, r.parents, r.ctx_len, kvs[b])
+        assert_logits(gl[off:off + n], ref, f"request {b} ({n} nodes)")
+        a, bonus, pth = O.greedy_accept(ref, r.tokens, r.parents)
+        if O.greedy_flagged(ref, pth):
+            ga = int(res["accept_len"][b])
+            assert greedy_valid(ref, r.tokens, r.parents, gpu_path(res, b, ga), int(res["bonus"][b]))
+        else:
+            assert (int(res["accept_len"][b]), int(res["bonus"][b])) == (a, bonus)
+        assert int(res["new_ctx_len"][b]) == r.ctx_len + 1 + int(res["accept_len"][b])
+        off += n
+    run.close()
+
+
+@pytest.mark.parametrize("path", PATHS)
 def test_all_layers_skipped_is_embedding_norm_lm_head(weights, path):
     w, wo, wg = weights
     run = make_runner(wg, n_slots=1, cap=64, path=path)
