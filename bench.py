@@ -139,13 +139,17 @@ class ClockSampler:
 
 
 def kernel_sources_hash():
-    """sha256 over the sources of the persistent verify kernel (an ncu traffic figure is only
-    valid for the kernel it was taken on)."""
+    """sha256 over the code of the persistent verify kernel's sources, comments and blank lines
+    left out (an ncu traffic figure is only valid for the kernel it was taken on)."""
     import hashlib
+    import re
     h = hashlib.sha256()
     for f in ("verify_mk.cu", "attn_body.cuh", "common.cuh", "internal.h"):
-        with open(os.path.join(ROOT, "paper_2609_26100_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2609_26100_gb300", "csrc", f), encoding="utf-8") as fh:
+            for line in fh:
+                code = re.sub(r"(^|\s)//.*$", "", line.rstrip("\n")).rstrip()
+                if code:
+                    h.update(code.encode() + b"\n")
     return h.hexdigest()
 
 

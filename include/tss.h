@@ -186,6 +186,9 @@ tss_status tss_active_layer_count(const tss_ctx* ctx, const tss_verify_batch* ba
  * not overlap on different streams (they share workspaces).
  * Default path: three launches -- a prologue (controller, embedding), one persistent cooperative
  * kernel for every active layer and the LM head, and a finish kernel (acceptance, compaction).
+ * When a step's context KV outweighs half a layer's weights (long contexts), the persistent kernel
+ * is launched once per span of GEMM phases between two attentions and each layer's attention
+ * runs as its own kernel (2 + 2 x active layers + 1 launches).
  * With the environment variable TSS_PATH=multi at tss_create, or when a step's rows do not fit the
  * persistent kernel's shared-memory plan, one kernel per operation runs instead (bf16 GEMM
  * activations, 6 + 7 x active layers launches). */

@@ -5,15 +5,19 @@
 // QKV, O, gate/up, down; then the LM head -- with the attention of a layer between its QKV and
 // O phases.  Each phase is split stream-K over the grid exactly as in gemm.cu.  Per CTA:
 //
-//   warp 0      TMA producer of weight tiles.  It walks the whole phase sequence and never waits
-//               for activations, so the weight stream does not stop at phase boundaries (it is
-//               bounded only by the shared-memory ring).
-//   warp 1      tcgen05.mma issuer (accumulators in TMEM, double-buffered).
+//   warp 0      TMA producer of weight tiles (lane 0).  It walks the whole phase sequence and
+//               never waits for activations, so the weight stream does not stop at phase
+//               boundaries (it is bounded only by the shared-memory ring).
+//   warp 1      tcgen05.mma issuer (lane 0; accumulators in TMEM, up to 8 buffers).
 //   warp 2      B-operand producer: for every k-block it waits until the activations it needs
 //               are final (flags polled 32 at a time), then loads the N x 64 bf16 tile by TMA --
 //               bf16(h * g) for QKV / gate-up / LM head, the attention output for O, the SwiGLU
 //               activations for down.
-//   warps 4-7   epilogues (TMEM -> registers, stream-K fixup, fused op) and the attention items.
+//   warp 3      attention only.
+//   warps 4-7   epilogues (TMEM -> registers, stream-K fixup, fused op).
+// All roles run one loop over the phases; at each O phase (when the attention runs in this
+// kernel) the eight warps first run the layer's attention items together, in the ring that every
+// role has stopped using by then.
 //
 // Phases hand data over through global memory and per-tile flags stamped with a sequence
 // number that grows monotonically over the step and across steps (seq = epoch*1024 + 8*(slot+1)
