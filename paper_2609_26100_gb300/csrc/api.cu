@@ -122,7 +122,7 @@ struct tss_ctx {
   int gemm_ctas_per_sm = 2;
   // persistent verify kernel
   bool use_mk = true;
-  int mk_kps = 4;  // weight k-blocks per ring stage of the persistent kernel
+  int mk_kps = 3;  // weight k-blocks per ring stage of the persistent kernel (48 KiB stages measured best)
   int attn_mode = 0;  // 0 auto, 1 attention inside the persistent kernel, 2 separate attention kernels
   int w_evict_first = 1;
   int mk_max_stages = 12;
