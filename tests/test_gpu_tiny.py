@@ -444,8 +444,27 @@ def test_host_validation_errors(weights):
     assert status([good], mode=native.TSS_MODE_SAMPLE) == native.TSS_ERR_INVALID_ARG  # no draft probs
     with pytest.raises(native.TssError):
         run.v.set_skip_config(0, 1 << ARCH.n_layers)
+    with pytest.raises(native.TssError):
+        run.v.set_skip_config(-1, 0)  # domain id out of range
+    # size limits: more nodes than a request may have, more rows than the context was created for,
+    # more requests than its batch limit, no request at all
+    big = synth.Request(0, synth.chain_parents(64), list(range(65)), 0)
+    assert status([big]) == native.TSS_ERR_INVALID_ARG
+    assert status([good] * 9, slots=list(range(9))) == native.TSS_ERR_INVALID_ARG
+    assert status([]) == native.TSS_ERR_INVALID_ARG
+    assert status([synth.Request(4, [-1, 0], [1, 2], 0)], slots=[2]) == native.TSS_ERR_INVALID_ARG  # slot range
+    assert status([good], mode=native.TSS_MODE_SAMPLE, temperature=0.0,
+                  draft_probs=torch.ones(2, ARCH.vocab, device="cuda")) == native.TSS_ERR_INVALID_ARG
     assert status([good]) == native.TSS_OK
     assert run.sync_status() == native.TSS_OK
+    run.close()
+    # more rows in one step than the context was created for
+    run = make_runner(wg, n_slots=3, cap=80, max_rows=128)
+    many = [synth.Request(0, synth.chain_parents(63), list(range(64)), 0) for _ in range(3)]
+    b = run.batch(many)
+    with pytest.raises(native.TssError) as err:
+        run.verify(b, run.alloc_results(3, 192))
+    assert err.value.status == native.TSS_ERR_INVALID_ARG
     run.close()
 
 
