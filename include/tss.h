@@ -195,6 +195,22 @@ tss_status tss_active_layer_count(const tss_ctx* ctx, const tss_verify_batch* ba
 tss_status tss_verify(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
                       const tss_verify_result* result, void* stream);
 
+/* Prefill: append tokens to the requests' KV caches under their skip configurations (the
+ * configuration is fixed for a whole request, prompt included: Sec. "Problem Formulation").
+ * Request b's tokens [ctx_len[b], ctx_len[b] + n_tokens[b]) run through the layers its domain
+ * does not skip, in chains of up to max_nodes tokens -- each chain one verification step on the
+ * same kernels, whose acceptance outputs are discarded -- and their K/V rows are written to the
+ * cache of every such layer; layers it skips are not touched.  Afterwards the caller's cache of
+ * request b holds ctx_len[b] + n_tokens[b] tokens.
+ *   n_tokens, ctx_len, domain_id, kv_slot: HOST arrays of n_req entries (n_tokens[b] >= 0;
+ *     kv_slot NULL means slot b).
+ *   tokens: the requests' tokens concatenated (sum(n_tokens) int32), DEVICE memory, or HOST
+ *     memory when io_host != 0.
+ * Asynchronous on `stream`, like tss_verify; host-detectable errors return before any launch. */
+tss_status tss_prefill(tss_ctx* ctx, int n_req, const int32_t* n_tokens, const int32_t* ctx_len,
+                       const int32_t* domain_id, const int32_t* kv_slot, const int32_t* tokens, int io_host,
+                       const tss_kv_cache* kv, void* stream);
+
 /* Synchronise `stream`, then return and clear the device status word (TSS_OK if no device-side
  * check failed since the last call). */
 tss_status tss_sync_status(tss_ctx* ctx, void* stream);

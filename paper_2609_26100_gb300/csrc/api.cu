@@ -1093,6 +1093,74 @@ tss_status tss_verify(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache
   return verify_impl(c, bt, kv, res, static_cast<cudaStream_t>(stream), nullptr);
 }
 
+tss_status tss_prefill(tss_ctx* c, int n_req, const int32_t* n_tokens, const int32_t* ctx_len,
+                       const int32_t* domain_id, const int32_t* kv_slot, const int32_t* tokens, int io_host,
+                       const tss_kv_cache* kv, void* stream) {
+  if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
+  if (n_req < 1 || n_req > c->a.max_batch) return fail(TSS_ERR_INVALID_ARG, "n_req must be in [1, max_batch]");
+  if (!n_tokens || !ctx_len || !domain_id || !tokens || !kv)
+    return fail(TSS_ERR_INVALID_ARG, "n_tokens, ctx_len, domain_id, tokens and kv are required");
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  std::vector<long long> off(n_req + 1, 0);
+  for (int b = 0; b < n_req; ++b) {
+    if (n_tokens[b] < 0 || ctx_len[b] < 0) return fail(TSS_ERR_INVALID_ARG, "n_tokens and ctx_len must be >= 0");
+    if (static_cast<long long>(ctx_len[b]) + n_tokens[b] > kv->cap)
+      return fail(TSS_ERR_KV_CAPACITY, "ctx_len + n_tokens exceeds KV capacity");
+    off[b + 1] = off[b] + n_tokens[b];
+  }
+  // Rounds of verification steps: each request still holding tokens adds a chain of up to
+  // max_nodes of them (row 0, the chain's root, is not yet cached, exactly like a draft block's
+  // root), within max_rows rows per step; the chains' K/V rows stay where the QKV epilogue wrote
+  // them (a chain's compaction moves nothing), and the acceptance outputs go to a scratch buffer.
+  std::vector<int> done(n_req, 0);
+  std::vector<int32_t> nn, cl, dom, slot, par;
+  tss_verify_result res{};
+  res.accept_len = c->io_res;
+  res.bonus = c->io_res + kMaxBatch;
+  res.new_ctx_len = c->io_res + 2 * kMaxBatch;
+  res.path = c->io_res + 3 * kMaxBatch;
+  res.path_stride = c->a.max_nodes + 1;
+  res.logits = nullptr;
+  for (;;) {
+    nn.clear();
+    cl.clear();
+    dom.clear();
+    slot.clear();
+    par.clear();
+    int rows = 0;
+    for (int b = 0; b < n_req && rows < c->a.max_rows; ++b) {
+      const int left = n_tokens[b] - done[b];
+      if (left <= 0) continue;
+      const int len = std::min(std::min(left, c->a.max_nodes), c->a.max_rows - rows);
+      const int32_t* src = tokens + off[b] + done[b];
+      TSS_CU(cudaMemcpyAsync(c->io_tokens + rows, src, sizeof(int32_t) * len,
+                             io_host ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToDevice, s));
+      nn.push_back(len);
+      cl.push_back(ctx_len[b] + done[b]);
+      dom.push_back(domain_id[b]);
+      slot.push_back(kv_slot ? kv_slot[b] : b);
+      for (int i = 0; i < len; ++i) par.push_back(i - 1);
+      done[b] += len;
+      rows += len;
+    }
+    if (nn.empty()) break;
+    tss_verify_batch bt{};
+    bt.n_req = static_cast<int>(nn.size());
+    bt.n_nodes = nn.data();
+    bt.ctx_len = cl.data();
+    bt.domain_id = dom.data();
+    bt.kv_slot = slot.data();
+    bt.parent_idx = par.data();
+    bt.positions = nullptr;
+    bt.tokens = c->io_tokens;
+    bt.mode = TSS_MODE_GREEDY;
+    bt.temperature = 1.f;
+    bt.io_host = 0;
+    TSS_TRY(verify_impl(c, &bt, kv, &res, s, nullptr));
+  }
+  return TSS_OK;
+}
+
 tss_status tss_verify_profiled(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache* kv,
                                const tss_verify_result* res, void* stream, tss_kernel_times* times) {
   if (!times) return fail(TSS_ERR_INVALID_ARG, "times is NULL");

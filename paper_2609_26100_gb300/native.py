@@ -25,8 +25,8 @@ TSS_MODE_SAMPLE = 1
 
 EXPORTS = (
     "tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
-    "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_sync_status", "tss_destroy", "tss_linear",
-    "tss_linear_static", "tss_read_trace", "tss_status_string", "tss_last_error",
+    "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status", "tss_destroy",
+    "tss_linear", "tss_linear_static", "tss_read_trace", "tss_status_string", "tss_last_error",
 )
 
 _P = ctypes.c_void_p
@@ -88,6 +88,8 @@ def lib() -> ctypes.CDLL:
                                  ctypes.POINTER(TssVerifyResult), _P]
         L.tss_verify_profiled.argtypes = [_P, ctypes.POINTER(TssVerifyBatch), ctypes.POINTER(TssKvCache),
                                           ctypes.POINTER(TssVerifyResult), _P, ctypes.POINTER(TssKernelTimes)]
+        L.tss_prefill.argtypes = [_P, ctypes.c_int, _I32P, _I32P, _I32P, _I32P, _P, ctypes.c_int,
+                                  ctypes.POINTER(TssKvCache), _P]
         L.tss_sync_status.argtypes = [_P, _P]
         L.tss_destroy.argtypes = [_P]
         L.tss_destroy.restype = None
@@ -99,8 +101,8 @@ def lib() -> ctypes.CDLL:
         L.tss_last_error.argtypes = []
         L.tss_last_error.restype = ctypes.c_char_p
         for name in ("tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
-                     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_sync_status", "tss_linear",
-                     "tss_linear_static", "tss_read_trace"):
+                     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status",
+                     "tss_linear", "tss_linear_static", "tss_read_trace"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -226,6 +228,14 @@ class Verifier:
     def verify(self, batch, kv, result, stream=None) -> None:
         check(lib().tss_verify(self.ctx, ctypes.byref(batch), ctypes.byref(kv), ctypes.byref(result), stream),
               "tss_verify")
+
+    def prefill(self, n_tokens: Sequence[int], ctx_len: Sequence[int], domain_id: Sequence[int], tokens, kv,
+                kv_slot=None, io_host: bool = False, stream=None) -> None:
+        """tss_prefill: tokens (int32, the requests' tokens concatenated) appended to the caches."""
+        keep = [_i32(n_tokens), _i32(ctx_len), _i32(domain_id), _i32(kv_slot) if kv_slot is not None else None]
+        cast = [ctypes.cast(a, _I32P) if a is not None else None for a in keep]
+        check(lib().tss_prefill(self.ctx, len(n_tokens), cast[0], cast[1], cast[2], cast[3], _ptr(tokens),
+                                1 if io_host else 0, ctypes.byref(kv), stream), "tss_prefill")
 
     def verify_profiled(self, batch, kv, result, times: "TssKernelTimes", stream=None) -> None:
         check(lib().tss_verify_profiled(self.ctx, ctypes.byref(batch), ctypes.byref(kv), ctypes.byref(result), stream,

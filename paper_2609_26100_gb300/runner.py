@@ -109,6 +109,16 @@ class TssRunner:
         s = stream if stream is not None else torch.cuda.current_stream().cuda_stream
         self.v.verify(batch, self.kv_struct, results["_struct"], s)
 
+    def prefill(self, prompts: Sequence[Sequence[int]], ctx_lens: Sequence[int], domains: Sequence[int], slots=None,
+                stream=None) -> None:
+        """Append each request's prompt tokens to its KV cache (tss_prefill) under its domain's
+        skip configuration; request b's cache then holds ctx_lens[b] + len(prompts[b]) tokens."""
+        toks = torch.tensor([t for pr in prompts for t in pr] or [0], dtype=torch.int32, device=self.device)
+        s = stream if stream is not None else torch.cuda.current_stream().cuda_stream
+        self.v.prefill([len(pr) for pr in prompts], list(ctx_lens), list(domains), toks, self.kv_struct, kv_slot=slots,
+                       stream=s)
+        self._prefill_tokens = toks  # alive until the stream has used it
+
     def sync_status(self, stream=None) -> int:
         s = stream if stream is not None else torch.cuda.current_stream().cuda_stream
         return self.v.sync_status(s)

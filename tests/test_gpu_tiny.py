@@ -266,6 +266,55 @@ def test_maximum_block_rows(weights, path):
 
 
 @pytest.mark.parametrize("path", PATHS)
+def test_gpu_prefill_matches_oracle_prefill(weights, path):
+    """tss_prefill under each request's skip set: a 150-token prompt on an empty cache, 40 tokens
+    appended to a 20-token context of another domain, and an empty prompt.  The K/V rows match
+    the oracle's prefill, skipped layers stay untouched, and a verification step on top of the
+    GPU-filled cache gives the oracle's logits."""
+    w, wo, wg = weights
+    phi = {0: O.set_to_mask({2}), 1: O.set_to_mask({0, 3})}
+    run = make_runner(wg, n_slots=3, cap=256, path=path)
+    run.set_phi(phi)
+    sentinel = 7.0
+    for t in run.kv:
+        t.fill_(sentinel)
+    doms = [0, 1, 0]
+    full = [synth.uniform_ints(150, ARCH.vocab, SEED, "pf.a").tolist(),
+            synth.uniform_ints(60, ARCH.vocab, SEED, "pf.b").tolist(),
+            synth.uniform_ints(12, ARCH.vocab, SEED, "pf.c").tolist()]
+    have = [0, 20, 12]  # tokens already in the cache (uploaded from the oracle)
+    skips = [O.skip_set({d: O.mask_to_set(m) for d, m in phi.items()}, d) for d in doms]
+    for b in (1, 2):
+        upload_context(run, O.prefill(wo, ARCH, skips[b], full[b][:have[b]]), b)
+    run.prefill([full[b][have[b]:] for b in range(3)], have, doms)
+    assert run.sync_status() == native.TSS_OK
+    torch.cuda.synchronize()
+    for b in range(3):
+        ref = O.prefill(wo, ARCH, skips[b], full[b])
+        C = len(full[b])
+        for l in range(ARCH.n_layers):
+            region = run.kv[l][b]
+            if l in skips[b]:
+                assert bool((region == sentinel).all()), f"request {b} skipped layer {l} was touched"
+                continue
+            gk = region[0, :, :C].float().cpu().numpy()
+            gv = region[1, :, :C].float().cpu().numpy()
+            np.testing.assert_allclose(gk, ref[l][0], atol=5e-2, rtol=3e-2)
+            np.testing.assert_allclose(gv, ref[l][1], atol=5e-2, rtol=3e-2)
+            assert float(np.abs(gk - ref[l][0]).mean()) < 2e-3
+            assert bool((region[:, :, C:] == sentinel).all())
+    # a verification step on the GPU-filled cache of request 0
+    C = len(full[0])
+    parents = synth.chain_parents(4)
+    toks = synth.draft_tokens(parents, ARCH.vocab, SEED, "pf.tok")
+    res, st = run_step(run, [synth.Request(C, parents, toks, doms[0])])
+    assert st == native.TSS_OK
+    ref, _ = O.verify_request(wo, ARCH, skips[0], toks, parents, C, O.prefill(wo, ARCH, skips[0], full[0]))
+    assert_logits(res["logits"].cpu().numpy(), ref, "verify after GPU prefill")
+    run.close()
+
+
+@pytest.mark.parametrize("path", PATHS)
 def test_all_layers_skipped_is_embedding_norm_lm_head(weights, path):
     w, wo, wg = weights
     run = make_runner(wg, n_slots=1, cap=64, path=path)
