@@ -44,6 +44,9 @@ def parse_args():
     p.add_argument("--sweep", default=None,
                    help="7b_long: comma-separated skipped-layer counts (e.g. 0,2,4,...,12); one process, one "
                         "weight and KV set, latency vs active layers with a least-squares line")
+    p.add_argument("--prefill", type=int, default=None,
+                   help="prompt tokens per request: time tss_prefill on the 7B chain's skip set (4 requests) "
+                        "instead of the verification step")
     p.add_argument("--traffic", default=os.path.join(ROOT, "profiles", "verify_persistent_7b_chain_traffic.txt"),
                    help="JSON summary of an ncu DRAM-traffic capture of the dominant kernel")
     return p.parse_args()
@@ -554,12 +557,67 @@ def run_sweep(args):
                       "data": "synthetic (seeded random-init weights, synthetic KV)"}))
 
 
+def run_prefill(args):
+    """Prompt prefill under the 7B chain workload's skip configuration: 4 requests of
+    args.prefill tokens each appended to empty caches with tss_prefill (chains of up to 64 tokens
+    per request, 256 rows per verification step on the same kernels), timed with CUDA events.
+    Prints one JSON line: prompt tokens per second and the weight bytes each step streams."""
+    import torch
+    from paper_2609_26100_gb300 import build as _build
+    from paper_2609_26100_gb300 import native, synth
+    from paper_2609_26100_gb300.runner import TssRunner
+    torch.cuda.set_device(0)
+    _build.build()
+    w = synth.workload_7b_chain()
+    a = w.arch
+    union = w.active_union()
+    n_req, n_tok = 4, args.prefill
+    weights = synth.make_weights(a, w.seed, device="cuda", layers=union)
+    for l in range(a.n_layers):
+        if weights["layers"][l] is None:
+            weights["layers"][l] = {k: torch.zeros(sh, dtype=torch.bfloat16, device="cuda")
+                                    for k, sh in synth.layer_shapes(a).items()}
+    run = TssRunner(a, weights, n_slots=n_req, kv_cap=n_tok + 8, max_batch=n_req, max_rows=256, max_nodes=64,
+                    kv_layers=union)
+    del weights
+    torch.cuda.empty_cache()
+    run.set_phi(w.phi)
+    prompts = [synth.uniform_ints(n_tok, a.vocab, w.seed, f"prefill.{b}").tolist() for b in range(n_req)]
+    doms = [w.requests[0].domain] * n_req
+    stream = torch.cuda.current_stream()
+    for _ in range(max(1, args.warmup)):
+        run.prefill(prompts, [0] * n_req, doms)
+    if run.sync_status() != native.TSS_OK:
+        raise RuntimeError("device status error in prefill")
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        run.prefill(prompts, [0] * n_req, doms)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    steps_per_prefill = -(-n_tok // 64)
+    ab = synth.algorithmic_bytes(w)
+    out = {"metric": "prompt prefill tokens/s under the 7B chain skip set (4 requests)", "value":
+           n_req * n_tok / (ms / 1e3), "unit": "tokens/s", "higher_is_better": True, "n_gpus": 1,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_prefill": ms, "dtype": "bf16",
+           "data": "synthetic (seeded random-init weights, uniform random prompt ids)",
+           "config": {"workload": f"7b_chain skip set, {n_req} requests x {n_tok} prompt tokens, "
+                                  f"{steps_per_prefill} verification steps of 256 rows", "active_layers": len(union)},
+           "weight_bytes_per_step": ab["weights"], "weight_gbs": steps_per_prefill * ab["weights"] / (ms / 1e3) / 1e9}
+    run.close()
+    print(json.dumps(out))
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
     elif args.sweep:
         run_sweep(args)
+    elif args.prefill:
+        run_prefill(args)
     else:
         run_tss(args)
 
