@@ -343,6 +343,11 @@ __device__ __forceinline__ void mma_f16_16816(float* d, const uint32_t* a, const
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
+__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
 // Two bf16 values (low half first) to two fp16 values, round to nearest.
 __device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t v) {
   const float lo = __uint_as_float(v << 16), hi = __uint_as_float(v & 0xffff0000u);

@@ -462,6 +462,168 @@ __device__ void mk_epilogue_chunk(const MkParams& p, const MkPhase& ph, const Mk
   }
 }
 
+// Stores of 4 consecutive features (k % 4 == 0) of row j into the split hi/lo layout: they are
+// adjacent in the swizzled 64-element rows, so each part is one 8-byte store.
+__device__ __forceinline__ void store_split4(__nv_bfloat16* buf, const XsLayout& L, int j, int k, const float* x) {
+  uint32_t hi[2], lo[2];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    hi[i] = pack_bf16(x[2 * i], x[2 * i + 1]);
+    const float h0 = __uint_as_float(hi[i] << 16), h1 = __uint_as_float(hi[i] & 0xffff0000u);
+    lo[i] = pack_bf16(x[2 * i] - h0, x[2 * i + 1] - h1);
+  }
+  *reinterpret_cast<uint2*>(buf + xs_elem(L, j, k, 0)) = make_uint2(hi[0], hi[1]);
+  *reinterpret_cast<uint2*>(buf + xs_elem(L, j, k, 1)) = make_uint2(lo[0], lo[1]);
+}
+
+// Fix-up of tile t from the partials of contributors cf..cl (in that order) when the tile has
+// more than one 16-row chunk: warp q takes chunks q, q + 4, ... and each lane 4 adjacent
+// features of all 128, so that the partner elements of RoPE and SwiGLU and the reductions over
+// the tile's features (sums of squares, argmax) stay within one warp -- no exchange between the
+// warps and no barrier per chunk -- and every load and store is a 16- or 8-byte vector.
+__device__ void mk_finalize_by_warps(const MkParams& p, const MkPhase& ph, const MkEpi& e, int t, int cf, int cl,
+                                     const float* partials, int n_pad) {
+  const int lane = e.lane, f0 = 4 * lane;  // features f0 .. f0 + 3 of the tile
+  const int n_ch = (e.M + 15) >> 4;
+  const bool resid = ph.kind == kMkO || ph.kind == kMkDown;
+  float4 gn = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (resid && e.direct_xn) gn = *reinterpret_cast<const float4*>(e.gnext + t * 128 + f0);
+  for (int ch = e.q; ch < n_ch; ch += 4) {
+#pragma unroll 1
+    for (int hh = 0; hh < 2; ++hh) {
+      const int j0 = ch * 16 + hh * 8;
+      if (j0 >= e.M) break;
+      float v[8][4], hv[8][4];
+#pragma unroll
+      for (int jj = 0; jj < 8; ++jj) {
+        const bool in = j0 + jj < e.M;
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (resid && in) x = __ldcg(reinterpret_cast<const float4*>(p.h + static_cast<size_t>(e.rows[j0 + jj]) * p.d + t * 128 + f0));
+        hv[jj][0] = x.x; hv[jj][1] = x.y; hv[jj][2] = x.z; hv[jj][3] = x.w;
+        v[jj][0] = v[jj][1] = v[jj][2] = v[jj][3] = 0.f;
+      }
+      // contributors in order (deterministic sum), two partials' loads in flight at once
+      for (int c0 = cf; c0 <= cl; c0 += 2) {
+        float4 a[8], b[8];
+        const float* pa = partials + static_cast<size_t>(c0 + t) * 128 * n_pad;
+        const float* pb = pa + static_cast<size_t>(128) * n_pad;
+        const bool two = c0 + 1 <= cl;
+#pragma unroll
+        for (int jj = 0; jj < 8; ++jj) {
+          const bool in = j0 + jj < e.M;
+          a[jj] = in ? __ldcg(reinterpret_cast<const float4*>(pa + (j0 + jj) * 128 + f0)) : make_float4(0.f, 0.f, 0.f, 0.f);
+          b[jj] = in && two ? __ldcg(reinterpret_cast<const float4*>(pb + (j0 + jj) * 128 + f0))
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int jj = 0; jj < 8; ++jj) {
+          v[jj][0] = (v[jj][0] + a[jj].x) + b[jj].x;
+          v[jj][1] = (v[jj][1] + a[jj].y) + b[jj].y;
+          v[jj][2] = (v[jj][2] + a[jj].z) + b[jj].z;
+          v[jj][3] = (v[jj][3] + a[jj].w) + b[jj].w;
+        }
+      }
+#pragma unroll
+      for (int jj = 0; jj < 8; ++jj) {
+        const int j = j0 + jj;
+        const bool in = j < e.M;  // uniform over the warp
+        if (ph.kind == kMkQkv) {
+          const int d = p.d, D = p.D, half = D >> 1;
+          const int sec = (t * 128) / d;  // q, k or v: one per tile
+          const int fs = t * 128 + f0 - sec * d;
+          const int head = fs / D, dim0 = fs - head * D;
+          const float rsj = in ? e.rs[j] : 0.f;
+          float val[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) val[i] = v[jj][i] * rsj;
+          if (sec < 2) {  // rotate-half RoPE: the partner feature dim ^ half sits in lane ^ half / 4
+            float rot[4];
+            const int pos = in ? e.pos[j] : 0;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const float pv = __shfl_xor_sync(0xffffffffu, val[i], half >> 2);
+              const int ii = (dim0 + i) & (half - 1);
+              const float c = j < 16 ? e.rcos[j * half + ii] : __ldg(&p.rope_cos[static_cast<size_t>(pos) * half + ii]);
+              const float sn = j < 16 ? e.rsin[j * half + ii] : __ldg(&p.rope_sin[static_cast<size_t>(pos) * half + ii]);
+              rot[i] = dim0 < half ? val[i] * c - pv * sn : val[i] * c + pv * sn;
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) val[i] = rot[i];
+          }
+          if (in) {
+            if (sec == 0) {  // q in fp16 (11 significant bits), split exactly into bf16 hi + lo by the attention
+              const uint32_t w0 = pack_f16(val[0], val[1]), w1 = pack_f16(val[2], val[3]);
+              *reinterpret_cast<uint2*>(reinterpret_cast<__half*>(p.qbuf) + static_cast<size_t>(j) * d + fs) =
+                  make_uint2(w0, w1);
+            } else {
+              const size_t off = ((static_cast<size_t>(e.kvslot[j]) * 2 + (sec - 1)) * p.H + head) * e.kv_cap + e.kvrow[j];
+              *reinterpret_cast<uint2*>(e.kv_base + off * D + dim0) =
+                  make_uint2(pack_bf16(val[0], val[1]), pack_bf16(val[2], val[3]));
+            }
+          }
+        } else if (resid) {
+          float nv[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) nv[i] = hv[jj][i] + v[jj][i];
+          float sq = (nv[0] * nv[0] + nv[1] * nv[1]) + (nv[2] * nv[2] + nv[3] * nv[3]);
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+          if (in) {
+            const int m = e.rows[j];
+            *reinterpret_cast<float4*>(p.h + static_cast<size_t>(m) * p.d + t * 128 + f0) =
+                make_float4(nv[0], nv[1], nv[2], nv[3]);
+            if (e.direct_xn) {
+              const float xg[4] = {nv[0] * gn.x, nv[1] * gn.y, nv[2] * gn.z, nv[3] * gn.w};
+              store_split4(p.xn, p.xs, j, t * 128 + f0, xg);
+            }
+            if (lane == 0) p.ssp[static_cast<size_t>(t) * kMaxRows + m] = sq;
+          }
+        } else if (ph.kind == kMkGu) {  // lanes 0-15: gate features, 16-31: the matching up features
+          const float rsj = in ? e.rs[j] : 0.f;
+          float x[4], act[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            x[i] = v[jj][i] * rsj;
+            const float u = __shfl_xor_sync(0xffffffffu, x[i], 16);
+            act[i] = x[i] / (1.f + expf(-x[i])) * u;
+          }
+          if (in && lane < 16) store_split4(p.act, p.xs, j, t * 64 + f0, act);
+        } else {  // LM head: logits and the tile's argmax of row j, lowest index on ties
+          const float rsj = in ? e.rs[j] : 0.f;
+          float bv = -INFINITY;
+          int bi = t * 128 + f0;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int o = t * 128 + f0 + i;
+            const float val = o < p.V && in ? v[jj][i] * rsj : -INFINITY;
+            if (o < p.V && in) {
+              if (e.logits) e.logits[static_cast<size_t>(e.rows[j]) * p.V + o] = val;
+              if (val != val) report(p.status, kStatusCheck);
+            }
+            if (val > bv) {
+              bv = val;
+              bi = o;
+            }
+          }
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+            if (ov > bv || (ov == bv && oi < bi)) {
+              bv = ov;
+              bi = oi;
+            }
+          }
+          if (in && lane == 0) {
+            p.amax_val[static_cast<size_t>(t) * kMaxRows + e.rows[j]] = bv;
+            p.amax_idx[static_cast<size_t>(t) * kMaxRows + e.rows[j]] = bi;
+          }
+        }
+      }
+    }
+  }
+}
+
 // After a residual phase finalised tile t of h: write the next norm phase's B operand
 // bf16(h * g_next) for features [128t, 128t+128) of every row that phase runs, in its compacted
 // order (O -> gate/up of the same layer; down -> QKV of the next layer, or the LM head).
@@ -1036,6 +1198,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
                 for (int jj = 0; jj < 8; ++jj) v[jj] += pv[q][jj];
               if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 7);
               mk_epilogue_chunk(p, ph, e, t, r, 0, v);
+            } else if (e.M > 16) {
+              mk_finalize_by_warps(p, ph, e, t, cf, cl, partials, n_pad);
             } else {
               // contributors in order (deterministic sum), four partials' loads in flight at once
               const bool pre_h = (ph.kind == kMkO || ph.kind == kMkDown) && t != e.hpre_tile;
