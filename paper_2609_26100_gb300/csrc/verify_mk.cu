@@ -476,55 +476,55 @@ __device__ __forceinline__ void store_split4(__nv_bfloat16* buf, const XsLayout&
   *reinterpret_cast<uint2*>(buf + xs_elem(L, j, k, 1)) = make_uint2(lo[0], lo[1]);
 }
 
-// Fix-up of tile t from the partials of contributors cf..cl (in that order) when the tile has
-// more than one 16-row chunk: warp q takes chunks q, q + 4, ... and each lane 4 adjacent
-// features of all 128, so that the partner elements of RoPE and SwiGLU and the reductions over
-// the tile's features (sums of squares, argmax) stay within one warp -- no exchange between the
-// warps and no barrier per chunk -- and every load and store is a 16- or 8-byte vector.
+// Fix-up of tile t from the partials of contributors cf..cl (in that order): warp q takes the
+// groups of G rows q, q + 4, ... and each lane 4 adjacent features of all 128, so that the
+// partner elements of RoPE and SwiGLU and the reductions over the tile's features (sums of
+// squares, argmax) stay within one warp -- no exchange between the warps and no barrier -- and
+// every load and store is a 16- or 8-byte vector.  CB contributors' partials per round of loads.
+template <int G, int CB>
 __device__ void mk_finalize_by_warps(const MkParams& p, const MkPhase& ph, const MkEpi& e, int t, int cf, int cl,
                                      const float* partials, int n_pad) {
   const int lane = e.lane, f0 = 4 * lane;  // features f0 .. f0 + 3 of the tile
-  const int n_ch = (e.M + 15) >> 4;
+  const int n_groups = (e.M + G - 1) / G;
   const bool resid = ph.kind == kMkO || ph.kind == kMkDown;
   float4 gn = make_float4(0.f, 0.f, 0.f, 0.f);
   if (resid && e.direct_xn) gn = *reinterpret_cast<const float4*>(e.gnext + t * 128 + f0);
-  for (int ch = e.q; ch < n_ch; ch += 4) {
-#pragma unroll 1
-    for (int hh = 0; hh < 2; ++hh) {
-      const int j0 = ch * 16 + hh * 8;
-      if (j0 >= e.M) break;
-      float v[8][4], hv[8][4];
+  for (int grp = e.q; grp < n_groups; grp += 4) {
+    {
+      const int j0 = grp * G;
+      float v[G][4], hv[G][4];
 #pragma unroll
-      for (int jj = 0; jj < 8; ++jj) {
+      for (int jj = 0; jj < G; ++jj) {
         const bool in = j0 + jj < e.M;
         float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
         if (resid && in) x = __ldcg(reinterpret_cast<const float4*>(p.h + static_cast<size_t>(e.rows[j0 + jj]) * p.d + t * 128 + f0));
         hv[jj][0] = x.x; hv[jj][1] = x.y; hv[jj][2] = x.z; hv[jj][3] = x.w;
         v[jj][0] = v[jj][1] = v[jj][2] = v[jj][3] = 0.f;
       }
-      // contributors in order (deterministic sum), two partials' loads in flight at once
-      for (int c0 = cf; c0 <= cl; c0 += 2) {
-        float4 a[8], b[8];
-        const float* pa = partials + static_cast<size_t>(c0 + t) * 128 * n_pad;
-        const float* pb = pa + static_cast<size_t>(128) * n_pad;
-        const bool two = c0 + 1 <= cl;
+      // contributors in order (deterministic sum), CB partials' loads in flight at once
+      for (int c0 = cf; c0 <= cl; c0 += CB) {
+        float4 a[CB][G];
 #pragma unroll
-        for (int jj = 0; jj < 8; ++jj) {
-          const bool in = j0 + jj < e.M;
-          a[jj] = in ? __ldcg(reinterpret_cast<const float4*>(pa + (j0 + jj) * 128 + f0)) : make_float4(0.f, 0.f, 0.f, 0.f);
-          b[jj] = in && two ? __ldcg(reinterpret_cast<const float4*>(pb + (j0 + jj) * 128 + f0))
-                            : make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int q = 0; q < CB; ++q) {
+          const bool cin = c0 + q <= cl;
+          const float* pa = partials + static_cast<size_t>(c0 + q + t) * 128 * n_pad;
+#pragma unroll
+          for (int jj = 0; jj < G; ++jj)
+            a[q][jj] = cin && j0 + jj < e.M ? __ldcg(reinterpret_cast<const float4*>(pa + (j0 + jj) * 128 + f0))
+                                            : make_float4(0.f, 0.f, 0.f, 0.f);
         }
 #pragma unroll
-        for (int jj = 0; jj < 8; ++jj) {
-          v[jj][0] = (v[jj][0] + a[jj].x) + b[jj].x;
-          v[jj][1] = (v[jj][1] + a[jj].y) + b[jj].y;
-          v[jj][2] = (v[jj][2] + a[jj].z) + b[jj].z;
-          v[jj][3] = (v[jj][3] + a[jj].w) + b[jj].w;
-        }
+        for (int q = 0; q < CB; ++q)
+#pragma unroll
+          for (int jj = 0; jj < G; ++jj) {
+            v[jj][0] += a[q][jj].x;
+            v[jj][1] += a[q][jj].y;
+            v[jj][2] += a[q][jj].z;
+            v[jj][3] += a[q][jj].w;
+          }
       }
 #pragma unroll
-      for (int jj = 0; jj < 8; ++jj) {
+      for (int jj = 0; jj < G; ++jj) {
         const int j = j0 + jj;
         const bool in = j < e.M;  // uniform over the warp
         if (ph.kind == kMkQkv) {
@@ -1179,27 +1179,11 @@ __global__ void __launch_bounds__(kMkThreads, 1)
             }
             if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 3);
             if (e.M <= 8 && cl - cf < 8) {
-              // up to 8 rows and 8 contributors: every partial in one round of loads, then the
-              // same sum in contributor order (an absent contributor adds an exact 0)
-              float pv[8][8];
-#pragma unroll
-              for (int q = 0; q < 8; ++q) {
-                const bool cin = cf + q <= cl;
-                const float* pa = partials + static_cast<size_t>(cf + q + t) * 128 * n_pad;
-#pragma unroll
-                for (int jj = 0; jj < 8; ++jj) pv[q][jj] = cin && jj < e.M ? __ldcg(&pa[jj * 128 + r]) : 0.f;
-              }
-              float v[16];
-#pragma unroll
-              for (int jj = 0; jj < 16; ++jj) v[jj] = 0.f;
-#pragma unroll
-              for (int q = 0; q < 8; ++q)
-#pragma unroll
-                for (int jj = 0; jj < 8; ++jj) v[jj] += pv[q][jj];
+              // up to 8 rows and 8 contributors: every partial in one round of loads, two rows a warp
+              mk_finalize_by_warps<2, 8>(p, ph, e, t, cf, cl, partials, n_pad);
               if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 7);
-              mk_epilogue_chunk(p, ph, e, t, r, 0, v);
             } else if (e.M > 16) {
-              mk_finalize_by_warps(p, ph, e, t, cf, cl, partials, n_pad);
+              mk_finalize_by_warps<8, 2>(p, ph, e, t, cf, cl, partials, n_pad);
             } else {
               // contributors in order (deterministic sum), four partials' loads in flight at once
               const bool pre_h = (ph.kind == kMkO || ph.kind == kMkDown) && t != e.hpre_tile;
