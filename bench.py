@@ -47,8 +47,9 @@ def parse_args():
     p.add_argument("--prefill", type=int, default=None,
                    help="prompt tokens per request: time tss_prefill on the 7B chain's skip set (4 requests) "
                         "instead of the verification step")
-    p.add_argument("--traffic", default=os.path.join(ROOT, "profiles", "verify_persistent_7b_chain_traffic.txt"),
-                   help="JSON summary of an ncu DRAM-traffic capture of the dominant kernel")
+    p.add_argument("--traffic", default=os.path.join(ROOT, "profiles"),
+                   help="JSON summary of an ncu DRAM-traffic capture of the dominant kernel, or a directory "
+                        "whose *_traffic.txt files are such summaries")
     return p.parse_args()
 
 
@@ -141,19 +142,43 @@ class ClockSampler:
                 "power_w_max": max(float(r[3]) for r in rows if r[3].replace(".", "").isdigit())}
 
 
-def kernel_sources_hash():
-    """sha256 over the code of the persistent verify kernel's sources, comments and blank lines
-    left out (an ncu traffic figure is only valid for the kernel it was taken on)."""
+# Sources of each kernel kind whose ncu traffic figure bench.py may reuse.
+KERNEL_SOURCES = {
+    "verify_persistent": ("verify_mk.cu", "attn_body.cuh", "common.cuh", "internal.h"),
+    "attention": ("attention.cu", "attn_body.cuh", "common.cuh", "internal.h"),
+}
+
+
+def kernel_sources_hash(kernel="verify_persistent"):
+    """sha256 over the code of a kernel's sources, comments and blank lines left out (an ncu
+    traffic figure is only valid for the kernel it was taken on)."""
     import hashlib
     import re
     h = hashlib.sha256()
-    for f in ("verify_mk.cu", "attn_body.cuh", "common.cuh", "internal.h"):
+    for f in KERNEL_SOURCES[kernel]:
         with open(os.path.join(ROOT, "paper_2609_26100_gb300", "csrc", f), encoding="utf-8") as fh:
             for line in fh:
                 code = re.sub(r"(^|\s)//.*$", "", line.rstrip("\n")).rstrip()
                 if code:
                     h.update(code.encode() + b"\n")
     return h.hexdigest()
+
+
+def find_traffic(path, kernel, workload):
+    """DRAM bytes per launch of `kernel` on `workload` from an ncu capture summary (JSON with
+    "kernel", "workload", "traffic_bytes" and "sources_sha256", the hash of the kernel sources
+    it was taken on); None unless one matches the workload and the unchanged sources."""
+    import glob
+    if not path or not os.path.exists(path) or kernel not in KERNEL_SOURCES:
+        return None
+    files = sorted(glob.glob(os.path.join(path, "*_traffic.txt"))) if os.path.isdir(path) else [path]
+    for fn in files:
+        with open(fn) as f:
+            tr = json.load(f)
+        if (tr.get("kernel") == kernel and tr.get("workload") == workload
+                and tr.get("sources_sha256") == kernel_sources_hash(kernel)):
+            return tr
+    return None
 
 
 def kernel_bytes(w, kinds):
@@ -453,15 +478,10 @@ def run_tss(args):
                     "frac": ach / peak, "peak_source": f"{peak_kind} copy bandwidth",
                     "frac_of_nominal_8TBs": ach / NOMINAL_HBM_GBS,
                     "bytes_per_launch": kb[dom] / kernels[dom]["launches_per_step"], "traffic": None}
-        if args.traffic and os.path.exists(args.traffic):
-            # DRAM bytes per launch of this kernel from an ncu capture (a summary with "kernel",
-            # "workload", "traffic_bytes" and the hash of the kernel sources it was taken on);
-            # used only for the same workload and unchanged kernel sources
-            with open(args.traffic) as f:
-                tr = json.load(f)
-            if tr.get("kernel") == dom and tr.get("workload") == w.name and tr.get("sources_sha256") == kernel_sources_hash():
-                roofline["traffic"] = tr["traffic_bytes"]
-                roofline["traffic_source"] = tr.get("source")
+        tr = find_traffic(args.traffic, dom, w.name)
+        if tr is not None:
+            roofline["traffic"] = tr["traffic_bytes"]
+            roofline["traffic_source"] = tr.get("source")
         if args.no_profile:
             kernels = None
             roofline = None

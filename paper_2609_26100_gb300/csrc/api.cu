@@ -127,6 +127,7 @@ struct tss_ctx {
   int w_evict_first = 1;
   int mk_max_stages = 12;
   int attn_plo = 1;
+  int attn_splits_force = 0;  // > 0: key splits of the separate attention kernel (TSS_ATTN_SPLITS)
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
   unsigned long long epoch = 0;
   float* ssp = nullptr;
@@ -381,6 +382,37 @@ int mk_attn_splits(const tss_ctx* c, int B, int tiles) {
     if (sl > 1 && sl > tiles) break;
     const long long waves = (static_cast<long long>(pairs) * sl + c->num_sms - 1) / c->num_sms;
     const long long cost = waves * ((tiles + sl - 1) / sl + 3);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = sl;
+    }
+  }
+  return best;
+}
+
+// Key splits per (request, head) for the separate attention kernel (two CTAs per SM).  In units
+// of one CTA scoring one 64-key tile, the launch takes about the larger of the mean load of a CTA
+// slot and the longest item, and every item costs about kItemTiles more for its set-up and the
+// merge of the splits.  The fewest splits on ties.  In a batch of ragged contexts this splits the
+// long requests' items so that they no longer set the length of the launch (13B batch of
+// contexts 644-3059: two splits, 98.6 vs 115.1 us per layer); equal long contexts keep one.
+int ext_attn_splits(const tss_ctx* c, const StepDesc* sd, int B) {
+  constexpr long long kItemTiles = 3;
+  const long long slots = 2LL * c->num_sms;
+  int max_tiles = 1;
+  for (int b = 0; b < B; ++b) max_tiles = std::max(max_tiles, (sd->req_ctx[b] + sd->req_nodes[b] + 63) / 64);
+  int best = 1;
+  long long best_cost = -1;
+  for (int sl = 1; sl <= c->max_splits && (sl == 1 || sl <= max_tiles); ++sl) {
+    long long work = 0, longest = 0;
+    for (int b = 0; b < B; ++b) {
+      const long long t = (sd->req_ctx[b] + sd->req_nodes[b] + 63) / 64;
+      const long long per = (t + sl - 1) / sl;
+      const long long items = per > 0 ? (t + per - 1) / per : 0;
+      work += c->H * (t + items * kItemTiles);
+      longest = std::max(longest, per + kItemTiles);
+    }
+    const long long cost = std::max((work + slots - 1) / slots, longest);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
       best = sl;
@@ -831,11 +863,8 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
   sd->off_lo = static_cast<uint32_t>(bt->philox_offset);
   sd->off_hi = static_cast<uint32_t>(bt->philox_offset >> 32);
   for (int l = 0; l < c->L; ++l) sd->kv_layer[l] = static_cast<__nv_bfloat16*>(kv->layer[l]);
-  // attention splits: aim for ~2 CTAs per SM; bucketed so graphs are reused as contexts grow
-  int tiles = (max_t + 63) / 64, tb = 1;
-  while (tb < tiles) tb <<= 1;
-  const int want = (2 * c->num_sms + B * c->H - 1) / (B * c->H);
-  int splits = std::max(1, std::min(std::min(want, c->max_splits), tb));
+  const int tiles = (max_t + 63) / 64;
+  const int splits = c->attn_splits_force > 0 ? std::min(c->attn_splits_force, c->max_splits) : ext_attn_splits(c, sd, B);
   sp->B = B;
   sp->M = M;
   sp->n_act = n_act;
@@ -903,6 +932,7 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_MK_KPS")) c->mk_kps = std::min(8, std::max(1, std::atoi(e)));
   if (const char* e = std::getenv("TSS_EVICT_FIRST")) c->w_evict_first = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ATTN_PLO")) c->attn_plo = std::atoi(e) != 0;
+  if (const char* e = std::getenv("TSS_ATTN_SPLITS")) c->attn_splits_force = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
   const char* trace_env = std::getenv("TSS_TRACE");
   tss_status s = build_workspaces(c);

@@ -249,13 +249,23 @@ __device__ __forceinline__ T block_reduce(T v, T* red, Op op) {
 // u * sum(w).  Each thread owns a contiguous chunk; chunk sums are scanned in thread order.
 // fp32 throughout: the sums over a 32k vocabulary are accurate to ~1e-6 of the mass, far inside
 // the 2e-4 band within which a draw counts as consistent, and fp64 is slow on this GPU.
+// Loads of the vocabulary passes are issued kLoadBatch at a time (one round trip per batch
+// instead of one per element); every sum keeps the element order of a plain loop.
+constexpr int kLoadBatch = 16;
+
 template <typename WFn>
 __device__ int inverse_cdf_block(int V, float u, WFn w, float* scan) {
   const int nt = blockDim.x, t = threadIdx.x;
   const int C = (V + nt - 1) / nt;
   const int v0 = min(V, t * C), v1 = min(V, v0 + C);
   float local = 0.f;
-  for (int v = v0; v < v1; ++v) local += w(v);
+  for (int b0 = v0; b0 < v1; b0 += kLoadBatch) {
+    float x[kLoadBatch];
+#pragma unroll
+    for (int j = 0; j < kLoadBatch; ++j) x[j] = b0 + j < v1 ? w(b0 + j) : 0.f;
+#pragma unroll
+    for (int j = 0; j < kLoadBatch; ++j) local += x[j];  // x + 0 == x: the order of a plain loop
+  }
   // exclusive scan of the chunk sums in thread order: warp scans, then the warp totals
   const int lane = t & 31, warp = t >> 5, nw = nt >> 5;
   float incl = local;
@@ -337,11 +347,25 @@ __device__ void accept_sample_body(const MiscParams& p, int b) {
   for (int i = 0; i < N; ++i) path[i] = i;
   for (int i = 1; i <= k + 1; ++i) {
     const float* lg = st->logits + static_cast<size_t>(off + i - 1) * V;
+    const int nt = blockDim.x;
     float mx = -INFINITY;
-    for (int v = threadIdx.x; v < V; v += blockDim.x) mx = fmx(mx, lg[v]);
+    for (int b0 = threadIdx.x; b0 < V; b0 += kLoadBatch * nt) {
+      float x[kLoadBatch];
+#pragma unroll
+      for (int j = 0; j < kLoadBatch; ++j) x[j] = b0 + j * nt < V ? lg[b0 + j * nt] : -INFINITY;
+#pragma unroll
+      for (int j = 0; j < kLoadBatch; ++j) mx = fmx(mx, x[j]);
+    }
     mx = block_reduce(mx, redf, fmx);
     float z = 0.f;
-    for (int v = threadIdx.x; v < V; v += blockDim.x) z += expf((lg[v] - mx) * invT);
+    for (int b0 = threadIdx.x; b0 < V; b0 += kLoadBatch * nt) {
+      float x[kLoadBatch];
+#pragma unroll
+      for (int j = 0; j < kLoadBatch; ++j) x[j] = b0 + j * nt < V ? lg[b0 + j * nt] : 0.f;
+#pragma unroll
+      for (int j = 0; j < kLoadBatch; ++j)
+        if (b0 + j * nt < V) z += expf((x[j] - mx) * invT);
+    }
     z = block_reduce(z, redf, fsum);
     const float invz = 1.f / z;
     auto pr = [&](int v) { return expf((lg[v] - mx) * invT) * invz; };
@@ -373,7 +397,7 @@ __device__ void accept_sample_body(const MiscParams& p, int b) {
   if (threadIdx.x == 0) write_result(p, b, a, bonus, path);
 }
 
-__global__ void accept_sample_kernel(const MiscParams p) {
+__global__ void __launch_bounds__(1024) accept_sample_kernel(const MiscParams p) {
   griddep_wait();
   griddep_launch();
   if (blockIdx.x >= p.step->B) return;
