@@ -21,7 +21,7 @@ Domain-Specific Large Language Models":
   sampling of the works the paper cites for speculative decoding (Leviathan et al. 2023,
   Chen et al. 2023).
 
-Readings of points the paper leaves open (each is listed in the design doc):
+Readings of points the paper leaves open:
 * layer indices are 0-based; RoPE uses the "rotate-half" pairing (i, i + D/2) with
   inv_freq_i = theta^(-2i/D), angles in float64;
 * new K and V rows are rounded to bf16 before they are stored or attended (storage precision);

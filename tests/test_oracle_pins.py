@@ -68,8 +68,10 @@ def test_rmsnorm_closed_forms():
     c = np.full((1, 64), -2.5)
     g = np.linspace(0.5, 1.5, 64)
     assert np.allclose(O.rms_norm(c, g, 0.0), -g, atol=1e-15)
-    # eps enters under the square root: a zero row stays zero, finite
+    # eps enters under the square root: a zero row stays zero, finite, and (3, 4) with eps = 0.5
+    # divides by sqrt(12.5 + 0.5), not by sqrt(12.5) + 0.5
     assert np.all(O.rms_norm(np.zeros((1, 8)), np.ones(8), 1e-5) == 0)
+    assert np.allclose(O.rms_norm(h, np.ones(2), 0.5), [[3 / math.sqrt(13.0), 4 / math.sqrt(13.0)]], rtol=0, atol=1e-15)
 
 
 def test_rope_is_complex_rotation_of_half_pairs():
