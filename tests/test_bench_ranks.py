@@ -53,3 +53,17 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
     args = bench.parse_args()
     bench.run_reference(args)
     assert capsys.readouterr().out == ""
+
+
+def test_traffic_record_needs_same_kernel_workload_and_sources(tmp_path):
+    rec = {"kernel": "attention", "workload": "7b_long", "traffic_bytes": 123,
+           "sources_sha256": bench.kernel_sources_hash("attention")}
+    (tmp_path / "a_traffic.txt").write_text(json.dumps(rec))
+    assert bench.find_traffic(str(tmp_path), "attention", "7b_long")["traffic_bytes"] == 123
+    assert bench.find_traffic(str(tmp_path / "a_traffic.txt"), "attention", "7b_long") is not None
+    assert bench.find_traffic(str(tmp_path), "attention", "13b_mixed") is None
+    assert bench.find_traffic(str(tmp_path), "verify_persistent", "7b_long") is None
+    (tmp_path / "a_traffic.txt").write_text(json.dumps(dict(rec, sources_sha256="0" * 64)))
+    assert bench.find_traffic(str(tmp_path), "attention", "7b_long") is None  # kernel changed since
+    # the hash ignores comments and blank lines but not code
+    assert bench.kernel_sources_hash("attention") != bench.kernel_sources_hash("verify_persistent")
