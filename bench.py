@@ -42,8 +42,8 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-profile", action="store_true")
     p.add_argument("--sweep", default=None,
-                   help="7b_long: comma-separated skipped-layer counts (e.g. 0,2,4,...,12); one process, one "
-                        "weight and KV set, latency vs active layers with a least-squares line")
+                   help="7b_long or 7b_chain: comma-separated skipped-layer counts (e.g. 0,2,4,...,12); one "
+                        "process, one weight and KV set, latency vs active layers with a least-squares line")
     p.add_argument("--prefill", type=int, default=None,
                    help="prompt tokens per request: time tss_prefill on the 7B chain's skip set (4 requests) "
                         "instead of the verification step")
@@ -519,12 +519,31 @@ def run_tss(args):
         dist.destroy_process_group()
 
 
+def sweep_workload(name, n_skip):
+    """Workload of a sweep point: the KV-bound 7B workload (B=16, ctx 16384, k=8) or the 7B chain
+    (B=1, ctx 1024, k=5), with the first n_skip layers of one seeded permutation of layers 1..31
+    skipped (nested sets, so each point adds layers to the previous one's skip set)."""
+    from paper_2609_26100_gb300 import synth
+    if name == "7b_long":
+        return synth.workload_7b_long(n_skip=n_skip)
+    if name == "7b_chain":
+        perm = synth.seeded_permutation(list(range(1, synth.LLAMA2_7B.n_layers)), synth.DEFAULT_SEED, "7b_long.perm")
+        return synth.workload_7b_chain(mask_layers=sorted(perm[:n_skip]))
+    raise ValueError(f"--sweep supports the 7b_long and 7b_chain workloads, not {name}")
+
+
+SWEEP_METRIC = {
+    "7b_long": "7B KV-bound verify latency vs active layers (B=16, ctx 16384, k=8)",
+    "7b_chain": "7B chain verify latency vs active layers (B=1, ctx 1024, k=5): the verification cost C_d(S)",
+}
+
+
 def run_sweep(args):
-    """Verify latency of the KV-bound 7B workload (B=16, ctx 16384, k=8) against the number of
-    active layers: the skip sets are nested prefixes of one seeded permutation, the weights and
-    the context KV of every layer are generated once, and each point is timed with CUDA events.
-    Prints one JSON line: the points, the least-squares line (slope, intercept, R^2) and each
-    point's bytes against the measured and nominal HBM peaks."""
+    """Verify latency against the number of active layers (the verification cost of a skip set,
+    the C_d term of the paper's search objective): the skip sets are nested prefixes of one seeded
+    permutation, the weights and the context KV of every layer are generated once, and each point
+    is timed with CUDA events.  Prints one JSON line: the points, the least-squares line (slope,
+    intercept, R^2) and each point's bytes against the measured and nominal HBM peaks."""
     import torch
     from paper_2609_26100_gb300 import build as _build
     from paper_2609_26100_gb300 import native, synth
@@ -532,13 +551,14 @@ def run_sweep(args):
     torch.cuda.set_device(0)
     _build.build()
     counts = [int(x) for x in args.sweep.split(",")]
-    dense = synth.workload_7b_long(n_skip=0)
+    name = args.workload if args.workload in SWEEP_METRIC else "7b_long"
+    dense = sweep_workload(name, 0)
     run = TssRunner.for_workload(dense)
     stream = torch.cuda.current_stream()
     peak, _ = measured_peak()
     points = []
     for n in counts:
-        w = synth.workload_7b_long(n_skip=n)
+        w = sweep_workload(name, n)
         run.set_phi(w.phi)
         res = run.alloc_results(len(w.requests), w.n_rows, logits=False)
         b = run.batch(w.requests)
@@ -571,7 +591,7 @@ def run_sweep(args):
     ss_tot = sum((y - my) ** 2 for y in ys)
     ss_res = sum((y - (icpt + slope * x)) ** 2 for x, y in zip(xs, ys))
     r2 = 1.0 - ss_res / ss_tot if ss_tot > 0 else 1.0
-    print(json.dumps({"metric": "7B KV-bound verify latency vs active layers (B=16, ctx 16384, k=8)",
+    print(json.dumps({"metric": SWEEP_METRIC[name], "workload": name,
                       "unit": "us/step", "higher_is_better": False, "steps": args.steps, "points": points,
                       "fit": {"slope_us_per_layer": slope, "intercept_us": icpt, "r2": r2},
                       "data": "synthetic (seeded random-init weights, synthetic KV)"}))

@@ -166,10 +166,13 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
 
 /* Phi(domain_id) = the set of layers whose bit is set in layer_bitmask (bit l = skip layer l;
  * 0 = dense).  Sec. "Domain-to-Configuration Mapping".  Bits >= n_layers must be clear.
- * Synchronous; affects verifies enqueued after it returns.  domain_id in [0, max_domains). */
+ * Synchronous: waits for all work on the device first (so a verify already enqueued runs under
+ * the configuration it was planned with), then affects verifies enqueued after it returns.
+ * domain_id in [0, max_domains).  Not for use during stream capture. */
 tss_status tss_set_skip_config(tss_ctx* ctx, int domain_id, uint64_t layer_bitmask);
 
-/* Remove domain_id from Phi: its requests then run the dense path (unsupported domain). */
+/* Remove domain_id from Phi: its requests then run the dense path (unsupported domain).
+ * Synchronises the device as tss_set_skip_config does. */
 tss_status tss_clear_skip_config(tss_ctx* ctx, int domain_id);
 
 /* Sparsity ratio R_d = |S_d| / L of a configured domain (0 for an unconfigured one), and the

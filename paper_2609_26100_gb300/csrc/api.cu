@@ -963,6 +963,9 @@ tss_status tss_set_skip_config(tss_ctx* c, int domain_id, uint64_t mask) {
   if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
   if (domain_id < 0 || domain_id >= c->a.max_domains) return fail(TSS_ERR_INVALID_ARG, "domain_id out of range");
   if (c->L < 64 && (mask >> c->L) != 0ull) return fail(TSS_ERR_INVALID_ARG, "skip mask names a layer >= n_layers");
+  // A step already enqueued reads Phi on the device when it runs, but planned its launches from
+  // the host copy when it was enqueued: let every such step finish before either copy changes.
+  TSS_CU(cudaDeviceSynchronize());
   c->phi[domain_id] = mask;
   c->phi_valid[domain_id] = 1;
   const int one = 1;
@@ -975,6 +978,7 @@ tss_status tss_set_skip_config(tss_ctx* c, int domain_id, uint64_t mask) {
 tss_status tss_clear_skip_config(tss_ctx* c, int domain_id) {
   if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
   if (domain_id < 0 || domain_id >= c->a.max_domains) return fail(TSS_ERR_INVALID_ARG, "domain_id out of range");
+  TSS_CU(cudaDeviceSynchronize());  // as in tss_set_skip_config
   c->phi[domain_id] = 0ull;
   c->phi_valid[domain_id] = 0;
   const int zero = 0;
