@@ -48,3 +48,36 @@ def test_status_strings_without_gpu(libtss):
 def test_library_built_for_sm103a_only():
     from paper_2609_26100_gb300 import build
     assert build.ARCH == ("-gencode", "arch=compute_103a,code=sm_103a")
+
+
+def test_header_is_c99_and_a_c_program_links_and_runs(libtss, tmp_path):
+    """A plain C program includes the header, takes the address of every declared entry point,
+    links against libtss.so and calls tss_status_string (no CUDA call)."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    from paper_2609_26100_gb300 import build
+    lib = build.build()
+    names = _declared()
+    src = ["#include \"tss.h\"", "#include <stdio.h>", "#include <string.h>",
+           "typedef void (*fnp)(void);",
+           "static const fnp table[] = {" + ", ".join(f"(fnp){n}" for n in names) + "};",
+           "int main(void) {",
+           "  if (strcmp(tss_status_string(TSS_OK), \"ok\") != 0) return 1;",
+           "  for (size_t i = 0; i < sizeof(table) / sizeof(table[0]); ++i) if (!table[i]) return 2;",
+           "  printf(\"%d\\n\", (int)(sizeof(table) / sizeof(table[0])));",
+           "  return 0;",
+           "}"]
+    c = tmp_path / "abi.c"
+    c.write_text("\n".join(src) + "\n")
+    exe = tmp_path / "abi"
+    libdir = os.path.dirname(lib)
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-I", os.path.join(ROOT, "include"), str(c),
+                        "-o", str(exe), "-L", libdir, "-l:libtss.so", f"-Wl,-rpath,{libdir}"],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    r = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    assert int(r.stdout) == len(names)
