@@ -161,7 +161,10 @@ typedef struct {
 
 /* Build a verifier on the current CUDA device (must be sm_103).  Copies and repacks the weights
  * into library-owned device memory, allocates every workspace for the limits in *arch, and
- * returns an opaque context.  Errors: INVALID_ARG, UNSUPPORTED_ARCH, OUT_OF_MEMORY, CUDA. */
+ * returns an opaque context.  Errors: INVALID_ARG, UNSUPPORTED_ARCH, OUT_OF_MEMORY, CUDA; on
+ * error everything allocated so far is freed and *out is NULL.  For failure injection, the
+ * environment variable TSS_ALLOC_LIMIT_BYTES=N makes the allocations fail with OUT_OF_MEMORY
+ * once they would pass N bytes. */
 tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx** out);
 
 /* Phi(domain_id) = the set of layers whose bit is set in layer_bitmask (bit l = skip layer l;

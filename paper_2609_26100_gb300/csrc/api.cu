@@ -137,15 +137,22 @@ struct tss_ctx {
   float *mk_part0 = nullptr, *mk_part1 = nullptr;
   size_t mk_part_floats = 0;
   std::vector<void*> allocs;
+  size_t allocated = 0;    // bytes allocated by alloc()
+  size_t alloc_limit = 0;  // > 0: alloc() fails beyond this many bytes (TSS_ALLOC_LIMIT_BYTES)
 
   template <typename T>
   tss_status alloc(T** p, size_t count) {
+    const size_t bytes = count * sizeof(T) + 16;
+    if (alloc_limit != 0 && allocated + bytes > alloc_limit)
+      return fail(TSS_ERR_OUT_OF_MEMORY, "allocating " + std::to_string(bytes) + " more bytes would exceed the limit of " +
+                                             std::to_string(alloc_limit) + " (TSS_ALLOC_LIMIT_BYTES)");
     void* q = nullptr;
-    if (cudaMalloc(&q, count * sizeof(T) + 16) != cudaSuccess) {
+    if (cudaMalloc(&q, bytes) != cudaSuccess) {
       cudaGetLastError();
       return fail(TSS_ERR_OUT_OF_MEMORY, "cudaMalloc of " + std::to_string(count * sizeof(T)) + " bytes failed");
     }
     allocs.push_back(q);
+    allocated += bytes;
     *p = static_cast<T*>(q);
     return TSS_OK;
   }
@@ -934,6 +941,7 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_ATTN_PLO")) c->attn_plo = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ATTN_SPLITS")) c->attn_splits_force = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
+  if (const char* e = std::getenv("TSS_ALLOC_LIMIT_BYTES")) c->alloc_limit = std::strtoull(e, nullptr, 10);
   const char* trace_env = std::getenv("TSS_TRACE");
   tss_status s = build_workspaces(c);
   if (s == TSS_OK) s = build_weights(c, weights);

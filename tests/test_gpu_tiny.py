@@ -538,3 +538,19 @@ def test_sparsity_ratio_and_active_layers(weights):
     run.v.clear_skip_config(1)
     assert run.v.active_layer_count(b) == 4
     run.close()
+
+
+def test_create_reports_out_of_memory_under_an_allocation_limit(weights, monkeypatch):
+    """Failure injection on the host: with TSS_ALLOC_LIMIT_BYTES below what tss_create needs, the
+    call returns TSS_ERR_OUT_OF_MEMORY, frees what it had allocated, and a later create without
+    the limit succeeds."""
+    _, _, wg = weights
+    monkeypatch.setenv("TSS_ALLOC_LIMIT_BYTES", str(1 << 20))
+    with pytest.raises(native.TssError) as err:
+        native.Verifier(wg, ARCH, max_batch=1, max_rows=8, max_nodes=8)
+    assert err.value.status == native.TSS_ERR_OUT_OF_MEMORY
+    assert "TSS_ALLOC_LIMIT_BYTES" in str(err.value)
+    monkeypatch.delenv("TSS_ALLOC_LIMIT_BYTES")
+    v = native.Verifier(wg, ARCH, max_batch=1, max_rows=8, max_nodes=8)
+    v.close()
+
