@@ -58,6 +58,14 @@ class TssRunner:
         for dom, mask in phi.items():
             self.v.set_skip_config(int(dom), int(mask))
 
+    def load_phi(self, path: str) -> Dict[int, int]:
+        """Apply the skip configurations of a configuration file (phi_config format) for this
+        model's layer count; returns the domain -> bitmask map that was set."""
+        from . import phi_config
+        phi = phi_config.masks(phi_config.load(path, self.arch.n_layers))
+        self.set_phi(phi)
+        return phi
+
     def write_kv(self, layer: int, slot: int, k: torch.Tensor, v: torch.Tensor, pos0: int = 0) -> None:
         """k, v: [H, n, D] values for positions [pos0, pos0 + n)."""
         n = k.shape[1]
