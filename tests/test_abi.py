@@ -81,3 +81,39 @@ def test_header_is_c99_and_a_c_program_links_and_runs(libtss, tmp_path):
     r = subprocess.run([str(exe)], capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
     assert int(r.stdout) == len(names)
+
+
+def test_binding_structs_match_the_c_layout(tmp_path):
+    """Every ctypes structure of the binding has the size and field offsets that a C compiler gives
+    the struct of the same name in tss.h (a field added, dropped or reordered on one side fails)."""
+    import shutil
+    import subprocess
+    from paper_2609_26100_gb300 import native
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    structs = {"tss_arch": native.TssArch, "tss_weights": native.TssWeights, "tss_verify_batch": native.TssVerifyBatch,
+               "tss_kv_cache": native.TssKvCache, "tss_verify_result": native.TssVerifyResult,
+               "tss_kernel_times": native.TssKernelTimes}
+    lines = ["#include \"tss.h\"", "#include <stdio.h>", "#include <stddef.h>", "int main(void) {"]
+    for cname, py in structs.items():
+        lines.append(f"  printf(\"{cname} size %zu\\n\", sizeof({cname}));")
+        for fname, _ in py._fields_:
+            lines.append(f"  printf(\"{cname} {fname} %zu\\n\", offsetof({cname}, {fname}));")
+    lines += ["  return 0;", "}"]
+    c = tmp_path / "layout.c"
+    c.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Werror", "-I", os.path.join(ROOT, "include"), str(c), "-o", str(exe)],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split("\n")
+    got = {}
+    for ln in out:
+        if ln:
+            cname, field, val = ln.split()
+            got[(cname, field)] = int(val)
+    for cname, py in structs.items():
+        assert got[(cname, "size")] == ctypes.sizeof(py), cname
+        for fname, _ in py._fields_:
+            assert got[(cname, fname)] == getattr(py, fname).offset, f"{cname}.{fname}"
