@@ -183,6 +183,24 @@ tss_status tss_clear_skip_config(tss_ctx* ctx, int domain_id);
 tss_status tss_sparsity_ratio(const tss_ctx* ctx, int domain_id, double* out);
 tss_status tss_active_layer_count(const tss_ctx* ctx, const tss_verify_batch* batch, int* out);
 
+/* Bytes a verification step must move through HBM, the numerator of its roofline.  On this
+ * memory-bound path the verification cost C_d(S) of Sec. "Problem Formulation" is proportional
+ * to it, so an offline search over skip sets can rank candidates without running them.
+ *   weights  = |union of the requests' active layers| x 2(4 d^2 + 3 d d_mlp)  +  vocab x d x 2
+ *              (every active layer's weights and the LM head, read once per step);
+ *   kv_read  = sum over requests of ctx_len x (layers it runs) x 4 d   (its context K and V);
+ *   kv_write = sum over requests of n_nodes x (layers it runs) x 4 d   (the rows it appends);
+ *   total    = weights + kv_read + kv_write; active_union = the size of the union.
+ * masks[n_req] (bit l set = request skips layer l, i.e. S(x)), ctx_len[n_req] and
+ * n_nodes[n_req] are HOST arrays.  Pure host arithmetic: no context and no CUDA call.  Errors:
+ * INVALID_ARG (NULL argument, n_req < 1, a mask bit >= n_layers, a negative length). */
+typedef struct {
+  uint64_t weights, kv_read, kv_write, total;
+  int active_union;
+} tss_step_bytes;
+tss_status tss_estimate_step_bytes(const tss_arch* arch, int n_req, const uint64_t* masks, const int32_t* ctx_len,
+                                   const int32_t* n_nodes, tss_step_bytes* out);
+
 /* One verification step, enqueued on `stream`: skip controller (per-request S(x), union of
  * active layers, per-layer compacted row lists) -> embedding -> for every layer in the union:
  * RMSNorm+QKV GEMM with RoPE and KV append, split-KV attention with the chain/tree mask,

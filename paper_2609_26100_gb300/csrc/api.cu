@@ -1002,6 +1002,35 @@ tss_status tss_sparsity_ratio(const tss_ctx* c, int domain_id, double* out) {
   return TSS_OK;
 }
 
+tss_status tss_estimate_step_bytes(const tss_arch* a, int n_req, const uint64_t* masks, const int32_t* ctx_len,
+                                   const int32_t* n_nodes, tss_step_bytes* out) {
+  if (!a || !masks || !ctx_len || !n_nodes || !out) return fail(TSS_ERR_INVALID_ARG, "NULL argument");
+  if (n_req < 1) return fail(TSS_ERR_INVALID_ARG, "n_req must be positive");
+  if (a->n_layers < 1 || a->n_layers > 64 || a->d_model < 1 || a->d_mlp < 1 || a->vocab < 1)
+    return fail(TSS_ERR_INVALID_ARG, "arch: n_layers in [1, 64], positive d_model, d_mlp and vocab");
+  const int L = a->n_layers;
+  const uint64_t d = static_cast<uint64_t>(a->d_model), f = static_cast<uint64_t>(a->d_mlp);
+  const uint64_t kv_token = 4 * d;  // K and V rows of one token in one layer, bf16
+  uint64_t runs = 0, kv_read = 0, kv_write = 0;
+  for (int b = 0; b < n_req; ++b) {
+    if (L < 64 && (masks[b] >> L) != 0) return fail(TSS_ERR_INVALID_ARG, "a skip mask names a layer >= n_layers");
+    if (ctx_len[b] < 0 || n_nodes[b] < 0) return fail(TSS_ERR_INVALID_ARG, "ctx_len and n_nodes must be >= 0");
+    const uint64_t all = L == 64 ? ~0ull : (1ull << L) - 1;
+    const uint64_t act = all & ~masks[b];
+    runs |= act;
+    const uint64_t n_act = static_cast<uint64_t>(__builtin_popcountll(act));
+    kv_read += static_cast<uint64_t>(ctx_len[b]) * n_act * kv_token;
+    kv_write += static_cast<uint64_t>(n_nodes[b]) * n_act * kv_token;
+  }
+  out->active_union = __builtin_popcountll(runs);
+  out->weights = static_cast<uint64_t>(out->active_union) * 2 * (4 * d * d + 3 * d * f) +
+                 static_cast<uint64_t>(a->vocab) * d * 2;
+  out->kv_read = kv_read;
+  out->kv_write = kv_write;
+  out->total = out->weights + kv_read + kv_write;
+  return TSS_OK;
+}
+
 tss_status tss_active_layer_count(const tss_ctx* c, const tss_verify_batch* bt, int* out) {
   if (!c || !bt || !out || !bt->domain_id) return fail(TSS_ERR_INVALID_ARG, "NULL argument");
   if (bt->n_req < 1 || bt->n_req > c->a.max_batch) return fail(TSS_ERR_INVALID_ARG, "n_req out of range");

@@ -27,6 +27,7 @@ EXPORTS = (
     "tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status", "tss_destroy",
     "tss_linear", "tss_linear_static", "tss_read_trace", "tss_status_string", "tss_last_error",
+    "tss_estimate_step_bytes",
 )
 
 _P = ctypes.c_void_p
@@ -62,6 +63,11 @@ KERNEL_KINDS = ("controller+embed+norms", "qkv_gemm", "attention", "o_gemm", "ga
 
 class TssKernelTimes(ctypes.Structure):
     _fields_ = [("ms", ctypes.c_float * 9), ("launches", ctypes.c_int * 9)]
+
+
+class TssStepBytes(ctypes.Structure):
+    _fields_ = [("weights", ctypes.c_uint64), ("kv_read", ctypes.c_uint64), ("kv_write", ctypes.c_uint64),
+                ("total", ctypes.c_uint64), ("active_union", ctypes.c_int)]
 
 
 class TssVerifyResult(ctypes.Structure):
@@ -100,9 +106,11 @@ def lib() -> ctypes.CDLL:
         L.tss_status_string.restype = ctypes.c_char_p
         L.tss_last_error.argtypes = []
         L.tss_last_error.restype = ctypes.c_char_p
+        L.tss_estimate_step_bytes.argtypes = [ctypes.POINTER(TssArch), ctypes.c_int, ctypes.POINTER(ctypes.c_uint64),
+                                              _I32P, _I32P, ctypes.POINTER(TssStepBytes)]
         for name in ("tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
                      "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status",
-                     "tss_linear", "tss_linear_static", "tss_read_trace"):
+                     "tss_linear", "tss_linear_static", "tss_read_trace", "tss_estimate_step_bytes"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -113,6 +121,19 @@ def linear_static(x, w, y, stream=None) -> None:
     m, k = x.shape
     check(lib().tss_linear_static(x.data_ptr(), w.data_ptr(), y.data_ptr(), m, k, w.shape[0], stream),
           "tss_linear_static")
+
+
+def estimate_step_bytes(arch, masks: Sequence[int], ctx_len: Sequence[int], n_nodes: Sequence[int]) -> Dict[str, int]:
+    """tss_estimate_step_bytes: HBM bytes of a verification step (host arithmetic, no GPU)."""
+    a = TssArch(arch.n_layers, arch.d_model, arch.n_heads, arch.head_dim, arch.d_mlp, arch.vocab,
+                arch.rms_eps, arch.rope_theta, 1, 1, 1, 1, 1)
+    n = len(masks)
+    m = (ctypes.c_uint64 * n)(*[int(x) for x in masks])
+    out = TssStepBytes()
+    check(lib().tss_estimate_step_bytes(ctypes.byref(a), n, m, ctypes.cast(_i32(ctx_len), _I32P),
+                                        ctypes.cast(_i32(n_nodes), _I32P), ctypes.byref(out)), "tss_estimate_step_bytes")
+    return {"weights": out.weights, "kv_read": out.kv_read, "kv_write": out.kv_write, "total": out.total,
+            "active_union": out.active_union}
 
 
 class TssError(RuntimeError):
