@@ -66,3 +66,27 @@ def test_layer_count_must_match_the_model():
     with pytest.raises(ValueError, match="40 layers"):
         PC.parse(json.dumps({"n_layers": 40, "domains": []}), 32)
     assert PC.parse(_doc(sparsity=2 / 32), 32)[0].skip == (1, 2)
+
+
+def test_runner_load_phi_sets_each_domain(tmp_path):
+    """TssRunner.load_phi hands every record's bitmask to tss_set_skip_config (the verifier is
+    replaced by a recorder, so no GPU is needed)."""
+    from paper_2609_26100_gb300 import synth
+    from paper_2609_26100_gb300.runner import TssRunner
+
+    class Recorder:
+        def __init__(self):
+            self.calls = []
+
+        def set_skip_config(self, domain, mask):
+            self.calls.append((domain, mask))
+
+    run = object.__new__(TssRunner)
+    run.arch, run.v = synth.TINY, Recorder()
+    path = tmp_path / "phi.json"
+    PC.save(str(path), synth.TINY.n_layers, [PC.DomainConfig(5, (2,)), PC.DomainConfig(1, (0, 3))])
+    assert run.load_phi(str(path)) == {1: 0b1001, 5: 0b100}
+    assert sorted(run.v.calls) == [(1, 0b1001), (5, 0b100)]
+    PC.save(str(path), 32, [PC.DomainConfig(0, (31,))])
+    with pytest.raises(ValueError, match="32 layers"):
+        run.load_phi(str(path))
