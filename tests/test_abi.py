@@ -117,3 +117,21 @@ def test_binding_structs_match_the_c_layout(tmp_path):
         assert got[(cname, "size")] == ctypes.sizeof(py), cname
         for fname, _ in py._fields_:
             assert got[(cname, fname)] == getattr(py, fname).offset, f"{cname}.{fname}"
+
+
+def test_readme_c_example_compiles(tmp_path):
+    """The C example in README.md compiles against tss.h as written."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    with open(os.path.join(ROOT, "README.md")) as f:
+        text = f.read()
+    blocks = re.findall(r"```c\n(.*?)```", text, flags=re.S)
+    assert blocks, "README has no C example"
+    c = tmp_path / "example.c"
+    c.write_text(blocks[0])
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-I",
+                        os.path.join(ROOT, "include"), str(c)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
