@@ -264,6 +264,40 @@ def verify_request(weights, arch, skip, tokens, parents, ctx_len: int, kv, dt=np
     return logits, new_kv
 
 
+def verify_requests(weights, arch, skips, blocks, kv, dt=np.float32):
+    """verify_request for several requests at once, layer by layer: block b = (tokens, parents,
+    ctx_len) runs under skip set skips[b], with context kv(b, l) = (K [H, >=ctx_len, D], V).
+
+    The arithmetic of each request is verify_request's, in the same order, so the results are the
+    same; only the loop order differs (layer-major: weights["layers"][l] is read once per batch).
+    Returns a list of (logits [N_b, V], new_kv_b).
+    """
+    h, pos, allowed = [], [], []
+    for tokens, parents, ctx_len in blocks:
+        check_parents(parents)
+        h.append(as_float(weights["embed"], dt)[np.asarray(tokens, dtype=np.int64)])
+        pos.append(ctx_len + depths(parents))
+        allowed.append(ancestor_or_self(parents))
+    new_kv = [{} for _ in blocks]
+    for l in range(arch.n_layers):
+        runs = [b for b in range(len(blocks)) if l not in skips[b]]
+        if not runs:
+            continue  # no request runs layer l
+        lw = weights["layers"][l]
+        for b in runs:
+            ctx_len = blocks[b][2]
+            k_ctx, v_ctx = kv(b, l)
+            k_ctx = as_float(k_ctx, dt)[:, :ctx_len, :]
+            v_ctx = as_float(v_ctx, dt)[:, :ctx_len, :]
+            h[b], k, v = llama_block(h[b], lw, arch, pos[b], allowed[b], k_ctx, v_ctx, dt)
+            new_kv[b][l] = (k, v)
+    out = []
+    for b in range(len(blocks)):
+        hf = rms_norm(h[b], as_float(weights["final_norm"], dt), arch.rms_eps)
+        out.append((hf @ as_float(weights["lm_head"], dt).T, new_kv[b]))
+    return out
+
+
 def prefill(weights, arch, skip, ctx_tokens, dt=np.float32):
     """KV of a context under the request's skip set: the causal (chain) forward of the context
     with an empty cache.  Returns kv[l] = (K [H, C, D], V) for active layers, None for skipped."""

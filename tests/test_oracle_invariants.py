@@ -299,3 +299,26 @@ def test_spec_sampling_monte_carlo_with_philox():
     chi2 = float(np.sum((counts - n * p0) ** 2 / (n * p0)))
     from scipy.stats import chi2 as chi2d
     assert chi2d.sf(chi2, V - 1) > 1e-3
+
+
+def test_layer_major_batch_equals_per_request_verification(tiny, tiny_ctx):
+    """verify_requests (layer by layer over a batch) gives each request exactly what
+    verify_request gives it alone: mixed skip sets (one dense, one skipping every layer), context
+    lengths and a tree block."""
+    arch, w = tiny
+    skips = [frozenset({1}), frozenset(), frozenset({0, 3}), frozenset(range(arch.n_layers))]
+    blocks, kvs = [], []
+    for b, skip in enumerate(skips):
+        ctx = tiny_ctx[: 24 - 5 * b]
+        parents = synth.eagle_tree(9, (3, 2, 1)) if b == 2 else synth.chain_parents(3 + b)
+        toks = synth.draft_tokens(parents, arch.vocab, 5, f"inv.batch{b}")
+        blocks.append((toks, parents, len(ctx)))
+        kvs.append(_kv(arch, w, skip, ctx))
+    got = O.verify_requests(w, arch, skips, blocks, lambda b, l: kvs[b][l], D64)
+    for b, skip in enumerate(skips):
+        toks, parents, C = blocks[b]
+        ref, nk = O.verify_request(w, arch, skip, toks, parents, C, kvs[b], D64)
+        assert np.array_equal(got[b][0], ref)
+        assert sorted(got[b][1]) == sorted(nk)
+        for l in nk:
+            assert np.array_equal(got[b][1][l][0], nk[l][0]) and np.array_equal(got[b][1][l][1], nk[l][1])
