@@ -25,6 +25,9 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "7B verify-step latency (us) & tokens/s at k=5, 4 skipped layers; % HBM roofline"
+# Bytes of the per-step descriptor tss_verify copies to the device (sizeof(tss::StepDesc);
+# tests/test_step_bytes.py compiles the struct and checks this number).
+STEP_DESC_BYTES = 7536
 NOMINAL_HBM_GBS = 8000.0
 
 
@@ -215,8 +218,100 @@ def kernel_bytes(w, kinds):
 
 
 # ----------------------------------------------------------------------------------------------
-# CPU oracle sample (cpu_baseline leg and --impl reference)
+# CPU oracle (cpu_baseline leg and --impl reference)
 # ----------------------------------------------------------------------------------------------
+def host_mem_available():
+    try:
+        with open("/proc/meminfo") as f:
+            for ln in f:
+                if ln.startswith("MemAvailable:"):
+                    return int(ln.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0
+
+
+def cpu_model():
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.startswith("Model name:"):
+                return ln.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    return "unknown"
+
+
+class OracleStep:
+    """The oracle timed on WHOLE verification steps of the workload: every request through
+    O.verify_requests (embedding, every layer it runs, final norm, LM head) and the acceptance
+    rule, one step per call.  The fp32 weights of the active layers and the requests' context KV
+    are generated (seeded, as the GPU run's) before any timing and stay in host memory, so a timed
+    step is the oracle's arithmetic only.  Raises MemoryError when they would take more than half
+    of the host's available memory."""
+
+    @staticmethod
+    def host_bytes(w):
+        a = w.arch
+        per_layer = 4 * (4 * a.d_model * a.d_model + 3 * a.d_model * a.d_mlp)
+        kv = sum(r.ctx_len * len([l for l in range(a.n_layers) if not (w.skip_mask(b) >> l) & 1])
+                 for b, r in enumerate(w.requests)) * 2 * a.d_model * 4
+        return len(w.active_union()) * per_layer + 2 * a.vocab * a.d_model * 4 + kv
+
+    def __init__(self, w, device):
+        from paper_2609_26100_gb300 import synth
+        if self.host_bytes(w) > 0.5 * host_mem_available():
+            raise MemoryError(f"oracle step needs {self.host_bytes(w) / 1e9:.1f} GB of host memory")
+        self.w = w
+        a = w.arch
+        f32 = lambda t: t.float().cpu().numpy()  # noqa: E731
+        g = synth.make_weights(a, w.seed, device=device, layers=[])
+        layers = [None] * a.n_layers
+        for l in w.active_union():
+            layers[l] = {k: f32(v) for k, v in synth.make_layer(a, l, w.seed, device=device).items()}
+        self.weights = {"embed": f32(g["embed"]), "lm_head": f32(g["lm_head"]), "final_norm": f32(g["final_norm"]),
+                        "layers": layers}
+        del g
+        self.skips = [frozenset(synth.layers_of(w.skip_mask(b))) for b in range(len(w.requests))]
+        self.kv = {}
+        for b, r in enumerate(w.requests):
+            for l in range(a.n_layers):
+                if l not in self.skips[b]:
+                    blk = f32(synth.kv_block(a, l, b, r.ctx_len, w.seed, device=device))
+                    self.kv[(b, l)] = (blk[0], blk[1])
+        if device != "cpu":
+            import torch
+            torch.cuda.empty_cache()
+
+    def step_seconds(self, i=0):
+        from oracle import tss_oracle as O
+        w = self.w
+        t = time.perf_counter()
+        outs = O.verify_requests(self.weights, w.arch, self.skips,
+                                 [(r.tokens, r.parents, r.ctx_len) for r in w.requests], lambda b, l: self.kv[(b, l)])
+        for b, r in enumerate(w.requests):
+            if w.mode == "sample":
+                u = O.philox_uniforms(w.seed, i, b, len(r.parents) - 1)
+                O.spec_sample_accept(outs[b][0], r.tokens, r.draft_probs.numpy(), u, w.temperature)
+            else:
+                O.greedy_accept(outs[b][0], r.tokens, r.parents)
+        return time.perf_counter() - t
+
+    def describe(self, n):
+        w = self.w
+        return (f"oracle (NumPy fp32) on whole verification steps of the workload ({len(w.requests)} request(s), "
+                f"{len(w.active_union())} active layers, {w.n_rows} rows, acceptance included), weights and context "
+                f"KV resident in host memory; median of {n} timed step(s); CPU {cpu_model()}")
+
+
+def make_oracle(w, device):
+    """Whole timed steps when their weights and KV fit in host memory, else the extrapolated sample."""
+    try:
+        return OracleStep(w, device)
+    except MemoryError:
+        return OracleSample(w, device)
+
+
 class OracleSample:
     """The oracle on a bounded sample of the workload: embedding + LM head with every layer
     skipped (t0), and with one sampled active layer (t1); a full step is estimated as
@@ -262,8 +357,9 @@ class OracleSample:
         return per_req * len(self.w.requests)
 
     def describe(self, n):
-        return (f"oracle (NumPy fp32) verify of request 0 with all layers skipped and with 1 sampled active layer, "
-                f"extrapolated to its active layers and scaled by the batch; {n} sample(s)")
+        return (f"EXTRAPOLATED (the workload's weights and KV do not fit in host memory): oracle (NumPy fp32) verify "
+                f"of request 0 with all layers skipped and with 1 sampled active layer, extrapolated to its active "
+                f"layers and scaled by the batch; {n} sample(s); CPU {cpu_model()}")
 
 
 def cores():
@@ -299,13 +395,14 @@ def run_reference(args):
     import torch
     w = make_workload(args.workload, args.skip)
     dev = "cuda" if torch.cuda.is_available() else "cpu"
-    s = OracleSample(w, dev)
+    s = make_oracle(w, dev)
     for i in range(args.warmup):
         s.step_seconds(i)
     times = [s.step_seconds(i) for i in range(args.steps)]
     sec = statistics.median(times)
     value = w.n_rows / sec
-    cb = {"value": value, "unit": "tokens/s", "cores": cores(), "kind": "oracle", "sample": s.describe(args.steps)}
+    cb = {"value": value, "unit": "tokens/s", "cores": cores(), "kind": "oracle", "sample": s.describe(args.steps),
+          "measured": isinstance(s, OracleStep), "timed_s_total": sum(times)}
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
@@ -344,7 +441,7 @@ def run_tss(args):
     # cpu baseline sample needs host copies of a few layers; take them before the GPU run
     sample = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        sample = OracleSample(w, "cuda")
+        sample = make_oracle(w, "cuda")
 
     run = TssRunner.for_workload(w)
     stream = torch.cuda.current_stream()
@@ -379,8 +476,9 @@ def run_tss(args):
             toks[i + 1] = g
         sel = synth.uniform_ints(n_var, 5, w.seed, "bench.prefix").tolist()
         for v in range(n_var):
-            if v % 5 == 4:  # one step in five
+            if v % 5 == 4:  # one step in five: variant 0's root followed by its greedy continuation
                 lp = sel[v] + 1
+                token_sets[v][0] = token_sets[0][0]
                 token_sets[v][1:1 + lp] = greedy[:lp]
     batches = []
     for v in range(n_var):
@@ -396,7 +494,6 @@ def run_tss(args):
 
     # ---------------- timed region (device-resident inputs) ----------------
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
-    accepts = []
     bus = torch.cuda.get_device_properties(local).pci_bus_id if hasattr(torch.cuda.get_device_properties(local), "pci_bus_id") else ""
     if world > 1:
         dist.barrier()
@@ -414,7 +511,6 @@ def run_tss(args):
     status = run.sync_status()
     if status != native.TSS_OK:
         raise RuntimeError(f"device status {status} in the timed region")
-    accepts.append(res["accept_len"].float().mean().item())
     total_ms = max_over_ranks(total_ms, "cuda")
     ms = total_ms / args.steps
     value = job_tokens_per_s(w.n_rows, args.steps, world, total_ms)
@@ -441,10 +537,15 @@ def run_tss(args):
             stream.synchronize()
             acc_sum += int(hres["accept_len"].sum())
         e2e_s = time.perf_counter() - t0
+        mean_accept = acc_sum / (n_e2e * len(w.requests))
         e2e = {"value": world * w.n_rows * n_e2e / e2e_s, "unit": "tokens/s",
-               "h2d_bytes_per_step": 4 * w.n_rows + (hprobs.numel() * 4 if sample_mode else 0),
+               "h2d_bytes_per_step": STEP_DESC_BYTES + 4 * w.n_rows + (hprobs.numel() * 4 if sample_mode else 0),
                "d2h_bytes_per_step": 4 * (3 * len(w.requests) + hres["path"].numel()),
-               "ms_per_step": e2e_s / n_e2e * 1e3, "steps": n_e2e}
+               "ms_per_step": e2e_s / n_e2e * 1e3, "steps": n_e2e,
+               "copies": "per step: the step descriptor and the draft tokens (and draft probabilities when sampling) "
+                         "host to device; accept_len, bonus, new_ctx_len and path device to host",
+               "committed_tokens_per_s": world * len(w.requests) * (1 + mean_accept) * n_e2e / e2e_s,
+               "mean_accept_len": mean_accept}
 
     # ---------------- per-kernel device times (CUDA events around every launch) ----------------
     roofline = None
@@ -504,14 +605,19 @@ def run_tss(args):
         "gpu_launches_per_step": launches_per_step,
         "clocks": clk.summary(),
     }
-    mean_acc = statistics.mean(accepts) if accepts else 0.0
-    out["committed_tokens_per_s"] = world * len(w.requests) * (1 + mean_acc) * args.steps / (total_ms / 1e3)
+    # committed tokens: the mean accept length over the e2e steps, which cycle through the same
+    # draft variants as the timed steps (the device-timed loop does not read results back)
+    if e2e is not None:
+        out["committed_tokens_per_s"] = world * len(w.requests) * (1 + e2e["mean_accept_len"]) * args.steps / (
+            total_ms / 1e3)
+        out["mean_accept_len"] = e2e["mean_accept_len"]
     if sample is not None:
         n_s = 3
         secs = [sample.step_seconds(i) for i in range(n_s)]
         sec = statistics.median(secs)
         out["cpu_baseline"] = {"value": w.n_rows / sec, "unit": "tokens/s", "cores": cores(), "kind": "oracle",
-                               "sample": sample.describe(n_s), "seconds_per_step": sec}
+                               "sample": sample.describe(n_s), "seconds_per_step": sec,
+                               "measured": isinstance(sample, OracleStep)}
     run.close()
     if rank == 0:
         print(json.dumps(out))

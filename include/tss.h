@@ -164,18 +164,21 @@ typedef struct {
  * returns an opaque context.  Errors: INVALID_ARG, UNSUPPORTED_ARCH, OUT_OF_MEMORY, CUDA; on
  * error everything allocated so far is freed and *out is NULL.  For failure injection, the
  * environment variable TSS_ALLOC_LIMIT_BYTES=N makes the allocations fail with OUT_OF_MEMORY
- * once they would pass N bytes. */
+ * once they would pass N bytes.  TSS_WAIT_LIMIT_MS=N (1..600000, default 2000) bounds every
+ * device-side wait of the persistent kernel (see tss_inject_timeout). */
 tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx** out);
 
 /* Phi(domain_id) = the set of layers whose bit is set in layer_bitmask (bit l = skip layer l;
  * 0 = dense).  Sec. "Domain-to-Configuration Mapping".  Bits >= n_layers must be clear.
- * Synchronous: waits for all work on the device first (so a verify already enqueued runs under
- * the configuration it was planned with), then affects verifies enqueued after it returns.
- * domain_id in [0, max_domains).  Not for use during stream capture. */
+ * Host-only and immediate: no device work and no wait.  tss_verify looks up each request's
+ * S(x) = Phi(d(x)) when it is called and passes the result to the device with the step, so a
+ * verify already enqueued runs under the map it was enqueued with and later verifies see the
+ * change.  domain_id in [0, max_domains).  Not thread-safe against concurrent calls on the same
+ * context (like every call taking a tss_ctx*). */
 tss_status tss_set_skip_config(tss_ctx* ctx, int domain_id, uint64_t layer_bitmask);
 
 /* Remove domain_id from Phi: its requests then run the dense path (unsupported domain).
- * Synchronises the device as tss_set_skip_config does. */
+ * Host-only and immediate, as tss_set_skip_config. */
 tss_status tss_clear_skip_config(tss_ctx* ctx, int domain_id);
 
 /* Sparsity ratio R_d = |S_d| / L of a configured domain (0 for an unconfigured one), and the
@@ -201,6 +204,22 @@ typedef struct {
 tss_status tss_estimate_step_bytes(const tss_arch* arch, int n_req, const uint64_t* masks, const int32_t* ctx_len,
                                    const int32_t* n_nodes, tss_step_bytes* out);
 
+/* Shared-memory plan of the persistent verify kernel for a step of n_req requests with n_rows
+ * draft-block rows in all, whose longest request spans max_keys keys (context + block), on a
+ * GPU with num_sms SMs, under the default switches: fits = 1 when the plan fits the 227 KiB a
+ * block may use (then tss_verify runs the step; otherwise it returns TSS_ERR_UNSUPPORTED_ARCH),
+ * with the weight k-blocks per ring stage, the ring stages, the attention's key splits, the
+ * dynamic shared memory of one block, and the weight stages held in tensor memory.  Pure host arithmetic: no context and no CUDA call.
+ * Errors: INVALID_ARG (NULL argument, head_dim not 64/128, n_req outside [1, 64], n_rows
+ * outside [n_req, 256], max_keys or num_sms < 1). */
+typedef struct {
+  int fits, kps, stages, attn_splits;
+  uint64_t smem_bytes;
+  int tmem_weight_slots; /* stages of streamed weights held in tensor memory (0: weights read from shared memory) */
+} tss_persistent_plan_info;
+tss_status tss_persistent_plan(const tss_arch* arch, int n_req, int n_rows, int max_keys, int num_sms,
+                               tss_persistent_plan_info* out);
+
 /* One verification step, enqueued on `stream`: skip controller (per-request S(x), union of
  * active layers, per-layer compacted row lists) -> embedding -> for every layer in the union:
  * RMSNorm+QKV GEMM with RoPE and KV append, split-KV attention with the chain/tree mask,
@@ -213,9 +232,11 @@ tss_status tss_estimate_step_bytes(const tss_arch* arch, int n_req, const uint64
  * When a step's context KV outweighs half a layer's weights (long contexts), the persistent kernel
  * is launched once per span of GEMM phases between two attentions and each layer's attention
  * runs as its own kernel (2 + 2 x active layers + 1 launches).
- * With the environment variable TSS_PATH=multi at tss_create, or when a step's rows do not fit the
- * persistent kernel's shared-memory plan, one kernel per operation runs instead (bf16 GEMM
- * activations, 6 + 7 x active layers launches). */
+ * A step that does not fit the persistent kernel's shared-memory plan (tss_persistent_plan) is
+ * rejected with TSS_ERR_UNSUPPORTED_ARCH before anything is enqueued.  With the environment
+ * variable TSS_PATH=multi at tss_create, one kernel per operation runs instead, a diagnostic path
+ * (bf16 GEMM activations: within the logit tolerance at the tiny test shape only; 6 + 7 x active
+ * layers launches). */
 tss_status tss_verify(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
                       const tss_verify_result* result, void* stream);
 
@@ -238,6 +259,27 @@ tss_status tss_prefill(tss_ctx* ctx, int n_req, const int32_t* n_tokens, const i
 /* Synchronise `stream`, then return and clear the device status word (TSS_OK if no device-side
  * check failed since the last call). */
 tss_status tss_sync_status(tss_ctx* ctx, void* stream);
+
+/* Fault injection for tests of the device-side timeout path; no GPU fault is involved.  The next
+ * n_steps verification steps of ctx on the persistent path do not publish one dataflow flag (the
+ * first 128-feature tile of the residual after the first active layer), so the waits that need
+ * it run out after the context's wait limit (environment variable TSS_WAIT_LIMIT_MS at
+ * tss_create, 1..600000, default 2000 ms): the kernel records TSS_ERR_TIMEOUT in the status word,
+ * every CTA leaves its loops and frees its tensor memory, and tss_sync_status reports the code.
+ * That step's outputs are undefined.  The context stays usable: every step starts with fresh
+ * counters and a clear abort word, so the next step runs normally.  A step with no active layer
+ * withholds nothing.  n_steps = 0 cancels. */
+tss_status tss_inject_timeout(tss_ctx* ctx, int n_steps);
+
+/* Diagnostic: the Philox4x32-10 stream that speculative sampling draws from when the batch gives
+ * no uniforms, for one (seed, offset): counter (slot, request, offset lo, offset hi), key
+ * (seed lo, seed hi), for requests [0, n_req) and slots [0, n_slots).
+ *   words: DEVICE uint32 [n_req][n_slots][4] (16-byte aligned), the generator's four output words;
+ *   uniforms: DEVICE fp32 [n_req][n_slots], (first word >> 8) * 2^-24, the value the acceptance
+ *   uses.  Either may be NULL (not both).  n_req * n_slots <= 2^28.  Asynchronous on `stream`;
+ *   uses the same device function as the acceptance kernels. */
+tss_status tss_philox_uniforms(uint64_t seed, uint64_t offset, int n_req, int n_slots, uint32_t* words,
+                               float* uniforms, void* stream);
 
 /* Release everything the context owns (after the caller's streams are idle). NULL is a no-op. */
 void tss_destroy(tss_ctx* ctx);
@@ -274,19 +316,30 @@ tss_status tss_verify_profiled(tss_ctx* ctx, const tss_verify_batch* batch, cons
  * framework that owns the whole device memory pool, a process with a memory budget fixed at
  * start-up, or a latency-critical loop that must not call cudaMalloc/cudaFree (they can
  * synchronise the device and stall unrelated streams).  It needs no tss_ctx and allocates
- * nothing: the stream-K scratch (partial tiles, per-tile counters) is a file-scope device array
- * of the library, 8 MiB + 1 KiB, held on every GPU that loads libtss.so until the process exits.
+ * nothing: the stream-K scratch (partial tiles, per-tile counters) and a status word are
+ * file-scope device arrays of the library, 8 MiB + 2 KiB in all.
  *   y[m][o] = sum_k x[m][k] * w[o][k]; x [m_rows][k_dim] bf16, w [n_out][k_dim] bf16,
  *   y [m_rows][n_out] fp32, device, row-major, 16-byte aligned; m_rows in [1, 64]; k_dim a
  *   multiple of 64; n_out a multiple of 128, at most 32768; and the scratch a problem needs,
  *   (min(#SMs, n_out/128 * k_dim/64) + n_out/128) * 128 * pad16(m_rows) * 4 bytes, at most 8 MiB
- *   -- larger requests return TSS_ERR_INVALID_ARG with a message.
- * The first call on a device (per process) looks up the array's device address and sets the
- * kernel's shared-memory limit; make that first call before any stream capture.  Every call on a
- * device shares the one array and the next call overwrites it (the counters are cleared on
- * `stream` at each call): calls that overlap on the GPU race, so serialise them on one stream.
- * Asynchronous on `stream`; no device status word is reported. */
+ *   -- larger requests return TSS_ERR_INVALID_ARG with a message.  The scratch bound caps n_out
+ *   further for many rows: on a 152-SM GB300 with 49..64 rows, n_out <= (256 - 152) * 128 = 13312;
+ *   with up to 16 rows the 32768 limit applies.
+ * The arrays live in a CUDA module that the runtime loads on a device at the first call there
+ * (CUDA's default lazy module loading), so the first call per device and process reserves the
+ * 8 MiB; a caller that later gives the rest of the device memory to its own pool should make that
+ * first call before, and before any stream capture (it also looks up the arrays' device addresses
+ * and sets the kernel's shared-memory limit).  Later calls allocate and reserve nothing.  Every
+ * call on a device shares the one array and the next call overwrites it (the counters are cleared
+ * on `stream` at each call): calls that overlap on the GPU race, so serialise them on one stream.
+ * Asynchronous on `stream`.  A device-side failure (a bounded wait that ran out) is recorded in
+ * the status word that tss_linear_static_status reports; the result is then undefined. */
 tss_status tss_linear_static(const void* x, const void* w, float* y, int m_rows, int k_dim, int n_out, void* stream);
+
+/* Synchronise `stream`, then return and clear the status word of tss_linear_static on the current
+ * device: TSS_OK, or TSS_ERR_TIMEOUT if a call since the last query gave up on a bounded wait
+ * (its y is then undefined).  Allocates nothing. */
+tss_status tss_linear_static_status(void* stream);
 
 /* Diagnostic timeline of the last persistent-path step, recorded when the environment variable
  * TSS_TRACE=1 was set at tss_create: globaltimer nanoseconds, per CTA (row of

@@ -69,6 +69,8 @@ struct GraphKey {
 };
 
 constexpr int kRing = 4;
+// Whether contexts stage the streamed weights in tensor memory by default (TSS_MK_TMEM overrides).
+constexpr bool kMkTmemDefault = false;
 constexpr int kMaxPathStride = 1024;
 
 }  // namespace
@@ -102,8 +104,6 @@ struct tss_ctx {
   bool ring_used[kRing] = {};
   int ring_i = 0;
   PlanDev* d_plan = nullptr;
-  unsigned long long* d_phi = nullptr;
-  int* d_phi_valid = nullptr;
   std::vector<unsigned long long> phi;
   std::vector<int> phi_valid;
   int* d_status = nullptr;
@@ -126,9 +126,12 @@ struct tss_ctx {
   int attn_mode = 0;  // 0 auto, 1 attention inside the persistent kernel, 2 separate attention kernels
   int w_evict_first = 1;
   int mk_max_stages = 12;
+  bool mk_tmem = kMkTmemDefault;  // stage the weights in tensor memory where it has room (TSS_MK_TMEM)
   int attn_plo = 1;
   int attn_splits_force = 0;  // > 0: key splits of the separate attention kernel (TSS_ATTN_SPLITS)
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
+  unsigned long long wait_ns = 2000000000ull;  // bound of the persistent kernel's waits (TSS_WAIT_LIMIT_MS)
+  int inject_timeouts = 0;  // steps left that withhold one dataflow flag (tss_inject_timeout)
   unsigned long long epoch = 0;
   float* ssp = nullptr;
   unsigned long long* flags = nullptr;  // hflag | qkvflag | guflag | attflag
@@ -202,9 +205,6 @@ MiscParams misc_params(tss_ctx* c) {
   MiscParams p{};
   p.step = c->d_step;
   p.plan = c->d_plan;
-  p.phi_mask = c->d_phi;
-  p.phi_valid = c->d_phi_valid;
-  p.max_domains = c->a.max_domains;
   p.n_layers = c->L;
   p.d_model = c->d;
   p.n_heads = c->H;
@@ -376,18 +376,39 @@ tss_status enqueue_step(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* pr
 struct MkConfig {
   int kps = 0, stages = 0, attn_splits = 1;
   size_t attn_extra = 0, smem = 0;
+  // tensor-memory staging of the weights: B-operand stages, weight slots, accumulator buffers
+  int ts = 0, x_stages = 0, tw_slots = 0, n_acc = 0;
 };
 
 // Key splits per (request, head) for the persistent kernel's attention: the fewest waves of
 // items over the grid times the tiles an item scores, plus a fixed per-item cost (flags, merge)
 // of about three tiles.  Short contexts get about one item per CTA.
-int mk_attn_splits(const tss_ctx* c, int B, int tiles) {
-  const int pairs = B * c->H;
+// What the persistent kernel's shared-memory plan depends on (a context's shape and switches).
+struct MkPlanIn {
+  int D, H, num_sms, kps_max, stages_max, max_splits, ts;
+};
+MkPlanIn mk_plan_in(const tss_ctx* c) {
+  return MkPlanIn{c->D, c->H, c->num_sms, c->mk_kps, c->mk_max_stages, c->max_splits, c->mk_tmem ? 1 : 0};
+}
+
+// Tensor-memory staging (TS) for an MMA width n_pad: accumulator buffers (2..8, about 128
+// columns of them) and the weight slots of kps k-blocks (32 columns each) that fit behind them
+// in the 512 columns; 0 slots when fewer than two fit.
+void mk_ts_slots(int n_pad, int kps, int* n_acc, int* slots) {
+  const int nb = std::max(2, std::min(8, 128 / n_pad));
+  const int free_cols = 512 - nb * n_pad;
+  const int tw = free_cols > 0 ? free_cols / (kps * 32) : 0;
+  *n_acc = nb;
+  *slots = tw >= 2 ? std::min(tw, 16) : 0;
+}
+
+int mk_attn_splits(const MkPlanIn& c, int B, int tiles) {
+  const int pairs = B * c.H;
   int best = 1;
   long long best_cost = -1;
-  for (int sl = 1; sl <= c->max_splits; ++sl) {
+  for (int sl = 1; sl <= c.max_splits; ++sl) {
     if (sl > 1 && sl > tiles) break;
-    const long long waves = (static_cast<long long>(pairs) * sl + c->num_sms - 1) / c->num_sms;
+    const long long waves = (static_cast<long long>(pairs) * sl + c.num_sms - 1) / c.num_sms;
     const long long cost = waves * ((tiles + sl - 1) / sl + 3);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
@@ -428,22 +449,32 @@ int ext_attn_splits(const tss_ctx* c, const StepDesc* sd, int B) {
   return best;
 }
 
-bool mk_config(const tss_ctx* c, const StepPlan& sp, MkConfig* out) {
+// B requests with M rows in all, the longest one spanning `tiles` 64-key tiles.
+bool mk_config_for(const MkPlanIn& c, int B, int M, int tiles, MkConfig* out) {
   constexpr size_t kLimit = 232448;  // per-block shared-memory maximum of sm_103 (227 KiB)
-  const size_t q = static_cast<size_t>(kMaxNodes) * (c->D + 8) * 2;
-  const size_t tile = static_cast<size_t>(2) * 64 * (c->D + 8) * 2;
-  const int splits = mk_attn_splits(c, sp.B, std::max(sp.tiles, 1));
-  const int per = std::max(1, (std::max(sp.tiles, 1) + splits - 1) / splits);
-  for (int kps = c->mk_kps; kps >= 1; --kps) {
-    const XsLayout xs = xs_layout(sp.M);
-    const size_t stage = static_cast<size_t>(kps) * (16384 + static_cast<size_t>(xs.rows) * xs.parts * 128);
-    for (int S = c->mk_max_stages; S >= 2; --S) {
-      const size_t ring = S * stage;
-      const size_t base = mk_smem_bytes(xs.rows, xs.parts, S, c->D, kps, 0);
+  const size_t q = static_cast<size_t>(kMaxNodes) * (c.D + 8) * 2;
+  const size_t tile = static_cast<size_t>(2) * 64 * (c.D + 8) * 2;
+  const int splits = mk_attn_splits(c, B, std::max(tiles, 1));
+  const int per = std::max(1, (std::max(tiles, 1) + splits - 1) / splits);
+  for (int kps = c.kps_max; kps >= 1; --kps) {
+    const XsLayout xs = xs_layout(M);
+    const size_t x_stage = static_cast<size_t>(kps) * xs.rows * xs.parts * 128;
+    const size_t stage = static_cast<size_t>(kps) * 16384 + x_stage;
+    int n_acc = 0, tw = 0;
+    if (c.ts) mk_ts_slots(xs.rows, kps, &n_acc, &tw);
+    for (int S = c.stages_max; S >= 2; --S) {
+      // TS: the B operand in its own ring of up to 8 stages (at least 2) behind S weight stages
+      int SX = 0;
+      if (tw >= 2) {
+        SX = 8;
+        while (SX > 2 && mk_smem_bytes(xs.rows, xs.parts, S, c.D, kps, 0, SX, tw) > kLimit) --SX;
+      }
+      const size_t ring = SX > 0 ? S * static_cast<size_t>(kps) * 16384 + SX * x_stage : S * stage;
+      const size_t base = mk_smem_bytes(xs.rows, xs.parts, S, c.D, kps, 0, SX, SX > 0 ? tw : 0);
       if (base > kLimit) continue;
       const size_t avail = kLimit - base;
       // at least Q + one tile, and Q + the warps' merge buffer (8 warps x 16 rows x D floats)
-      const size_t first = q + std::max(tile, static_cast<size_t>(8) * 16 * c->D * 4);
+      const size_t first = q + std::max(tile, static_cast<size_t>(8) * 16 * c.D * 4);
       const size_t need_min = ring >= first ? 0 : first - ring;
       if (need_min > avail) continue;
       const size_t want = q + per * tile > ring ? q + per * tile - ring : 0;
@@ -455,10 +486,18 @@ bool mk_config(const tss_ctx* c, const StepPlan& sp, MkConfig* out) {
       out->attn_splits = splits;
       out->attn_extra = extra;
       out->smem = base + extra;
+      out->ts = SX > 0 ? 1 : 0;
+      out->x_stages = SX;
+      out->tw_slots = SX > 0 ? tw : 0;
+      out->n_acc = SX > 0 ? n_acc : 0;
       return true;
     }
   }
   return false;
+}
+
+bool mk_config(const tss_ctx* c, const StepPlan& sp, MkConfig* out) {
+  return mk_config_for(mk_plan_in(c), sp.B, sp.M, sp.tiles, out);
 }
 
 // One verification step on the persistent path: prologue (controller, embedding, sums of
@@ -488,6 +527,10 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.stages = stages;
   p.kps = kps;
   p.xs = xs;
+  p.ts = cfg.ts;
+  p.x_stages = cfg.x_stages;
+  p.tw_slots = cfg.tw_slots;
+  p.n_acc = cfg.n_acc;
   p.attn_plo = c->attn_plo;
   p.attn_extra = static_cast<int>(cfg.attn_extra);
   p.w_evict_first = c->w_evict_first;
@@ -530,6 +573,9 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.rope_cos = c->rope_cos;
   p.rope_sin = c->rope_sin;
   p.status = c->d_status;
+  p.wait_ns = c->wait_ns;
+  p.withhold_flag = c->inject_timeouts > 0 && sp.n_act > 0 ? 1 : 0;
+  if (p.withhold_flag) --c->inject_timeouts;
 #define TSS_MK(kind, expr)                 \
   do {                                     \
     if (prof) TSS_TRY(prof->begin(kind));  \
@@ -586,7 +632,7 @@ bool mk_supported(const tss_ctx* c, const StepPlan& sp) {
   if (!c->use_mk) return false;
   MkConfig cfg;
   if (!mk_config(c, sp, &cfg)) return false;
-  return mk_max_blocks_per_sm(c->D, cfg.smem) >= 1;
+  return mk_max_blocks_per_sm(c->D, cfg.ts != 0, cfg.smem) >= 1;
 }
 
 tss_status validate_arch(const tss_arch* a) {
@@ -699,15 +745,9 @@ tss_status build_workspaces(tss_ctx* c) {
   const size_t ph = static_cast<size_t>(c->a.max_batch) * c->H * c->max_splits * kMaxNodes;
   TSS_TRY(c->alloc(&c->attn_po, ph * c->D));
   TSS_TRY(c->alloc(&c->attn_pml, ph * 2));
-  TSS_TRY(c->alloc(&c->attn_cnt, static_cast<size_t>(c->a.max_batch) * c->H));
-  TSS_CU(cudaMemset(c->attn_cnt, 0, static_cast<size_t>(c->a.max_batch) * c->H * sizeof(int)));
   TSS_TRY(c->alloc(&c->d_step, 1));
   TSS_TRY(c->alloc(&c->d_plan, 1));
   TSS_CU(cudaMemset(c->d_plan, 0, sizeof(PlanDev)));
-  TSS_TRY(c->alloc(&c->d_phi, c->a.max_domains));
-  TSS_TRY(c->alloc(&c->d_phi_valid, c->a.max_domains));
-  TSS_CU(cudaMemset(c->d_phi, 0, sizeof(unsigned long long) * c->a.max_domains));
-  TSS_CU(cudaMemset(c->d_phi_valid, 0, sizeof(int) * c->a.max_domains));
   c->phi.assign(c->a.max_domains, 0ull);
   c->phi_valid.assign(c->a.max_domains, 0);
   TSS_TRY(c->alloc(&c->d_status, 1));
@@ -751,9 +791,12 @@ tss_status build_workspaces(tss_ctx* c) {
     const size_t nflags = static_cast<size_t>(nt) + 3 * nt + c->Ft + static_cast<size_t>(c->a.max_batch) * c->H;
     TSS_TRY(c->alloc(&c->flags, nflags));
     TSS_CU(cudaMemset(c->flags, 0, nflags * sizeof(unsigned long long)));
-    c->mk_n_zero = 7 * max_tiles + 1;
+    // stream-K counters, the abort word and the attention's split counters: zeroed by every
+    // step's prologue, so that a step after one that gave up on a timeout starts clean
+    c->mk_n_zero = 7 * max_tiles + 1 + c->a.max_batch * c->H;
     TSS_TRY(c->alloc(&c->mk_zero, static_cast<size_t>(c->mk_n_zero)));
     TSS_CU(cudaMemset(c->mk_zero, 0, static_cast<size_t>(c->mk_n_zero) * sizeof(int)));
+    c->attn_cnt = c->mk_zero + 7 * max_tiles + 1;
     // partial tiles are strided by the MMA width of the split B operand (up to 256 rows)
     int xs_rows_max = 16;
     for (int m = 1; m <= c->a.max_rows; ++m) xs_rows_max = std::max(xs_rows_max, xs_layout(m).rows);
@@ -813,6 +856,7 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
     sd->req_rowoff[b] = M;
     sd->req_slot[b] = slot;
     sd->req_domain[b] = dom;
+    sd->req_phi[b] = mask;
     unsigned long long anc[kMaxNodes];
     int depth[kMaxNodes];
     for (int i = 0; i < n; ++i) {
@@ -941,7 +985,12 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_ATTN_PLO")) c->attn_plo = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ATTN_SPLITS")) c->attn_splits_force = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
+  if (const char* e = std::getenv("TSS_MK_TMEM")) c->mk_tmem = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ALLOC_LIMIT_BYTES")) c->alloc_limit = std::strtoull(e, nullptr, 10);
+  if (const char* e = std::getenv("TSS_WAIT_LIMIT_MS")) {
+    const long long ms = std::atoll(e);
+    if (ms >= 1 && ms <= 600000) c->wait_ns = static_cast<unsigned long long>(ms) * 1000000ull;
+  }
   const char* trace_env = std::getenv("TSS_TRACE");
   tss_status s = build_workspaces(c);
   if (s == TSS_OK) s = build_weights(c, weights);
@@ -971,26 +1020,18 @@ tss_status tss_set_skip_config(tss_ctx* c, int domain_id, uint64_t mask) {
   if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
   if (domain_id < 0 || domain_id >= c->a.max_domains) return fail(TSS_ERR_INVALID_ARG, "domain_id out of range");
   if (c->L < 64 && (mask >> c->L) != 0ull) return fail(TSS_ERR_INVALID_ARG, "skip mask names a layer >= n_layers");
-  // A step already enqueued reads Phi on the device when it runs, but planned its launches from
-  // the host copy when it was enqueued: let every such step finish before either copy changes.
-  TSS_CU(cudaDeviceSynchronize());
+  // Host-only: a step takes each request's S(x) from this map when it is enqueued (into its
+  // descriptor), so steps already enqueued keep the map they were planned with and nothing waits.
   c->phi[domain_id] = mask;
   c->phi_valid[domain_id] = 1;
-  const int one = 1;
-  const unsigned long long m = mask;
-  TSS_CU(cudaMemcpy(c->d_phi + domain_id, &m, sizeof(m), cudaMemcpyHostToDevice));
-  TSS_CU(cudaMemcpy(c->d_phi_valid + domain_id, &one, sizeof(int), cudaMemcpyHostToDevice));
   return TSS_OK;
 }
 
 tss_status tss_clear_skip_config(tss_ctx* c, int domain_id) {
   if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
   if (domain_id < 0 || domain_id >= c->a.max_domains) return fail(TSS_ERR_INVALID_ARG, "domain_id out of range");
-  TSS_CU(cudaDeviceSynchronize());  // as in tss_set_skip_config
-  c->phi[domain_id] = 0ull;
+  c->phi[domain_id] = 0ull;  // host-only, as in tss_set_skip_config
   c->phi_valid[domain_id] = 0;
-  const int zero = 0;
-  TSS_CU(cudaMemcpy(c->d_phi_valid + domain_id, &zero, sizeof(int), cudaMemcpyHostToDevice));
   return TSS_OK;
 }
 
@@ -1028,6 +1069,25 @@ tss_status tss_estimate_step_bytes(const tss_arch* a, int n_req, const uint64_t*
   out->kv_read = kv_read;
   out->kv_write = kv_write;
   out->total = out->weights + kv_read + kv_write;
+  return TSS_OK;
+}
+
+tss_status tss_persistent_plan(const tss_arch* a, int n_req, int n_rows, int max_keys, int num_sms,
+                               tss_persistent_plan_info* out) {
+  if (!a || !out) return fail(TSS_ERR_INVALID_ARG, "NULL argument");
+  if ((a->head_dim != 64 && a->head_dim != 128) || a->n_heads < 1)
+    return fail(TSS_ERR_INVALID_ARG, "arch: head_dim 64 or 128 and n_heads >= 1");
+  if (n_req < 1 || n_req > kMaxBatch || n_rows < n_req || n_rows > kMaxRows || max_keys < 1 || num_sms < 1)
+    return fail(TSS_ERR_INVALID_ARG, "n_req in [1, 64], n_rows in [n_req, 256], max_keys and num_sms positive");
+  const MkPlanIn in{a->head_dim, a->n_heads, num_sms, 3, 12, kMaxSplits, kMkTmemDefault ? 1 : 0};
+  MkConfig cfg;
+  const bool fits = mk_config_for(in, n_req, n_rows, (max_keys + 63) / 64, &cfg);
+  out->fits = fits ? 1 : 0;
+  out->kps = fits ? cfg.kps : 0;
+  out->stages = fits ? cfg.stages : 0;
+  out->attn_splits = fits ? cfg.attn_splits : 0;
+  out->smem_bytes = fits ? static_cast<uint64_t>(cfg.smem) : 0;
+  out->tmem_weight_slots = fits ? cfg.tw_slots : 0;
   return TSS_OK;
 }
 
@@ -1093,7 +1153,12 @@ tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cach
         TSS_CU(cudaMemcpyAsync(c->io_unif, bt->uniforms, sizeof(float) * B * bt->uniform_stride, cudaMemcpyHostToDevice, s));
     }
   }
-  if (mk_supported(c, sp)) {
+  const bool mk = mk_supported(c, sp);
+  if (c->use_mk && !mk)
+    return fail(TSS_ERR_UNSUPPORTED_ARCH,
+                "the step does not fit the persistent kernel's shared-memory plan (and the kernel-per-operation path, "
+                "TSS_PATH=multi, does not meet the logit tolerance at 7B/13B widths)");
+  if (mk) {
     // Persistent path: three launches per step (the verify kernel is a cooperative launch), so no
     // graph is needed; with a Prof the events bracket each launch directly.
     if (prof) prof->s = s;
@@ -1266,6 +1331,23 @@ tss_status tss_sync_status(tss_ctx* c, void* stream) {
   TSS_CU(cudaStreamSynchronize(s));
   const int v = *c->h_status;
   if (v != 0) return fail(v, std::string("device status: ") + tss_status_string(v));
+  return TSS_OK;
+}
+
+tss_status tss_philox_uniforms(uint64_t seed, uint64_t offset, int n_req, int n_slots, uint32_t* words, float* uniforms,
+                               void* stream) {
+  if (n_req < 1 || n_slots < 1 || static_cast<long long>(n_req) * n_slots > (1LL << 28))
+    return fail(TSS_ERR_INVALID_ARG, "n_req and n_slots must be positive, n_req * n_slots at most 2^28");
+  if (!words && !uniforms) return fail(TSS_ERR_INVALID_ARG, "words and uniforms are both NULL");
+  if (words && !aligned16(words)) return fail(TSS_ERR_INVALID_ARG, "words must be 16-byte aligned");
+  TSS_CU(launch_philox_fill(seed, offset, n_req, n_slots, words, uniforms, static_cast<cudaStream_t>(stream)));
+  return TSS_OK;
+}
+
+tss_status tss_inject_timeout(tss_ctx* c, int n_steps) {
+  if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
+  if (n_steps < 0) return fail(TSS_ERR_INVALID_ARG, "n_steps must be >= 0");
+  c->inject_timeouts = n_steps;
   return TSS_OK;
 }
 

@@ -41,6 +41,10 @@ struct StepDesc {
   int req_rowoff[kMaxBatch];
   int req_slot[kMaxBatch];
   int req_domain[kMaxBatch];
+  // S(x) of every request: the domain map's entry for its domain when the step was enqueued (the
+  // lookup S(x) = Phi(d(x)) runs on the host, so a later change of the map affects later steps
+  // only), 0 (dense) for a domain that is not configured.
+  unsigned long long req_phi[kMaxBatch];
   int row_req[kMaxRows];
   int row_pos[kMaxRows];
   int row_parent[kMaxRows];  // request-local parent, -1 for the root
@@ -303,6 +307,25 @@ __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint6
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
+}
+
+// The same MMA with the A operand (128 rows x 16 bf16 of K) read from tensor memory: row i in lane
+// i, two K elements per 32-bit column, so one K=16 step spans 8 columns from a_tmem.
+__device__ __forceinline__ void umma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                             uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Asynchronous copy shared -> tensor memory of a 128-row x 256-bit matrix (one K=16 slice of a
+// 128-row bf16 operand) described by a shared-memory matrix descriptor: row i lands in lane i,
+// columns taddr .. taddr + 7.  Completion is tracked by tcgen05.commit like an MMA's.
+__device__ __forceinline__ void tmem_cp_128x256b(uint32_t taddr, uint64_t sdesc) {
+  asm volatile("tcgen05.cp.cta_group::1.128x256b [%0], %1;" ::"r"(taddr), "l"(sdesc) : "memory");
 }
 
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {

@@ -79,9 +79,7 @@ cudaError_t launch_attention(const AttnParams& p, int B, cudaStream_t s, bool pd
 struct MiscParams {
   const StepDesc* step;
   PlanDev* plan;
-  const unsigned long long* phi_mask;
-  const int* phi_valid;
-  int max_domains, n_layers, d_model, n_heads, head_dim, vocab;
+  int n_layers, d_model, n_heads, head_dim, vocab;
   float rms_eps;
   const __nv_bfloat16* embed;   // [vocab][d]
   float* h;                     // [kMaxRows][d]
@@ -107,6 +105,10 @@ cudaError_t launch_accept_greedy(const MiscParams& p, int B, cudaStream_t s, boo
 cudaError_t launch_accept_sample(const MiscParams& p, int B, cudaStream_t s, bool pdl);
 cudaError_t launch_compact(const MiscParams& p, int B, int n_act, cudaStream_t s, bool pdl);
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* src, float* dst, size_t n, cudaStream_t s);
+// The acceptance's Philox4x32-10 stream for one (seed, offset): words [n_req][n_slots][4] and/or
+// uniforms [n_req][n_slots] (either may be null).
+cudaError_t launch_philox_fill(uint64_t seed, uint64_t offset, int n_req, int n_slots, uint32_t* words, float* unif,
+                               cudaStream_t s);
 // Row-major [rows][cols] bf16 (rows % 128 == 0, cols % 64 == 0) -> pre-tiled, pre-swizzled blocks.
 cudaError_t launch_tile_weights(const __nv_bfloat16* src, __nv_bfloat16* dst, int rows, int cols, cudaStream_t s);
 
@@ -157,11 +159,20 @@ struct MkParams {
   const float* rope_sin;
   int* status;
   int* abort_word;
+  unsigned long long wait_ns;  // bound of every wait of the kernel
+  int withhold_flag;  // fault injection: withhold one dataflow flag so that a bounded wait runs out
+  // Tensor-memory staging of the weights (ts != 0): x_stages B-operand stages in their own ring,
+  // tw_slots weight slots of kps k-blocks in tensor memory behind n_acc accumulators of n_pad
+  // columns (n_acc * n_pad + tw_slots * kps * 32 <= 512).
+  int ts, x_stages, tw_slots, n_acc;
 };
-size_t mk_smem_bytes(int n_pad, int parts, int stages, int head_dim, int kps, size_t attn_extra);
+// x_stages > 0: the TS layout (weight ring of `stages` stages, B ring of x_stages, tw_slots
+// tensor-memory slots); 0: weights and B operand share `stages` ring stages.
+size_t mk_smem_bytes(int n_pad, int parts, int stages, int head_dim, int kps, size_t attn_extra, int x_stages = 0,
+                     int tw_slots = 0);
 size_t mk_trace_slots();
 cudaError_t mk_prepare();
-int mk_max_blocks_per_sm(int head_dim, size_t smem);
+int mk_max_blocks_per_sm(int head_dim, bool ts, size_t smem);
 cudaError_t launch_verify_mk(const MkParams& p, int grid, size_t smem, cudaStream_t s);
 
 // Records the message tss_last_error() returns on the calling thread.

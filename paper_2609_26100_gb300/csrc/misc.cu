@@ -7,8 +7,9 @@ namespace tss {
 // ------------------------------------------------------------------------------------------
 // Skip controller (Sec. "Domain-Aware Skip Controller", first equation; Sec.
 // "Domain-to-Configuration Mapping"): S(x) = Phi(d(x)) if the domain is configured, else the
-// empty set.  From the requests' skip sets it builds, on the device, the ascending list of layers
-// that at least one request runs (the only layers that get launches) and, per layer, the
+// empty set -- looked up on the host when the step is enqueued and passed in the step
+// descriptor.  From the requests' skip sets it builds, on the device, the ascending list of
+// layers that at least one request runs (the only layers that get launches) and, per layer, the
 // compacted list of rows of the requests that run it.
 // ------------------------------------------------------------------------------------------
 __device__ void controller_body(const MiscParams& p) {
@@ -19,9 +20,7 @@ __device__ void controller_body(const MiscParams& p) {
   __shared__ int s_n;
   const int B = st->B, L = p.n_layers;
   for (int b = threadIdx.x; b < B; b += blockDim.x) {
-    const int dom = st->req_domain[b];
-    const unsigned long long m =
-        (dom >= 0 && dom < p.max_domains && p.phi_valid[dom]) ? p.phi_mask[dom] : 0ull;  // dense fallback
+    const unsigned long long m = st->req_phi[b];
     smask[b] = m;
     pl->req_mask[b] = m;
   }
@@ -225,11 +224,42 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1
   return c;
 }
 
+// The generator's output for uniform slot `slot` of request b: counter (slot, request, offset lo,
+// offset hi), key (seed lo, seed hi); the uniform is (first word >> 8) * 2^-24, exact in fp32.
+__device__ __forceinline__ uint4 philox_slot(uint32_t seed_lo, uint32_t seed_hi, uint32_t off_lo, uint32_t off_hi,
+                                             int b, int slot) {
+  return philox4x32_10(make_uint4(static_cast<uint32_t>(slot), static_cast<uint32_t>(b), off_lo, off_hi), seed_lo,
+                       seed_hi);
+}
+__device__ __forceinline__ float uniform24(uint32_t x) { return static_cast<float>(x >> 8) * (1.f / 16777216.f); }
+
 __device__ __forceinline__ double draw_uniform(const StepDesc* st, int b, int slot) {
   if (st->uniforms) return static_cast<double>(st->uniforms[static_cast<size_t>(b) * st->uniform_stride + slot]);
-  const uint4 x = philox4x32_10(make_uint4(static_cast<uint32_t>(slot), static_cast<uint32_t>(b), st->off_lo, st->off_hi),
-                                st->seed_lo, st->seed_hi);
-  return static_cast<double>(x.x >> 8) * (1.0 / 16777216.0);
+  return static_cast<double>(uniform24(philox_slot(st->seed_lo, st->seed_hi, st->off_lo, st->off_hi, b, slot).x));
+}
+
+// Diagnostic: the generator's words and uniforms for requests [0, n_req) and slots [0, n_slots)
+// of one (seed, offset), laid out [request][slot] (the stream the acceptance draws from).
+__global__ void philox_fill_kernel(uint32_t seed_lo, uint32_t seed_hi, uint32_t off_lo, uint32_t off_hi, int n_req,
+                                   int n_slots, uint4* words, float* unif) {
+  const size_t n = static_cast<size_t>(n_req) * n_slots;
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const int b = static_cast<int>(i / n_slots), slot = static_cast<int>(i - static_cast<size_t>(b) * n_slots);
+    const uint4 x = philox_slot(seed_lo, seed_hi, off_lo, off_hi, b, slot);
+    if (words) words[i] = x;
+    if (unif) unif[i] = uniform24(x.x);
+  }
+}
+
+cudaError_t launch_philox_fill(uint64_t seed, uint64_t offset, int n_req, int n_slots, uint32_t* words, float* unif,
+                               cudaStream_t s) {
+  const size_t n = static_cast<size_t>(n_req) * n_slots;
+  const int blocks = static_cast<int>((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
+  philox_fill_kernel<<<blocks, 256, 0, s>>>(static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32),
+                                            static_cast<uint32_t>(offset), static_cast<uint32_t>(offset >> 32), n_req,
+                                            n_slots, reinterpret_cast<uint4*>(words), unif);
+  return cudaGetLastError();
 }
 
 template <typename T, typename Op>
@@ -432,10 +462,7 @@ __global__ void __launch_bounds__(256) prologue_kernel(const MiscParams p, float
   __shared__ int s_l0, s_crow;
   // The first norm phase is the QKV of the union's first layer (or the LM head when every layer
   // is skipped); find this row's compacted position in it, as the controller does.
-  for (int b = threadIdx.x; b < st->B; b += blockDim.x) {
-    const int dom = st->req_domain[b];
-    smask[b] = (dom >= 0 && dom < p.max_domains && p.phi_valid[dom]) ? p.phi_mask[dom] : 0ull;
-  }
+  for (int b = threadIdx.x; b < st->B; b += blockDim.x) smask[b] = st->req_phi[b];
   __syncthreads();
   if (threadIdx.x == 0) {
     int l0 = -1;

@@ -8,10 +8,12 @@
 // This entry point runs the same GEMM kernel with that scratch taken from file-scope device
 // arrays instead, so it needs no context and allocates nothing.
 //
-// The arrays are part of the library image: every GPU that loads libtss.so holds them
-// (kStaticPartialBytes + counters) until the process exits.  Every call on a device shares them,
-// so two calls that overlap on the GPU (different streams, or different host threads) race and
-// may return wrong results; serialise them on one stream.
+// The arrays belong to this file's CUDA module, which the runtime loads on a device (lazily, at
+// the first call on that device, under CUDA's default lazy module loading): from then on the GPU
+// holds them (kStaticPartialBytes + counters + a status word) until the process exits.  A caller
+// that hands the rest of the device memory to its own pool should make one call first.  Every
+// call on a device shares them, so two calls that overlap on the GPU (different streams, or
+// different host threads) race and may return wrong results; serialise them on one stream.
 #include <cudaTypedefs.h>
 
 #include <mutex>
@@ -29,26 +31,32 @@ constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) float g_static_partials[kStaticPartialFloats];
 static __device__ __align__(256) int g_static_counters[kStaticCounters];
+// First failure of a device-side check or bounded wait since the last tss_linear_static_status
+// (0: none); the GEMM kernel records it and never traps.
+static __device__ __align__(256) int g_static_status;
 
 struct DeviceScratch {
   bool ready = false;
   float* partials = nullptr;  // device addresses of the arrays above on this device
   int* counters = nullptr;
+  int* status = nullptr;
   int num_sms = 0;
 };
 DeviceScratch g_dev[kMaxDevices];
 std::mutex g_mu;
+std::once_flag g_encode_once;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 bool encode(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows, int rank) {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
+  std::call_once(g_encode_once, [] {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
-        q != cudaDriverEntryPointSuccess)
-      return false;
-    fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  const PFN_cuTensorMapEncodeTiled_v12000 fn = g_encode;
+  if (!fn) return false;
   cuuint64_t dims[3] = {inner, rows, 1};
   cuuint64_t strides[2] = {inner * 2, inner * rows * 2};
   cuuint32_t box[3] = {64, box_rows, 1};
@@ -79,6 +87,8 @@ tss_status setup_device(int dev, DeviceScratch** out) {
     e = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.partials), g_static_partials);
     if (e != cudaSuccess) return reject(TSS_ERR_CUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e));
     e = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.counters), g_static_counters);
+    if (e != cudaSuccess) return reject(TSS_ERR_CUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e));
+    e = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.status), g_static_status);
     if (e != cudaSuccess) return reject(TSS_ERR_CUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e));
     e = tss::gemm_prepare(232448);  // the per-block shared-memory maximum of sm_103 (227 KiB)
     if (e != cudaSuccess) return reject(TSS_ERR_CUDA, std::string("cudaFuncSetAttribute: ") + cudaGetErrorString(e));
@@ -135,11 +145,30 @@ extern "C" tss_status tss_linear_static(const void* x, const void* w, float* y, 
   g.layer_fixed = 0;
   g.partials = ds->partials;
   g.counters = ds->counters;
-  g.status = nullptr;
+  g.status = ds->status;
   g.out = y;
   g.out_ld = n_out;
   g.o_real = n_out;
   e = tss::launch_gemm(tss::kEpiStore, tw, tx, g, grid, tss::gemm_smem_bytes(n_pad, stages), s, false);
   if (e != cudaSuccess) return reject(TSS_ERR_CUDA, std::string("launch: ") + cudaGetErrorString(e));
+  return TSS_OK;
+}
+
+// Synchronise `stream`, then return and clear the status word of the current device.
+extern "C" tss_status tss_linear_static_status(void* stream) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return reject(TSS_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
+  if (dev < 0 || dev >= kMaxDevices) return reject(TSS_ERR_UNSUPPORTED_ARCH, "device index beyond 63");
+  DeviceScratch* ds = nullptr;
+  tss_status st = setup_device(dev, &ds);
+  if (st != TSS_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int v = 0;
+  e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess) e = cudaMemcpy(&v, ds->status, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemset(ds->status, 0, sizeof(int));
+  if (e != cudaSuccess) return reject(TSS_ERR_CUDA, std::string("status read: ") + cudaGetErrorString(e));
+  if (v != 0) return reject(v, std::string("device status of tss_linear_static: ") + tss_status_string(v));
   return TSS_OK;
 }

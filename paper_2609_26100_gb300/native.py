@@ -27,7 +27,8 @@ EXPORTS = (
     "tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status", "tss_destroy",
     "tss_linear", "tss_linear_static", "tss_read_trace", "tss_status_string", "tss_last_error",
-    "tss_estimate_step_bytes",
+    "tss_estimate_step_bytes", "tss_persistent_plan", "tss_inject_timeout", "tss_philox_uniforms",
+    "tss_linear_static_status",
 )
 
 _P = ctypes.c_void_p
@@ -70,6 +71,11 @@ class TssStepBytes(ctypes.Structure):
                 ("total", ctypes.c_uint64), ("active_union", ctypes.c_int)]
 
 
+class TssPersistentPlanInfo(ctypes.Structure):
+    _fields_ = [("fits", ctypes.c_int), ("kps", ctypes.c_int), ("stages", ctypes.c_int), ("attn_splits", ctypes.c_int),
+                ("smem_bytes", ctypes.c_uint64), ("tmem_weight_slots", ctypes.c_int)]
+
+
 class TssVerifyResult(ctypes.Structure):
     _fields_ = [("accept_len", _P), ("bonus", _P), ("path", _P), ("path_stride", ctypes.c_int),
                 ("new_ctx_len", _P), ("logits", _P)]
@@ -108,9 +114,15 @@ def lib() -> ctypes.CDLL:
         L.tss_last_error.restype = ctypes.c_char_p
         L.tss_estimate_step_bytes.argtypes = [ctypes.POINTER(TssArch), ctypes.c_int, ctypes.POINTER(ctypes.c_uint64),
                                               _I32P, _I32P, ctypes.POINTER(TssStepBytes)]
+        L.tss_persistent_plan.argtypes = [ctypes.POINTER(TssArch), ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                          ctypes.c_int, ctypes.POINTER(TssPersistentPlanInfo)]
+        L.tss_inject_timeout.argtypes = [_P, ctypes.c_int]
+        L.tss_philox_uniforms.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int, ctypes.c_int, _P, _P, _P]
+        L.tss_linear_static_status.argtypes = [_P]
         for name in ("tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
                      "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status",
-                     "tss_linear", "tss_linear_static", "tss_read_trace", "tss_estimate_step_bytes"):
+                     "tss_linear", "tss_linear_static", "tss_read_trace", "tss_estimate_step_bytes",
+                     "tss_persistent_plan", "tss_inject_timeout", "tss_philox_uniforms", "tss_linear_static_status"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -121,6 +133,31 @@ def linear_static(x, w, y, stream=None) -> None:
     m, k = x.shape
     check(lib().tss_linear_static(x.data_ptr(), w.data_ptr(), y.data_ptr(), m, k, w.shape[0], stream),
           "tss_linear_static")
+
+
+def linear_static_status(stream=None) -> int:
+    """tss_linear_static_status: synchronise, return and clear the static linear layer's status."""
+    return lib().tss_linear_static_status(stream)
+
+
+def philox_uniforms(seed: int, offset: int, words=None, uniforms=None, stream=None) -> None:
+    """tss_philox_uniforms into device tensors words [n_req][n_slots][4] (int32 or uint32 bits)
+    and/or uniforms [n_req][n_slots] (float32)."""
+    t = words if words is not None else uniforms
+    n_req, n_slots = int(t.shape[0]), int(t.shape[1])
+    check(lib().tss_philox_uniforms(int(seed), int(offset), n_req, n_slots, _ptr(words), _ptr(uniforms), stream),
+          "tss_philox_uniforms")
+
+
+def persistent_plan(arch, n_req: int, n_rows: int, max_keys: int, num_sms: int) -> Dict[str, int]:
+    """tss_persistent_plan: the persistent kernel's shared-memory plan for a step (host only)."""
+    a = TssArch(arch.n_layers, arch.d_model, arch.n_heads, arch.head_dim, arch.d_mlp, arch.vocab,
+                arch.rms_eps, arch.rope_theta, 1, 1, 1, 1, 1)
+    out = TssPersistentPlanInfo()
+    check(lib().tss_persistent_plan(ctypes.byref(a), n_req, n_rows, max_keys, num_sms, ctypes.byref(out)),
+          "tss_persistent_plan")
+    return {"fits": bool(out.fits), "kps": out.kps, "stages": out.stages, "attn_splits": out.attn_splits,
+            "smem_bytes": out.smem_bytes, "tmem_weight_slots": out.tmem_weight_slots}
 
 
 def estimate_step_bytes(arch, masks: Sequence[int], ctx_len: Sequence[int], n_nodes: Sequence[int]) -> Dict[str, int]:
@@ -208,6 +245,9 @@ class Verifier:
 
     def sync_status(self, stream=None) -> int:
         return lib().tss_sync_status(self.ctx, stream)
+
+    def inject_timeout(self, n_steps: int) -> None:
+        check(lib().tss_inject_timeout(self.ctx, n_steps), "tss_inject_timeout")
 
     def linear(self, x, w, y, stream=None) -> None:
         m, k = x.shape

@@ -29,10 +29,11 @@ class TssRunner:
         self.kv_struct = self.v.make_kv([t.data_ptr() if t is not None else None for t in self.kv], n_slots, kv_cap)
 
     @classmethod
-    def for_workload(cls, w: synth.Workload, device: str = "cuda") -> "TssRunner":
+    def for_workload(cls, w: synth.Workload, device: str = "cuda", extra_cap: int = 0) -> "TssRunner":
         """The configuration bench.py times for workload w: seeded weights of the layers some
         request runs (generated on the device), one KV slot per request sized to its context plus
-        the draft block, synthetic context KV, and the workload's skip configurations."""
+        the draft block (plus extra_cap positions for runs of several steps), synthetic context
+        KV, and the workload's skip configurations."""
         a = w.arch
         union = w.active_union()
         max_ctx = max(r.ctx_len for r in w.requests)
@@ -42,7 +43,7 @@ class TssRunner:
             if weights["layers"][l] is None:
                 weights["layers"][l] = {k: torch.zeros(s, dtype=torch.bfloat16, device=device)
                                         for k, s in synth.layer_shapes(a).items()}
-        run = cls(a, weights, n_slots=len(w.requests), kv_cap=max_ctx + max_n + 8, max_batch=len(w.requests),
+        run = cls(a, weights, n_slots=len(w.requests), kv_cap=max_ctx + max_n + 8 + extra_cap, max_batch=len(w.requests),
                   max_rows=max(16, w.n_rows), max_nodes=max_n, kv_layers=union, device=device)
         del weights
         if device != "cpu":

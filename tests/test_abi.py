@@ -94,7 +94,8 @@ def test_binding_structs_match_the_c_layout(tmp_path):
         pytest.skip("no C compiler")
     structs = {"tss_arch": native.TssArch, "tss_weights": native.TssWeights, "tss_verify_batch": native.TssVerifyBatch,
                "tss_kv_cache": native.TssKvCache, "tss_verify_result": native.TssVerifyResult,
-               "tss_kernel_times": native.TssKernelTimes}
+               "tss_kernel_times": native.TssKernelTimes, "tss_step_bytes": native.TssStepBytes,
+               "tss_persistent_plan_info": native.TssPersistentPlanInfo}
     lines = ["#include \"tss.h\"", "#include <stdio.h>", "#include <stddef.h>", "int main(void) {"]
     for cname, py in structs.items():
         lines.append(f"  printf(\"{cname} size %zu\\n\", sizeof({cname}));")

@@ -2,11 +2,14 @@
 uses for its roofline (synth.algorithmic_bytes, a separate Python implementation): the five
 benchmark workloads, random mixed batches, and the argument checks."""
 import dataclasses
+import os
 
 import numpy as np
 import pytest
 
 from paper_2609_26100_gb300 import native, synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 def _c_bytes(w):
@@ -60,3 +63,23 @@ def test_argument_checks():
         native.estimate_step_bytes(a, [0], [-1], [1])
     with pytest.raises(native.TssError):
         native.estimate_step_bytes(a, [], [], [])
+
+
+def test_bench_counts_the_step_descriptor_it_uploads(tmp_path):
+    """bench.py's e2e copy count includes the per-step descriptor: its constant equals the size of
+    the struct tss_verify copies (compiled here with nvcc, host code only)."""
+    import shutil
+    import subprocess
+    import bench
+    nvcc = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
+    if not os.path.exists(nvcc) and not shutil.which("nvcc"):
+        pytest.skip("no nvcc")
+    src = tmp_path / "sd.cu"
+    src.write_text('#include "common.cuh"\n#include <cstdio>\n'
+                   'int main() { printf("%zu\\n", sizeof(tss::StepDesc)); return 0; }\n')
+    exe = tmp_path / "sd"
+    csrc = os.path.join(ROOT, "paper_2609_26100_gb300", "csrc")
+    r = subprocess.run([nvcc, "-std=c++17", "-I", csrc, str(src), "-o", str(exe)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
+    assert int(out) == bench.STEP_DESC_BYTES
