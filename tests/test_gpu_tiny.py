@@ -657,3 +657,22 @@ def test_device_philox_matches_the_oracle_generator():
     assert np.array_equal(O.philox_uniforms(42, 3, 7, 5), P.to_uniform24(
         P.philox4x32_10(np.stack([np.arange(11, dtype=np.uint64), np.full(11, 7, np.uint64), np.full(11, 3, np.uint64),
                                   np.zeros(11, np.uint64)], -1), np.array([42, 0], np.uint64))[:, 0]))
+
+
+def test_search_with_measured_verification_latency(weights):
+    """Algorithm 1 with the verification cost C_d(S) measured by tss_verify on the GPU (tiny model,
+    every subset of its 4 layers up to depth 2, synthetic acceptance and metric): the dense step
+    is slower than every 2-layer skip, and the chosen set is feasible."""
+    w, wo, wg = weights
+    from paper_2609_26100_gb300 import search
+    run = make_runner(wg, n_slots=1, cap=128)
+    reqs = [synth.Request(64, synth.chain_parents(4), [1, 2, 3, 4, 5], 0)]
+    cost = search.latency_cost(run, reqs, steps=20)
+    res = search.breadth_search(ARCH.n_layers, search.combine(search.SyntheticObjective(ARCH.n_layers, 7), cost), 2,
+                                0.3, 0.05, 0.3, 0.05)
+    lat = {s: e.cost for s, e in res.log}
+    print(f"[search] latency us by skip set: { {str(s): round(v, 1) for s, v in lat.items()} }")
+    assert all(lat[()] > v for s, v in lat.items() if len(s) == 2)
+    assert res.best in [s for k in res.feasible for s in res.feasible[k]]
+    assert run.sync_status() == native.TSS_OK
+    run.close()
