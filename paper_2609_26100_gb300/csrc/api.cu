@@ -127,6 +127,10 @@ struct tss_ctx {
   int w_evict_first = 1;
   int mk_max_stages = 12;
   bool mk_tmem = kMkTmemDefault;  // stage the weights in tensor memory where it has room (TSS_MK_TMEM)
+  int mk_tw_max = 16, mk_sx_max = 8;  // caps on its weight slots and B-operand stages (TSS_MK_TW, TSS_MK_SX)
+  int mk_ts_pre = 1;  // stage the first O-phase weights before the attention (TSS_MK_TS_PRE)
+  int mk_spin_roles = 0;  // warps that poll mbarriers without the suspend hint (TSS_MK_SPIN, bit mask)
+  int mk_dp_tail = 1;  // whole-tile tails for phases with a tile per CTA (TSS_MK_DP)
   int attn_plo = 1;
   int attn_splits_force = 0;  // > 0: key splits of the separate attention kernel (TSS_ATTN_SPLITS)
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
@@ -386,9 +390,13 @@ struct MkConfig {
 // What the persistent kernel's shared-memory plan depends on (a context's shape and switches).
 struct MkPlanIn {
   int D, H, num_sms, kps_max, stages_max, max_splits, ts;
+  int tw_max = 16, sx_max = 8;  // caps on tensor-memory weight slots and B-operand stages
 };
 MkPlanIn mk_plan_in(const tss_ctx* c) {
-  return MkPlanIn{c->D, c->H, c->num_sms, c->mk_kps, c->mk_max_stages, c->max_splits, c->mk_tmem ? 1 : 0};
+  MkPlanIn in{c->D, c->H, c->num_sms, c->mk_kps, c->mk_max_stages, c->max_splits, c->mk_tmem ? 1 : 0};
+  in.tw_max = c->mk_tw_max;
+  in.sx_max = c->mk_sx_max;
+  return in;
 }
 
 // Tensor-memory staging (TS) for an MMA width n_pad: accumulator buffers (2..8, about 128
@@ -462,11 +470,12 @@ bool mk_config_for(const MkPlanIn& c, int B, int M, int tiles, MkConfig* out) {
     const size_t stage = static_cast<size_t>(kps) * 16384 + x_stage;
     int n_acc = 0, tw = 0;
     if (c.ts) mk_ts_slots(xs.rows, kps, &n_acc, &tw);
+    tw = std::min(tw, c.tw_max);
     for (int S = c.stages_max; S >= 2; --S) {
       // TS: the B operand in its own ring of up to 8 stages (at least 2) behind S weight stages
       int SX = 0;
       if (tw >= 2) {
-        SX = 8;
+        SX = std::max(2, c.sx_max);
         while (SX > 2 && mk_smem_bytes(xs.rows, xs.parts, S, c.D, kps, 0, SX, tw) > kLimit) --SX;
       }
       const size_t ring = SX > 0 ? S * static_cast<size_t>(kps) * 16384 + SX * x_stage : S * stage;
@@ -528,6 +537,9 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.kps = kps;
   p.xs = xs;
   p.ts = cfg.ts;
+  p.ts_pre = c->mk_ts_pre;
+  p.spin_roles = c->mk_spin_roles;
+  p.dp_tail = c->mk_dp_tail;
   p.x_stages = cfg.x_stages;
   p.tw_slots = cfg.tw_slots;
   p.n_acc = cfg.n_acc;
@@ -986,6 +998,11 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_ATTN_SPLITS")) c->attn_splits_force = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
   if (const char* e = std::getenv("TSS_MK_TMEM")) c->mk_tmem = std::atoi(e) != 0;
+  if (const char* e = std::getenv("TSS_MK_TW")) c->mk_tw_max = std::max(2, std::min(16, std::atoi(e)));
+  if (const char* e = std::getenv("TSS_MK_SX")) c->mk_sx_max = std::max(2, std::min(8, std::atoi(e)));
+  if (const char* e = std::getenv("TSS_MK_TS_PRE")) c->mk_ts_pre = std::atoi(e) != 0;
+  if (const char* e = std::getenv("TSS_MK_SPIN")) c->mk_spin_roles = std::atoi(e) & 0xff;
+  if (const char* e = std::getenv("TSS_MK_DP")) c->mk_dp_tail = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ALLOC_LIMIT_BYTES")) c->alloc_limit = std::strtoull(e, nullptr, 10);
   if (const char* e = std::getenv("TSS_WAIT_LIMIT_MS")) {
     const long long ms = std::atoll(e);

@@ -165,6 +165,9 @@ struct MkParams {
   // tw_slots weight slots of kps k-blocks in tensor memory behind n_acc accumulators of n_pad
   // columns (n_acc * n_pad + tw_slots * kps * 32 <= 512).
   int ts, x_stages, tw_slots, n_acc;
+  int ts_pre;  // TS: the first O-phase weight stages reach tensor memory before the attention
+  int spin_roles;  // bit w: warp w polls mbarriers without the suspend hint
+  int dp_tail;     // phases with a tile per CTA end with one whole tile per CTA (no fix-up on their tail)
 };
 // x_stages > 0: the TS layout (weight ring of `stages` stages, B ring of x_stages, tw_slots
 // tensor-memory slots); 0: weights and B operand share `stages` ring stages.

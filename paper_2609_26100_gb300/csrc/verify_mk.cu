@@ -86,6 +86,7 @@ struct MkShared {
   int* abort_g;
   int* status;
   uint64_t limit_ns;  // bound of every wait (create-time setting, 2 s by default)
+  bool spin;          // poll mbarriers without the suspend hint
 };
 
 __device__ __forceinline__ bool mk_aborted(const MkShared& sh) {
@@ -125,7 +126,7 @@ __device__ bool mk_wait_bar(uint64_t* bar, uint32_t parity, const MkShared& sh) 
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (sh.spin ? mbar_try_wait(bar, parity) : mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     if ((i & 255) == 0) {
       if (mk_aborted(sh)) return false;
       if (globaltimer_ns() - t0 > sh.limit_ns) {
@@ -192,16 +193,39 @@ __device__ __forceinline__ const __nv_bfloat16* mk_weights(const MkParams& p, co
   return base + static_cast<size_t>(ph.layer) * blocks * kTileElems;
 }
 
-// CTA c's stream-K range of a phase over geff = min(grid, iterations) CTAs.
-__device__ __forceinline__ void mk_range(const MkPhase& ph, int c, int G, long long& it0, long long& it1, int& geff) {
-  const long long T = static_cast<long long>(ph.n_tiles) * ph.kb;
-  geff = static_cast<int>(T < G ? T : G);
-  if (c >= geff) {
-    it0 = it1 = 0;
-    return;
+// CTA c's share of a phase as a sequence of segments (tile t, k-blocks [k0, k1)): stream-K over
+// every iteration (tile x k-block) of the phase; or, when the phase has at least one tile per CTA
+// and p.dp_tail is set, stream-K over its first n_tiles - G tiles followed by one whole tile per
+// CTA, so that the phase ends with whole-tile epilogues (no partial tiles, no arrival counter,
+// no reload of other CTAs' partials on its critical tail).  Residual phases keep plain stream-K.
+struct MkSeg {
+  long long it, it1;  // stream-K iterations of this CTA still to take
+  long long T;        // stream-K iterations of the phase (the fix-up contributor arithmetic)
+  int geff;           // CTAs sharing them
+  int kb, whole;      // this CTA's whole tile after them, -1: none
+  __device__ __forceinline__ bool next(int& t, int& k0, int& k1);
+  __device__ __forceinline__ bool done() const { return it >= it1 && whole < 0; }
+  __device__ __forceinline__ long long start() const { return it; }
+};
+
+__device__ __forceinline__ MkSeg mk_seg(const MkParams& p, const MkPhase& ph, int c, int G) {
+  MkSeg s;
+  s.kb = ph.kb;
+  s.whole = -1;
+  int n_split = ph.n_tiles;
+  if (p.dp_tail && ph.n_tiles >= G && ph.kind != kMkO && ph.kind != kMkDown) {
+    n_split = ph.n_tiles - G;
+    s.whole = n_split + c;
   }
-  it0 = T * c / geff;
-  it1 = T * (c + 1) / geff;
+  s.T = static_cast<long long>(n_split) * ph.kb;
+  s.geff = static_cast<int>(s.T < G ? s.T : G);
+  if (c >= s.geff) {
+    s.it = s.it1 = 0;
+  } else {
+    s.it = s.T * c / s.geff;
+    s.it1 = s.T * (c + 1) / s.geff;
+  }
+  return s;
 }
 
 __device__ __forceinline__ int mk_cta_of(long long i, long long T, int G) {
@@ -216,6 +240,16 @@ __device__ __forceinline__ bool mk_next_segment(long long& it, long long end, in
   const long long e = end < tile_end ? end : tile_end;
   k1 = static_cast<int>(e - static_cast<long long>(t) * kb);
   it = e;
+  return true;
+}
+
+__device__ __forceinline__ bool MkSeg::next(int& t, int& k0, int& k1) {
+  if (mk_next_segment(it, it1, kb, t, k0, k1)) return true;
+  if (whole < 0) return false;
+  t = whole;
+  k0 = 0;
+  k1 = kb;
+  whole = -1;
   return true;
 }
 
@@ -773,6 +807,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   sh.abort_g = p.abort_word;
   sh.status = p.status;
   sh.limit_ns = p.wait_ns;
+  sh.spin = (p.spin_roles >> (threadIdx.x >> 5)) & 1;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -859,20 +894,18 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   // weight stages [j_lo, j_hi) of this CTA's range of a phase (j counts its stages in order):
   // warp 0 lane 0 issues their bulk copies into the ring
   auto produce = [&](const MkPhase& ph, int pi, int j_lo, int j_hi) -> bool {
-    long long it0, it1;
-    int geff;
-    mk_range(ph, c, G, it0, it1, geff);
+    MkSeg seg = mk_seg(p, ph, c, G);
     const __nv_bfloat16* wl = mk_weights(p, ph);
-    long long it = it0;
     int t, k0, k1, j = 0;
-    while (j < j_hi && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
+    while (j < j_hi && seg.next(t, k0, k1)) {
+      const bool last_seg = seg.done();
       for (int kc = k0; kc < k1 && j < j_hi; kc += KPS, ++j) {
         if (j < j_lo) continue;
         const int nk = min(KPS, k1 - kc);
         const int s = static_cast<int>(i % S);
         if (!mk_wait_bar(&empty[s], static_cast<uint32_t>((i / S) & 1) ^ 1u, sh)) return false;
-        if (static_cast<long long>(t) * ph.kb + kc == it0) mk_trace(p, pi * 8 + 0);
-        if (static_cast<long long>(t) * ph.kb + kc + nk == it1) mk_trace(p, pi * 8 + 1);
+        if (j == 0) mk_trace(p, pi * 8 + 0);
+        if (last_seg && kc + nk == k1) mk_trace(p, pi * 8 + 1);
         mbar_arrive_expect_tx(&full[s], nk * kMkWBytes);
         if (p.w_evict_first)
           bulk_load_hint(sW + static_cast<size_t>(s) * sw_bytes,
@@ -892,12 +925,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   int last_empty = -1;  // ring slot and phase parity of the copier's latest release
   uint32_t last_par = 0;
   auto copy_stages = [&](const MkPhase& ph, int j_lo, int j_hi, bool drain) -> bool {
-    long long it0, it1;
-    int geff;
-    mk_range(ph, c, G, it0, it1, geff);
-    long long it = it0;
+    MkSeg seg = mk_seg(p, ph, c, G);
     int t, k0, k1, j = 0;
-    while (j < j_hi && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
+    while (j < j_hi && seg.next(t, k0, k1)) {
       for (int kc = k0; kc < k1 && j < j_hi; kc += KPS, ++j) {
         if (j < j_lo) continue;
         const int nk = min(KPS, k1 - kc);
@@ -923,12 +953,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   };
   // stages of this CTA's range of a phase
   auto stage_count = [&](const MkPhase& ph) -> int {
-    long long it0, it1;
-    int geff;
-    mk_range(ph, c, G, it0, it1, geff);
-    long long it = it0;
+    MkSeg seg = mk_seg(p, ph, c, G);
     int t, k0, k1, n = 0;
-    while (mk_next_segment(it, it1, ph.kb, t, k0, k1)) n += (k1 - k0 + KPS - 1) / KPS;
+    while (seg.next(t, k0, k1)) n += (k1 - k0 + KPS - 1) / KPS;
     return n;
   };
 
@@ -937,8 +964,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     const bool att = ph.kind == kMkO && !p.attn_external;
     // TS: before a layer's attention borrows the ring, the weight stream already brings the first
     // O-phase stages (as many as the tensor-memory slots hold) into tensor memory
-    const int npre = TS && att && (warp == 0 || warp == 3) ? min(TW, stage_count(ph)) : 0;
-    if (TS && att && (warp == 0 || warp == 3)) {
+    const int npre = TS && att && p.ts_pre && (warp == 0 || warp == 3) ? min(TW, stage_count(ph)) : 0;
+    if (TS && att && p.ts_pre && (warp == 0 || warp == 3)) {
       bool good = true;
       if (lane == 0) good = warp == 0 ? produce(ph, pi, 0, npre) : copy_stages(ph, 0, npre, true);
       ok = __shfl_sync(0xffffffffu, good, 0);
@@ -963,12 +990,10 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     } else if (warp == 1) {
       // ---------------- MMA issuer (lane 0) ----------------
       if (lane == 0) {
-        long long it0, it1;
-        int geff;
-        mk_range(ph, c, G, it0, it1, geff);
-        long long it = it0;
+        MkSeg seg = mk_seg(p, ph, c, G);
         int t, k0, k1;
-        while (ok && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
+        bool first = true;
+        while (ok && seg.next(t, k0, k1)) {
           const int buf = use % NB;
           if (!mk_wait_bar(&acce[buf], static_cast<uint32_t>((use / NB) & 1) ^ 1u, sh)) {
             ok = false;
@@ -986,7 +1011,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
                 break;
               }
               tc_fence_after();
-              if (kc == k0 && static_cast<long long>(t) * ph.kb + k0 == it0) mk_trace(p, pi * 8 + 4);
+              if (first) mk_trace(p, pi * 8 + 4);
+              first = false;
               const uint32_t acol = tmem_base + tw_col + static_cast<uint32_t>(ts * KPS * 32);
               for (int j = 0; j < nk; ++j) {
                 const uint32_t b0 = smem_u32(sX + static_cast<size_t>(sx) * sx_bytes + j * XP * x_bytes);
@@ -1014,7 +1040,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
               break;
             }
             tc_fence_after();
-            if (kc == k0 && static_cast<long long>(t) * ph.kb + k0 == it0) mk_trace(p, pi * 8 + 4);
+            if (first) mk_trace(p, pi * 8 + 4);
+            first = false;
             for (int j = 0; j < nk; ++j) {
               const uint32_t a0 = smem_u32(sW + static_cast<size_t>(s) * sw_bytes + j * kMkWBytes);
               const uint32_t b0 = smem_u32(sX + static_cast<size_t>(s) * sx_bytes + j * XP * x_bytes);
@@ -1038,17 +1065,15 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           }
           if (!ok) break;
           umma_commit(&accf[buf]);
-          if (it >= it1) mk_trace(p, pi * 8 + 5);
+          if (seg.done()) mk_trace(p, pi * 8 + 5);
           ++use;
         }
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
     } else if (warp == 2) {
       // ---------------- B-operand producer: TMA after the producing tiles are flagged ----------------
-      long long it0, it1;
-      int geff;
-      mk_range(ph, c, G, it0, it1, geff);
-      if (it0 >= it1) continue;
+      MkSeg seg = mk_seg(p, ph, c, G);
+      if (seg.done()) continue;
       // dependency index space of this phase: h tiles, heads, or gate/up tiles
       const unsigned long long* flags;
       unsigned long long want;
@@ -1076,9 +1101,10 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           if (pl->slot_crow[ph.slot][b] >= 0 && ld_acquire_u64(&flags[b * p.H + x]) < want) return false;
         return true;
       };
-      long long it = it0;
       int t, k0, k1;
-      while (ok && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
+      bool first = true;
+      while (ok && seg.next(t, k0, k1)) {
+       const bool last_seg = seg.done();
        for (int kc = k0; ok && kc < k1; kc += KPS, ++i) {
         const int nk = min(KPS, k1 - kc);
         const int s = static_cast<int>(i % SX);
@@ -1121,22 +1147,20 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         }
         if (!ok) break;
         if (lane == 0) {
-          const long long g0 = static_cast<long long>(t) * ph.kb + kc;
-          if (g0 == it0) mk_trace(p, pi * 8 + 2);
-          if (g0 + nk == it1) mk_trace(p, pi * 8 + 3);
+          if (first) mk_trace(p, pi * 8 + 2);
+          if (last_seg && kc + nk == k1) mk_trace(p, pi * 8 + 3);
           fence_proxy_async_global();
           mbar_arrive_expect_tx(xf, nk * XP * x_bytes);
           bulk_load(sX + static_cast<size_t>(s) * sx_bytes, xsrc + static_cast<size_t>(kc) * XP * n_pad * 64, nk * XP * x_bytes,
                     xf);
         }
+        first = false;
        }
       }
     } else if (warp >= 4) {
       // ---------------- epilogues ----------------
-      long long it0, it1;
-      int geff;
-      mk_range(ph, c, G, it0, it1, geff);
-      if (it0 >= it1 && ph.kind != kMkQkv) continue;
+      MkSeg seg = mk_seg(p, ph, c, G);
+      if (seg.done() && ph.kind != kMkQkv) continue;
       // per-phase row metadata in shared memory (loaded while the first accumulator is pending)
       const int rslot = mk_row_slot(ph);
       e.M = pl->slot_M[rslot];
@@ -1173,12 +1197,12 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       e.kvrow = s_kvrow;
       e.nrows = s_nrows;
       e.hpre_tile = -1;
-      if ((ph.kind == kMkO || ph.kind == kMkDown) && it1 > it0 && e.M <= 16) {
+      if ((ph.kind == kMkO || ph.kind == kMkDown) && !seg.done() && e.M <= 16) {
         // h is final for this phase (only this phase's finaliser of a tile writes it): load the
         // rows of the CTA's last tile now, one thread per feature, into xch (unused by residual
         // epilogues), so that finalising that tile -- typically the phase's last -- skips a
         // memory round trip
-        const int tl = static_cast<int>((it1 - 1) / ph.kb);
+        const int tl = static_cast<int>((seg.it1 - 1) / ph.kb);  // (residual phases: plain stream-K)
         float hv[16];
 #pragma unroll
         for (int jj = 0; jj < 16; ++jj)
@@ -1226,7 +1250,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         named_bar_sync(1, 128);
       }
       bool rs_ready = false;
-      const long long T = static_cast<long long>(ph.n_tiles) * ph.kb;
+      const long long T = seg.T;
+      const int geff = seg.geff;
       float* partials = (pi & 1) ? p.partials1 : p.partials0;
       int* counters = p.counters + static_cast<size_t>(ph.kind) * p.max_tiles;
       const bool needs_rs = ph.kind == kMkQkv || ph.kind == kMkGu || ph.kind == kMkLm;
@@ -1236,20 +1261,21 @@ __global__ void __launch_bounds__(kMkThreads, 1)
         ok = false;
         break;
       }
-      long long it = it0;
       int t, k0, k1;
-      while (ok && mk_next_segment(it, it1, ph.kb, t, k0, k1)) {
+      bool first = true;
+      while (ok && seg.next(t, k0, k1)) {
         const int buf = use % NB;
         const bool got = e.et == 0 ? mk_wait_bar(&accf[buf], static_cast<uint32_t>((use / NB) & 1), sh) : true;
         if (!bar_and(1, 128, got)) {
           ok = false;
           break;
         }
-        if (e.et == 0 && static_cast<long long>(t) * ph.kb + k0 == it0) mk_trace(p, pi * 8 + 6);
+        if (e.et == 0 && first) mk_trace(p, pi * 8 + 6);
+        first = false;
         tc_fence_after();
         const uint32_t tb = tmem_base + (static_cast<uint32_t>(e.q * 32) << 16) + static_cast<uint32_t>(buf * n_pad);
         const int n_ch = (e.M + 15) >> 4;  // 16-token chunks of the accumulator
-        const bool tr_last = e.et == 0 && it >= it1;
+        const bool tr_last = e.et == 0 && seg.done();
         if (tr_last) mk_trace(p, kMkTraceSub + pi * 8 + 0);
         bool finalize = false;
         int cf = 0, cl = 0;
@@ -1354,7 +1380,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           const bool withheld = p.withhold_flag && ph.kind == kMkDown && ph.slot == 0 && t == 0;
           if (flag && e.et == 0 && !withheld) st_release_u64(flag, mk_seq(p.seq_base, ph.slot, ph.kind));
         }
-        if (e.et == 0 && it >= it1) mk_trace(p, pi * 8 + 7);
+        if (e.et == 0 && seg.done()) mk_trace(p, pi * 8 + 7);
         ++use;
       }
     }
