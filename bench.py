@@ -27,7 +27,7 @@ if ROOT not in sys.path:
 METRIC = "7B verify-step latency (us) & tokens/s at k=5, 4 skipped layers; % HBM roofline"
 # Bytes of the per-step descriptor tss_verify copies to the device (sizeof(tss::StepDesc);
 # tests/test_step_bytes.py compiles the struct and checks this number).
-STEP_DESC_BYTES = 7536
+STEP_DESC_BYTES = 9584
 NOMINAL_HBM_GBS = 8000.0
 
 

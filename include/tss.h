@@ -63,8 +63,10 @@ typedef struct tss_ctx tss_ctx; /* opaque; owns repacked weights and all workspa
  *   n_layers <= 64; head_dim 64 or 128; d_model = n_heads * head_dim, a multiple of 128 and at
  *   most 8192.
  *   max_batch: requests per verify (<= 64).  max_rows: total draft-block rows per verify
- *   (<= 256).  max_nodes: rows per request, root included (<= 64).  max_domains: size of the
- *   domain table Phi.  max_positions: RoPE positions must be < max_positions. */
+ *   (<= 256).  max_nodes: rows per request, root included (<= 128; a step with a block of more than 64 rows runs
+ *   each layer's attention as a separate kernel, the persistent kernel's in-kernel attention taking
+ *   blocks of up to 64).  max_domains: size of the domain table Phi.
+ *   max_positions: RoPE positions must be < max_positions. */
 typedef struct {
   int n_layers, d_model, n_heads, head_dim, d_mlp, vocab;
   float rms_eps, rope_theta;
@@ -96,7 +98,7 @@ typedef struct {
  * in request order; M = sum(n_nodes).  Row 0 of each block is the root (the last committed
  * token, whose KV is not yet cached); rows 1.. are draft nodes.
  *   n_nodes, ctx_len, domain_id, kv_slot, parent_idx, positions: HOST arrays.
- *     n_nodes[b]   in [1, max_nodes]
+ *     n_nodes[b]   in [1, max_nodes] (max_nodes <= 128)
  *     ctx_len[b]   tokens of request b already in its KV cache (>= 0)
  *     domain_id[b] key into Phi; an id never configured (or out of range) means dense
  *     kv_slot[b]   cache slot of request b (distinct); NULL means slot b
@@ -208,14 +210,13 @@ tss_status tss_estimate_step_bytes(const tss_arch* arch, int n_req, const uint64
  * draft-block rows in all, whose longest request spans max_keys keys (context + block), on a
  * GPU with num_sms SMs, under the default switches: fits = 1 when the plan fits the 227 KiB a
  * block may use (then tss_verify runs the step; otherwise it returns TSS_ERR_UNSUPPORTED_ARCH),
- * with the weight k-blocks per ring stage, the ring stages, the attention's key splits, the
- * dynamic shared memory of one block, and the weight stages held in tensor memory.  Pure host arithmetic: no context and no CUDA call.
+ * with the weight k-blocks per ring stage, the ring stages, the attention's key splits and the
+ * dynamic shared memory of one block.  Pure host arithmetic: no context and no CUDA call.
  * Errors: INVALID_ARG (NULL argument, head_dim not 64/128, n_req outside [1, 64], n_rows
  * outside [n_req, 256], max_keys or num_sms < 1). */
 typedef struct {
   int fits, kps, stages, attn_splits;
   uint64_t smem_bytes;
-  int tmem_weight_slots; /* stages of streamed weights held in tensor memory (0: weights read from shared memory) */
 } tss_persistent_plan_info;
 tss_status tss_persistent_plan(const tss_arch* arch, int n_req, int n_rows, int max_keys, int num_sms,
                                tss_persistent_plan_info* out);

@@ -69,8 +69,6 @@ struct GraphKey {
 };
 
 constexpr int kRing = 4;
-// Whether contexts stage the streamed weights in tensor memory by default (TSS_MK_TMEM overrides).
-constexpr bool kMkTmemDefault = false;
 constexpr int kMaxPathStride = 1024;
 
 }  // namespace
@@ -126,10 +124,6 @@ struct tss_ctx {
   int attn_mode = 0;  // 0 auto, 1 attention inside the persistent kernel, 2 separate attention kernels
   int w_evict_first = 1;
   int mk_max_stages = 12;
-  bool mk_tmem = kMkTmemDefault;  // stage the weights in tensor memory where it has room (TSS_MK_TMEM)
-  int mk_tw_max = 16, mk_sx_max = 8;  // caps on its weight slots and B-operand stages (TSS_MK_TW, TSS_MK_SX)
-  int mk_ts_pre = 1;  // stage the first O-phase weights before the attention (TSS_MK_TS_PRE)
-  int mk_spin_roles = 0;  // warps that poll mbarriers without the suspend hint (TSS_MK_SPIN, bit mask)
   int mk_dp_tail = 1;  // whole-tile tails for phases with a tile per CTA (TSS_MK_DP)
   int attn_plo = 1;
   int attn_splits_force = 0;  // > 0: key splits of the separate attention kernel (TSS_ATTN_SPLITS)
@@ -269,6 +263,7 @@ tss_status run_gemm(tss_ctx* c, int epi, const CUtensorMap& tmW, const CUtensorM
 
 struct StepPlan {
   int B, M, n_act, mode, splits, n_pad;
+  int max_nodes;      // rows of the largest request's block
   int tiles;          // 64-key tiles of the longest request (context + block)
   long long ctx_sum;  // context tokens over the batch
 };
@@ -331,6 +326,7 @@ tss_status enqueue_step(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* pr
   ap.o = c->obuf;
   ap.part_o = c->attn_po;
   ap.part_ml = c->attn_pml;
+  ap.wide = sp.max_nodes > kNarrowNodes ? 1 : 0;
   ap.counters = c->attn_cnt;
   ap.status = c->d_status;
   const int kbd = c->d / 64;
@@ -380,8 +376,6 @@ tss_status enqueue_step(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* pr
 struct MkConfig {
   int kps = 0, stages = 0, attn_splits = 1;
   size_t attn_extra = 0, smem = 0;
-  // tensor-memory staging of the weights: B-operand stages, weight slots, accumulator buffers
-  int ts = 0, x_stages = 0, tw_slots = 0, n_acc = 0;
 };
 
 // Key splits per (request, head) for the persistent kernel's attention: the fewest waves of
@@ -389,25 +383,10 @@ struct MkConfig {
 // of about three tiles.  Short contexts get about one item per CTA.
 // What the persistent kernel's shared-memory plan depends on (a context's shape and switches).
 struct MkPlanIn {
-  int D, H, num_sms, kps_max, stages_max, max_splits, ts;
-  int tw_max = 16, sx_max = 8;  // caps on tensor-memory weight slots and B-operand stages
+  int D, H, num_sms, kps_max, stages_max, max_splits;
 };
 MkPlanIn mk_plan_in(const tss_ctx* c) {
-  MkPlanIn in{c->D, c->H, c->num_sms, c->mk_kps, c->mk_max_stages, c->max_splits, c->mk_tmem ? 1 : 0};
-  in.tw_max = c->mk_tw_max;
-  in.sx_max = c->mk_sx_max;
-  return in;
-}
-
-// Tensor-memory staging (TS) for an MMA width n_pad: accumulator buffers (2..8, about 128
-// columns of them) and the weight slots of kps k-blocks (32 columns each) that fit behind them
-// in the 512 columns; 0 slots when fewer than two fit.
-void mk_ts_slots(int n_pad, int kps, int* n_acc, int* slots) {
-  const int nb = std::max(2, std::min(8, 128 / n_pad));
-  const int free_cols = 512 - nb * n_pad;
-  const int tw = free_cols > 0 ? free_cols / (kps * 32) : 0;
-  *n_acc = nb;
-  *slots = tw >= 2 ? std::min(tw, 16) : 0;
+  return MkPlanIn{c->D, c->H, c->num_sms, c->mk_kps, c->mk_max_stages, c->max_splits};
 }
 
 int mk_attn_splits(const MkPlanIn& c, int B, int tiles) {
@@ -460,26 +439,16 @@ int ext_attn_splits(const tss_ctx* c, const StepDesc* sd, int B) {
 // B requests with M rows in all, the longest one spanning `tiles` 64-key tiles.
 bool mk_config_for(const MkPlanIn& c, int B, int M, int tiles, MkConfig* out) {
   constexpr size_t kLimit = 232448;  // per-block shared-memory maximum of sm_103 (227 KiB)
-  const size_t q = static_cast<size_t>(kMaxNodes) * (c.D + 8) * 2;
+  const size_t q = static_cast<size_t>(kNarrowNodes) * (c.D + 8) * 2;
   const size_t tile = static_cast<size_t>(2) * 64 * (c.D + 8) * 2;
   const int splits = mk_attn_splits(c, B, std::max(tiles, 1));
   const int per = std::max(1, (std::max(tiles, 1) + splits - 1) / splits);
   for (int kps = c.kps_max; kps >= 1; --kps) {
     const XsLayout xs = xs_layout(M);
-    const size_t x_stage = static_cast<size_t>(kps) * xs.rows * xs.parts * 128;
-    const size_t stage = static_cast<size_t>(kps) * 16384 + x_stage;
-    int n_acc = 0, tw = 0;
-    if (c.ts) mk_ts_slots(xs.rows, kps, &n_acc, &tw);
-    tw = std::min(tw, c.tw_max);
+    const size_t stage = static_cast<size_t>(kps) * (16384 + static_cast<size_t>(xs.rows) * xs.parts * 128);
     for (int S = c.stages_max; S >= 2; --S) {
-      // TS: the B operand in its own ring of up to 8 stages (at least 2) behind S weight stages
-      int SX = 0;
-      if (tw >= 2) {
-        SX = std::max(2, c.sx_max);
-        while (SX > 2 && mk_smem_bytes(xs.rows, xs.parts, S, c.D, kps, 0, SX, tw) > kLimit) --SX;
-      }
-      const size_t ring = SX > 0 ? S * static_cast<size_t>(kps) * 16384 + SX * x_stage : S * stage;
-      const size_t base = mk_smem_bytes(xs.rows, xs.parts, S, c.D, kps, 0, SX, SX > 0 ? tw : 0);
+      const size_t ring = S * stage;
+      const size_t base = mk_smem_bytes(xs.rows, xs.parts, S, c.D, kps, 0);
       if (base > kLimit) continue;
       const size_t avail = kLimit - base;
       // at least Q + one tile, and Q + the warps' merge buffer (8 warps x 16 rows x D floats)
@@ -495,10 +464,6 @@ bool mk_config_for(const MkPlanIn& c, int B, int M, int tiles, MkConfig* out) {
       out->attn_splits = splits;
       out->attn_extra = extra;
       out->smem = base + extra;
-      out->ts = SX > 0 ? 1 : 0;
-      out->x_stages = SX;
-      out->tw_slots = SX > 0 ? tw : 0;
-      out->n_acc = SX > 0 ? n_acc : 0;
       return true;
     }
   }
@@ -536,13 +501,7 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   p.stages = stages;
   p.kps = kps;
   p.xs = xs;
-  p.ts = cfg.ts;
-  p.ts_pre = c->mk_ts_pre;
-  p.spin_roles = c->mk_spin_roles;
   p.dp_tail = c->mk_dp_tail;
-  p.x_stages = cfg.x_stages;
-  p.tw_slots = cfg.tw_slots;
-  p.n_acc = cfg.n_acc;
   p.attn_plo = c->attn_plo;
   p.attn_extra = static_cast<int>(cfg.attn_extra);
   p.w_evict_first = c->w_evict_first;
@@ -599,7 +558,10 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   // launches of the persistent kernel over the GEMM phases in between.
   const double layer_bytes = (4.0 * c->d * c->d + 3.0 * c->d * c->a.d_mlp) * 2.0;
   const double kv_bytes = static_cast<double>(sp.ctx_sum) * 4.0 * c->d;
-  const bool ext = c->attn_mode == 2 || (c->attn_mode == 0 && kv_bytes >= 0.5 * layer_bytes);
+  // (blocks of more than 64 rows always take the separate kernels: their wide variant has the eight
+  // query tiles and 128-row buffers; the attention inside the persistent kernel keeps 64)
+  const bool ext = sp.max_nodes > kNarrowNodes || c->attn_mode == 2 ||
+                   (c->attn_mode == 0 && kv_bytes >= 0.5 * layer_bytes);
   p.attn_external = ext ? 1 : 0;
   TSS_MK(0, TSS_CU(launch_prologue(mp, c->ssp, c->mk_zero, c->mk_n_zero, sp.M, s, false)));
   if (!ext) {
@@ -620,6 +582,7 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
     ap.o_xs = xs;  // fp16 q, hi/lo output: the persistent kernel's operands
     ap.part_o = c->attn_po;
     ap.part_ml = c->attn_pml;
+    ap.wide = sp.max_nodes > kNarrowNodes ? 1 : 0;
     ap.counters = c->attn_cnt;
     ap.status = c->d_status;
     int pb = 0;
@@ -644,7 +607,7 @@ bool mk_supported(const tss_ctx* c, const StepPlan& sp) {
   if (!c->use_mk) return false;
   MkConfig cfg;
   if (!mk_config(c, sp, &cfg)) return false;
-  return mk_max_blocks_per_sm(c->D, cfg.ts != 0, cfg.smem) >= 1;
+  return mk_max_blocks_per_sm(c->D, cfg.smem) >= 1;
 }
 
 tss_status validate_arch(const tss_arch* a) {
@@ -659,7 +622,7 @@ tss_status validate_arch(const tss_arch* a) {
   if (a->d_mlp % 8 != 0) return fail(TSS_ERR_UNSUPPORTED_ARCH, "d_mlp must be a multiple of 8");
   if (a->max_batch < 1 || a->max_batch > kMaxBatch) return fail(TSS_ERR_INVALID_ARG, "max_batch must be in [1, 64]");
   if (a->max_rows < 1 || a->max_rows > kMaxRows) return fail(TSS_ERR_INVALID_ARG, "max_rows must be in [1, 256]");
-  if (a->max_nodes < 1 || a->max_nodes > kMaxNodes) return fail(TSS_ERR_INVALID_ARG, "max_nodes must be in [1, 64]");
+  if (a->max_nodes < 1 || a->max_nodes > kMaxNodes) return fail(TSS_ERR_INVALID_ARG, "max_nodes must be in [1, 128]");
   if (a->max_domains < 1 || a->max_domains > (1 << 20)) return fail(TSS_ERR_INVALID_ARG, "max_domains out of range");
   if (a->max_positions < 1) return fail(TSS_ERR_INVALID_ARG, "max_positions must be positive");
   if (!(a->rms_eps >= 0.f) || !(a->rope_theta > 0.f)) return fail(TSS_ERR_INVALID_ARG, "rms_eps / rope_theta invalid");
@@ -754,7 +717,9 @@ tss_status build_workspaces(tss_ctx* c) {
   TSS_CU(cudaMemset(c->counters, 0, (max_tiles + 64) * sizeof(int)));
   TSS_TRY(c->alloc(&c->amax_val, static_cast<size_t>(c->V_pad / 128) * kMaxRows));
   TSS_TRY(c->alloc(&c->amax_idx, static_cast<size_t>(c->V_pad / 128) * kMaxRows));
-  const size_t ph = static_cast<size_t>(c->a.max_batch) * c->H * c->max_splits * kMaxNodes;
+  // partials of the split attention: 64 rows per (request, head, split), 128 for wide blocks
+  const size_t ph = static_cast<size_t>(c->a.max_batch) * c->H * c->max_splits *
+                    (c->a.max_nodes > kNarrowNodes ? kMaxNodes : kNarrowNodes);
   TSS_TRY(c->alloc(&c->attn_po, ph * c->D));
   TSS_TRY(c->alloc(&c->attn_pml, ph * 2));
   TSS_TRY(c->alloc(&c->d_step, 1));
@@ -869,7 +834,7 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
     sd->req_slot[b] = slot;
     sd->req_domain[b] = dom;
     sd->req_phi[b] = mask;
-    unsigned long long anc[kMaxNodes];
+    unsigned long long anc[kMaxNodes], anc_hi[kMaxNodes];  // ancestor-or-self bits of rows 0..63, 64..127
     int depth[kMaxNodes];
     for (int i = 0; i < n; ++i) {
       const int par = bt->parent_idx[M + i];
@@ -878,7 +843,8 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
       if (bt->mode == TSS_MODE_SAMPLE && i > 0 && par != i - 1)
         return fail(TSS_ERR_INVALID_ARG, "speculative sampling verifies chain drafts only");
       depth[i] = i == 0 ? 0 : depth[par] + 1;
-      anc[i] = (i == 0 ? 0ull : anc[par]) | (1ull << i);
+      anc[i] = (i == 0 ? 0ull : anc[par]) | (i < 64 ? 1ull << i : 0ull);
+      anc_hi[i] = (i == 0 ? 0ull : anc_hi[par]) | (i >= 64 ? 1ull << (i - 64) : 0ull);
       const int pos = ctx + depth[i];
       if (bt->positions && bt->positions[M + i] != pos)
         return fail(TSS_ERR_INVALID_ARG, "positions must equal ctx_len + depth");
@@ -887,6 +853,7 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
       sd->row_pos[M + i] = pos;
       sd->row_parent[M + i] = par;
       sd->row_anc[M + i] = anc[i];
+      sd->row_anc_hi[M + i] = anc_hi[i];
       if (depth[i] > max_depth) max_depth = depth[i];
     }
     max_t = std::max(max_t, ctx + n);
@@ -934,6 +901,8 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
   sp->mode = bt->mode;
   sp->splits = splits;
   sp->n_pad = pad_to(M, 16);
+  sp->max_nodes = 1;
+  for (int b = 0; b < B; ++b) sp->max_nodes = std::max(sp->max_nodes, bt->n_nodes[b]);
   sp->tiles = tiles;
   sp->ctx_sum = 0;
   for (int b = 0; b < B; ++b) sp->ctx_sum += bt->ctx_len[b];
@@ -997,11 +966,6 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_ATTN_PLO")) c->attn_plo = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ATTN_SPLITS")) c->attn_splits_force = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
-  if (const char* e = std::getenv("TSS_MK_TMEM")) c->mk_tmem = std::atoi(e) != 0;
-  if (const char* e = std::getenv("TSS_MK_TW")) c->mk_tw_max = std::max(2, std::min(16, std::atoi(e)));
-  if (const char* e = std::getenv("TSS_MK_SX")) c->mk_sx_max = std::max(2, std::min(8, std::atoi(e)));
-  if (const char* e = std::getenv("TSS_MK_TS_PRE")) c->mk_ts_pre = std::atoi(e) != 0;
-  if (const char* e = std::getenv("TSS_MK_SPIN")) c->mk_spin_roles = std::atoi(e) & 0xff;
   if (const char* e = std::getenv("TSS_MK_DP")) c->mk_dp_tail = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ALLOC_LIMIT_BYTES")) c->alloc_limit = std::strtoull(e, nullptr, 10);
   if (const char* e = std::getenv("TSS_WAIT_LIMIT_MS")) {
@@ -1096,7 +1060,7 @@ tss_status tss_persistent_plan(const tss_arch* a, int n_req, int n_rows, int max
     return fail(TSS_ERR_INVALID_ARG, "arch: head_dim 64 or 128 and n_heads >= 1");
   if (n_req < 1 || n_req > kMaxBatch || n_rows < n_req || n_rows > kMaxRows || max_keys < 1 || num_sms < 1)
     return fail(TSS_ERR_INVALID_ARG, "n_req in [1, 64], n_rows in [n_req, 256], max_keys and num_sms positive");
-  const MkPlanIn in{a->head_dim, a->n_heads, num_sms, 3, 12, kMaxSplits, kMkTmemDefault ? 1 : 0};
+  const MkPlanIn in{a->head_dim, a->n_heads, num_sms, 3, 12, kMaxSplits};
   MkConfig cfg;
   const bool fits = mk_config_for(in, n_req, n_rows, (max_keys + 63) / 64, &cfg);
   out->fits = fits ? 1 : 0;
@@ -1104,7 +1068,6 @@ tss_status tss_persistent_plan(const tss_arch* a, int n_req, int n_rows, int max
   out->stages = fits ? cfg.stages : 0;
   out->attn_splits = fits ? cfg.attn_splits : 0;
   out->smem_bytes = fits ? static_cast<uint64_t>(cfg.smem) : 0;
-  out->tmem_weight_slots = fits ? cfg.tw_slots : 0;
   return TSS_OK;
 }
 

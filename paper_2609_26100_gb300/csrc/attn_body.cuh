@@ -15,12 +15,17 @@ constexpr int attn_ld() {
 }
 
 __host__ __device__ inline size_t attn_qlo_bytes(int head_dim) {
-  return static_cast<size_t>(kMaxNodes) * (head_dim + 8) * 2;  // lo parts of q
+  return static_cast<size_t>(kNarrowNodes) * (head_dim + 8) * 2;  // lo parts of q
 }
 
+// The separate kernel's wide variant (blocks of up to 128 rows): Q of 128 rows, and its lo part.
+__host__ __device__ inline size_t attn_wide_smem_bytes(int head_dim) {
+  const size_t ld = head_dim + 8;
+  return static_cast<size_t>(2 * kMaxNodes + 4 * kKeyTile) * ld * 2;
+}
 __host__ __device__ inline size_t attn_smem_bytes_impl(int head_dim) {
   const int ld = head_dim + 8;
-  return static_cast<size_t>(kMaxNodes + 4 * kKeyTile) * ld * 2;  // Q + double-buffered K and V
+  return static_cast<size_t>(kNarrowNodes + 4 * kKeyTile) * ld * 2;  // Q + double-buffered K and V
 }
 
 // Keys [k0, k1) that split `split` of n_splits covers in a block of T keys (whole 64-key tiles,
@@ -41,11 +46,13 @@ struct AttnItem {
   const __nv_bfloat16* Vg;
   int crow, N, ctx, T, t0, t1, mt, wm, wk, ksplit, kpw, g, tq, warp, lane;
   unsigned long long anc0, anc1;
+  const unsigned long long* anc_hi;  // blocks of more than 64 rows: ancestor bits of block rows 64..127 by row
 };
 
 // Fills `it` for thread `tid` of a team of NT threads; false when the request does not run this
 // layer or the item is out of range.
-template <int D, int NT = kAttnThreads>
+// NB: block rows the item's buffers hold (64, or 128 for the separate kernel's wide variant).
+template <int D, int NT = kAttnThreads, int NB = kNarrowNodes>
 __device__ __forceinline__ bool attn_item_setup(const AttnParams& p, int split, int head, int b, int tid,
                                                 AttnItem<D>& it) {
   const StepDesc* st = p.step;
@@ -68,7 +75,7 @@ __device__ __forceinline__ bool attn_item_setup(const AttnParams& p, int split, 
   it.Vg = it.Kg + static_cast<size_t>(H) * cap * D;
   it.warp = tid >> 5;
   it.lane = tid & 31;
-  it.mt = it.N <= 16 ? 1 : (it.N <= 32 ? 2 : 4);  // 16-row query tiles
+  it.mt = it.N <= 16 ? 1 : (it.N <= 32 ? 2 : (NB > kNarrowNodes && it.N > kNarrowNodes ? 8 : 4));  // 16-row query tiles
   it.ksplit = NT / 32 / it.mt;  // warps sharing one query tile
   it.wm = it.warp % it.mt;
   it.wk = it.warp / it.mt;
@@ -78,6 +85,7 @@ __device__ __forceinline__ bool attn_item_setup(const AttnParams& p, int split, 
   const int qr0 = it.wm * 16 + it.g, qr1 = qr0 + 8;
   it.anc0 = qr0 < it.N ? st->row_anc[row0 + qr0] : 0ull;
   it.anc1 = qr1 < it.N ? st->row_anc[row0 + qr1] : 0ull;
+  if constexpr (NB > kNarrowNodes) it.anc_hi = st->row_anc_hi + row0;
   return true;
 }
 
@@ -141,10 +149,10 @@ __device__ __forceinline__ void attn_load_qfrag(const AttnItem<D>& it, const __n
 
 // q arrives in fp16 (11 significant bits) and is split exactly into two bf16 parts: hi in place
 // of q, lo into sQlo (rows of the warps' query tiles).
-template <int D>
+template <int D, int NT = kAttnThreads>
 __device__ __forceinline__ void attn_split_q(const AttnItem<D>& it, __nv_bfloat16* sQ, __nv_bfloat16* sQlo, int tid) {
   constexpr int LD = attn_ld<D>(), C2 = D / 2;
-  for (int idx = tid; idx < 16 * it.mt * C2; idx += kAttnThreads) {
+  for (int idx = tid; idx < 16 * it.mt * C2; idx += NT) {
     const int row = idx / C2, c2 = idx - row * C2;
     uint32_t* qw = reinterpret_cast<uint32_t*>(sQ + row * LD) + c2;
     const __half2 hq = *reinterpret_cast<const __half2*>(qw);
@@ -174,7 +182,8 @@ __device__ __forceinline__ void attn_load_qfrag_hilo(const AttnItem<D>& it, cons
 // registers (exact for |k| in [6.1e-5, 65504]).  PLO: P.V with P as two bf16 parts,
 // hi = bf16(p) and lo = bf16(p - hi), both multiplied by the bf16 values (else P in bf16).
 // QLO: bf16 scores with q as two bf16 parts (a.qf hi, a.qlo lo), keys as stored.
-template <int D, bool QK16 = false, bool PLO = false, bool QLO = false>
+// WIDE: blocks of more than 64 rows (the ancestor bits of block rows 64..127 come from it.anc_hi).
+template <int D, bool QK16 = false, bool PLO = false, bool QLO = false, bool WIDE = false>
 __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __nv_bfloat16* const (&kp)[4],
                                                  const __nv_bfloat16* const (&vp)[4], const int (&key0)[4], int n,
                                                  float scale_log2, AttnAcc<D>& a) {
@@ -219,8 +228,15 @@ __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __
         float val = s[nt][e2] * scale_log2;
         if (need_mask) {
           const int key = kb0 + it.tq * 2 + (e2 & 1);
-          const unsigned long long anc = e2 < 2 ? it.anc0 : it.anc1;
-          if (key >= it.T || (key >= it.ctx && !((anc >> (key - it.ctx)) & 1ull))) val = -INFINITY;
+          if constexpr (WIDE) {
+            const int j = key - it.ctx;  // block row of the key
+            const int qr = it.wm * 16 + it.g + (e2 < 2 ? 0 : 8);
+            const unsigned long long anc = j < 64 ? (e2 < 2 ? it.anc0 : it.anc1) : (qr < it.N ? it.anc_hi[qr] : 0ull);
+            if (key >= it.T || (j >= 0 && !((anc >> (j & 63)) & 1ull))) val = -INFINITY;
+          } else {
+            const unsigned long long anc = e2 < 2 ? it.anc0 : it.anc1;
+            if (key >= it.T || (key >= it.ctx && !((anc >> (key - it.ctx)) & 1ull))) val = -INFINITY;
+          }
         }
         s[nt][e2] = val;
       }
@@ -293,7 +309,7 @@ __device__ __forceinline__ void attn_blocks_step(const AttnItem<D>& it, const __
 }
 
 // This warp's keys of one resident 64-key tile (K / V buffers sK, sV).
-template <int D, bool QK16 = false, bool PLO = false, bool QLO = false>
+template <int D, bool QK16 = false, bool PLO = false, bool QLO = false, bool WIDE = false>
 __device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, const __nv_bfloat16* sK,
                                                const __nv_bfloat16* sV, float scale_log2, AttnAcc<D>& a) {
   constexpr int LD = attn_ld<D>();
@@ -307,13 +323,13 @@ __device__ __forceinline__ void attn_tile_step(const AttnItem<D>& it, int tile, 
     vp[np] = sV + (kbase + np * 16) * LD;
     key0[np] = tile * kKeyTile + kbase + np * 16;
   }
-  attn_blocks_step<D, QK16, PLO, QLO>(it, kp, vp, key0, it.kpw / 16, scale_log2, a);
+  attn_blocks_step<D, QK16, PLO, QLO, WIDE>(it, kp, vp, key0, it.kpw / 16, scale_log2, a);
 }
 
 // Weighted sum over the splits of every output element of a (request, head): each thread takes
 // kU elements per round with the partial outputs of all (<= kS) splits loaded together; the first
 // round's loads are issued before `weights()` (which computes wgt) so that they overlap.
-template <int D, int NT, int kU, int kS, typename Weights, typename Put>
+template <int D, int NT, int kU, int kS, typename Weights, typename Put, int NB = kNarrowNodes>
 __device__ __forceinline__ void attn_merge_rounds(const AttnParams& p, size_t ph, int N, int ns, int tid,
                                                   const float* wgt, Weights weights, Put put) {
   float po[kU][kS];
@@ -324,7 +340,7 @@ __device__ __forceinline__ void attn_merge_rounds(const AttnParams& p, size_t ph
       const int i = idx / D, dd = idx - i * D;
 #pragma unroll
       for (int sp = 0; sp < kS; ++sp)
-        po[u][sp] = idx < N * D && sp < ns ? __ldcg(&p.part_o[((ph + sp) * kMaxNodes + i) * D + dd]) : 0.f;
+        po[u][sp] = idx < N * D && sp < ns ? __ldcg(&p.part_o[((ph + sp) * NB + i) * D + dd]) : 0.f;
     }
   };
   load(tid);
@@ -352,7 +368,7 @@ __device__ __forceinline__ void attn_merge_rounds(const AttnParams& p, size_t ph
 // final output rows.  `stamp(k)` records diagnostics (k = 9, 2, 3, 4 in that order).
 // kFastMerge: the merge's loads in one round (attn_merge_rounds), used by the persistent
 // kernel; the standalone kernel keeps the plain loop, which measured faster there.
-template <int D, int BAR, int NT, bool kFastMerge, typename Stamp>
+template <int D, int BAR, int NT, bool kFastMerge, typename Stamp, int NB = kNarrowNodes>
 __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<D>& it, AttnAcc<D>& a, int split,
                                             int head, int b, int tid, float* sO, float (*sM)[16], float (*sL)[16],
                                             int* s_last, Stamp stamp) {
@@ -401,7 +417,7 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
     if (p.n_splits == 1) {
       if (!(L > 0.f)) report(p.status, kStatusCheck);
     } else {
-      const size_t pi = (ph + split) * kMaxNodes + i;
+      const size_t pi = (ph + split) * NB + i;
       __stcg(&p.part_ml[pi * 2 + 0], M);
       __stcg(&p.part_ml[pi * 2 + 1], L);
     }
@@ -421,7 +437,7 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
       else
         p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
     } else {
-      __stcg(&p.part_o[((ph + split) * kMaxNodes + i) * D + dd], O);
+      __stcg(&p.part_o[((ph + split) * NB + i) * D + dd], O);
     }
   }
   if (p.n_splits == 1) return true;
@@ -445,10 +461,10 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
     // flight, so that the merge of a small block costs one round of loads.
     const int ns = p.n_splits;
     float* wgt = sO;                          // [N][ns]
-    float* sml = sO + kMaxNodes * kMaxSplits;  // [N][ns] x (m, l)
+    float* sml = sO + NB * kMaxSplits;  // [N][ns] x (m, l)
     for (int x = tid; x < N * ns; x += NT) {
       const int i = x / ns, sp = x - i * ns;
-      const size_t pi = (ph + sp) * kMaxNodes + i;
+      const size_t pi = (ph + sp) * NB + i;
       sml[2 * x] = __ldcg(&p.part_ml[pi * 2]);
       sml[2 * x + 1] = __ldcg(&p.part_ml[pi * 2 + 1]);
     }
@@ -478,11 +494,11 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
         p.o[static_cast<size_t>(crow + i) * d + head * D + dd] = __float2bfloat16_rn(val);
     };
     if (ns <= 4)
-      attn_merge_rounds<D, NT, 8, 4>(p, ph, N, ns, tid, wgt, weights, put);
+      attn_merge_rounds<D, NT, 8, 4, decltype(weights), decltype(put), NB>(p, ph, N, ns, tid, wgt, weights, put);
     else if (ns <= 8)
-      attn_merge_rounds<D, NT, 4, 8>(p, ph, N, ns, tid, wgt, weights, put);
+      attn_merge_rounds<D, NT, 4, 8, decltype(weights), decltype(put), NB>(p, ph, N, ns, tid, wgt, weights, put);
     else
-      attn_merge_rounds<D, NT, 2, 16>(p, ph, N, ns, tid, wgt, weights, put);
+      attn_merge_rounds<D, NT, 2, 16, decltype(weights), decltype(put), NB>(p, ph, N, ns, tid, wgt, weights, put);
   } else {
     // Merge weights per (row, split) first -- w = 2^(m_s - M) / L with L = sum 2^(m_s - M) l_s, in
     // split order -- into shared memory (sO is free again), then every output element is a
@@ -491,11 +507,11 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
     const int ns = p.n_splits;
     for (int i = tid; i < N; i += NT) {
       float M = -INFINITY;
-      for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, __ldcg(&p.part_ml[((ph + sp) * kMaxNodes + i) * 2]));
+      for (int sp = 0; sp < ns; ++sp) M = fmaxf(M, __ldcg(&p.part_ml[((ph + sp) * NB + i) * 2]));
       const float base = M == -INFINITY ? 0.f : M;
       float L = 0.f;
       for (int sp = 0; sp < ns; ++sp) {
-        const size_t pi = (ph + sp) * kMaxNodes + i;
+        const size_t pi = (ph + sp) * NB + i;
         const float f = exp2f(__ldcg(&p.part_ml[pi * 2]) - base);
         L += f * __ldcg(&p.part_ml[pi * 2 + 1]);
         wgt[i * ns + sp] = f;
@@ -516,7 +532,7 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
         for (int u = 0; u < kU; ++u) {
           const int idx = idx0 + u * NT;
           const int i = idx / D, dd = idx - i * D;
-          po[u] = idx < N * D ? __ldcg(&p.part_o[((ph + sp) * kMaxNodes + i) * D + dd]) : 0.f;
+          po[u] = idx < N * D ? __ldcg(&p.part_o[((ph + sp) * NB + i) * D + dd]) : 0.f;
         }
   #pragma unroll
         for (int u = 0; u < kU; ++u) {
@@ -548,48 +564,52 @@ __device__ __forceinline__ bool attn_finish(const AttnParams& p, const AttnItem<
 // once into bf16 hi/lo parts for the score MMAs, so the bf16 keys need no conversion; P as hi/lo
 // bf16 parts in P.V; output split hi/lo); else all bf16.  With P16 the kernel needs
 // attn_smem_bytes(D) + attn_qlo_bytes(D) of shared memory.
-template <int D, int BAR, bool P16 = false>
+// NB / NT: block rows the buffers hold and threads of the item -- 64 and 128, or the wide variant
+// for blocks of up to 128 rows, 128 and 256 (eight query tiles, one warp each).
+template <int D, int BAR, bool P16 = false, int NB = kNarrowNodes, int NT = kAttnThreads>
 __device__ bool attention_item(const AttnParams& p, int split, int head, int b, int tid, uint8_t* smem,
                                float (*sM)[16], float (*sL)[16], int* s_last) {
   constexpr int LD = attn_ld<D>();
-  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [kMaxNodes][LD]
-  __nv_bfloat16* sK = sQ + kMaxNodes * LD;                       // [2][kKeyTile][LD]
+  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [NB][LD]
+  __nv_bfloat16* sK = sQ + NB * LD;                              // [2][kKeyTile][LD]
   __nv_bfloat16* sV = sK + 2 * kKeyTile * LD;                    // [2][kKeyTile][LD]
   AttnItem<D> it;
-  if (!attn_item_setup<D>(p, split, head, b, tid, it)) return false;
-  attn_load_q<D>(p, it, head, tid, sQ);
-  if (it.t0 < it.t1) attn_load_tile<D>(it, it.t0, tid, sK, sV);
+  if (!attn_item_setup<D, NT, NB>(p, split, head, b, tid, it)) return false;
+  attn_load_q<D, NT>(p, it, head, tid, sQ);
+  if (it.t0 < it.t1) attn_load_tile<D, NT>(it, it.t0, tid, sK, sV);
   cp_async_commit();
   AttnAcc<D> a;
   attn_acc_init<D>(a);
   for (int tile = it.t0; tile < it.t1; ++tile) {
     const int buf = (tile - it.t0) & 1;
     if (tile + 1 < it.t1)
-      attn_load_tile<D>(it, tile + 1, tid, sK + (buf ^ 1) * kKeyTile * LD, sV + (buf ^ 1) * kKeyTile * LD);
+      attn_load_tile<D, NT>(it, tile + 1, tid, sK + (buf ^ 1) * kKeyTile * LD, sV + (buf ^ 1) * kKeyTile * LD);
     cp_async_commit();
     cp_async_wait<1>();
-    named_bar_sync(BAR, kAttnThreads);
+    named_bar_sync(BAR, NT);
     if (tile == it.t0) {
       if (P16) {
         __nv_bfloat16* sQlo = sV + 2 * kKeyTile * LD;
-        attn_split_q<D>(it, sQ, sQlo, tid);
-        named_bar_sync(BAR, kAttnThreads);
+        attn_split_q<D, NT>(it, sQ, sQlo, tid);
+        named_bar_sync(BAR, NT);
         attn_load_qfrag_hilo<D>(it, sQ, sQlo, a);
       } else {
         attn_load_qfrag<D>(it, sQ, a);
       }
     }
-    attn_tile_step<D, false, P16, P16>(it, tile, sK + buf * kKeyTile * LD, sV + buf * kKeyTile * LD, p.scale_log2, a);
-    named_bar_sync(BAR, kAttnThreads);
+    attn_tile_step<D, false, P16, P16, (NB > kNarrowNodes)>(it, tile, sK + buf * kKeyTile * LD, sV + buf * kKeyTile * LD,
+                                                          p.scale_log2, a);
+    named_bar_sync(BAR, NT);
   }
   cp_async_wait<0>();
-  return attn_finish<D, BAR, kAttnThreads, false>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sK), sM, sL, s_last,
-                             [](int) {});
+  auto no_stamp = [](int) {};
+  return attn_finish<D, BAR, NT, false, decltype(no_stamp), NB>(p, it, a, split, head, b, tid, reinterpret_cast<float*>(sK),
+                                                             sM, sL, s_last, no_stamp);
 }
 
 // Tiles of K and V that attention_item_resident keeps resident in `smem_bytes` of shared memory.
 __host__ __device__ inline int attn_resident_tiles(int head_dim, size_t smem_bytes) {
-  const size_t ld = head_dim + 8, q = static_cast<size_t>(kMaxNodes) * ld * 2, tile = 2ull * kKeyTile * ld * 2;
+  const size_t ld = head_dim + 8, q = static_cast<size_t>(kNarrowNodes) * ld * 2, tile = 2ull * kKeyTile * ld * 2;
   return smem_bytes > q ? static_cast<int>((smem_bytes - q) / tile) : 0;
 }
 
@@ -611,8 +631,8 @@ __device__ bool attention_item_resident(const AttnParams& p, int split, int head
     if (trace && tid == 0) trace[k] = globaltimer_ns();
   };
   failed = false;
-  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [kMaxNodes][LD] (q in fp16)
-  __nv_bfloat16* sKV = sQ + kMaxNodes * LD;                      // per tile slot: K [kKeyTile][LD], V [kKeyTile][LD]
+  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);  // [kNarrowNodes][LD] (q in fp16)
+  __nv_bfloat16* sKV = sQ + kNarrowNodes * LD;                   // per tile slot: K [kKeyTile][LD], V [kKeyTile][LD]
   const int R = attn_resident_tiles(D, smem_bytes);
   AttnItem<D> it;
   const bool run = attn_item_setup<D, NT>(p, split, head, b, tid, it);

@@ -19,7 +19,9 @@ namespace tss {
 constexpr int kMaxLayers = 64;
 constexpr int kMaxBatch = 64;
 constexpr int kMaxRows = 256;
-constexpr int kMaxNodes = 64;
+constexpr int kMaxNodes = 128;    // rows of one request's draft block (root included)
+constexpr int kNarrowNodes = 64;  // blocks the attention inside the persistent kernel takes (larger: the
+                                  // separate attention kernel's wide variant)
 constexpr int kMaxSplits = 16;  // key splits of one (request, head) in the attention
 constexpr int kFinalSlot = kMaxLayers;  // plan slot of the final norm + LM head (all rows)
 constexpr int kPathStride = kMaxNodes;  // internal copy of each request's accepted path
@@ -48,7 +50,8 @@ struct StepDesc {
   int row_req[kMaxRows];
   int row_pos[kMaxRows];
   int row_parent[kMaxRows];  // request-local parent, -1 for the root
-  unsigned long long row_anc[kMaxRows];  // request-local ancestor-or-self bits
+  unsigned long long row_anc[kMaxRows];     // request-local ancestor-or-self bits of block rows 0..63
+  unsigned long long row_anc_hi[kMaxRows];  // ... and of block rows 64..127
   const int* tokens;
   const float* draft_probs;
   const float* uniforms;
@@ -307,25 +310,6 @@ __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint6
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
-}
-
-// The same MMA with the A operand (128 rows x 16 bf16 of K) read from tensor memory: row i in lane
-// i, two K elements per 32-bit column, so one K=16 step spans 8 columns from a_tmem.
-__device__ __forceinline__ void umma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
-                                             uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// Asynchronous copy shared -> tensor memory of a 128-row x 256-bit matrix (one K=16 slice of a
-// 128-row bf16 operand) described by a shared-memory matrix descriptor: row i lands in lane i,
-// columns taddr .. taddr + 7.  Completion is tracked by tcgen05.commit like an MMA's.
-__device__ __forceinline__ void tmem_cp_128x256b(uint32_t taddr, uint64_t sdesc) {
-  asm volatile("tcgen05.cp.cta_group::1.128x256b [%0], %1;" ::"r"(taddr), "l"(sdesc) : "memory");
 }
 
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {

@@ -66,8 +66,9 @@ struct AttnParams {
   const StepDesc* step;
   const __nv_bfloat16* q;  // [kMaxRows][d_model] compacted rows of the slot
   __nv_bfloat16* o;        // [kMaxRows][d_model]
-  float* part_o;           // [B][H][n_splits][kMaxNodes][head_dim]
-  float* part_ml;          // [B][H][n_splits][kMaxNodes][2]
+  float* part_o;           // [B][H][n_splits][64 or 128][head_dim]
+  float* part_ml;          // [B][H][n_splits][64 or 128][2]
+  int wide;                // separate kernel: blocks of up to 128 rows (partials strided by 128, else 64)
   int* counters;           // [B][H], self-resetting
   int* status;
   XsLayout o_xs;           // o_xs.rows == 0: o row-major [row][d]; else split k-block tiled
@@ -161,21 +162,12 @@ struct MkParams {
   int* abort_word;
   unsigned long long wait_ns;  // bound of every wait of the kernel
   int withhold_flag;  // fault injection: withhold one dataflow flag so that a bounded wait runs out
-  // Tensor-memory staging of the weights (ts != 0): x_stages B-operand stages in their own ring,
-  // tw_slots weight slots of kps k-blocks in tensor memory behind n_acc accumulators of n_pad
-  // columns (n_acc * n_pad + tw_slots * kps * 32 <= 512).
-  int ts, x_stages, tw_slots, n_acc;
-  int ts_pre;  // TS: the first O-phase weight stages reach tensor memory before the attention
-  int spin_roles;  // bit w: warp w polls mbarriers without the suspend hint
   int dp_tail;     // phases with a tile per CTA end with one whole tile per CTA (no fix-up on their tail)
 };
-// x_stages > 0: the TS layout (weight ring of `stages` stages, B ring of x_stages, tw_slots
-// tensor-memory slots); 0: weights and B operand share `stages` ring stages.
-size_t mk_smem_bytes(int n_pad, int parts, int stages, int head_dim, int kps, size_t attn_extra, int x_stages = 0,
-                     int tw_slots = 0);
+size_t mk_smem_bytes(int n_pad, int parts, int stages, int head_dim, int kps, size_t attn_extra);
 size_t mk_trace_slots();
 cudaError_t mk_prepare();
-int mk_max_blocks_per_sm(int head_dim, bool ts, size_t smem);
+int mk_max_blocks_per_sm(int head_dim, size_t smem);
 cudaError_t launch_verify_mk(const MkParams& p, int grid, size_t smem, cudaStream_t s);
 
 // Records the message tss_last_error() returns on the calling thread.

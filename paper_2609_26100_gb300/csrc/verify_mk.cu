@@ -86,7 +86,6 @@ struct MkShared {
   int* abort_g;
   int* status;
   uint64_t limit_ns;  // bound of every wait (create-time setting, 2 s by default)
-  bool spin;          // poll mbarriers without the suspend hint
 };
 
 __device__ __forceinline__ bool mk_aborted(const MkShared& sh) {
@@ -126,7 +125,7 @@ __device__ bool mk_wait_bar(uint64_t* bar, uint32_t parity, const MkShared& sh) 
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
-    if (sh.spin ? mbar_try_wait(bar, parity) : mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     if ((i & 255) == 0) {
       if (mk_aborted(sh)) return false;
       if (globaltimer_ns() - t0 > sh.limit_ns) {
@@ -751,35 +750,21 @@ __device__ __forceinline__ bool mk_team_attention(const MkParams& p, const AttnP
   return mk_team_sync(team, team_n, sh) && ok;
 }
 
-// TS (tensor-memory staging of the weights): the weight ring in shared memory is only the landing
-// area of the bulk copies; warp 3 moves each landed stage into one of TW slots of tensor memory
-// (tcgen05.cp) and frees the ring slot, and the MMA reads A from tensor memory.  The weight
-// stream then runs ahead of the MMA by the ring plus the slots (7 x 48 KiB for the 7B chain
-// instead of 3), which covers most of a phase hand-over; the B operand has its own small ring.
-// Without TS, weights and B share the ring stages and the MMA reads A from shared memory.
-template <int D, bool TS>
+template <int D>
 __global__ void __launch_bounds__(kMkThreads, 1)
     verify_mk_kernel(const MkParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = p.stages, n_pad = p.n_pad, KPS = p.kps;
-  const int SX = TS ? p.x_stages : S;  // B-operand stages
-  const int TW = TS ? p.tw_slots : 1;  // tensor-memory weight slots
   const int XP = p.xs.parts;
   const uint32_t x_bytes = static_cast<uint32_t>(n_pad) * 128u;  // one block of one k-block of the B operand
   const uint32_t sw_bytes = KPS * kMkWBytes, sx_bytes = KPS * XP * x_bytes;
   uint8_t* sW = base;
   uint8_t* sX = sW + static_cast<size_t>(S) * sw_bytes;
-  uint8_t* s_attn = sX + static_cast<size_t>(SX) * sx_bytes;
-  // full/empty: the ring stages (TS: weights only; arrivals 1 and 1, the copier releasing), xfull /
-  // xempty: the B-operand stages (TS), tfull / tempty: the tensor-memory weight slots (TS)
+  uint8_t* s_attn = sX + static_cast<size_t>(S) * sx_bytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(s_attn + p.attn_extra);
   uint64_t* empty = full + S;
-  uint64_t* xfull = empty + S;
-  uint64_t* xempty = xfull + (TS ? SX : 0);
-  uint64_t* tfull = xempty + (TS ? SX : 0);
-  uint64_t* tempty = tfull + (TS ? TW : 0);
-  uint64_t* accf = tempty + (TS ? TW : 0);
+  uint64_t* accf = empty + S;
   uint64_t* acce = accf + kMkMaxAcc;
   uint64_t* team = acce + kMkMaxAcc;  // all 256 threads: entry to / exit from a layer's attention
   int* misc = reinterpret_cast<int*>(team + 1);  // [0] tmem addr, [1] abort, [2..4] bcast, [5] s_last
@@ -797,9 +782,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   float* s_rope = reinterpret_cast<float*>(s_nrows + kMaxRows);  // [2][16][64]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int NB = TS ? p.n_acc : mk_acc_bufs(n_pad);
-  const uint32_t ncols = TS ? 512u : gemm_tmem_cols(n_pad, NB);
-  const uint32_t tw_col = static_cast<uint32_t>(NB * n_pad);  // TS: first column of the weight slots
+  const int NB = mk_acc_bufs(n_pad);
+  const uint32_t ncols = gemm_tmem_cols(n_pad, NB);
   const PlanDev* pl = p.plan;
   const size_t ring_attn_bytes = static_cast<size_t>(s_attn - base) + p.attn_extra;
   MkShared sh;
@@ -807,22 +791,11 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   sh.abort_g = p.abort_word;
   sh.status = p.status;
   sh.limit_ns = p.wait_ns;
-  sh.spin = (p.spin_roles >> (threadIdx.x >> 5)) & 1;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
-      mbar_init(&full[i], TS ? 1 : 2);  // weight TMA arrival (+ B-operand arrival without TS)
+      mbar_init(&full[i], 2);  // weight TMA arrival + B-operand arrival
       mbar_init(&empty[i], 1);
-    }
-    if (TS) {
-      for (int i = 0; i < SX; ++i) {
-        mbar_init(&xfull[i], 1);
-        mbar_init(&xempty[i], 1);
-      }
-      for (int i = 0; i < TW; ++i) {
-        mbar_init(&tfull[i], 1);
-        mbar_init(&tempty[i], 1);
-      }
     }
     for (int i = 0; i < kMkMaxAcc; ++i) {
       mbar_init(&accf[i], 1);
@@ -891,16 +864,15 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   e.rsin = s_rope + 16 * 64;
   const int r = e.q * 32 + lane;
   int* bcast = misc + 2;
-  // weight stages [j_lo, j_hi) of this CTA's range of a phase (j counts its stages in order):
-  // warp 0 lane 0 issues their bulk copies into the ring
-  auto produce = [&](const MkPhase& ph, int pi, int j_lo, int j_hi) -> bool {
+  // the weight stages of this CTA's share of a phase: warp 0 lane 0 issues their bulk copies into
+  // the ring (it never waits for activations, only for free ring stages)
+  auto produce = [&](const MkPhase& ph, int pi) -> bool {
     MkSeg seg = mk_seg(p, ph, c, G);
     const __nv_bfloat16* wl = mk_weights(p, ph);
     int t, k0, k1, j = 0;
-    while (j < j_hi && seg.next(t, k0, k1)) {
+    while (seg.next(t, k0, k1)) {
       const bool last_seg = seg.done();
-      for (int kc = k0; kc < k1 && j < j_hi; kc += KPS, ++j) {
-        if (j < j_lo) continue;
+      for (int kc = k0; kc < k1; kc += KPS, ++j) {
         const int nk = min(KPS, k1 - kc);
         const int s = static_cast<int>(i % S);
         if (!mk_wait_bar(&empty[s], static_cast<uint32_t>((i / S) & 1) ^ 1u, sh)) return false;
@@ -918,74 +890,19 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     }
     return true;
   };
-  // TS: warp 3 lane 0 moves landed ring stages [j_lo, j_hi) of a phase into tensor-memory slots,
-  // releasing each ring slot (and filling its tensor-memory slot) when its copies complete; with
-  // `drain` it then waits until its copies so far have read their ring slots (before the
-  // attention reuses the ring)
-  int last_empty = -1;  // ring slot and phase parity of the copier's latest release
-  uint32_t last_par = 0;
-  auto copy_stages = [&](const MkPhase& ph, int j_lo, int j_hi, bool drain) -> bool {
-    MkSeg seg = mk_seg(p, ph, c, G);
-    int t, k0, k1, j = 0;
-    while (j < j_hi && seg.next(t, k0, k1)) {
-      for (int kc = k0; kc < k1 && j < j_hi; kc += KPS, ++j) {
-        if (j < j_lo) continue;
-        const int nk = min(KPS, k1 - kc);
-        const int s = static_cast<int>(i % S), ts = static_cast<int>(i % TW);
-        if (!mk_wait_bar(&full[s], static_cast<uint32_t>((i / S) & 1), sh)) return false;
-        if (!mk_wait_bar(&tempty[ts], static_cast<uint32_t>((i / TW) & 1) ^ 1u, sh)) return false;
-        tc_fence_after();
-        const uint32_t a0 = smem_u32(sW + static_cast<size_t>(s) * sw_bytes);
-        const uint32_t tcol = tmem_base + tw_col + static_cast<uint32_t>(ts * KPS * 32);
-        for (int jj = 0; jj < nk; ++jj)
-#pragma unroll
-          for (int k16 = 0; k16 < 4; ++k16)
-            tmem_cp_128x256b(tcol + jj * 32 + k16 * 8, sdesc_sw128(a0 + jj * kMkWBytes + k16 * 32));
-        umma_commit(&empty[s]);
-        umma_commit(&tfull[ts]);
-        last_empty = s;
-        last_par = static_cast<uint32_t>((i / S) & 1);
-        ++i;
-      }
-    }
-    if (drain && last_empty >= 0 && !mk_wait_bar(&empty[last_empty], last_par, sh)) return false;
-    return true;
-  };
-  // stages of this CTA's range of a phase
-  auto stage_count = [&](const MkPhase& ph) -> int {
-    MkSeg seg = mk_seg(p, ph, c, G);
-    int t, k0, k1, n = 0;
-    while (seg.next(t, k0, k1)) n += (k1 - k0 + KPS - 1) / KPS;
-    return n;
-  };
-
   for (int pi = ph0; ok && pi < n_phases; ++pi) {
     const MkPhase ph = mk_phase(p, pl, pi);
-    const bool att = ph.kind == kMkO && !p.attn_external;
-    // TS: before a layer's attention borrows the ring, the weight stream already brings the first
-    // O-phase stages (as many as the tensor-memory slots hold) into tensor memory
-    const int npre = TS && att && p.ts_pre && (warp == 0 || warp == 3) ? min(TW, stage_count(ph)) : 0;
-    if (TS && att && p.ts_pre && (warp == 0 || warp == 3)) {
-      bool good = true;
-      if (lane == 0) good = warp == 0 ? produce(ph, pi, 0, npre) : copy_stages(ph, 0, npre, true);
-      ok = __shfl_sync(0xffffffffu, good, 0);
-    }
-    if (att) {
+    if (ph.kind == kMkO && !p.attn_external) {
       // this layer's attention: the epilogue warps come after the QKV epilogues (every QKV MMA of
       // this CTA has completed), the other warps before they start the O phase
-      const bool t = team_attention(ph.slot) && ok;
+      const bool t = team_attention(ph.slot);
       ok = warp >= 4 ? bar_and(1, 128, t) : __shfl_sync(0xffffffffu, t, 0);
       if (!ok) break;
     }
     if (warp == 0) {
       // ---------------- weight TMA producer (lane 0): never waits for activations ----------------
       bool good = true;
-      if (lane == 0) good = produce(ph, pi, npre, 1 << 30);
-      ok = __shfl_sync(0xffffffffu, good, 0);
-    } else if (TS && warp == 3) {
-      // ---------------- shared -> tensor memory copier of the weight stages (lane 0) ----------------
-      bool good = true;
-      if (lane == 0) good = copy_stages(ph, npre, 1 << 30, false);
+      if (lane == 0) good = produce(ph, pi);
       ok = __shfl_sync(0xffffffffu, good, 0);
     } else if (warp == 1) {
       // ---------------- MMA issuer (lane 0) ----------------
@@ -1003,37 +920,6 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * n_pad);
           for (int kc = k0; kc < k1; kc += KPS, ++i) {
             const int nk = min(KPS, k1 - kc);
-            if constexpr (TS) {
-              const int sx = static_cast<int>(i % SX), ts = static_cast<int>(i % TW);
-              if (!mk_wait_bar(&tfull[ts], static_cast<uint32_t>((i / TW) & 1), sh) ||
-                  !mk_wait_bar(&xfull[sx], static_cast<uint32_t>((i / SX) & 1), sh)) {
-                ok = false;
-                break;
-              }
-              tc_fence_after();
-              if (first) mk_trace(p, pi * 8 + 4);
-              first = false;
-              const uint32_t acol = tmem_base + tw_col + static_cast<uint32_t>(ts * KPS * 32);
-              for (int j = 0; j < nk; ++j) {
-                const uint32_t b0 = smem_u32(sX + static_cast<size_t>(sx) * sx_bytes + j * XP * x_bytes);
-                if (XP == 1) {
-#pragma unroll
-                  for (int k16 = 0; k16 < 4; ++k16)
-                    umma_bf16_ts(d_tmem, acol + j * 32 + k16 * 8, sdesc_sw128(b0 + k16 * 32), idesc,
-                                 (kc + j > k0 || k16 > 0) ? 1u : 0u);
-                } else {
-#pragma unroll
-                  for (int k16 = 0; k16 < 4; ++k16) {
-                    umma_bf16_ts(d_tmem, acol + j * 32 + k16 * 8, sdesc_sw128(b0 + k16 * 32), idesc,
-                                 (kc + j > k0 || k16 > 0) ? 1u : 0u);
-                    umma_bf16_ts(d_tmem, acol + j * 32 + k16 * 8, sdesc_sw128(b0 + x_bytes + k16 * 32), idesc, 1u);
-                  }
-                }
-              }
-              umma_commit(&xempty[sx]);
-              umma_commit(&tempty[ts]);
-              continue;
-            }
             const int s = static_cast<int>(i % S);
             if (!mk_wait_bar(&full[s], static_cast<uint32_t>((i / S) & 1), sh)) {
               ok = false;
@@ -1107,9 +993,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
        const bool last_seg = seg.done();
        for (int kc = k0; ok && kc < k1; kc += KPS, ++i) {
         const int nk = min(KPS, k1 - kc);
-        const int s = static_cast<int>(i % SX);
-        uint64_t* xf = TS ? &xfull[s] : &full[s];
-        if (lane == 0) ok = mk_wait_bar(TS ? &xempty[s] : &empty[s], static_cast<uint32_t>((i / SX) & 1) ^ 1u, sh);
+        const int s = static_cast<int>(i % S);
+        if (lane == 0) ok = mk_wait_bar(&empty[s], static_cast<uint32_t>((i / S) & 1) ^ 1u, sh);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) break;
         for (int kk = kc; kk < kc + nk; ++kk) {
@@ -1150,9 +1035,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           if (first) mk_trace(p, pi * 8 + 2);
           if (last_seg && kc + nk == k1) mk_trace(p, pi * 8 + 3);
           fence_proxy_async_global();
-          mbar_arrive_expect_tx(xf, nk * XP * x_bytes);
+          mbar_arrive_expect_tx(&full[s], nk * XP * x_bytes);
           bulk_load(sX + static_cast<size_t>(s) * sx_bytes, xsrc + static_cast<size_t>(kc) * XP * n_pad * 64, nk * XP * x_bytes,
-                    xf);
+                    &full[s]);
         }
         first = false;
        }
@@ -1402,26 +1287,16 @@ __global__ void __launch_bounds__(kMkThreads, 1)
 
 size_t mk_trace_slots() { return kMkTraceSlots; }
 
-size_t mk_smem_bytes(int n_pad, int parts, int stages, int head_dim, int kps, size_t attn_extra, int x_stages,
-                     int tw_slots) {
-  const size_t x_stage = static_cast<size_t>(kps) * n_pad * parts * 128;
-  const size_t ring = x_stages > 0 ? static_cast<size_t>(stages) * kps * kMkWBytes + x_stages * x_stage
-                                   : static_cast<size_t>(stages) * (kps * kMkWBytes + x_stage);
-  const int bars = 2 * stages + 2 * x_stages + 2 * tw_slots + 2 * kMkMaxAcc + 1;
-  return 1024 + ring + attn_extra + static_cast<size_t>(bars) * 8 + 64 + 16 * 128 * 4 + 64 * 4 * 2 + kMaxRows * 4 +
-         256 * 4 + 5 * kMaxRows * 4 + 2 * 16 * 64 * 4 + 64;
-}
-
-template <int D, bool TS>
-cudaError_t mk_prepare_one() {
-  return cudaFuncSetAttribute(verify_mk_kernel<D, TS>, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+size_t mk_smem_bytes(int n_pad, int parts, int stages, int head_dim, int kps, size_t attn_extra) {
+  return 1024 + static_cast<size_t>(stages) * kps * (kMkWBytes + static_cast<size_t>(n_pad) * parts * 128) +
+         attn_extra + static_cast<size_t>(2 * stages + 2 * kMkMaxAcc + 1) * 8 + 64 + 16 * 128 * 4 +
+         64 * 4 * 2 + kMaxRows * 4 + 256 * 4 + 5 * kMaxRows * 4 + 2 * 16 * 64 * 4 + 64;
 }
 
 cudaError_t mk_prepare() {
-  cudaError_t e = mk_prepare_one<64, false>();
-  if (e == cudaSuccess) e = mk_prepare_one<128, false>();
-  if (e == cudaSuccess) e = mk_prepare_one<64, true>();
-  if (e == cudaSuccess) e = mk_prepare_one<128, true>();
+  cudaError_t e = cudaFuncSetAttribute(verify_mk_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(verify_mk_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
   return e;
 }
 
@@ -1436,19 +1311,17 @@ cudaError_t launch_verify_mk(const MkParams& p, int grid, size_t smem, cudaStrea
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (p.D == 64) return cudaLaunchKernelEx(&cfg, p.ts ? verify_mk_kernel<64, true> : verify_mk_kernel<64, false>, p);
-  if (p.D == 128) return cudaLaunchKernelEx(&cfg, p.ts ? verify_mk_kernel<128, true> : verify_mk_kernel<128, false>, p);
+  if (p.D == 64) return cudaLaunchKernelEx(&cfg, verify_mk_kernel<64>, p);
+  if (p.D == 128) return cudaLaunchKernelEx(&cfg, verify_mk_kernel<128>, p);
   return cudaErrorInvalidValue;
 }
 
-int mk_max_blocks_per_sm(int head_dim, bool ts, size_t smem) {
+int mk_max_blocks_per_sm(int head_dim, size_t smem) {
   int n = 0;
   if (head_dim == 64)
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, ts ? verify_mk_kernel<64, true> : verify_mk_kernel<64, false>,
-                                                  kMkThreads, smem);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, verify_mk_kernel<64>, kMkThreads, smem);
   else
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, ts ? verify_mk_kernel<128, true> : verify_mk_kernel<128, false>,
-                                                  kMkThreads, smem);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, verify_mk_kernel<128>, kMkThreads, smem);
   return n;
 }
 

@@ -73,7 +73,7 @@ class TssStepBytes(ctypes.Structure):
 
 class TssPersistentPlanInfo(ctypes.Structure):
     _fields_ = [("fits", ctypes.c_int), ("kps", ctypes.c_int), ("stages", ctypes.c_int), ("attn_splits", ctypes.c_int),
-                ("smem_bytes", ctypes.c_uint64), ("tmem_weight_slots", ctypes.c_int)]
+                ("smem_bytes", ctypes.c_uint64)]
 
 
 class TssVerifyResult(ctypes.Structure):
@@ -157,7 +157,7 @@ def persistent_plan(arch, n_req: int, n_rows: int, max_keys: int, num_sms: int) 
     check(lib().tss_persistent_plan(ctypes.byref(a), n_req, n_rows, max_keys, num_sms, ctypes.byref(out)),
           "tss_persistent_plan")
     return {"fits": bool(out.fits), "kps": out.kps, "stages": out.stages, "attn_splits": out.attn_splits,
-            "smem_bytes": out.smem_bytes, "tmem_weight_slots": out.tmem_weight_slots}
+            "smem_bytes": out.smem_bytes}
 
 
 def estimate_step_bytes(arch, masks: Sequence[int], ctx_len: Sequence[int], n_nodes: Sequence[int]) -> Dict[str, int]:

@@ -60,7 +60,8 @@ def greedy_ar(wo, skip, kv, root, C, n):
 
 
 def run_step(run, reqs, **kw):
-    res = run.alloc_results(len(reqs), sum(len(r.parents) for r in reqs))
+    depth = max(max(synth.depths_of(r.parents)) for r in reqs)
+    res = run.alloc_results(len(reqs), sum(len(r.parents) for r in reqs), path_stride=max(64, depth + 1))
     b = run.batch(reqs, **kw)
     run.verify(b, res)
     st = run.sync_status()
@@ -675,4 +676,75 @@ def test_search_with_measured_verification_latency(weights):
     assert all(lat[()] > v for s, v in lat.items() if len(s) == 2)
     assert res.best in [s for k in res.feasible for s in res.feasible[k]]
     assert run.sync_status() == native.TSS_OK
+    run.close()
+
+
+WIDE = (8, 4, 3, 2, 2, 1, 1, 1)  # a wide static draft tree (SAMD / token-recycling style), beyond 64 nodes
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_blocks_beyond_64_rows(weights, path):
+    """A 127-node wide draft tree (128 rows) with a planted greedy path and a 99-draft chain (100
+    rows) in one 228-row step: logits of every row, the tree walk and the chain's acceptance, the
+    tree's KV compacted to its path, and a skipped layer left untouched.  Blocks over 64 rows take
+    the separate attention kernel's wide variant (two-word ancestor mask, eight 16-row query tiles)
+    on every path."""
+    w, wo, wg = weights
+    run = make_runner(wg, n_slots=2, cap=400, path=path, max_nodes=128)
+    phi = {0: O.set_to_mask({2}), 1: 0}
+    run.set_phi(phi)
+    sentinel = 7.0
+    for t in run.kv:
+        t.fill_(sentinel)
+    skips = [frozenset({2}), frozenset()]
+    ctxs = [150, 90]
+    kvs = []
+    for b in range(2):
+        kv = O.prefill(wo, ARCH, skips[b], synth.uniform_ints(ctxs[b], ARCH.vocab, SEED, f"wide.ctx{b}").tolist())
+        upload_context(run, kv, b)
+        kvs.append(kv)
+    tree = synth.eagle_tree(127, WIDE)
+    assert len(tree) == 128 and max(synth.depths_of(tree)) >= 5
+    toks = synth.draft_tokens(tree, ARCH.vocab, SEED, "wide.tok")
+    toks[0] = 23
+    greedy = greedy_ar(wo, skips[0], kvs[0], toks[0], ctxs[0], 5)
+    ch = O.children_of(tree)
+    cur = 0
+    for rank, g in zip((3, 0, 0, 0, 0), greedy):  # the path's first node is row 110 of the block
+        if len(ch[cur]) <= rank:
+            break
+        nxt = ch[cur][rank]
+        for sib in ch[cur]:
+            if toks[sib] == g:
+                toks[sib] = (g + 7) % ARCH.vocab
+        toks[nxt] = g
+        cur = nxt
+    chain = synth.chain_parents(99)
+    ctoks = synth.draft_tokens(chain, ARCH.vocab, SEED, "wide.chain")
+    reqs = [synth.Request(ctxs[0], tree, toks, 0), synth.Request(ctxs[1], chain, ctoks, 1)]
+    res, st = run_step(run, reqs)
+    assert st == native.TSS_OK
+    gl = res["logits"].cpu().numpy()
+    ref_t, nk_t = O.verify_request(wo, ARCH, skips[0], toks, tree, ctxs[0], kvs[0])
+    ref_c, _ = O.verify_request(wo, ARCH, skips[1], ctoks, chain, ctxs[1], kvs[1])
+    assert_logits(gl[:128], ref_t, "127-node tree")
+    assert_logits(gl[128:], ref_c, "100-row chain")
+    for b, (ref, tk, par) in enumerate([(ref_t, toks, tree), (ref_c, ctoks, chain)]):
+        a, bonus, pth = O.greedy_accept(ref, tk, par)
+        ga, gb = int(res["accept_len"][b]), int(res["bonus"][b])
+        gp = gpu_path(res, b, ga)
+        if O.greedy_flagged(ref, pth):
+            assert greedy_valid(ref, tk, par, gp, gb)
+        else:
+            assert (ga, gb, gp) == (a, bonus, pth)
+            if b == 0:
+                assert a >= 1 and gp[1] > 64
+    ga = int(res["accept_len"][0])
+    gp = gpu_path(res, 0, ga)
+    C = ctxs[0]
+    for l in nk_t:
+        gk = run.kv[l][0, 0, :, C:C + ga + 1].float().cpu().numpy()
+        np.testing.assert_allclose(gk, np.transpose(O.compact_block_rows(nk_t[l][0], gp), (1, 0, 2)), atol=3e-2,
+                                   rtol=2e-2)
+    assert bool((run.kv[2][0] == sentinel).all())  # request 0 skips layer 2
     run.close()

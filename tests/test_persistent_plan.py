@@ -15,8 +15,8 @@ def test_plan_fits_every_row_count(arch):
     request) fits, at short (the chain and tree workloads) and long (16k) contexts."""
     seen = set()
     for M in range(1, 257):
-        for B in sorted({1, (M + 63) // 64, min(M, 8), min(M, 16), min(M, 64)}):
-            if B < (M + 63) // 64 or B > M:
+        for B in sorted({1, (M + 127) // 128, (M + 63) // 64, min(M, 8), min(M, 16), min(M, 64)}):
+            if B < (M + 127) // 128 or B > M:
                 continue
             for keys in (1, 1030, 2109, 4101, 16393):
                 plan = native.persistent_plan(arch, B, M, keys, SMS)
@@ -35,6 +35,8 @@ def test_plan_of_the_benchmark_steps():
     assert tree["fits"]
     mixed = native.persistent_plan(synth.LLAMA2_13B, 8, 48, 4101, SMS)
     assert mixed["fits"]
+    wide = native.persistent_plan(synth.LLAMA2_7B, 2, 228, 2109, SMS)
+    assert wide["fits"]
 
 
 def test_plan_rejects_bad_arguments():
