@@ -27,7 +27,7 @@ if ROOT not in sys.path:
 METRIC = "7B verify-step latency (us) & tokens/s at k=5, 4 skipped layers; % HBM roofline"
 # Bytes of the per-step descriptor tss_verify copies to the device (sizeof(tss::StepDesc);
 # tests/test_step_bytes.py compiles the struct and checks this number).
-STEP_DESC_BYTES = 9584
+STEP_DESC_BYTES = 9840
 NOMINAL_HBM_GBS = 8000.0
 
 
@@ -50,6 +50,9 @@ def parse_args():
     p.add_argument("--prefill", type=int, default=None,
                    help="prompt tokens per request: time tss_prefill on the 7B chain's skip set (4 requests) "
                         "instead of the verification step")
+    p.add_argument("--grouped", action="store_true",
+                   help="time tss_verify_grouped (one step per skip set, fewest active layers first) against the "
+                        "mixed step on the workload (13b_mixed by default): per-request completion times")
     p.add_argument("--traffic", default=os.path.join(ROOT, "profiles"),
                    help="JSON summary of an ncu DRAM-traffic capture of the dominant kernel, or a directory "
                         "whose *_traffic.txt files are such summaries")
@@ -756,6 +759,79 @@ def run_prefill(args):
     print(json.dumps(out))
 
 
+def run_grouped(args):
+    """Domain-grouped verification against the mixed step: the same batch verified as one mixed
+    step (every request completes when the union of active layers has streamed) and as one step per
+    skip set (tss_verify_grouped, fewest active layers first); CUDA events give each group's
+    completion time.  Prints one JSON line: per-request completion times of both, their means, and
+    each group's layer count and bytes."""
+    import torch
+    from paper_2609_26100_gb300 import build as _build
+    from paper_2609_26100_gb300 import native, synth
+    from paper_2609_26100_gb300.runner import TssRunner
+    torch.cuda.set_device(0)
+    _build.build()
+    name = args.workload if args.workload != "7b_chain" else "13b_mixed"
+    w = make_workload(name, args.skip)
+    run = TssRunner.for_workload(w)
+    stream = torch.cuda.current_stream()
+    sample = w.mode == "sample"
+    kw = {}
+    if sample:
+        kw = dict(mode=native.TSS_MODE_SAMPLE, temperature=w.temperature,
+                  draft_probs=torch.cat([r.draft_probs for r in w.requests], 0).cuda(), philox_seed=w.seed)
+    B = len(w.requests)
+    b = run.batch(w.requests, **kw)
+    res = run.alloc_results(B, w.n_rows, logits=False)
+    for _ in range(max(2, args.warmup)):
+        run.verify(b, res)
+        run.verify_grouped(b, res)
+    if run.sync_status() != native.TSS_OK:
+        raise RuntimeError("device status error")
+    steps = max(3, min(args.steps, 50))
+    mixed_ms, group_ms = [], []
+    n_groups = 0
+    for _ in range(steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        run.verify(b, res)
+        e1.record(stream)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(B)]
+        g0 = torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        n_groups = run.verify_grouped(b, res, events=ev)
+        torch.cuda.synchronize()
+        mixed_ms.append(e0.elapsed_time(e1))
+        group_ms.append([g0.elapsed_time(ev[g]) for g in range(n_groups)])
+    if run.sync_status() != native.TSS_OK:
+        raise RuntimeError("device status error in the timed region")
+    mixed = statistics.median(mixed_ms)
+    gdone = [statistics.median(x[g] for x in group_ms) for g in range(n_groups)]
+    # group of each request: skip sets ordered as the library orders them
+    masks = [w.skip_mask(i) for i in range(B)]
+    order = []
+    for m in masks:
+        if m not in order:
+            order.append(m)
+    order.sort(key=lambda m: w.arch.n_layers - bin(m).count("1"))
+    per_req = [gdone[order.index(m)] for m in masks]
+    groups = []
+    for g, m in enumerate(order):
+        members = [i for i in range(B) if masks[i] == m]
+        ab = native.estimate_step_bytes(w.arch, [m] * len(members), [w.requests[i].ctx_len for i in members],
+                                        [len(w.requests[i].parents) for i in members])
+        groups.append({"skip": synth.layers_of(m), "requests": members, "active_layers": ab["active_union"],
+                       "bytes": ab["total"], "done_us": gdone[g] * 1e3})
+    run.close()
+    print(json.dumps({
+        "metric": "per-request completion time: mixed step vs domain-grouped steps", "workload": w.name,
+        "unit": "us", "steps": steps, "mixed_step_us": mixed * 1e3,
+        "grouped_total_us": gdone[-1] * 1e3, "grouped_request_us": [x * 1e3 for x in per_req],
+        "mixed_request_mean_us": mixed * 1e3, "grouped_request_mean_us": statistics.mean(per_req) * 1e3,
+        "requests_sooner_than_mixed": sum(1 for x in per_req if x < mixed), "groups": groups,
+        "data": "synthetic (seeded random-init weights, synthetic KV)"}))
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -764,6 +840,8 @@ def main():
         run_sweep(args)
     elif args.prefill:
         run_prefill(args)
+    elif args.grouped:
+        run_grouped(args)
     else:
         run_tss(args)
 

@@ -241,6 +241,28 @@ tss_status tss_persistent_plan(const tss_arch* arch, int n_req, int n_rows, int 
 tss_status tss_verify(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
                       const tss_verify_result* result, void* stream);
 
+/* Domain-grouped verification (a latency option for mixed-domain batches): the requests of the
+ * batch are grouped by their skip set S(x) = Phi(d(x)) (Sec. "Domain-to-Configuration Mapping":
+ * one model serves several domain-specific sparse paths), and one verification step per group is
+ * enqueued on `stream`, the group with the fewest active layers first.  Each group's step streams
+ * the weights of its own active layers only, so the requests of a domain that skips many layers
+ * complete sooner than in the mixed step -- which streams the union of every request's active
+ * layers once -- while the batch as a whole takes longer (the groups' layer counts add up to at
+ * least the union).  Results land in the caller's arrays at each request's position, and every
+ * request draws the same Philox uniforms as in tss_verify (counter request index = its index in
+ * the whole batch), so the outputs equal tss_verify's up to the rounding of the GEMM partition.
+ *   batch, kv, result: as tss_verify, DEVICE arrays only (io_host = 0).
+ *   n_groups (optional, HOST): the number of groups (steps) enqueued.
+ *   group_events (optional, HOST array of cudaEvent_t passed as void*, one per request, entries
+ *   may be NULL): event g is recorded on `stream` when group g's results are in place, so a caller
+ *   can time or wait for each group.
+ * Uses the context's staging buffers: do not overlap with another call on the same context.
+ * Errors: those of tss_verify (all checked for the whole batch before anything is enqueued);
+ * INVALID_ARG for io_host != 0 or a uniform_stride above 512. */
+tss_status tss_verify_grouped(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
+                              const tss_verify_result* result, void* stream, int* n_groups,
+                              void* const* group_events);
+
 /* Prefill: append tokens to the requests' KV caches under their skip configurations (the
  * configuration is fixed for a whole request, prompt included: Sec. "Problem Formulation").
  * Request b's tokens [ctx_len[b], ctx_len[b] + n_tokens[b]) run through the layers its domain

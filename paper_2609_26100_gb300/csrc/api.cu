@@ -3,6 +3,7 @@
 // and CUDA-graph capture of that plan.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -560,8 +561,11 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   const double kv_bytes = static_cast<double>(sp.ctx_sum) * 4.0 * c->d;
   // (blocks of more than 64 rows always take the separate kernels: their wide variant has the eight
   // query tiles and 128-row buffers; the attention inside the persistent kernel keeps 64)
+  // Also when the (request, head) items outnumber the CTAs: inside the persistent kernel they
+  // would run in more than one wave, one CTA per SM (13B, 4 requests x 40 heads, contexts ~2000:
+  // 7.6 ms with separate kernels vs 11.2 ms inside).
   const bool ext = sp.max_nodes > kNarrowNodes || c->attn_mode == 2 ||
-                   (c->attn_mode == 0 && kv_bytes >= 0.5 * layer_bytes);
+                   (c->attn_mode == 0 && (kv_bytes >= 0.5 * layer_bytes || sp.B * c->H > c->num_sms));
   p.attn_external = ext ? 1 : 0;
   TSS_MK(0, TSS_CU(launch_prologue(mp, c->ssp, c->mk_zero, c->mk_n_zero, sp.M, s, false)));
   if (!ext) {
@@ -799,8 +803,9 @@ void destroy_ctx(tss_ctx* c) {
 }
 
 // Host-side per-step checks and the descriptor contents.  Nothing is enqueued here.
+// rng_ids (optional): the Philox request index of each request (default: its index in the batch).
 tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache* kv,
-                        const tss_verify_result* res, StepDesc* sd, StepPlan* sp) {
+                        const tss_verify_result* res, StepDesc* sd, StepPlan* sp, const int* rng_ids = nullptr) {
   if (!bt || !kv || !res) return fail(TSS_ERR_INVALID_ARG, "batch, kv or result is NULL");
   const int B = bt->n_req;
   if (B < 1 || B > c->a.max_batch) return fail(TSS_ERR_INVALID_ARG, "n_req must be in [1, max_batch]");
@@ -833,6 +838,7 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
     sd->req_rowoff[b] = M;
     sd->req_slot[b] = slot;
     sd->req_domain[b] = dom;
+    sd->req_rng[b] = rng_ids ? rng_ids[b] : b;
     sd->req_phi[b] = mask;
     unsigned long long anc[kMaxNodes], anc_hi[kMaxNodes];  // ancestor-or-self bits of rows 0..63, 64..127
     int depth[kMaxNodes];
@@ -1090,13 +1096,13 @@ tss_status tss_active_layer_count(const tss_ctx* c, const tss_verify_batch* bt, 
 namespace {
 
 tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache* kv, const tss_verify_result* res,
-                       cudaStream_t s, Prof* prof) {
+                       cudaStream_t s, Prof* prof, const int* rng_ids = nullptr) {
   if (!c) return fail(TSS_ERR_INVALID_ARG, "ctx is NULL");
   const int ri = c->ring_i;
   if (c->ring_used[ri]) TSS_CU(cudaEventSynchronize(c->ring_ev[ri]));
   StepDesc* sd = c->h_ring[ri];
   StepPlan sp;
-  TSS_TRY(prepare_step(c, bt, kv, res, sd, &sp));
+  TSS_TRY(prepare_step(c, bt, kv, res, sd, &sp, rng_ids));
   const int M = sp.M, B = sp.B;
   const bool host_io = bt->io_host != 0;
   if (host_io) {
@@ -1207,6 +1213,102 @@ extern "C" {
 tss_status tss_verify(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache* kv, const tss_verify_result* res,
                       void* stream) {
   return verify_impl(c, bt, kv, res, static_cast<cudaStream_t>(stream), nullptr);
+}
+
+tss_status tss_verify_grouped(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cache* kv,
+                              const tss_verify_result* res, void* stream, int* n_groups, void* const* group_events) {
+  if (!c || !bt || !kv || !res) return fail(TSS_ERR_INVALID_ARG, "ctx, batch, kv or result is NULL");
+  if (bt->io_host) return fail(TSS_ERR_INVALID_ARG, "grouped verification takes device arrays (io_host = 0)");
+  if (bt->mode == TSS_MODE_SAMPLE && bt->uniforms && bt->uniform_stride > 4 * kMaxNodes)
+    return fail(TSS_ERR_INVALID_ARG, "uniform_stride too large for grouped verification");
+  // every host-side check of the whole batch first: nothing is enqueued for an invalid batch
+  std::vector<StepDesc> scratch(1);
+  StepPlan all;
+  TSS_TRY(prepare_step(c, bt, kv, res, scratch.data(), &all));
+  const int B = bt->n_req;
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // groups: requests with the same S(x), fewest active layers first (their requests complete first),
+  // ties in order of first appearance
+  std::vector<unsigned long long> masks(B);
+  std::vector<int> off(B + 1, 0);
+  for (int b = 0; b < B; ++b) {
+    masks[b] = scratch[0].req_phi[b];
+    off[b + 1] = off[b] + bt->n_nodes[b];
+  }
+  std::vector<unsigned long long> keys;
+  for (int b = 0; b < B; ++b)
+    if (std::find(keys.begin(), keys.end(), masks[b]) == keys.end()) keys.push_back(masks[b]);
+  const uint64_t all_layers = c->L == 64 ? ~0ull : (1ull << c->L) - 1;
+  std::stable_sort(keys.begin(), keys.end(), [&](unsigned long long x, unsigned long long y) {
+    return __builtin_popcountll(all_layers & ~x) < __builtin_popcountll(all_layers & ~y);
+  });
+  const size_t V = static_cast<size_t>(c->V);
+  for (size_t g = 0; g < keys.size(); ++g) {
+    std::vector<int32_t> nn, cl, dom, slot, par, pos;
+    std::vector<int> orig;
+    int rows = 0;
+    for (int b = 0; b < B; ++b) {
+      if (masks[b] != keys[g]) continue;
+      const int n = bt->n_nodes[b];
+      orig.push_back(b);
+      nn.push_back(n);
+      cl.push_back(bt->ctx_len[b]);
+      dom.push_back(bt->domain_id[b]);
+      slot.push_back(bt->kv_slot ? bt->kv_slot[b] : b);
+      for (int i = 0; i < n; ++i) {
+        par.push_back(bt->parent_idx[off[b] + i]);
+        if (bt->positions) pos.push_back(bt->positions[off[b] + i]);
+      }
+      // inputs of the group, contiguous in the context's staging buffers
+      TSS_CU(cudaMemcpyAsync(c->io_tokens + rows, bt->tokens + off[b], sizeof(int32_t) * n, cudaMemcpyDeviceToDevice, s));
+      if (bt->mode == TSS_MODE_SAMPLE) {
+        TSS_CU(cudaMemcpyAsync(c->io_probs + rows * V, bt->draft_probs + off[b] * V, sizeof(float) * n * V,
+                               cudaMemcpyDeviceToDevice, s));
+        if (bt->uniforms)
+          TSS_CU(cudaMemcpyAsync(c->io_unif + (orig.size() - 1) * bt->uniform_stride,
+                                 bt->uniforms + static_cast<size_t>(b) * bt->uniform_stride,
+                                 sizeof(float) * bt->uniform_stride, cudaMemcpyDeviceToDevice, s));
+      }
+      rows += n;
+    }
+    tss_verify_batch sub = *bt;
+    sub.n_req = static_cast<int>(nn.size());
+    sub.n_nodes = nn.data();
+    sub.ctx_len = cl.data();
+    sub.domain_id = dom.data();
+    sub.kv_slot = slot.data();
+    sub.parent_idx = par.data();
+    sub.positions = bt->positions ? pos.data() : nullptr;
+    sub.tokens = c->io_tokens;
+    sub.draft_probs = bt->mode == TSS_MODE_SAMPLE ? c->io_probs : nullptr;
+    sub.uniforms = bt->mode == TSS_MODE_SAMPLE && bt->uniforms ? c->io_unif : nullptr;
+    tss_verify_result sr{};
+    sr.accept_len = c->io_res;
+    sr.bonus = c->io_res + kMaxBatch;
+    sr.new_ctx_len = c->io_res + 2 * kMaxBatch;
+    sr.path = c->io_res + 3 * kMaxBatch;
+    sr.path_stride = res->path_stride;
+    sr.logits = res->logits ? c->logits_ws : nullptr;
+    TSS_TRY(verify_impl(c, &sub, kv, &sr, s, nullptr, orig.data()));
+    // results back to the caller's request positions
+    int r = 0;
+    for (size_t j = 0; j < orig.size(); ++j) {
+      const int b = orig[j], n = nn[j];
+      TSS_CU(cudaMemcpyAsync(res->accept_len + b, sr.accept_len + j, sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+      TSS_CU(cudaMemcpyAsync(res->bonus + b, sr.bonus + j, sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+      TSS_CU(cudaMemcpyAsync(res->new_ctx_len + b, sr.new_ctx_len + j, sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+      TSS_CU(cudaMemcpyAsync(res->path + static_cast<size_t>(b) * res->path_stride,
+                             sr.path + j * static_cast<size_t>(res->path_stride), sizeof(int32_t) * res->path_stride,
+                             cudaMemcpyDeviceToDevice, s));
+      if (res->logits)
+        TSS_CU(cudaMemcpyAsync(res->logits + off[b] * V, c->logits_ws + r * V, sizeof(float) * n * V,
+                               cudaMemcpyDeviceToDevice, s));
+      r += n;
+    }
+    if (group_events && group_events[g]) TSS_CU(cudaEventRecord(static_cast<cudaEvent_t>(group_events[g]), s));
+  }
+  if (n_groups) *n_groups = static_cast<int>(keys.size());
+  return TSS_OK;
 }
 
 tss_status tss_prefill(tss_ctx* c, int n_req, const int32_t* n_tokens, const int32_t* ctx_len,

@@ -47,6 +47,7 @@ struct StepDesc {
   // lookup S(x) = Phi(d(x)) runs on the host, so a later change of the map affects later steps
   // only), 0 (dense) for a domain that is not configured.
   unsigned long long req_phi[kMaxBatch];
+  int req_rng[kMaxBatch];  // request index of the Philox counter (the caller's index when a batch is split)
   int row_req[kMaxRows];
   int row_pos[kMaxRows];
   int row_parent[kMaxRows];  // request-local parent, -1 for the root

@@ -235,7 +235,8 @@ __device__ __forceinline__ float uniform24(uint32_t x) { return static_cast<floa
 
 __device__ __forceinline__ double draw_uniform(const StepDesc* st, int b, int slot) {
   if (st->uniforms) return static_cast<double>(st->uniforms[static_cast<size_t>(b) * st->uniform_stride + slot]);
-  return static_cast<double>(uniform24(philox_slot(st->seed_lo, st->seed_hi, st->off_lo, st->off_hi, b, slot).x));
+  return static_cast<double>(
+      uniform24(philox_slot(st->seed_lo, st->seed_hi, st->off_lo, st->off_hi, st->req_rng[b], slot).x));
 }
 
 // Diagnostic: the generator's words and uniforms for requests [0, n_req) and slots [0, n_slots)

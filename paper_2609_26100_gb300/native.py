@@ -28,7 +28,7 @@ EXPORTS = (
     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status", "tss_destroy",
     "tss_linear", "tss_linear_static", "tss_read_trace", "tss_status_string", "tss_last_error",
     "tss_estimate_step_bytes", "tss_persistent_plan", "tss_inject_timeout", "tss_philox_uniforms",
-    "tss_linear_static_status",
+    "tss_linear_static_status", "tss_verify_grouped",
 )
 
 _P = ctypes.c_void_p
@@ -119,10 +119,14 @@ def lib() -> ctypes.CDLL:
         L.tss_inject_timeout.argtypes = [_P, ctypes.c_int]
         L.tss_philox_uniforms.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int, ctypes.c_int, _P, _P, _P]
         L.tss_linear_static_status.argtypes = [_P]
+        L.tss_verify_grouped.argtypes = [_P, ctypes.POINTER(TssVerifyBatch), ctypes.POINTER(TssKvCache),
+                                         ctypes.POINTER(TssVerifyResult), _P, ctypes.POINTER(ctypes.c_int),
+                                         ctypes.POINTER(_P)]
         for name in ("tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
                      "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status",
                      "tss_linear", "tss_linear_static", "tss_read_trace", "tss_estimate_step_bytes",
-                     "tss_persistent_plan", "tss_inject_timeout", "tss_philox_uniforms", "tss_linear_static_status"):
+                     "tss_persistent_plan", "tss_inject_timeout", "tss_philox_uniforms", "tss_linear_static_status",
+                     "tss_verify_grouped"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -289,6 +293,20 @@ class Verifier:
     def verify(self, batch, kv, result, stream=None) -> None:
         check(lib().tss_verify(self.ctx, ctypes.byref(batch), ctypes.byref(kv), ctypes.byref(result), stream),
               "tss_verify")
+
+    def verify_grouped(self, batch, kv, result, stream=None, events=None) -> int:
+        """tss_verify_grouped; events: optional list of torch.cuda.Event (one per request, the first
+        n_groups are recorded).  Returns the number of groups."""
+        n = ctypes.c_int()
+        ev = None
+        if events is not None:
+            for e in events:  # torch creates an event at its first record
+                if e is not None and not e.cuda_event:
+                    e.record()
+            ev = (_P * len(events))(*[e.cuda_event if e is not None else None for e in events])
+        check(lib().tss_verify_grouped(self.ctx, ctypes.byref(batch), ctypes.byref(kv), ctypes.byref(result), stream,
+                                       ctypes.byref(n), ev), "tss_verify_grouped")
+        return n.value
 
     def prefill(self, n_tokens: Sequence[int], ctx_len: Sequence[int], domain_id: Sequence[int], tokens, kv,
                 kv_slot=None, io_host: bool = False, stream=None) -> None:

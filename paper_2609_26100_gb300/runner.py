@@ -128,6 +128,11 @@ class TssRunner:
                        stream=s)
         self._prefill_tokens = toks  # alive until the stream has used it
 
+    def verify_grouped(self, batch, results, stream=None, events=None) -> int:
+        """tss_verify_grouped: one step per group of requests sharing a skip set; returns the groups."""
+        s = stream if stream is not None else torch.cuda.current_stream().cuda_stream
+        return self.v.verify_grouped(batch, self.kv_struct, results["_struct"], s, events)
+
     def sync_status(self, stream=None) -> int:
         s = stream if stream is not None else torch.cuda.current_stream().cuda_stream
         return self.v.sync_status(s)

@@ -748,3 +748,63 @@ def test_blocks_beyond_64_rows(weights, path):
                                    rtol=2e-2)
     assert bool((run.kv[2][0] == sentinel).all())  # request 0 skips layer 2
     run.close()
+
+
+@pytest.mark.parametrize("mode", ["greedy", "sample"])
+def test_grouped_verification_equals_mixed_step_and_oracle(weights, mode):
+    """tss_verify_grouped on a mixed batch of four requests (two skip sets, one dense domain and one
+    unconfigured domain, which share the dense path): three groups, the one with the most skipped
+    layers first; every request's logits, acceptance and path equal the oracle's and the mixed
+    step's (sampling: the same Philox uniforms per request), and the groups' events complete in
+    order."""
+    w, wo, wg = weights
+    phi = {0: O.set_to_mask({2}), 1: O.set_to_mask({0, 3}), 2: 0}
+    doms = [2, 1, 0, 7]
+    ctxs = [60, 33, 90, 12]
+    ks = [3, 4, 2, 5]
+    run = make_runner(wg, n_slots=4, cap=160)
+    run.set_phi(phi)
+    reqs, kvs, skips, qs = [], [], [], []
+    for b in range(4):
+        skip = O.skip_set({d: O.mask_to_set(m) for d, m in phi.items()}, doms[b])
+        kv = O.prefill(wo, ARCH, skip, synth.uniform_ints(ctxs[b], ARCH.vocab, SEED, f"grp.ctx{b}").tolist())
+        upload_context(run, kv, b)
+        q, samp = synth.draft_probs_and_samples(ks[b] + 1, ARCH.vocab, SEED, f"grp.q{b}")
+        toks = [int(synth.uniform_ints(1, ARCH.vocab, SEED, f"grp.root{b}").item())] + samp[1:]
+        reqs.append(synth.Request(ctxs[b], synth.chain_parents(ks[b]), toks, doms[b], q))
+        kvs.append(kv)
+        skips.append(skip)
+        qs.append(q)
+    kw = {}
+    if mode == "sample":
+        kw = dict(mode=native.TSS_MODE_SAMPLE, temperature=1.0, draft_probs=torch.cat(qs, 0).cuda(), philox_seed=77,
+                  philox_offset=5)
+    rows = sum(len(r.parents) for r in reqs)
+    mixed = run.alloc_results(4, rows)
+    run.verify(run.batch(reqs, **kw), mixed)
+    grouped = run.alloc_results(4, rows)
+    events = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    n_groups = run.verify_grouped(run.batch(reqs, **kw), grouped, events=events)
+    assert run.sync_status() == native.TSS_OK
+    torch.cuda.synchronize()
+    assert n_groups == 3
+    assert events[0].elapsed_time(events[1]) > 0 and events[1].elapsed_time(events[2]) > 0
+    for key in ("accept_len", "bonus", "new_ctx_len", "path"):
+        assert torch.equal(grouped[key], mixed[key]), key
+    gl = grouped["logits"].cpu().numpy()
+    assert np.abs(gl - mixed["logits"].cpu().numpy()).max() < 1e-3
+    off = 0
+    for b, r in enumerate(reqs):
+        n = len(r.parents)
+        ref, _ = O.verify_request(wo, ARCH, skips[b], r.tokens, r.parents, r.ctx_len, kvs[b])
+        assert_logits(gl[off:off + n], ref, f"grouped request {b}")
+        ga, gb = int(grouped["accept_len"][b]), int(grouped["bonus"][b])
+        if mode == "greedy":
+            a, bonus, pth = O.greedy_accept(ref, r.tokens, r.parents)
+            if not O.greedy_flagged(ref, pth):
+                assert (ga, gb) == (a, bonus)
+        else:
+            u = O.philox_uniforms(77, 5, b, ks[b])
+            check_sample(ref, gl[off:off + n], r.tokens, qs[b].numpy(), u, 1.0, ga, gb, f"grouped request {b}")
+        off += n
+    run.close()
