@@ -241,6 +241,17 @@ tss_status tss_persistent_plan(const tss_arch* arch, int n_req, int n_rows, int 
 tss_status tss_verify(tss_ctx* ctx, const tss_verify_batch* batch, const tss_kv_cache* kv,
                       const tss_verify_result* result, void* stream);
 
+/* The attention kernel of the last step enqueued on ctx (tss_verify, tss_verify_grouped's last
+ * group, tss_verify_profiled):
+ *   0  the separate split-KV attention kernel (warp-level MMA; blocks of up to 64 rows),
+ *   1  the tcgen05 attention kernel: blocks of at most 16 rows and head_dim 128, the keys on the
+ *      MMA's 128-row side, K/V tiles by TMA, scores and outputs in tensor memory (the default for
+ *      such steps; the environment variable TSS_ATTN_TC=0 at tss_create turns it off),
+ *   2  the separate kernel's variant for blocks of more than 64 rows,
+ *   3  the attention inside the persistent verify kernel;
+ * -1 before the first step or for a NULL ctx.  Host state only: no CUDA call. */
+int tss_attention_kernel(const tss_ctx* ctx);
+
 /* Domain-grouped verification (a latency option for mixed-domain batches): the requests of the
  * batch are grouped by their skip set S(x) = Phi(d(x)) (Sec. "Domain-to-Configuration Mapping":
  * one model serves several domain-specific sparse paths), and one verification step per group is

@@ -63,9 +63,9 @@ bool make_tmap(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint6
 int pad_to(int x, int m) { return (x + m - 1) / m * m; }
 
 struct GraphKey {
-  int B, M, n_act, mode, splits;
+  int B, M, n_act, mode, splits, attn;  // attn: the attention kernel variant (attn_variant)
   bool operator<(const GraphKey& o) const {
-    return std::tie(B, M, n_act, mode, splits) < std::tie(o.B, o.M, o.n_act, o.mode, o.splits);
+    return std::tie(B, M, n_act, mode, splits, attn) < std::tie(o.B, o.M, o.n_act, o.mode, o.splits, o.attn);
   }
 };
 
@@ -128,6 +128,15 @@ struct tss_ctx {
   int mk_dp_tail = 1;  // whole-tile tails for phases with a tile per CTA (TSS_MK_DP)
   int attn_plo = 1;
   int attn_splits_force = 0;  // > 0: key splits of the separate attention kernel (TSS_ATTN_SPLITS)
+  // tcgen05 attention of blocks of at most 16 rows (head_dim 128; TSS_ATTN_TC=0 turns it off)
+  int attn_tc = 1;
+  int last_attn = -1;                    // attention kernel of the last step (tss_attention_kernel)
+  CUtensorMap* d_kvmaps = nullptr;       // [L] each layer's KV cache as a 2-D tensor
+  std::vector<CUtensorMap> h_kvmaps;     // host copy of the last maps uploaded
+  std::vector<const void*> kvmap_ptr;    // the layer pointers they were made for
+  int kvmap_slots = -1, kvmap_cap = -1;  // ... and the cache shape
+  bool kvmap_ok = false;                 // the maps describe the current cache
+  float *tc_po = nullptr, *tc_pml = nullptr;
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
   unsigned long long wait_ns = 2000000000ull;  // bound of the persistent kernel's waits (TSS_WAIT_LIMIT_MS)
   int inject_timeouts = 0;  // steps left that withhold one dataflow flag (tss_inject_timeout)
@@ -269,6 +278,57 @@ struct StepPlan {
   long long ctx_sum;  // context tokens over the batch
 };
 
+// The attention kernel of a step: 2 the separate kernel's wide variant (blocks over 64 rows), 1
+// the tcgen05 kernel (blocks of at most kTcMaxNodes rows, head_dim 128, KV tensor maps of the
+// current cache uploaded), 0 the separate kernel's narrow variant.
+int attn_variant(const tss_ctx* c, const StepPlan& sp) {
+  if (sp.max_nodes > kNarrowNodes) return 2;
+  if (c->attn_tc && c->D == 128 && sp.max_nodes <= kTcMaxNodes && c->kvmap_ok) return 1;
+  return 0;
+}
+
+AttnTcParams tc_params(const tss_ctx* c, float scale_log2) {
+  AttnTcParams tp{};
+  tp.n_heads = c->H;
+  tp.d_model = c->d;
+  tp.scale_log2 = scale_log2;
+  tp.plan = c->d_plan;
+  tp.step = c->d_step;
+  tp.kv_maps = c->d_kvmaps;
+  tp.q = c->qbuf;
+  tp.o = c->obuf;
+  tp.part_o = c->tc_po;
+  tp.part_ml = c->tc_pml;
+  tp.counters = c->attn_cnt;
+  tp.status = c->d_status;
+  return tp;
+}
+
+// Tensor maps of the KV cache for the tcgen05 attention, one per layer: the layer's buffer as a
+// 2-D bf16 tensor of n_slots * 2 * n_heads * cap rows of 128 elements.  Encoded and uploaded (in
+// stream order, before the step's kernels) only when the cache's pointers or shape change, so a
+// captured graph keeps reading the maps from the same device array.
+tss_status sync_kv_maps(tss_ctx* c, const tss_kv_cache* kv, cudaStream_t s) {
+  if (!c->attn_tc || !c->d_kvmaps) return TSS_OK;
+  bool same = c->kvmap_slots == kv->n_slots && c->kvmap_cap == kv->cap;
+  for (int l = 0; l < c->L && same; ++l) same = c->kvmap_ptr[l] == kv->layer[l];
+  if (same) return TSS_OK;
+  const unsigned long long rows = static_cast<unsigned long long>(kv->n_slots) * 2ull * c->H * kv->cap;
+  c->kvmap_ok = false;
+  c->kvmap_slots = kv->n_slots;
+  c->kvmap_cap = kv->cap;
+  for (int l = 0; l < c->L; ++l) c->kvmap_ptr[l] = kv->layer[l];
+  if (rows == 0 || rows + kTcMaxKeyTile > 0x7fffffffull) return TSS_OK;  // (row coordinates are 32-bit)
+  for (int l = 0; l < c->L; ++l) {
+    std::memset(&c->h_kvmaps[l], 0, sizeof(CUtensorMap));
+    if (kv->layer[l] && !make_tmap(&c->h_kvmaps[l], kv->layer[l], 128, rows, 1, 128, 2))
+      return fail(TSS_ERR_CUDA, "cuTensorMapEncodeTiled failed for a KV cache layer");
+  }
+  TSS_CU(cudaMemcpyAsync(c->d_kvmaps, c->h_kvmaps.data(), sizeof(CUtensorMap) * c->L, cudaMemcpyHostToDevice, s));
+  c->kvmap_ok = true;
+  return TSS_OK;
+}
+
 // Optional per-launch event timing (tss_verify_profiled).
 struct Prof {
   std::vector<cudaEvent_t> ev;
@@ -330,6 +390,8 @@ tss_status enqueue_step(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* pr
   ap.wide = sp.max_nodes > kNarrowNodes ? 1 : 0;
   ap.counters = c->attn_cnt;
   ap.status = c->d_status;
+  const bool tc = attn_variant(c, sp) == 1;
+  AttnTcParams tp = tc_params(c, ap.scale_log2);
   const int kbd = c->d / 64;
   for (int j = 0; j < sp.n_act; ++j) {
     // attention sub-block: h_{l+1} = f_l(h_l) only for layers in the union; others get no launch
@@ -340,8 +402,13 @@ tss_status enqueue_step(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof* pr
     g.w_tiled = c->wqkv;
     g.w_layer_elems = static_cast<long long>(3 * dd);
     TSS_K(1, TSS_TRY(run_gemm(c, kEpiQkv, *txn, *txn, g, 3 * c->d / 128, kbd, s, pdl)));
-    ap.slot = j;
-    TSS_K(2, TSS_CU(launch_attention(ap, sp.B, s, pdl)));
+    if (tc) {
+      tp.slot = j;
+      TSS_K(2, TSS_CU(launch_attention_tc(tp, c->num_sms, s, pdl)));
+    } else {
+      ap.slot = j;
+      TSS_K(2, TSS_CU(launch_attention(ap, sp.B, s, pdl)));
+    }
     g.w_tiled = c->wo;
     g.w_layer_elems = static_cast<long long>(dd);
     TSS_K(3, TSS_TRY(run_gemm(c, kEpiResid, *to, *to, g, c->d / 128, kbd, s, pdl)));
@@ -567,6 +634,7 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
   const bool ext = sp.max_nodes > kNarrowNodes || c->attn_mode == 2 ||
                    (c->attn_mode == 0 && (kv_bytes >= 0.5 * layer_bytes || sp.B * c->H > c->num_sms));
   p.attn_external = ext ? 1 : 0;
+  c->last_attn = ext ? attn_variant(c, sp) : 3;
   TSS_MK(0, TSS_CU(launch_prologue(mp, c->ssp, c->mk_zero, c->mk_n_zero, sp.M, s, false)));
   if (!ext) {
     p.ph_begin = 0;
@@ -589,13 +657,21 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
     ap.wide = sp.max_nodes > kNarrowNodes ? 1 : 0;
     ap.counters = c->attn_cnt;
     ap.status = c->d_status;
+    const bool tc = attn_variant(c, sp) == 1;
+    AttnTcParams tp = tc_params(c, p.scale_log2);
+    tp.o_xs = xs;
     int pb = 0;
     for (int j = 0; j < sp.n_act; ++j) {
       p.ph_begin = pb;  // phases 4j .. 4j+3 are QKV, O, gate/up, down of slot j; 4 n_act the LM head
       p.ph_end = 4 * j + 1;
       TSS_MK(8, TSS_CU(launch_verify_mk(p, c->num_sms, smem, s)));
-      ap.slot = j;
-      TSS_MK(2, TSS_CU(launch_attention(ap, sp.B, s, false)));
+      if (tc) {
+        tp.slot = j;
+        TSS_MK(2, TSS_CU(launch_attention_tc(tp, c->num_sms, s, false)));
+      } else {
+        ap.slot = j;
+        TSS_MK(2, TSS_CU(launch_attention(ap, sp.B, s, false)));
+      }
       pb = 4 * j + 1;
     }
     p.ph_begin = pb;
@@ -726,6 +802,14 @@ tss_status build_workspaces(tss_ctx* c) {
                     (c->a.max_nodes > kNarrowNodes ? kMaxNodes : kNarrowNodes);
   TSS_TRY(c->alloc(&c->attn_po, ph * c->D));
   TSS_TRY(c->alloc(&c->attn_pml, ph * 2));
+  if (c->D == 128 && c->attn_tc) {
+    TSS_TRY(c->alloc(&c->d_kvmaps, c->L));
+    c->h_kvmaps.assign(c->L, CUtensorMap{});
+    c->kvmap_ptr.assign(c->L, nullptr);
+    const size_t tr = attn_tc_partial_rows(c->a.max_batch, c->H, c->num_sms);
+    TSS_TRY(c->alloc(&c->tc_po, tr * 128));
+    TSS_TRY(c->alloc(&c->tc_pml, tr * 2));
+  }
   TSS_TRY(c->alloc(&c->d_step, 1));
   TSS_TRY(c->alloc(&c->d_plan, 1));
   TSS_CU(cudaMemset(c->d_plan, 0, sizeof(PlanDev)));
@@ -763,6 +847,7 @@ tss_status build_workspaces(tss_ctx* c) {
   if (max_smem > 232448) max_smem = 232448;
   TSS_CU(gemm_prepare(max_smem));
   TSS_CU(attn_prepare());
+  TSS_CU(attn_tc_prepare());
   TSS_CU(mk_prepare());
   {
     const int nt = d / 128;
@@ -935,6 +1020,8 @@ const char* tss_status_string(tss_status s) {
 
 const char* tss_last_error(void) { return g_err.c_str(); }
 
+int tss_attention_kernel(const tss_ctx* c) { return c ? c->last_attn : -1; }
+
 tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx** out) {
   if (!out) return fail(TSS_ERR_INVALID_ARG, "out is NULL");
   *out = nullptr;
@@ -971,6 +1058,7 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_EVICT_FIRST")) c->w_evict_first = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ATTN_PLO")) c->attn_plo = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ATTN_SPLITS")) c->attn_splits_force = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("TSS_ATTN_TC")) c->attn_tc = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
   if (const char* e = std::getenv("TSS_MK_DP")) c->mk_dp_tail = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ALLOC_LIMIT_BYTES")) c->alloc_limit = std::strtoull(e, nullptr, 10);
@@ -1128,6 +1216,7 @@ tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cach
   sd->logits = logits_dev;
 
   TSS_CU(cudaMemcpyAsync(c->d_step, sd, sizeof(StepDesc), cudaMemcpyHostToDevice, s));
+  TSS_TRY(sync_kv_maps(c, kv, s));
   TSS_CU(cudaEventRecord(c->ring_ev[ri], s));
   c->ring_used[ri] = true;
   c->ring_i = (ri + 1) % kRing;
@@ -1150,6 +1239,7 @@ tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cach
     if (prof) prof->s = s;
     TSS_TRY(enqueue_step_mk(c, sp, s, prof));
   } else if (prof) {
+    c->last_attn = attn_variant(c, sp);
     // Launches bracketed by events, captured into a graph so that the device runs them back to
     // back: the events then time device work only, not host launch latency.
     prof->s = c->cap_stream;
@@ -1172,7 +1262,8 @@ tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cach
     cudaGraphExecDestroy(exec);
     if (ce != cudaSuccess) return fail(TSS_ERR_CUDA, std::string("profile launch: ") + cudaGetErrorString(ce));
   } else if (c->use_graphs) {
-    const GraphKey key{sp.B, sp.M, sp.n_act, sp.mode, sp.splits};
+    c->last_attn = attn_variant(c, sp);
+    const GraphKey key{sp.B, sp.M, sp.n_act, sp.mode, sp.splits, attn_variant(c, sp)};
     auto it = c->graphs.find(key);
     if (it == c->graphs.end()) {
       cudaGraph_t graph = nullptr;
@@ -1192,6 +1283,7 @@ tss_status verify_impl(tss_ctx* c, const tss_verify_batch* bt, const tss_kv_cach
     }
     TSS_CU(cudaGraphLaunch(it->second, s));
   } else {
+    c->last_attn = attn_variant(c, sp);
     TSS_TRY(enqueue_step(c, sp, s));
   }
   if (host_io) {

@@ -74,6 +74,30 @@ struct AttnParams {
   XsLayout o_xs;           // o_xs.rows == 0: o row-major [row][d]; else split k-block tiled
 };
 size_t attn_smem_bytes(int head_dim);
+
+// The tcgen05 attention for blocks of at most 16 rows and head_dim 128 (attn_tc.cu): one CTA per
+// SM over the items' 128-key tiles laid end to end.
+constexpr int kTcMaxNodes = 16;
+constexpr int kTcMaxKeyTile = 128;
+struct AttnTcParams {
+  int slot, n_heads, d_model;
+  float scale_log2;              // log2(e) / sqrt(head_dim)
+  const PlanDev* plan;
+  const StepDesc* step;
+  const CUtensorMap* kv_maps;    // [n_layers] in device memory: each layer's cache as a 2-D bf16
+                                 // tensor [n_slots * 2 * n_heads * cap rows][128], boxes 64 x 128, 128-byte swizzle
+  const __nv_bfloat16* q;        // [kMaxRows][d_model] compacted rows (fp16 bits when o_xs.rows != 0)
+  __nv_bfloat16* o;              // [kMaxRows][d_model], or the split tiled operand o_xs
+  XsLayout o_xs;
+  float* part_o;                 // [attn_tc_partial_rows][128]
+  float* part_ml;                // [attn_tc_partial_rows][2]
+  int* counters;                 // [B][H], self-resetting
+  int* status;
+};
+size_t attn_tc_smem_bytes();
+size_t attn_tc_partial_rows(int max_batch, int n_heads, int grid);
+cudaError_t attn_tc_prepare();
+cudaError_t launch_attention_tc(const AttnTcParams& p, int grid, cudaStream_t s, bool pdl);
 cudaError_t attn_prepare();
 cudaError_t launch_attention(const AttnParams& p, int B, cudaStream_t s, bool pdl);
 

@@ -28,7 +28,7 @@ EXPORTS = (
     "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status", "tss_destroy",
     "tss_linear", "tss_linear_static", "tss_read_trace", "tss_status_string", "tss_last_error",
     "tss_estimate_step_bytes", "tss_persistent_plan", "tss_inject_timeout", "tss_philox_uniforms",
-    "tss_linear_static_status", "tss_verify_grouped",
+    "tss_linear_static_status", "tss_verify_grouped", "tss_attention_kernel",
 )
 
 _P = ctypes.c_void_p
@@ -122,6 +122,8 @@ def lib() -> ctypes.CDLL:
         L.tss_verify_grouped.argtypes = [_P, ctypes.POINTER(TssVerifyBatch), ctypes.POINTER(TssKvCache),
                                          ctypes.POINTER(TssVerifyResult), _P, ctypes.POINTER(ctypes.c_int),
                                          ctypes.POINTER(_P)]
+        L.tss_attention_kernel.argtypes = [_P]
+        L.tss_attention_kernel.restype = ctypes.c_int
         for name in ("tss_create", "tss_set_skip_config", "tss_clear_skip_config", "tss_sparsity_ratio",
                      "tss_active_layer_count", "tss_verify", "tss_verify_profiled", "tss_prefill", "tss_sync_status",
                      "tss_linear", "tss_linear_static", "tss_read_trace", "tss_estimate_step_bytes",
@@ -249,6 +251,11 @@ class Verifier:
 
     def sync_status(self, stream=None) -> int:
         return lib().tss_sync_status(self.ctx, stream)
+
+    def attention_kernel(self) -> int:
+        """tss_attention_kernel: the attention kernel of the last step (0 split-KV warp-MMA kernel,
+        1 tcgen05 kernel, 2 its wide variant, 3 inside the persistent kernel, -1 none yet)."""
+        return int(lib().tss_attention_kernel(self.ctx))
 
     def inject_timeout(self, n_steps: int) -> None:
         check(lib().tss_inject_timeout(self.ctx, n_steps), "tss_inject_timeout")
