@@ -7,20 +7,26 @@
 //   key ctx_len + t for which block row t is row q itself or one of its ancestors,
 // for blocks of at most 16 rows and head_dim 128.  With so few query rows the keys take the
 // 128-row (M) side of the MMA:
-//   S^T [128 keys x 16 rows]  = K [128 keys x D] . Q^T           (A: K tile, K-major, from TMA)
-//   O^T [D x 16 rows]        += V^T [D x 128 keys] . P^T         (A: V tile read MN-major)
-// with S^T and O^T in tensor memory.  One thread per key turns its lane of S^T into softmax
-// weights; the running maximum of each query row is raised only when a tile's score exceeds it
-// by more than 2^8 (the weights stay finite and exact up to rounding; the sums are rescaled
-// then), so a typical tile needs no reduction across keys.
+//   S^T [128 keys x NQ]  = K [128 keys x D] . Qop^T        (A: K tile, K-major, from TMA)
+//   O^T [D x NQ]        += V^T [D x 128 keys] . Pop^T      (A: V tile read MN-major)
+// with S^T and O^T in tensor memory.  Operands in two bf16 parts (fp16 q of the persistent
+// plan split exactly into hi + lo, and the softmax weights P as hi + lo) stack the parts as rows
+// 0-15 and 16-31 of one NQ = 32-row operand, so one MMA per k-step yields both products in
+// separate accumulator columns, added in fp32 when read; single-part operands use NQ = 16.
+// One thread per key turns its lane of S^T into weights; the running maximum of each query row
+// is raised only when a tile's score exceeds it by more than 2^8 (the weights stay finite; the
+// sums and O are rescaled then), so a typical tile needs no reduction across keys.
 //
 // Work split: the (request, head) items of the requests that run this layer, each cut into
-// 128-key tiles, are laid end to end and cut into one equal range per CTA (one CTA per SM);
-// a CTA streams its range through a three-stage TMA ring, writes one partial (O, max, sum) for
-// each item it covers in part, and the last CTA to finish an item merges its partials in CTA
-// order.  Roles: warps 0-3 softmax and epilogue (warp w owns TMEM lanes 32w..32w+31), warp 4 the
-// TMA producer, warp 5 the MMA issuer.  Every wait is bounded; on expiry the kernel records a
-// timeout, drains its copies and MMAs and returns.
+// 128-key tiles, are laid end to end and cut into min(grid, tiles) equal ranges, one per CTA
+// (one CTA per SM).  A CTA streams its range through two three-slot TMA rings -- keys, released
+// as soon as their score product completes, and values, released after P.V -- and produces one
+// result per item it covers: the output itself when it holds the whole item, else a partial
+// (O, max, sum) that the last CTA to finish the item merges with the others in CTA order.
+// Roles (320 threads): warps 0-3 softmax (warp w: TMEM lanes 32w..32w+31 = keys), warps 4-7
+// epilogue (the same lanes of O^T = head dimensions; double-buffered O so the next item's P.V
+// proceeds meanwhile), warp 8 the TMA producer, warp 9 the MMA issuer.  Every wait is bounded;
+// on expiry the kernel records a timeout, drains its copies and MMAs and returns.
 #include "internal.h"
 
 namespace tss {
@@ -28,32 +34,35 @@ namespace tss {
 namespace {
 
 constexpr int kTcKeys = 128;    // keys per tile (MMA M of the score product)
-constexpr int kTcRows = 16;     // query rows (MMA N)
-constexpr int kTcStages = 3;    // K/V ring depth
+constexpr int kTcRows = 16;     // query rows of a block
+constexpr int kTcStages = 3;    // slots of each of the K and V rings
 constexpr int kTcD = 128;       // head dimension
-constexpr int kTcThreads = 192;
-constexpr uint32_t kBox = kTcKeys * 64 * 2;        // one 128-key x 64-column swizzled box: 16 KiB
-constexpr uint32_t kStageBytes = 4 * kBox;         // K box 0, K box 1, V box 0, V box 1
-constexpr uint32_t kOpBytes = kTcRows * 128;       // one 16-row x 64-column swizzled operand block: 2 KiB
-constexpr uint32_t kQBytes = 2 * 2 * kOpBytes;     // Q: 2 column blocks x (hi, lo)
-constexpr uint32_t kPBytes = 2 * 2 * kOpBytes;     // P: 2 key blocks x (hi, lo)
-constexpr uint32_t kTmemCols = 64;                 // S^T x 2 (cols 0-31), O^T (cols 32-47)
-constexpr float kRaise = 8.f;                      // log2 headroom before the running max is raised
+constexpr int kTcThreads = 320;
+constexpr uint32_t kBox = kTcKeys * 64 * 2;   // one 128-key x 64-column swizzled box: 16 KiB
+constexpr uint32_t kSlotBytes = 2 * kBox;     // one tile's K (or V): both 64-column boxes
+constexpr uint32_t kOpRows = 32;              // operand rows: part hi in rows 0-15, lo in 16-31
+constexpr uint32_t kOpBytes = kOpRows * 128;  // one 64-column block of an operand: 4 KiB
+constexpr uint32_t kQBytes = 2 * kOpBytes;    // Q operand: 128 columns
+constexpr uint32_t kPBytes = 2 * kOpBytes;    // P operand: 128 keys
+constexpr uint32_t kTmemCols = 128;           // S^T x 2 (cols 0-63), O^T x 2 (cols 64-127), 32 each
+constexpr uint32_t kOCol = 64;
+constexpr float kRaise = 8.f;                 // log2 headroom before the running max is raised
 
 struct TcShared {
-  uint64_t full[kTcStages], empty[kTcStages];
+  uint64_t kfull[kTcStages], kempty[kTcStages], vfull[kTcStages], vempty[kTcStages];
   uint64_t s_full[2], s_free[2], p_full[2], p_free[2], q_full[2];
-  uint64_t o_full, o_free, drain;
+  uint64_t o_full[2], o_free[2], h_full[2], h_free[2], drain;
   uint32_t tmem;
   int abort;
   int last;
-  int cum[kMaxBatch + 1];  // prefix sums of the (request, head) tiles over the requests
-  float red[4][kTcRows];
-  float m[kTcRows];
+  int cum[kMaxBatch + 1];   // prefix sums of the (request, head) tiles over the requests
+  float red[4][kTcRows];    // softmax: per-warp column maxima
+  float hm[2][kTcRows];     // softmax -> epilogue: running maxima of an item's part
+  float hl[2][4][kTcRows];  // ... and the per-warp sums of its weights
 };
 
 __host__ __device__ inline size_t tc_dyn_smem() {
-  return static_cast<size_t>(kTcStages) * kStageBytes + 2 * kQBytes + 2 * kPBytes + 1024;
+  return static_cast<size_t>(2 * kTcStages) * kSlotBytes + 2 * kQBytes + 2 * kPBytes + 1024;
 }
 
 // Descriptor of an MN-major operand in 128-byte-swizzled atoms of 64 elements along M (or N):
@@ -68,26 +77,28 @@ __device__ __forceinline__ uint64_t sdesc_sw128_mn(uint32_t saddr, uint32_t lbo)
   return d;
 }
 
-// Byte offset of element (row r, column k) of a 16-row operand block group in K-major 128-byte
-// swizzle: 64-column blocks of kOpBytes, rows of 128 B, 16-byte chunks permuted by the row.
+// Byte offset of element (row r, column k) of a 32-row operand in K-major 128-byte swizzle:
+// 64-column blocks of kOpBytes, rows of 128 B, 16-byte chunks permuted by the row.
 __device__ __forceinline__ uint32_t op_off(int r, int k) {
   return static_cast<uint32_t>((k >> 6) * kOpBytes + r * 128 + ((((k & 63) >> 3) ^ (r & 7)) << 4) + (k & 7) * 2);
 }
 
+// OR of v over the 128 threads of named barrier ID (which it also synchronises).
+template <int ID>
 __device__ __forceinline__ bool bar_or(bool v) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred p, q;\n\t"
       "setp.ne.u32 q, %1, 0;\n\t"
-      "bar.red.or.pred p, 1, 128, q;\n\t"
+      "bar.red.or.pred p, %2, 128, q;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}\n"
       : "=r"(r)
-      : "r"(v ? 1u : 0u)
+      : "r"(v ? 1u : 0u), "n"(ID)
       : "memory");
   return r != 0;
 }
 
-__device__ __forceinline__ void sm_sync() { named_bar_sync(1, 128); }
+constexpr int kBarSoftmax = 1, kBarEpi = 2;
 
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float* v) {
   asm volatile(
@@ -120,7 +131,6 @@ struct TcCursor {
   __device__ void start(const TcShared& sh, int B, int H, long long g) {
     b = 0;
     while (b + 1 < B && sh.cum[b + 1] <= g) ++b;
-    while (sh.cum[b + 1] == sh.cum[b]) ++b;  // (g lies in a request with tiles)
     nt = (sh.cum[b + 1] - sh.cum[b]) / H;
     const int r = static_cast<int>(g - sh.cum[b]);
     h = r / nt;
@@ -138,18 +148,15 @@ struct TcCursor {
   }
 };
 
-}  // namespace
-
-// Q rows of (request b, head h) as the B operand of the score product: 16 rows (rows >= N zero)
-// x 128 columns, K-major 128-byte swizzle, hi part then (P16) lo part.  P16: q arrives in fp16
-// and is split exactly into bf16 hi + lo; else q is bf16 and only hi is used.
+// Q rows of (request b, head h) as the B operand of the score product: rows >= N zero, 128
+// columns, K-major 128-byte swizzle.  P16: q arrives in fp16 and is split exactly into bf16 hi
+// (rows 0-15) + lo (rows 16-31); else q is bf16 (rows 0-15).
 template <bool P16>
 __device__ __forceinline__ void tc_write_q(const AttnTcParams& p, int crow, int N, int h, uint8_t* qb, int tid) {
   for (int x = tid; x < kTcRows * (kTcD / 8); x += 128) {
     const int r = x >> 4, c8 = x & 15;
     uint4 raw = make_uint4(0, 0, 0, 0);
     if (r < N) raw = *reinterpret_cast<const uint4*>(p.q + static_cast<size_t>(crow + r) * p.d_model + h * kTcD + c8 * 8);
-    const uint32_t off = op_off(r, c8 * 8);
     if (P16) {
       const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
       uint32_t hi[4], lo[4];
@@ -160,10 +167,10 @@ __device__ __forceinline__ void tc_write_q(const AttnTcParams& p, int crow, int 
         const float hx = __uint_as_float(hi[i] << 16), hy = __uint_as_float(hi[i] & 0xffff0000u);
         lo[i] = pack_bf16(f.x - hx, f.y - hy);
       }
-      *reinterpret_cast<uint4*>(qb + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-      *reinterpret_cast<uint4*>(qb + 2 * kOpBytes + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+      *reinterpret_cast<uint4*>(qb + op_off(r, c8 * 8)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+      *reinterpret_cast<uint4*>(qb + op_off(kTcRows + r, c8 * 8)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
     } else {
-      *reinterpret_cast<uint4*>(qb + off) = raw;
+      *reinterpret_cast<uint4*>(qb + op_off(r, c8 * 8)) = raw;
     }
   }
 }
@@ -175,12 +182,28 @@ __device__ __forceinline__ void tc_store_out(const AttnTcParams& p, int row, int
     p.o[static_cast<size_t>(row) * p.d_model + col] = __float2bfloat16_rn(v);
 }
 
-// Softmax, epilogue and merge: warps 0-3, thread k owns key row k of every tile (TMEM lane k of
-// S^T) and head-dimension element k of the output (TMEM lane k of O^T).
+// NQ columns of a 32-lane TMEM block (thread i: lane i) to or from v[NQ]
+template <int NQ>
+__device__ __forceinline__ void tmem_ld_nq(uint32_t taddr, float* v) {
+  tmem_ld16(taddr, v);
+  if (NQ == 32) tmem_ld16(taddr + 16, v + 16);
+}
+template <int NQ>
+__device__ __forceinline__ void tmem_st_nq(uint32_t taddr, const float* v) {
+  tmem_st16(taddr, v);
+  if (NQ == 32) tmem_st16(taddr + 16, v + 16);
+}
+
+}  // namespace
+
+// Softmax: warps 0-3, thread k owns key row k of every tile (TMEM lane k of S^T).  Per tile:
+// scores -> weights P (both parts) into the P operand; at the end of each item's part, its
+// running maxima and weight sums go to the epilogue warps.
 template <bool P16>
 __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, uint32_t tm, uint8_t* qbuf,
-                                           uint8_t* pbuf, uint8_t* ring, int n, long long g0, long long T, int C,
-                                           int c, int tid, int warp, int lane) {
+                                           uint8_t* pbuf, uint8_t* vring, int n, long long g0, int tid, int warp,
+                                           int lane) {
+  constexpr int NQ = P16 ? 32 : 16;
   const StepDesc* st = p.step;
   const PlanDev* pl = p.plan;
   const int B = st->B, H = p.n_heads;
@@ -191,7 +214,7 @@ __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, 
   cur.start(sh, B, H, g0);
   tc_write_q<P16>(p, pl->slot_crow[p.slot][cur.b], st->req_nodes[cur.b], cur.h, qbuf, tid);
   fence_async_smem();
-  sm_sync();
+  named_bar_sync(kBarSoftmax, 128);
   if (tid == 0) mbar_arrive(&sh.q_full[0]);
   float m[kTcRows], l[kTcRows];
 #pragma unroll
@@ -201,22 +224,24 @@ __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, 
   }
   int seg = 0;
   for (int t = 0; t < n; ++t) {
-    const int b = cur.b, h = cur.h, kt = cur.kt, nt = cur.nt;
+    const int b = cur.b, kt = cur.kt, nt = cur.nt;
     const bool first = t == 0 || kt == 0;
     const bool last = t == n - 1 || kt == nt - 1;
     const int ctx = st->req_ctx[b], N = st->req_nodes[b], Tk = ctx + N;
-    const int crow = pl->slot_crow[p.slot][b];
     const int key = kt * kTcKeys + k;
 
-    // scores of this key for the 16 rows
+    // scores of this key for the block's rows (hi and lo products added)
     bool ok = mbar_wait(&sh.s_full[t & 1], (t >> 1) & 1, abort, p.status);
-    if (bar_or(!ok)) break;
+    if (bar_or<kBarSoftmax>(!ok)) break;
     tc_fence_after();
-    float s[kTcRows];
-    tmem_ld16(tm + lanes + (t & 1) * kTcRows, s);
+    float a[NQ];
+    tmem_ld_nq<NQ>(tm + lanes + (t & 1) * 32, a);
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(&sh.s_free[t & 1]);
+    float s[kTcRows];
+#pragma unroll
+    for (int q = 0; q < kTcRows; ++q) s[q] = P16 ? a[q] + a[kTcRows + q] : a[q];
 
     // Q of the next item into the other buffer (the score products of the item before this one,
     // which read it, are complete: their commit preceded this tile's)
@@ -251,17 +276,17 @@ __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, 
     if (t >= 2) ok = mbar_wait(&sh.p_free[t & 1], ((t >> 1) - 1) & 1, abort, p.status);
     if (ok && kt == nt - 1) {
       const int s_ = t % kTcStages;
-      ok = mbar_wait(&sh.full[s_], (t / kTcStages) & 1, abort, p.status);
+      ok = mbar_wait(&sh.vfull[s_], (t / kTcStages) & 1, abort, p.status);
       if (ok && key >= Tk) {
-        uint4* v0 = reinterpret_cast<uint4*>(ring + s_ * kStageBytes + 2 * kBox + k * 128);
-        uint4* v1 = reinterpret_cast<uint4*>(ring + s_ * kStageBytes + 3 * kBox + k * 128);
+        uint4* v0 = reinterpret_cast<uint4*>(vring + s_ * kSlotBytes + k * 128);
+        uint4* v1 = reinterpret_cast<uint4*>(vring + s_ * kSlotBytes + kBox + k * 128);
 #pragma unroll
         for (int i = 0; i < 8; ++i) v0[i] = v1[i] = make_uint4(0, 0, 0, 0);
       }
     }
-    if (bar_or(!ok)) break;
+    if (bar_or<kBarSoftmax>(!ok)) break;
 
-    if (bar_or(raise)) {
+    if (bar_or<kBarSoftmax>(raise)) {
       // new running maxima: the column maxima of the tile over the 128 keys
 #pragma unroll
       for (int q = 0; q < kTcRows; ++q) {
@@ -270,7 +295,7 @@ __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, 
         for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
         if (lane == 0) sh.red[warp][q] = v;
       }
-      sm_sync();
+      named_bar_sync(kBarSoftmax, 128);
       float alpha[kTcRows];
       bool rescale = false;
 #pragma unroll
@@ -281,24 +306,25 @@ __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, 
         rescale |= alpha[q] != 1.f;
         m[q] = mn;
       }
-      sm_sync();  // (sh.red is rewritten later)
+      named_bar_sync(kBarSoftmax, 128);  // (sh.red is rewritten by the next raise)
       if (!first && rescale) {
-        // O^T *= alpha column by column once PV(t - 1) has completed
+        // O^T *= alpha column by column (both parts) once PV(t - 1) has completed
         ok = mbar_wait(&sh.p_free[(t - 1) & 1], ((t - 1) >> 1) & 1, abort, p.status);
-        if (bar_or(!ok)) break;
+        if (bar_or<kBarSoftmax>(!ok)) break;
         tc_fence_after();
-        float o[kTcRows];
-        tmem_ld16(tm + lanes + 2 * kTcRows, o);
+        float o[NQ];
+        const uint32_t oaddr = tm + lanes + kOCol + (seg & 1) * 32;
+        tmem_ld_nq<NQ>(oaddr, o);
 #pragma unroll
-        for (int q = 0; q < kTcRows; ++q) o[q] *= alpha[q];
-        tmem_st16(tm + lanes + 2 * kTcRows, o);
+        for (int q = 0; q < NQ; ++q) o[q] *= alpha[q & (kTcRows - 1)];
+        tmem_st_nq<NQ>(oaddr, o);
         tc_fence_before();
       }
 #pragma unroll
       for (int q = 0; q < kTcRows; ++q) l[q] *= alpha[q];
     }
 
-    // weights 2^(s - m) of this key: hi (and lo) bf16 parts into P^T (row q, key k)
+    // weights 2^(s - m) of this key: hi (row q) and lo (row 16 + q) bf16 parts into the P operand
     uint8_t* pb = pbuf + (t & 1) * kPBytes;
 #pragma unroll
     for (int q = 0; q < kTcRows; ++q) {
@@ -307,86 +333,30 @@ __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, 
       l[q] += w;
       const __nv_bfloat16 hi = __float2bfloat16_rn(w);
       *reinterpret_cast<__nv_bfloat16*>(pb + op_off(q, k)) = hi;
-      if (P16) *reinterpret_cast<__nv_bfloat16*>(pb + 2 * kOpBytes + op_off(q, k)) = __float2bfloat16_rn(w - __bfloat162float(hi));
+      if (P16) *reinterpret_cast<__nv_bfloat16*>(pb + op_off(kTcRows + q, k)) = __float2bfloat16_rn(w - __bfloat162float(hi));
     }
     fence_async_smem();
-    sm_sync();
+    named_bar_sync(kBarSoftmax, 128);
     if (tid == 0) {
       mbar_arrive(&sh.p_full[t & 1]);
       if (next_q) mbar_arrive(&sh.q_full[(seg + 1) & 1]);
     }
 
     if (last) {
-      // ---- end of this CTA's part of item (b, h) ----
-      ok = mbar_wait(&sh.o_full, seg & 1, abort, p.status);
-      if (bar_or(!ok)) break;
-      tc_fence_after();
-      float o[kTcRows];
-      tmem_ld16(tm + lanes + 2 * kTcRows, o);
-      tc_fence_before();
-      sm_sync();
-      if (tid == 0) mbar_arrive(&sh.o_free);
-      // sums over the 128 keys of every row
+      // end of this CTA's part of the item: maxima and per-warp sums to the epilogue (buffer seg & 1,
+      // free once the epilogue has taken the part two before)
+      ok = seg < 2 || mbar_wait(&sh.h_free[seg & 1], ((seg >> 1) - 1) & 1, abort, p.status);
+      if (bar_or<kBarSoftmax>(!ok)) break;
 #pragma unroll
       for (int q = 0; q < kTcRows; ++q) {
         float v = l[q];
 #pragma unroll
-        for (int o2 = 16; o2 > 0; o2 >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o2);
-        if (lane == 0) sh.red[warp][q] = v;
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0) sh.hl[seg & 1][warp][q] = v;
+        if (q == k) sh.hm[seg & 1][q] = m[q];
       }
-      sm_sync();
-      float L[kTcRows];
-#pragma unroll
-      for (int q = 0; q < kTcRows; ++q) L[q] = ((sh.red[0][q] + sh.red[1][q]) + sh.red[2][q]) + sh.red[3][q];
-      const int item = b * H + h;
-      const long long gi0 = sh.cum[b] + static_cast<long long>(h) * nt;
-      const int cf = tc_cta_of(gi0, T, C), cl = tc_cta_of(gi0 + nt - 1, T, C);
-      const int col = h * kTcD + k;
-      if (cf == cl) {
-#pragma unroll
-        for (int q = 0; q < kTcRows; ++q)
-          if (q < N) {
-            if (!(L[q] > 0.f)) report(p.status, kStatusCheck);
-            tc_store_out(p, crow + q, col, L[q] > 0.f ? o[q] / L[q] : 0.f);
-          }
-      } else {
-        const size_t sg = static_cast<size_t>(item + c);
-#pragma unroll
-        for (int q = 0; q < kTcRows; ++q)
-          if (q < N) __stcg(&p.part_o[(sg * kTcRows + q) * kTcD + k], o[q]);
-#pragma unroll
-        for (int q = 0; q < kTcRows; ++q)
-          if (q == k && q < N) {
-            __stcg(&p.part_ml[(sg * kTcRows + q) * 2], m[q]);
-            __stcg(&p.part_ml[(sg * kTcRows + q) * 2 + 1], L[q]);
-          }
-        __threadfence();
-        sm_sync();
-        if (tid == 0) {
-          int* cnt = p.counters + item;
-          const int old = atom_add_acq_rel_gpu(cnt, 1);
-          sh.last = old == cl - cf;
-          if (sh.last) atomicExch(cnt, 0);
-        }
-        sm_sync();
-        if (sh.last) {
-          // all partials of the item, merged in CTA order: weights 2^(m_s - M), divided by L
-          for (int q = 0; q < N; ++q) {
-            float M = -INFINITY;
-            for (int cc = cf; cc <= cl; ++cc) M = fmaxf(M, __ldcg(&p.part_ml[((static_cast<size_t>(item + cc)) * kTcRows + q) * 2]));
-            const float mb = M == -INFINITY ? 0.f : M;
-            float Ls = 0.f, O = 0.f;
-            for (int cc = cf; cc <= cl; ++cc) {
-              const size_t sq = static_cast<size_t>(item + cc) * kTcRows + q;
-              const float w = exp2f(__ldcg(&p.part_ml[sq * 2]) - mb);
-              Ls += w * __ldcg(&p.part_ml[sq * 2 + 1]);
-              O += w * __ldcg(&p.part_o[sq * kTcD + k]);
-            }
-            if (!(Ls > 0.f)) report(p.status, kStatusCheck);
-            tc_store_out(p, crow + q, col, Ls > 0.f ? O / Ls : 0.f);
-          }
-        }
-      }
+      named_bar_sync(kBarSoftmax, 128);
+      if (tid == 0) mbar_arrive(&sh.h_full[seg & 1]);
 #pragma unroll
       for (int q = 0; q < kTcRows; ++q) {
         m[q] = -INFINITY;
@@ -398,14 +368,131 @@ __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, 
   }
 }
 
+// Epilogue: warps 4-7, thread e owns head-dimension element e (TMEM lane e of O^T).  For each
+// item part of the CTA, in order: O (both parts added), the softmax's maxima and sums, then the
+// output (whole item), or a partial and -- by the last CTA to finish the item -- the merge of
+// all its partials in CTA order.
+template <bool P16>
+__device__ __forceinline__ void tc_epilogue(const AttnTcParams& p, TcShared& sh, uint32_t tm, int n, long long g0,
+                                            long long T, int C, int c, int e, int warp) {
+  constexpr int NQ = P16 ? 32 : 16;
+  const StepDesc* st = p.step;
+  const PlanDev* pl = p.plan;
+  const int B = st->B, H = p.n_heads;
+  volatile int* abort = &sh.abort;
+  const uint32_t lanes = static_cast<uint32_t>((warp & 3) * 32) << 16;
+  TcCursor cur;
+  cur.start(sh, B, H, g0);
+  int t = 0;
+  for (int j = 0; t < n; ++j) {
+    const int b = cur.b, h = cur.h, nt = cur.nt;
+    const int len = min(nt - cur.kt, n - t);  // tiles of this part
+    const int N = st->req_nodes[b], crow = pl->slot_crow[p.slot][b];
+    bool ok = mbar_wait(&sh.o_full[j & 1], (j >> 1) & 1, abort, p.status);
+    ok = ok && mbar_wait(&sh.h_full[j & 1], (j >> 1) & 1, abort, p.status);
+    if (bar_or<kBarEpi>(!ok)) break;
+    tc_fence_after();
+    float a[NQ];
+    tmem_ld_nq<NQ>(tm + lanes + kOCol + (j & 1) * 32, a);
+    float o[kTcRows], m[kTcRows], L[kTcRows];
+#pragma unroll
+    for (int q = 0; q < kTcRows; ++q) {
+      o[q] = P16 ? a[q] + a[kTcRows + q] : a[q];
+      m[q] = sh.hm[j & 1][q];
+      L[q] = ((sh.hl[j & 1][0][q] + sh.hl[j & 1][1][q]) + sh.hl[j & 1][2][q]) + sh.hl[j & 1][3][q];
+    }
+    tc_fence_before();
+    named_bar_sync(kBarEpi, 128);
+    if (e == 0) {
+      mbar_arrive(&sh.o_free[j & 1]);
+      mbar_arrive(&sh.h_free[j & 1]);
+    }
+    const int item = b * H + h;
+    const long long gi0 = sh.cum[b] + static_cast<long long>(h) * nt;
+    const int cf = tc_cta_of(gi0, T, C), cl = tc_cta_of(gi0 + nt - 1, T, C);
+    const int col = h * kTcD + e;
+    if (cf == cl) {
+#pragma unroll
+      for (int q = 0; q < kTcRows; ++q)
+        if (q < N) {
+          if (!(L[q] > 0.f)) report(p.status, kStatusCheck);
+          tc_store_out(p, crow + q, col, L[q] > 0.f ? o[q] / L[q] : 0.f);
+        }
+    } else {
+      const size_t sg = static_cast<size_t>(item + c);
+#pragma unroll
+      for (int q = 0; q < kTcRows; ++q)
+        if (q < N) __stcg(&p.part_o[(sg * kTcRows + q) * kTcD + e], o[q]);
+#pragma unroll
+      for (int q = 0; q < kTcRows; ++q)
+        if (q == e && q < N) {
+          __stcg(&p.part_ml[(sg * kTcRows + q) * 2], m[q]);
+          __stcg(&p.part_ml[(sg * kTcRows + q) * 2 + 1], L[q]);
+        }
+      __threadfence();
+      named_bar_sync(kBarEpi, 128);
+      if (e == 0) {
+        int* cnt = p.counters + item;
+        const int old = atom_add_acq_rel_gpu(cnt, 1);
+        sh.last = old == cl - cf;
+        if (sh.last) atomicExch(cnt, 0);
+      }
+      named_bar_sync(kBarEpi, 128);
+      if (sh.last) {
+        // online merge of the item's partials in CTA order (one round of loads per partial)
+        float M[kTcRows], Ls[kTcRows], O[kTcRows];
+#pragma unroll
+        for (int q = 0; q < kTcRows; ++q) {
+          M[q] = -INFINITY;
+          Ls[q] = O[q] = 0.f;
+        }
+        for (int cc = cf; cc <= cl; ++cc) {
+          const size_t s0 = static_cast<size_t>(item + cc) * kTcRows;
+          float pm[kTcRows], pl_[kTcRows], po[kTcRows];
+#pragma unroll
+          for (int q = 0; q < kTcRows; ++q)
+            if (q < N) {
+              pm[q] = __ldcg(&p.part_ml[(s0 + q) * 2]);
+              pl_[q] = __ldcg(&p.part_ml[(s0 + q) * 2 + 1]);
+              po[q] = __ldcg(&p.part_o[(s0 + q) * kTcD + e]);
+            }
+#pragma unroll
+          for (int q = 0; q < kTcRows; ++q)
+            if (q < N) {
+              const float mn = fmaxf(M[q], pm[q]);
+              const float mb = mn == -INFINITY ? 0.f : mn;
+              const float wa = exp2f(M[q] - mb), wb = exp2f(pm[q] - mb);
+              O[q] = O[q] * wa + po[q] * wb;
+              Ls[q] = Ls[q] * wa + pl_[q] * wb;
+              M[q] = mn;
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < kTcRows; ++q)
+          if (q < N) {
+            if (!(Ls[q] > 0.f)) report(p.status, kStatusCheck);
+            tc_store_out(p, crow + q, col, Ls[q] > 0.f ? O[q] / Ls[q] : 0.f);
+          }
+      }
+    }
+    t += len;
+    if (t < n) {
+      cur.kt = cur.nt - 1;
+      cur.next(sh, B, H);
+    }
+  }
+}
+
 template <bool P16>
 __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const AttnTcParams p) {
+  constexpr int NQ = P16 ? 32 : 16;
   extern __shared__ uint8_t tc_dyn[];
   __shared__ TcShared sh;
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tc_dyn) + 1023) & ~uintptr_t(1023));
-  uint8_t* ring = base;                           // [stage] K box 0, K box 1, V box 0, V box 1
-  uint8_t* qbuf = base + kTcStages * kStageBytes;  // [2] Q operand (hi, lo)
-  uint8_t* pbuf = qbuf + 2 * kQBytes;              // [2] P operand (hi, lo)
+  uint8_t* kring = base;                            // [slot] K box 0, K box 1
+  uint8_t* vring = kring + kTcStages * kSlotBytes;  // [slot] V box 0, V box 1
+  uint8_t* qbuf = vring + kTcStages * kSlotBytes;   // [2] Q operand
+  uint8_t* pbuf = qbuf + 2 * kQBytes;               // [2] P operand
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const StepDesc* st = p.step;
   const PlanDev* pl = p.plan;
@@ -421,8 +508,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const AttnTcPara
     }
     sh.abort = 0;
     for (int i = 0; i < kTcStages; ++i) {
-      mbar_init(&sh.full[i], 1);
-      mbar_init(&sh.empty[i], 1);
+      mbar_init(&sh.kfull[i], 1);
+      mbar_init(&sh.kempty[i], 1);
+      mbar_init(&sh.vfull[i], 1);
+      mbar_init(&sh.vempty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sh.s_full[i], 1);
@@ -430,9 +519,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const AttnTcPara
       mbar_init(&sh.p_full[i], 1);
       mbar_init(&sh.p_free[i], 1);
       mbar_init(&sh.q_full[i], 1);
+      mbar_init(&sh.o_full[i], 1);
+      mbar_init(&sh.o_free[i], 1);
+      mbar_init(&sh.h_full[i], 1);
+      mbar_init(&sh.h_free[i], 1);
     }
-    mbar_init(&sh.o_full, 1);
-    mbar_init(&sh.o_free, 1);
     mbar_init(&sh.drain, 1);
     fence_mbar_init();
   }
@@ -455,36 +546,52 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const AttnTcPara
   const CUtensorMap* map = p.kv_maps + pl->act_layer[p.slot];
   volatile int* abort = &sh.abort;
 
-  if (warp == 4) {
-    // ---------------- TMA producer ----------------
+  if (warp == 8) {
+    // ---------------- TMA producer: K of tile i, then V of tile i - 1 ----------------
     if (lane == 0) {
       prefetch_tmap(map);
-      TcCursor cur;
-      cur.start(sh, B, H, g0);
+      TcCursor ck, cv;
+      ck.start(sh, B, H, g0);
+      cv = ck;
       const size_t cap = static_cast<size_t>(st->kv_cap);
-      int t = 0;
-      for (; t < n; ++t) {
-        const int s = t % kTcStages;
-        if (t >= kTcStages && !mbar_wait(&sh.empty[s], ((t / kTcStages) - 1) & 1, abort, p.status)) break;
-        const int rowK = static_cast<int>(((static_cast<size_t>(st->req_slot[cur.b]) * 2) * H + cur.h) * cap) +
-                         cur.kt * kTcKeys;
-        const int rowV = rowK + static_cast<int>(static_cast<size_t>(H) * cap);
-        uint8_t* dst = ring + s * kStageBytes;
-        mbar_arrive_expect_tx(&sh.full[s], kStageBytes);
-        tma_load_2d(dst, map, &sh.full[s], 0, rowK);
-        tma_load_2d(dst + kBox, map, &sh.full[s], 64, rowK);
-        tma_load_2d(dst + 2 * kBox, map, &sh.full[s], 0, rowV);
-        tma_load_2d(dst + 3 * kBox, map, &sh.full[s], 64, rowV);
-        cur.next(sh, B, H);
+      auto row_of = [&](const TcCursor& cu, int kv) {
+        return static_cast<int>(((static_cast<size_t>(st->req_slot[cu.b]) * 2 + kv) * H + cu.h) * cap) +
+               cu.kt * kTcKeys;
+      };
+      int nk = 0, nv = 0;  // tiles whose K / V copies were issued
+      for (int i = 0; i <= n; ++i) {
+        if (i < n) {
+          const int s = i % kTcStages;
+          if (i >= kTcStages && !mbar_wait(&sh.kempty[s], ((i / kTcStages) - 1) & 1, abort, p.status)) break;
+          uint8_t* dst = kring + s * kSlotBytes;
+          const int row = row_of(ck, 0);
+          mbar_arrive_expect_tx(&sh.kfull[s], kSlotBytes);
+          tma_load_2d(dst, map, &sh.kfull[s], 0, row);
+          tma_load_2d(dst + kBox, map, &sh.kfull[s], 64, row);
+          ++nk;
+          ck.next(sh, B, H);
+        }
+        if (i >= 1) {
+          const int u = i - 1, s = u % kTcStages;
+          if (u >= kTcStages && !mbar_wait(&sh.vempty[s], ((u / kTcStages) - 1) & 1, abort, p.status)) break;
+          uint8_t* dst = vring + s * kSlotBytes;
+          const int row = row_of(cv, 1);
+          mbar_arrive_expect_tx(&sh.vfull[s], kSlotBytes);
+          tma_load_2d(dst, map, &sh.vfull[s], 0, row);
+          tma_load_2d(dst + kBox, map, &sh.vfull[s], 64, row);
+          ++nv;
+          cv.next(sh, B, H);
+        }
       }
-      // the copies issued last into each stage have landed before the kernel returns
-      for (int u = t - 1; u >= 0 && u >= t - kTcStages; --u) mbar_drain(&sh.full[u % kTcStages], (u / kTcStages) & 1);
+      // the copies issued last into each slot have landed before the kernel returns
+      for (int u = nk - 1; u >= 0 && u >= nk - kTcStages; --u) mbar_drain(&sh.kfull[u % kTcStages], (u / kTcStages) & 1);
+      for (int u = nv - 1; u >= 0 && u >= nv - kTcStages; --u) mbar_drain(&sh.vfull[u % kTcStages], (u / kTcStages) & 1);
     }
-  } else if (warp == 5) {
-    // ---------------- MMA issuer ----------------
+  } else if (warp == 9) {
+    // ---------------- MMA issuer: S(t), then PV(t - 1) ----------------
     if (lane == 0) {
-      const uint32_t idS = idesc_bf16_m128(kTcRows), idPV = idesc_bf16_m128(kTcRows) | (1u << 15);  // (A MN-major)
-      const uint32_t ring_a = smem_u32(ring), q_a = smem_u32(qbuf), p_a = smem_u32(pbuf);
+      const uint32_t idS = idesc_bf16_m128(NQ), idPV = idesc_bf16_m128(NQ) | (1u << 15);  // (A MN-major)
+      const uint32_t k_a = smem_u32(kring), v_a = smem_u32(vring), q_a = smem_u32(qbuf), p_a = smem_u32(pbuf);
       TcCursor cur;
       cur.start(sh, B, H, g0);
       int seg_s = -1, pv_seg = 0;
@@ -492,45 +599,41 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const AttnTcPara
       for (int t = 0; t <= n; ++t) {
         bool first = false, last = false;
         if (t < n) {
-          // S^T(t) = K(t) . Q^T into S buffer t & 1
           first = t == 0 || cur.kt == 0;
           last = t == n - 1 || cur.kt == cur.nt - 1;
           if (first) ++seg_s;
           const int s = t % kTcStages;
-          if (!mbar_wait(&sh.full[s], (t / kTcStages) & 1, abort, p.status)) break;
+          if (!mbar_wait(&sh.kfull[s], (t / kTcStages) & 1, abort, p.status)) break;
           if (t >= 2 && !mbar_wait(&sh.s_free[t & 1], ((t >> 1) - 1) & 1, abort, p.status)) break;
           if (first && !mbar_wait(&sh.q_full[seg_s & 1], (seg_s >> 1) & 1, abort, p.status)) break;
           tc_fence_after();
-          const uint32_t kb_a = ring_a + s * kStageBytes, qb_a = q_a + (seg_s & 1) * kQBytes;
-          const uint32_t dS = tm + (t & 1) * kTcRows;
+          const uint32_t kb_a = k_a + s * kSlotBytes, qb_a = q_a + (seg_s & 1) * kQBytes;
+          const uint32_t dS = tm + (t & 1) * 32;
 #pragma unroll
           for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
-            for (int k16 = 0; k16 < 4; ++k16) {
-              const uint64_t a = sdesc_sw128(kb_a + kb * kBox + k16 * 32);
-              umma_bf16(dS, a, sdesc_sw128(qb_a + kb * kOpBytes + k16 * 32), idS, (kb | k16) ? 1u : 0u);
-              if (P16) umma_bf16(dS, a, sdesc_sw128(qb_a + 2 * kOpBytes + kb * kOpBytes + k16 * 32), idS, 1u);
-            }
+            for (int k16 = 0; k16 < 4; ++k16)
+              umma_bf16(dS, sdesc_sw128(kb_a + kb * kBox + k16 * 32), sdesc_sw128(qb_a + kb * kOpBytes + k16 * 32), idS,
+                        (kb | k16) ? 1u : 0u);
           umma_commit(&sh.s_full[t & 1]);
+          umma_commit(&sh.kempty[s]);
         }
         if (t >= 1) {
-          // O^T += V^T(u) . P^T(u) for the previous tile u
           const int u = t - 1, s = u % kTcStages;
+          if (!mbar_wait(&sh.vfull[s], (u / kTcStages) & 1, abort, p.status)) break;
           if (!mbar_wait(&sh.p_full[u & 1], (u >> 1) & 1, abort, p.status)) break;
-          if (pv_first && pv_seg > 0 && !mbar_wait(&sh.o_free, (pv_seg - 1) & 1, abort, p.status)) break;
+          if (pv_first && pv_seg >= 2 && !mbar_wait(&sh.o_free[pv_seg & 1], ((pv_seg >> 1) - 1) & 1, abort, p.status))
+            break;
           tc_fence_after();
-          const uint32_t v_a = ring_a + s * kStageBytes + 2 * kBox, pb_a = p_a + (u & 1) * kPBytes;
-          const uint32_t dO = tm + 2 * kTcRows;
+          const uint32_t vb_a = v_a + s * kSlotBytes, pb_a = p_a + (u & 1) * kPBytes;
+          const uint32_t dO = tm + kOCol + (pv_seg & 1) * 32;
 #pragma unroll
-          for (int kk = 0; kk < kTcKeys / 16; ++kk) {
-            const uint64_t a = sdesc_sw128_mn(v_a + kk * 16 * 128, kBox);
-            const uint32_t poff = (kk >> 2) * kOpBytes + (kk & 3) * 32;
-            umma_bf16(dO, a, sdesc_sw128(pb_a + poff), idPV, (pv_first && kk == 0) ? 0u : 1u);
-            if (P16) umma_bf16(dO, a, sdesc_sw128(pb_a + 2 * kOpBytes + poff), idPV, 1u);
-          }
-          umma_commit(&sh.empty[s]);
+          for (int kk = 0; kk < kTcKeys / 16; ++kk)
+            umma_bf16(dO, sdesc_sw128_mn(vb_a + kk * 16 * 128, kBox),
+                      sdesc_sw128(pb_a + (kk >> 2) * kOpBytes + (kk & 3) * 32), idPV, (pv_first && kk == 0) ? 0u : 1u);
+          umma_commit(&sh.vempty[s]);
           umma_commit(&sh.p_free[u & 1]);
-          if (pv_last) umma_commit(&sh.o_full);
+          if (pv_last) umma_commit(&sh.o_full[pv_seg & 1]);
         }
         pv_first = first;
         pv_last = last;
@@ -541,8 +644,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const AttnTcPara
       umma_commit(&sh.drain);
       mbar_drain(&sh.drain, 0);
     }
+  } else if (warp < 4) {
+    tc_softmax<P16>(p, sh, tm, qbuf, pbuf, vring, n, g0, tid, warp, lane);
   } else {
-    tc_softmax<P16>(p, sh, tm, qbuf, pbuf, ring, n, g0, T, C, c, tid, warp, lane);
+    tc_epilogue<P16>(p, sh, tm, n, g0, T, C, c, tid - 128, warp);
   }
   __syncwarp();
   tc_fence_before();
@@ -552,6 +657,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const AttnTcPara
     tmem_dealloc(tm, kTmemCols);
   }
 }
+
 
 size_t attn_tc_smem_bytes() { return tc_dyn_smem(); }
 
