@@ -152,7 +152,11 @@ class ClockSampler:
 KERNEL_SOURCES = {
     "verify_persistent": ("verify_mk.cu", "attn_body.cuh", "common.cuh", "internal.h"),
     "attention": ("attention.cu", "attn_body.cuh", "common.cuh", "internal.h"),
+    "attention_tc": ("attn_tc.cu", "common.cuh", "internal.h"),
 }
+
+# tss_attention_kernel -> the KERNEL_SOURCES entry of the separate attention kernel that ran
+ATTENTION_IMPL = {0: "attention", 1: "attention_tc", 2: "attention"}
 
 
 def kernel_sources_hash(kernel="verify_persistent"):
@@ -578,11 +582,14 @@ def run_tss(args):
             v["share"] = v["ms_per_step"] / tot
         dom = max((n for n in kernels if n in kb), key=lambda n: kernels[n]["ms_per_step"])
         ach = kernels[dom]["gbs"]
-        roofline = {"kernel": dom, "bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
+        if "attention" in kernels:
+            kernels["attention"]["impl"] = ATTENTION_IMPL.get(run.v.attention_kernel(), "attention")
+        impl = kernels[dom].get("impl", dom)
+        roofline = {"kernel": impl, "bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
                     "frac": ach / peak, "peak_source": f"{peak_kind} copy bandwidth",
                     "frac_of_nominal_8TBs": ach / NOMINAL_HBM_GBS,
                     "bytes_per_launch": kb[dom] / kernels[dom]["launches_per_step"], "traffic": None}
-        tr = find_traffic(args.traffic, dom, w.name)
+        tr = find_traffic(args.traffic, impl, w.name)
         if tr is not None:
             roofline["traffic"] = tr["traffic_bytes"]
             roofline["traffic_source"] = tr.get("source")
