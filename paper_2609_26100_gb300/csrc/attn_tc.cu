@@ -151,12 +151,23 @@ struct TcCursor {
 // Q rows of (request b, head h) as the B operand of the score product: rows >= N zero, 128
 // columns, K-major 128-byte swizzle.  P16: q arrives in fp16 and is split exactly into bf16 hi
 // (rows 0-15) + lo (rows 16-31); else q is bf16 (rows 0-15).
+// Each of 128 threads holds two 16-byte chunks (8 columns of one row): tc_load_q reads them
+// from the q rows, tc_store_q writes them (split into parts) into an operand buffer.
+__device__ __forceinline__ void tc_load_q(const AttnTcParams& p, int crow, int N, int h, int tid, uint4 (&raw)[2]) {
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int x = tid + 128 * i, r = x >> 4, c8 = x & 15;
+    raw[i] = make_uint4(0, 0, 0, 0);
+    if (r < N) raw[i] = *reinterpret_cast<const uint4*>(p.q + static_cast<size_t>(crow + r) * p.d_model + h * kTcD + c8 * 8);
+  }
+}
+
 template <bool P16>
-__device__ __forceinline__ void tc_write_q(const AttnTcParams& p, int crow, int N, int h, uint8_t* qb, int tid) {
-  for (int x = tid; x < kTcRows * (kTcD / 8); x += 128) {
-    const int r = x >> 4, c8 = x & 15;
-    uint4 raw = make_uint4(0, 0, 0, 0);
-    if (r < N) raw = *reinterpret_cast<const uint4*>(p.q + static_cast<size_t>(crow + r) * p.d_model + h * kTcD + c8 * 8);
+__device__ __forceinline__ void tc_store_q(uint8_t* qb, int tid, const uint4 (&rawq)[2]) {
+#pragma unroll
+  for (int i2 = 0; i2 < 2; ++i2) {
+    const int x = tid + 128 * i2, r = x >> 4, c8 = x & 15;
+    const uint4 raw = rawq[i2];
     if (P16) {
       const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
       uint32_t hi[4], lo[4];
@@ -173,6 +184,13 @@ __device__ __forceinline__ void tc_write_q(const AttnTcParams& p, int crow, int 
       *reinterpret_cast<uint4*>(qb + op_off(r, c8 * 8)) = raw;
     }
   }
+}
+
+template <bool P16>
+__device__ __forceinline__ void tc_write_q(const AttnTcParams& p, int crow, int N, int h, uint8_t* qb, int tid) {
+  uint4 raw[2];
+  tc_load_q(p, crow, N, h, tid, raw);
+  tc_store_q<P16>(qb, tid, raw);
 }
 
 __device__ __forceinline__ void tc_store_out(const AttnTcParams& p, int row, int col, float v) {
@@ -230,6 +248,17 @@ __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, 
     const int ctx = st->req_ctx[b], N = st->req_nodes[b], Tk = ctx + N;
     const int key = kt * kTcKeys + k;
 
+    // the next item's q rows are read now, while this tile's scores are being computed, and
+    // written into the other Q buffer below
+    const bool next_q = first && t + (nt - kt) < n;
+    uint4 qraw[2];
+    if (next_q) {
+      TcCursor nx = cur;
+      nx.kt = nx.nt - 1;
+      nx.next(sh, B, H);
+      tc_load_q(p, pl->slot_crow[p.slot][nx.b], st->req_nodes[nx.b], nx.h, tid, qraw);
+    }
+
     // scores of this key for the block's rows (hi and lo products added)
     bool ok = mbar_wait(&sh.s_full[t & 1], (t >> 1) & 1, abort, p.status);
     if (bar_or<kBarSoftmax>(!ok)) break;
@@ -245,14 +274,7 @@ __device__ __forceinline__ void tc_softmax(const AttnTcParams& p, TcShared& sh, 
 
     // Q of the next item into the other buffer (the score products of the item before this one,
     // which read it, are complete: their commit preceded this tile's)
-    bool next_q = false;
-    if (first && t + (nt - kt) < n) {
-      TcCursor nx = cur;
-      nx.kt = nx.nt - 1;
-      nx.next(sh, B, H);
-      tc_write_q<P16>(p, pl->slot_crow[p.slot][nx.b], st->req_nodes[nx.b], nx.h, qbuf + ((seg + 1) & 1) * kQBytes, tid);
-      next_q = true;
-    }
+    if (next_q) tc_store_q<P16>(qbuf + ((seg + 1) & 1) * kQBytes, tid, qraw);
 
     // context / ancestor mask (vis bit q: row q sees this key), scale to log2 units
     uint32_t vis = 0;
