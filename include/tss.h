@@ -167,7 +167,8 @@ typedef struct {
  * error everything allocated so far is freed and *out is NULL.  For failure injection, the
  * environment variable TSS_ALLOC_LIMIT_BYTES=N makes the allocations fail with OUT_OF_MEMORY
  * once they would pass N bytes.  TSS_WAIT_LIMIT_MS=N (1..600000, default 2000) bounds every
- * device-side wait of the persistent kernel (see tss_inject_timeout). */
+ * device-side wait of the persistent kernel (see tss_inject_timeout); the tcgen05 attention's
+ * waits are bounded by 2 s. */
 tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx** out);
 
 /* Phi(domain_id) = the set of layers whose bit is set in layer_bitmask (bit l = skip layer l;
@@ -302,7 +303,10 @@ tss_status tss_sync_status(tss_ctx* ctx, void* stream);
  * every CTA leaves its loops and frees its tensor memory, and tss_sync_status reports the code.
  * That step's outputs are undefined.  The context stays usable: every step starts with fresh
  * counters and a clear abort word, so the next step runs normally.  A step with no active layer
- * withholds nothing.  n_steps = 0 cancels. */
+ * withholds nothing.  n_steps = 0 cancels.  When the step's attention runs in the tcgen05 kernel
+ * (tss_attention_kernel = 1), the first CTA of the step's first attention launch issues no MMA
+ * instead, so that kernel's waits run out (after its fixed 2 s bound) and it takes the same
+ * abort path; the next step's prologue resets its counters. */
 tss_status tss_inject_timeout(tss_ctx* ctx, int n_steps);
 
 /* Diagnostic: the Philox4x32-10 stream that speculative sampling draws from when the batch gives

@@ -660,6 +660,10 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
     const bool tc = attn_variant(c, sp) == 1;
     AttnTcParams tp = tc_params(c, p.scale_log2);
     tp.o_xs = xs;
+    // fault injection: with the tcgen05 attention the first attention launch withholds the signal
+    // (the persistent launches then withhold nothing)
+    const int inject_attn = tc ? p.withhold_flag : 0;
+    if (tc) p.withhold_flag = 0;
     int pb = 0;
     for (int j = 0; j < sp.n_act; ++j) {
       p.ph_begin = pb;  // phases 4j .. 4j+3 are QKV, O, gate/up, down of slot j; 4 n_act the LM head
@@ -667,6 +671,7 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
       TSS_MK(8, TSS_CU(launch_verify_mk(p, c->num_sms, smem, s)));
       if (tc) {
         tp.slot = j;
+        tp.withhold = j == 0 ? inject_attn : 0;
         TSS_MK(2, TSS_CU(launch_attention_tc(tp, c->num_sms, s, false)));
       } else {
         ap.slot = j;

@@ -618,7 +618,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const AttnTcPara
       cur.start(sh, B, H, g0);
       int seg_s = -1, pv_seg = 0;
       bool pv_first = false, pv_last = false;
-      for (int t = 0; t <= n; ++t) {
+      // fault injection: CTA 0 issues no MMA, so its softmax's first wait runs out
+      const int n_issue = p.withhold && blockIdx.x == 0 ? -1 : n;
+      for (int t = 0; t <= n_issue; ++t) {
         bool first = false, last = false;
         if (t < n) {
           first = t == 0 || cur.kt == 0;

@@ -93,6 +93,7 @@ struct AttnTcParams {
   float* part_ml;                // [attn_tc_partial_rows][2]
   int* counters;                 // [B][H], self-resetting
   int* status;
+  int withhold;                  // fault injection: CTA 0 issues no MMA (its first wait runs out)
 };
 size_t attn_tc_smem_bytes();
 size_t attn_tc_partial_rows(int max_batch, int n_heads, int grid);

@@ -182,3 +182,30 @@ def test_tc_not_used_for_larger_blocks_or_when_off(weights):
     assert run.v.attention_kernel() == NARROW
     case.check(wo, res, "20 rows")
     run.close()
+
+
+def test_tc_bounded_wait_times_out_and_the_context_recovers(weights):
+    """Failure injection without a GPU fault, in the tcgen05 attention kernel: a step whose first
+    attention launch has CTA 0 issue no MMA (tss_inject_timeout) ends with TSS_ERR_TIMEOUT from
+    that kernel's bounded waits (2 s), every CTA drains its copies and frees its tensor memory,
+    and the next steps on the same context run normally and match the oracle."""
+    wo, wg = weights
+    reqs = [chain(1000, 5, "tc.to0"), chain(300, 3, "tc.to1")]
+    run = make_runner(wg, n_slots=2, cap=1024, path="hybrid")
+    case = Case(run, reqs, {0: 0})
+    run.v.inject_timeout(1)
+    depth = max(max(synth.depths_of(r.parents)) for r in reqs)
+    res = run.alloc_results(len(reqs), sum(len(r.parents) for r in reqs), path_stride=max(64, depth + 1))
+    run.verify(run.batch(reqs), res)
+    st = run.sync_status()
+    torch.cuda.synchronize()
+    assert st == native.TSS_ERR_TIMEOUT
+    assert run.v.attention_kernel() == TC
+    assert run.sync_status() == native.TSS_OK  # reported once, then cleared
+    for _ in range(2):
+        for l in range(ARCH.n_layers):  # the failed step's appends are discarded
+            for b, r in enumerate(reqs):
+                run.kv[l][b, :, :, r.ctx_len:].fill_(float("nan"))
+        res = case.step()
+        case.check(wo, res, "after a timeout")
+    run.close()
