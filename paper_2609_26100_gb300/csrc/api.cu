@@ -128,6 +128,7 @@ struct tss_ctx {
   int mk_dp_tail = 1;  // whole-tile tails for phases with a tile per CTA (TSS_MK_DP)
   int attn_plo = 1;
   int attn_splits_force = 0;  // > 0: key splits of the separate attention kernel (TSS_ATTN_SPLITS)
+  int mk_splits_force = 0;    // > 0: key splits of the persistent kernel's attention (TSS_MK_ATTN_SPLITS)
   // tcgen05 attention of blocks of at most 16 rows (head_dim 128; TSS_ATTN_TC=0 turns it off)
   int attn_tc = 1;
   int last_attn = -1;                    // attention kernel of the last step (tss_attention_kernel)
@@ -452,9 +453,10 @@ struct MkConfig {
 // What the persistent kernel's shared-memory plan depends on (a context's shape and switches).
 struct MkPlanIn {
   int D, H, num_sms, kps_max, stages_max, max_splits;
+  int splits_force;  // > 0: key splits of the persistent kernel's attention (TSS_MK_ATTN_SPLITS)
 };
 MkPlanIn mk_plan_in(const tss_ctx* c) {
-  return MkPlanIn{c->D, c->H, c->num_sms, c->mk_kps, c->mk_max_stages, c->max_splits};
+  return MkPlanIn{c->D, c->H, c->num_sms, c->mk_kps, c->mk_max_stages, c->max_splits, c->mk_splits_force};
 }
 
 int mk_attn_splits(const MkPlanIn& c, int B, int tiles) {
@@ -509,7 +511,7 @@ bool mk_config_for(const MkPlanIn& c, int B, int M, int tiles, MkConfig* out) {
   constexpr size_t kLimit = 232448;  // per-block shared-memory maximum of sm_103 (227 KiB)
   const size_t q = static_cast<size_t>(kNarrowNodes) * (c.D + 8) * 2;
   const size_t tile = static_cast<size_t>(2) * 64 * (c.D + 8) * 2;
-  const int splits = mk_attn_splits(c, B, std::max(tiles, 1));
+  const int splits = c.splits_force > 0 ? std::min(c.splits_force, c.max_splits) : mk_attn_splits(c, B, std::max(tiles, 1));
   const int per = std::max(1, (std::max(tiles, 1) + splits - 1) / splits);
   for (int kps = c.kps_max; kps >= 1; --kps) {
     const XsLayout xs = xs_layout(M);
@@ -1064,6 +1066,7 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_ATTN_PLO")) c->attn_plo = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ATTN_SPLITS")) c->attn_splits_force = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_ATTN_TC")) c->attn_tc = std::atoi(e) != 0;
+  if (const char* e = std::getenv("TSS_MK_ATTN_SPLITS")) c->mk_splits_force = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
   if (const char* e = std::getenv("TSS_MK_DP")) c->mk_dp_tail = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ALLOC_LIMIT_BYTES")) c->alloc_limit = std::strtoull(e, nullptr, 10);
@@ -1159,7 +1162,7 @@ tss_status tss_persistent_plan(const tss_arch* a, int n_req, int n_rows, int max
     return fail(TSS_ERR_INVALID_ARG, "arch: head_dim 64 or 128 and n_heads >= 1");
   if (n_req < 1 || n_req > kMaxBatch || n_rows < n_req || n_rows > kMaxRows || max_keys < 1 || num_sms < 1)
     return fail(TSS_ERR_INVALID_ARG, "n_req in [1, 64], n_rows in [n_req, 256], max_keys and num_sms positive");
-  const MkPlanIn in{a->head_dim, a->n_heads, num_sms, 3, 12, kMaxSplits};
+  const MkPlanIn in{a->head_dim, a->n_heads, num_sms, 3, 12, kMaxSplits, 0};
   MkConfig cfg;
   const bool fits = mk_config_for(in, n_req, n_rows, (max_keys + 63) / 64, &cfg);
   out->fits = fits ? 1 : 0;
