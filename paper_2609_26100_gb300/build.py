@@ -10,7 +10,7 @@ import sys
 HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 LIB = os.path.join(HERE, "libtss.so")
-SOURCES = ("api.cu", "gemm.cu", "attention.cu", "attn_tc.cu", "misc.cu", "noalloc.cu", "verify_mk.cu")
+SOURCES = ("api.cu", "gemm.cu", "attention.cu", "attn_tc.cu", "misc.cu", "noalloc.cu", "prefill.cu", "verify_mk.cu")
 HEADERS = ("common.cuh", "internal.h", "attn_body.cuh")
 ARCH = ("-gencode", "arch=compute_103a,code=sm_103a")
 FLAGS = ("-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr")

@@ -138,6 +138,14 @@ struct tss_ctx {
   int kvmap_slots = -1, kvmap_cap = -1;  // ... and the cache shape
   bool kvmap_ok = false;                 // the maps describe the current cache
   float *tc_po = nullptr, *tc_pml = nullptr;
+  // compute-bound prefill (prefill.cu; head_dim 128, TSS_PREFILL=steps turns it off)
+  bool pf_enabled = true;
+  int pf_tmax = 0;  // tokens per chunk; 0 until the workspaces exist
+  float* pf_h = nullptr;
+  __nv_bfloat16 *pf_xh = nullptr, *pf_xl = nullptr, *pf_qh = nullptr, *pf_ql = nullptr, *pf_ah = nullptr,
+                *pf_al = nullptr, *pf_uh = nullptr, *pf_ul = nullptr;
+  int* pf_tok = nullptr;
+  CUtensorMap pf_tm_xh, pf_tm_xl, pf_tm_qh, pf_tm_ql, pf_tm_ah, pf_tm_al, pf_tm_uh, pf_tm_ul;
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
   unsigned long long wait_ns = 2000000000ull;  // bound of the persistent kernel's waits (TSS_WAIT_LIMIT_MS)
   int inject_timeouts = 0;  // steps left that withhold one dataflow flag (tss_inject_timeout)
@@ -855,6 +863,7 @@ tss_status build_workspaces(tss_ctx* c) {
   TSS_CU(gemm_prepare(max_smem));
   TSS_CU(attn_prepare());
   TSS_CU(attn_tc_prepare());
+  TSS_CU(pf_prepare());
   TSS_CU(mk_prepare());
   {
     const int nt = d / 128;
@@ -1007,6 +1016,97 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
   return TSS_OK;
 }
 
+// Workspaces of the compute-bound prefill, made at the first call: chunks of up to 1024 tokens.
+tss_status pf_workspaces(tss_ctx* c) {
+  if (c->pf_tmax) return TSS_OK;
+  const int T = 1024;
+  const size_t d = c->d, F = c->F_pad;
+  TSS_TRY(c->alloc(&c->pf_h, T * d));
+  TSS_TRY(c->alloc(&c->pf_xh, T * d));
+  TSS_TRY(c->alloc(&c->pf_xl, T * d));
+  TSS_TRY(c->alloc(&c->pf_qh, T * d));
+  TSS_TRY(c->alloc(&c->pf_ql, T * d));
+  TSS_TRY(c->alloc(&c->pf_ah, T * d));
+  TSS_TRY(c->alloc(&c->pf_al, T * d));
+  TSS_TRY(c->alloc(&c->pf_uh, T * F));
+  TSS_TRY(c->alloc(&c->pf_ul, T * F));
+  TSS_TRY(c->alloc(&c->pf_tok, T));
+  // (rows past a chunk's tokens are read by the last tile of each GEMM and attention: finite)
+  TSS_CU(cudaMemset(c->pf_xh, 0, T * d * 2));
+  TSS_CU(cudaMemset(c->pf_xl, 0, T * d * 2));
+  TSS_CU(cudaMemset(c->pf_qh, 0, T * d * 2));
+  TSS_CU(cudaMemset(c->pf_ql, 0, T * d * 2));
+  TSS_CU(cudaMemset(c->pf_ah, 0, T * d * 2));
+  TSS_CU(cudaMemset(c->pf_al, 0, T * d * 2));
+  TSS_CU(cudaMemset(c->pf_uh, 0, T * F * 2));
+  TSS_CU(cudaMemset(c->pf_ul, 0, T * F * 2));
+  const struct {
+    CUtensorMap* m;
+    const void* p;
+    size_t k;
+  } maps[] = {{&c->pf_tm_xh, c->pf_xh, d}, {&c->pf_tm_xl, c->pf_xl, d}, {&c->pf_tm_qh, c->pf_qh, d},
+              {&c->pf_tm_ql, c->pf_ql, d}, {&c->pf_tm_ah, c->pf_ah, d}, {&c->pf_tm_al, c->pf_al, d},
+              {&c->pf_tm_uh, c->pf_uh, F}, {&c->pf_tm_ul, c->pf_ul, F}};
+  for (const auto& m : maps)
+    if (!make_tmap(m.m, m.p, m.k, T, 1, 128, 2)) return fail(TSS_ERR_CUDA, "cuTensorMapEncodeTiled failed (prefill)");
+  c->pf_tmax = T;
+  return TSS_OK;
+}
+
+// One request's chunk of T (<= pf_tmax) prompt tokens at positions pos0.. through every layer its
+// skip set keeps (Sec. "Domain-Aware Skip Controller": h_{l+1} = h_l for a skipped layer, which
+// writes no KV).  d_tokens: DEVICE, already in c->pf_tok.
+tss_status pf_chunk(tss_ctx* c, int slot, int pos0, int T, unsigned long long skip, const tss_kv_cache* kv,
+                    cudaStream_t s) {
+  PfParams p{};
+  p.T = T;
+  p.pos0 = pos0;
+  p.slot = slot;
+  p.d_model = c->d;
+  p.n_heads = c->H;
+  p.head_dim = c->D;
+  p.vocab = c->V;
+  p.kv_cap = kv->cap;
+  p.rms_eps = c->a.rms_eps;
+  p.tokens = c->pf_tok;
+  p.embed = c->embed;
+  p.h = c->pf_h;
+  p.xh = c->pf_xh;
+  p.xl = c->pf_xl;
+  p.x_ld = c->d;
+  p.qh = c->pf_qh;
+  p.ql = c->pf_ql;
+  p.ah = c->pf_ah;
+  p.al = c->pf_al;
+  p.uh = c->pf_uh;
+  p.ul = c->pf_ul;
+  p.u_ld = c->F_pad;
+  p.rope_cos = c->rope_cos;
+  p.rope_sin = c->rope_sin;
+  p.status = c->d_status;
+  const unsigned long long rows = static_cast<unsigned long long>(kv->n_slots) * 2ull * c->H * kv->cap;
+  if (rows + 64 > 0x7fffffffull) return fail(TSS_ERR_INVALID_ARG, "KV cache too large for the prefill's tensor maps");
+  TSS_CU(launch_pf_embed(p, s));
+  const int d = c->d, kbd = d / 64, G = c->num_sms;
+  const size_t dd = static_cast<size_t>(d) * d;
+  for (int l = 0; l < c->L; ++l) {
+    if ((skip >> l) & 1ull) continue;
+    CUtensorMap tkv;
+    if (!make_tmap(&tkv, kv->layer[l], 128, rows, 1, 64, 2)) return fail(TSS_ERR_CUDA, "cuTensorMapEncodeTiled failed (prefill KV)");
+    p.kv = static_cast<__nv_bfloat16*>(kv->layer[l]);
+    TSS_CU(launch_pf_norm(p, c->g_attn + static_cast<size_t>(l) * d, s));
+    TSS_CU(launch_pf_gemm(kPfEpiQkv, c->pf_tm_xh, c->pf_tm_xl, p, PfGemm{c->wqkv, static_cast<long long>(3 * dd), l, 3 * d / 128, kbd}, G, s));
+    TSS_CU(launch_pf_attn(c->pf_tm_qh, c->pf_tm_ql, tkv, p, s));
+    TSS_CU(launch_pf_gemm(kPfEpiResid, c->pf_tm_ah, c->pf_tm_al, p, PfGemm{c->wo, static_cast<long long>(dd), l, d / 128, kbd}, G, s));
+    TSS_CU(launch_pf_norm(p, c->g_mlp + static_cast<size_t>(l) * d, s));
+    TSS_CU(launch_pf_gemm(kPfEpiSwiglu, c->pf_tm_xh, c->pf_tm_xl, p,
+                          PfGemm{c->wgu, static_cast<long long>(c->Ft) * 128 * d, l, c->Ft, kbd}, G, s));
+    TSS_CU(launch_pf_gemm(kPfEpiResid, c->pf_tm_uh, c->pf_tm_ul, p,
+                          PfGemm{c->wdown, static_cast<long long>(d) * c->F_pad, l, d / 128, c->F_pad / 64}, G, s));
+  }
+  return TSS_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -1067,6 +1167,7 @@ tss_status tss_create(const tss_weights* weights, const tss_arch* arch, tss_ctx*
   if (const char* e = std::getenv("TSS_ATTN_SPLITS")) c->attn_splits_force = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("TSS_ATTN_TC")) c->attn_tc = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_MK_ATTN_SPLITS")) c->mk_splits_force = std::max(0, std::atoi(e));
+  if (const char* e = std::getenv("TSS_PREFILL")) c->pf_enabled = std::string(e) != "steps";
   if (const char* e = std::getenv("TSS_MK_STAGES")) c->mk_max_stages = std::min(12, std::max(2, std::atoi(e)));
   if (const char* e = std::getenv("TSS_MK_DP")) c->mk_dp_tail = std::atoi(e) != 0;
   if (const char* e = std::getenv("TSS_ALLOC_LIMIT_BYTES")) c->alloc_limit = std::strtoull(e, nullptr, 10);
@@ -1425,6 +1526,28 @@ tss_status tss_prefill(tss_ctx* c, int n_req, const int32_t* n_tokens, const int
     if (static_cast<long long>(ctx_len[b]) + n_tokens[b] > kv->cap)
       return fail(TSS_ERR_KV_CAPACITY, "ctx_len + n_tokens exceeds KV capacity");
     off[b + 1] = off[b] + n_tokens[b];
+  }
+  if (c->pf_enabled && c->D == 128) {
+    // compute-bound path: each request's tokens in chunks of up to pf_tmax, all at once per chunk
+    for (int l = 0; l < c->L; ++l)
+      if (kv->layer[l] && !aligned16(kv->layer[l])) return fail(TSS_ERR_INVALID_ARG, "KV buffers must be 16-byte aligned");
+    TSS_TRY(pf_workspaces(c));
+    for (int b = 0; b < n_req; ++b) {
+      const int dom = domain_id[b];
+      const bool configured = dom >= 0 && dom < c->a.max_domains && c->phi_valid[dom];
+      const unsigned long long skip = configured ? c->phi[dom] : 0ull;
+      for (int l = 0; l < c->L; ++l)
+        if (!((skip >> l) & 1ull) && !kv->layer[l]) return fail(TSS_ERR_INVALID_ARG, "KV buffer of an active layer is NULL");
+      const int slot = kv_slot ? kv_slot[b] : b;
+      if (slot < 0 || slot >= kv->n_slots) return fail(TSS_ERR_INVALID_ARG, "kv_slot out of range");
+      for (int done = 0; done < n_tokens[b]; done += c->pf_tmax) {
+        const int T = std::min(c->pf_tmax, n_tokens[b] - done);
+        TSS_CU(cudaMemcpyAsync(c->pf_tok, tokens + off[b] + done, sizeof(int32_t) * T,
+                               io_host ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToDevice, s));
+        TSS_TRY(pf_chunk(c, slot, ctx_len[b] + done, T, skip, kv, s));
+      }
+    }
+    return TSS_OK;
   }
   // Rounds of verification steps: each request still holding tokens adds a chain of up to
   // max_nodes of them (row 0, the chain's root, is not yet cached, exactly like a draft block's

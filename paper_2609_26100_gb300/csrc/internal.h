@@ -95,6 +95,39 @@ struct AttnTcParams {
   int* status;
   int withhold;                  // fault injection: CTA 0 issues no MMA (its first wait runs out)
 };
+// Compute-bound prefill (prefill.cu): one request's chunk of T prompt tokens at positions
+// pos0 .. pos0 + T - 1 (head_dim 128).
+constexpr int kPfEpiQkv = 0, kPfEpiResid = 1, kPfEpiSwiglu = 2;
+struct PfParams {
+  int T, pos0, slot, d_model, n_heads, head_dim, vocab, kv_cap;
+  float rms_eps;
+  const int* tokens;               // [T] device
+  const __nv_bfloat16* embed;      // [vocab][d]
+  float* h;                        // [T_max][d] residual stream
+  __nv_bfloat16 *xh, *xl;          // [T_max][x_ld] normed activations (hi, lo): the B operand of QKV and gate/up
+  int x_ld;
+  __nv_bfloat16 *qh, *ql;          // [T_max][d] q after RoPE (hi, lo)
+  __nv_bfloat16 *ah, *al;          // [T_max][d] attention output (hi, lo): the B operand of O
+  __nv_bfloat16 *uh, *ul;          // [T_max][u_ld] SwiGLU output (hi, lo): the B operand of down
+  int u_ld;
+  __nv_bfloat16* kv;               // this layer's cache [n_slots][2][H][cap][D]
+  const float* rope_cos;           // [max_positions][D / 2]
+  const float* rope_sin;
+  int* status;
+};
+struct PfGemm {
+  const __nv_bfloat16* w;          // pre-tiled weights (16 KiB blocks [layer][row tile][k-block])
+  long long w_layer_elems;
+  int layer, n_o, kb;              // layer, 128-row weight tiles, 64-column k-blocks
+};
+cudaError_t pf_prepare();
+cudaError_t launch_pf_embed(const PfParams& p, cudaStream_t s);
+cudaError_t launch_pf_norm(const PfParams& p, const float* g, cudaStream_t s);
+cudaError_t launch_pf_gemm(int epi, const CUtensorMap& xh, const CUtensorMap& xl, const PfParams& p, const PfGemm& g,
+                           int grid, cudaStream_t s);
+cudaError_t launch_pf_attn(const CUtensorMap& qh, const CUtensorMap& ql, const CUtensorMap& kv, const PfParams& p,
+                           cudaStream_t s);
+
 size_t attn_tc_smem_bytes();
 size_t attn_tc_partial_rows(int max_batch, int n_heads, int grid);
 cudaError_t attn_tc_prepare();
