@@ -728,6 +728,10 @@ def run_prefill(args):
     torch.cuda.set_device(0)
     _build.build()
     w = synth.workload_7b_chain()
+    if args.layers:  # a cut of the model (profiling): the first args.layers layers
+        import dataclasses
+        w.arch = dataclasses.replace(w.arch, n_layers=args.layers)
+        w.phi = {d: m & ((1 << args.layers) - 1) for d, m in w.phi.items()}
     a = w.arch
     union = w.active_union()
     n_req, n_tok = 4, args.prefill

@@ -9,9 +9,10 @@
 //
 // GEMMs (pf_gemm_kernel): out[t][o] = sum_k X[t][k] W[o][k] with the weights on the MMA's M side
 // (128-row tiles, the pre-tiled 128-byte-swizzled images the verification kernels stream) and
-// 128 tokens on the N side; every tile runs its whole K loop in one CTA (no split), tiles are
-// taken weight-row-major by a persistent grid so that the CTAs working at the same time share a
-// weight tile through L2.  X is held as two bf16 parts (hi = bf16(x), lo = bf16(x - hi)), both
+// 128 tokens on the N side; a CTA takes two weight tiles against one token tile at a time (two
+// accumulators sharing the token operand) through its whole K loop (no split); items are taken
+// weight-row-major by a persistent grid so that the CTAs working at the same time share weight
+// tiles through L2.  X is held as two bf16 parts (hi = bf16(x), lo = bf16(x - hi)), both
 // multiplied by the weights into one fp32 accumulator in tensor memory, as on the verification
 // path.  Attention (pf_attn_kernel): one CTA per (128-query tile, head), queries on the MMA's M
 // side, 64-key tiles of the cache by TMA, S = Q K^T and O += P V in tensor memory, one thread
@@ -22,15 +23,17 @@ namespace tss {
 
 namespace {
 
-constexpr int kPfThreads = 192;  // warp 0: TMA / bulk copies, warp 1: MMA (+ TMEM), warps 2-5: epilogue
-constexpr int kPfStages = 4;
+constexpr int kPfThreads = 192;  // attention: warp 0 TMA, warp 1 MMA (+ TMEM), warps 2-5 softmax
+constexpr int kPgGroups = 4;     // GEMM epilogue groups of four warps (one per TMEM lane quarter)
+constexpr int kPgThreads = 64 + 128 * kPgGroups;  // warp 0 copies, warp 1 MMA (+ TMEM), then the epilogue groups
+constexpr int kPfStages = 3;
 constexpr uint32_t kPfA = 128 * 64 * 2;      // weight block: 16 KiB
 constexpr uint32_t kPfB = 128 * 64 * 2;      // 128 tokens x 64 columns of one part: 16 KiB
-constexpr uint32_t kPfStage = kPfA + 2 * kPfB;
+constexpr uint32_t kPfStage = 2 * kPfA + 2 * kPfB;  // two weight blocks, the token block's two parts
 constexpr uint32_t kPfAccCols = 128;         // one accumulator: 128 token columns
 
 __host__ __device__ inline size_t pf_gemm_smem() {
-  return 1024 + static_cast<size_t>(kPfStages) * kPfStage + 16 * 128 * 4;  // + epilogue exchange
+  return 1024 + static_cast<size_t>(kPfStages) * kPfStage + kPgGroups * 16 * 128 * 4;  // + exchange per group
 }
 
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
@@ -85,26 +88,26 @@ __global__ void pf_norm_kernel(const PfParams p, const float* g) {
 // ---------------------------------------------------------------------------------------------
 namespace {
 
-// OR of v over the 128 epilogue threads (named barrier 2), which it also synchronises.
+// OR of v over the epilogue threads (named barrier 2), which it also synchronises.
 __device__ __forceinline__ bool pf_epi_or(bool v) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred p, q;\n\t"
       "setp.ne.u32 q, %1, 0;\n\t"
-      "bar.red.or.pred p, 2, 128, q;\n\t"
+      "bar.red.or.pred p, 2, %2, q;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}\n"
       : "=r"(r)
-      : "r"(v ? 1u : 0u)
+      : "r"(v ? 1u : 0u), "n"(128 * kPgGroups)
       : "memory");
   return r != 0;
 }
 
 // One 16-token chunk (tokens j0 .. j0 + 15) of output row r of weight tile t; xch: [16][128]
-// exchange for the row pairs of RoPE (r, r ^ head_dim / 2) and SwiGLU (gate r, up r + 64).
+// exchange (the group's own, synchronised by named barrier `bar` of its 128 threads) for the row
+// pairs of RoPE (r, r ^ head_dim / 2) and SwiGLU (gate r, up r + 64).
 template <int EPI>
 __device__ __forceinline__ void pf_epilogue(const PfParams& p, const PfGemm& g, float* xch, int t, int r, int j0,
-                                            const float* v, int et) {
-  (void)et;
+                                            const float* v, int bar) {
   if constexpr (EPI == kPfEpiResid) {
     const int o = t * 128 + r;
 #pragma unroll
@@ -122,7 +125,7 @@ __device__ __forceinline__ void pf_epilogue(const PfParams& p, const PfGemm& g, 
     if (sec < 2) {
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) xch[jj * 128 + r] = v[jj];
-      named_bar_sync(1, 128);
+      named_bar_sync(bar, 128);
       const int pr = r ^ half, i = dim & (half - 1);
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) {
@@ -135,7 +138,7 @@ __device__ __forceinline__ void pf_epilogue(const PfParams& p, const PfGemm& g, 
           out[jj] = dim < half ? v[jj] * c - pv * s : v[jj] * c + pv * s;
         }
       }
-      named_bar_sync(1, 128);
+      named_bar_sync(bar, 128);
     } else {
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) out[jj] = v[jj];
@@ -155,7 +158,7 @@ __device__ __forceinline__ void pf_epilogue(const PfParams& p, const PfGemm& g, 
   } else if constexpr (EPI == kPfEpiSwiglu) {
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) xch[jj * 128 + r] = v[jj];
-    named_bar_sync(1, 128);
+    named_bar_sync(bar, 128);
     if (r < 64) {
       const int fcol = t * 64 + r;
 #pragma unroll
@@ -167,26 +170,30 @@ __device__ __forceinline__ void pf_epilogue(const PfParams& p, const PfGemm& g, 
         }
       }
     }
-    named_bar_sync(1, 128);
+    named_bar_sync(bar, 128);
   }
   (void)g;
 }
 
 }  // namespace
 
+// Work item = (pair of weight tiles 2w, 2w + 1; token tile u): the two weight tiles share every
+// stage's token operand, so a stage of 64 KiB feeds 4 MMAs of 128 x 128 x 16 per k16 step (the
+// copy bytes per MMA are half those of one weight tile per item, which L2 bandwidth binds).
 template <int EPI>
-__global__ void __launch_bounds__(kPfThreads, 1) pf_gemm_kernel(const __grid_constant__ CUtensorMap tm_xh,
+__global__ void __launch_bounds__(kPgThreads, 1) pf_gemm_kernel(const __grid_constant__ CUtensorMap tm_xh,
                                                                  const __grid_constant__ CUtensorMap tm_xl,
                                                                  const PfParams p, const PfGemm g) {
   extern __shared__ uint8_t pf_dyn[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(pf_dyn) + 1023) & ~uintptr_t(1023));
-  float* xch = reinterpret_cast<float*>(base + kPfStages * kPfStage);  // [16][128]
+  float* xch0 = reinterpret_cast<float*>(base + kPfStages * kPfStage);  // [group][16][128]
   __shared__ uint64_t full[kPfStages], empty[kPfStages], acc_full[2], acc_empty[2], drain;
   __shared__ uint32_t tslot;
   __shared__ int abort_s;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int n_u = (p.T + 127) >> 7;  // token tiles
-  const long long n_tiles = static_cast<long long>(g.n_o) * n_u;
+  const int n_u = (p.T + 127) >> 7;         // token tiles
+  const int n_w = (g.n_o + 1) >> 1;         // weight-tile pairs (the last may hold one tile)
+  const long long n_items = static_cast<long long>(n_w) * n_u;
   if (tid == 0) {
     for (int i = 0; i < kPfStages; ++i) {
       mbar_init(&full[i], 1);
@@ -194,14 +201,14 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_gemm_kernel(const __grid_con
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&acc_full[i], 1);
-      mbar_init(&acc_empty[i], 4);
+      mbar_init(&acc_empty[i], 4 * kPgGroups);
     }
     mbar_init(&drain, 1);
     abort_s = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(&tslot, 2 * kPfAccCols);
+    tmem_alloc(&tslot, 4 * kPfAccCols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -212,13 +219,16 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_gemm_kernel(const __grid_con
   const __nv_bfloat16* wl = g.w + static_cast<size_t>(g.layer) * g.w_layer_elems;
 
   if (warp == 0) {
+    // ---------------- producer: both weight blocks and both token parts of each k-block ----------------
     if (lane == 0) {
       prefetch_tmap(&tm_xh);
       prefetch_tmap(&tm_xl);
-      long long it = 0;  // (tile, k-block) iterations of this CTA
+      long long it = 0;
       bool ok = true;
-      for (long long tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-        const int t = static_cast<int>(tile / n_u), u = static_cast<int>(tile - static_cast<long long>(t) * n_u);
+      for (long long item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+        const int w = static_cast<int>(item / n_u), u = static_cast<int>(item - static_cast<long long>(w) * n_u);
+        const int t0 = 2 * w;
+        const bool two = t0 + 1 < g.n_o;
         for (int k = 0; k < g.kb; ++k, ++it) {
           const int s = static_cast<int>(it % kPfStages);
           if (it >= kPfStages && !mbar_wait(&empty[s], static_cast<uint32_t>((it / kPfStages) - 1) & 1u, abort, p.status)) {
@@ -226,13 +236,13 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_gemm_kernel(const __grid_con
             break;
           }
           uint8_t* st = base + s * kPfStage;
-          mbar_arrive_expect_tx(&full[s], kPfStage);
-          bulk_load(st, wl + (static_cast<size_t>(t) * g.kb + k) * kTileElems, kPfA, &full[s]);
-          tma_load_2d(st + kPfA, &tm_xh, &full[s], k * 64, u * 128);
-          tma_load_2d(st + kPfA + kPfB, &tm_xl, &full[s], k * 64, u * 128);
+          mbar_arrive_expect_tx(&full[s], (two ? 2 : 1) * kPfA + 2 * kPfB);
+          bulk_load(st, wl + (static_cast<size_t>(t0) * g.kb + k) * kTileElems, kPfA, &full[s]);
+          if (two) bulk_load(st + kPfA, wl + (static_cast<size_t>(t0 + 1) * g.kb + k) * kTileElems, kPfA, &full[s]);
+          tma_load_2d(st + 2 * kPfA, &tm_xh, &full[s], k * 64, u * 128);
+          tma_load_2d(st + 2 * kPfA + kPfB, &tm_xl, &full[s], k * 64, u * 128);
         }
       }
-      // the copies issued last have landed before the kernel returns
       for (long long v = it - 1; v >= 0 && v >= it - kPfStages; --v) {
         const uint64_t t0 = globaltimer_ns();
         while (!mbar_try_wait(&full[v % kPfStages], static_cast<uint32_t>(v / kPfStages) & 1u))
@@ -240,16 +250,19 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_gemm_kernel(const __grid_con
       }
     }
   } else if (warp == 1) {
+    // ---------------- MMA issuer: per k16 step, (A0, A1) x (hi, lo) into two accumulators ----------------
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_m128(128);
       long long it = 0;
-      int n = 0;  // tiles of this CTA
+      int n = 0;
       bool ok = true;
-      for (long long tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++n) {
+      for (long long item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++n) {
+        const int w = static_cast<int>(item / n_u);
+        const bool two = 2 * w + 1 < g.n_o;
         const int buf = n & 1;
         if (n >= 2 && !mbar_wait(&acc_empty[buf], static_cast<uint32_t>((n >> 1) - 1) & 1u, abort, p.status)) break;
         tc_fence_after();
-        const uint32_t d = tm + buf * kPfAccCols;
+        const uint32_t d0 = tm + buf * 2 * kPfAccCols, d1 = d0 + kPfAccCols;
         for (int k = 0; k < g.kb; ++k, ++it) {
           const int s = static_cast<int>(it % kPfStages);
           if (!mbar_wait(&full[s], static_cast<uint32_t>(it / kPfStages) & 1u, abort, p.status)) {
@@ -257,12 +270,18 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_gemm_kernel(const __grid_con
             break;
           }
           tc_fence_after();
-          const uint32_t a = smem_u32(base + s * kPfStage);
+          const uint32_t a = smem_u32(base + s * kPfStage), b = a + 2 * kPfA;
 #pragma unroll
           for (int k16 = 0; k16 < 4; ++k16) {
-            const uint64_t ad = sdesc_sw128(a + k16 * 32);
-            umma_bf16(d, ad, sdesc_sw128(a + kPfA + k16 * 32), idesc, (k | k16) ? 1u : 0u);
-            umma_bf16(d, ad, sdesc_sw128(a + kPfA + kPfB + k16 * 32), idesc, 1u);
+            const uint64_t bh = sdesc_sw128(b + k16 * 32), bl = sdesc_sw128(b + kPfB + k16 * 32);
+            const uint64_t a0 = sdesc_sw128(a + k16 * 32);
+            umma_bf16(d0, a0, bh, idesc, (k | k16) ? 1u : 0u);
+            umma_bf16(d0, a0, bl, idesc, 1u);
+            if (two) {
+              const uint64_t a1 = sdesc_sw128(a + kPfA + k16 * 32);
+              umma_bf16(d1, a1, bh, idesc, (k | k16) ? 1u : 0u);
+              umma_bf16(d1, a1, bl, idesc, 1u);
+            }
           }
           umma_commit(&empty[s]);
         }
@@ -275,21 +294,28 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_gemm_kernel(const __grid_con
         if (globaltimer_ns() - t0 > kWaitLimitNs) break;
     }
   } else {
-    // epilogue warps 2-5: TMEM lane quarter = warp & 3, thread r = weight row of the tile
-    const int q = warp & 3, r = q * 32 + lane, et = tid - 64;
+    // ---------------- epilogue warps: TMEM lane quarter = warp & 3, thread r = weight row; group
+    // (warp - 2) / 4 takes its share of the 8 token chunks of each accumulator ----------------
+    constexpr int kCh = 8 / kPgGroups;
+    const int q = warp & 3, r = q * 32 + lane, grp = (warp - 2) >> 2;
+    float* xch = xch0 + grp * 16 * 128;
+    const int bar = grp == 0 ? 1 : 2 + grp;  // (2 is the vote barrier)
     int n = 0;
-    for (long long tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++n) {
-      const int t = static_cast<int>(tile / n_u), u = static_cast<int>(tile - static_cast<long long>(t) * n_u);
+    for (long long item = blockIdx.x; item < n_items; item += gridDim.x, ++n) {
+      const int w = static_cast<int>(item / n_u), u = static_cast<int>(item - static_cast<long long>(w) * n_u);
       const int buf = n & 1;
       const bool ok = mbar_wait(&acc_full[buf], static_cast<uint32_t>(n >> 1) & 1u, abort, p.status);
       if (pf_epi_or(!ok)) break;
       tc_fence_after();
-      const uint32_t tb = tm + (static_cast<uint32_t>(q * 32) << 16) + buf * kPfAccCols;
-      for (int ch = 0; ch < 8; ++ch) {
-        float v[16];
-        tmem_ld16(tb + ch * 16, v);
-        const int j0 = u * 128 + ch * 16;
-        pf_epilogue<EPI>(p, g, xch, t, r, j0, v, et);
+      for (int a = 0; a < 2; ++a) {
+        const int t = 2 * w + a;
+        if (t >= g.n_o) break;
+        const uint32_t tb = tm + (static_cast<uint32_t>(q * 32) << 16) + (buf * 2 + a) * kPfAccCols;
+        for (int ch = kCh * grp; ch < kCh * grp + kCh; ++ch) {
+          float v[16];
+          tmem_ld16(tb + ch * 16, v);
+          pf_epilogue<EPI>(p, g, xch, t, r, u * 128 + ch * 16, v, bar);
+        }
       }
       tc_fence_before();
       __syncwarp();
@@ -301,7 +327,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_gemm_kernel(const __grid_con
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tm, 2 * kPfAccCols);
+    tmem_dealloc(tm, 4 * kPfAccCols);
   }
 }
 
@@ -630,8 +656,8 @@ cudaError_t launch_pf_norm(const PfParams& p, const float* g, cudaStream_t s) {
 
 cudaError_t launch_pf_gemm(int epi, const CUtensorMap& xh, const CUtensorMap& xl, const PfParams& p, const PfGemm& g,
                            int grid, cudaStream_t s) {
-  const long long tiles = static_cast<long long>(g.n_o) * ((p.T + 127) / 128);
-  const dim3 gr(static_cast<unsigned>(tiles < grid ? tiles : grid)), blk(kPfThreads);
+  const long long tiles = static_cast<long long>((g.n_o + 1) / 2) * ((p.T + 127) / 128);
+  const dim3 gr(static_cast<unsigned>(tiles < grid ? tiles : grid)), blk(kPgThreads);
   switch (epi) {
     case kPfEpiQkv: return launch_k(pf_gemm_kernel<kPfEpiQkv>, gr, blk, pf_gemm_smem(), s, false, xh, xl, p, g);
     case kPfEpiResid: return launch_k(pf_gemm_kernel<kPfEpiResid>, gr, blk, pf_gemm_smem(), s, false, xh, xl, p, g);
