@@ -278,10 +278,15 @@ tss_status tss_verify_grouped(tss_ctx* ctx, const tss_verify_batch* batch, const
 /* Prefill: append tokens to the requests' KV caches under their skip configurations (the
  * configuration is fixed for a whole request, prompt included: Sec. "Problem Formulation").
  * Request b's tokens [ctx_len[b], ctx_len[b] + n_tokens[b]) run through the layers its domain
- * does not skip, in chains of up to max_nodes tokens -- each chain one verification step on the
- * same kernels, whose acceptance outputs are discarded -- and their K/V rows are written to the
- * cache of every such layer; layers it skips are not touched.  Afterwards the caller's cache of
- * request b holds ctx_len[b] + n_tokens[b] tokens.
+ * does not skip, and their K/V rows are written to the cache of every such layer; layers it skips
+ * are not touched.  Afterwards the caller's cache of request b holds ctx_len[b] + n_tokens[b]
+ * tokens.  With head_dim 128 the requests of one skip set share passes of up to 4096 rows (each
+ * request's next chunk at a multiple of 128 rows), every layer's projections run as tokens-tiled
+ * tcgen05 GEMMs and its attention as a causal tcgen05 kernel (the environment variable
+ * TSS_PREFILL=steps at tss_create selects the other path); otherwise the prompt runs in chains of
+ * up to max_nodes tokens, each chain one verification step on the same kernels, whose acceptance
+ * outputs are discarded.  The first call on the tcgen05 path allocates its workspaces (about
+ * 0.45 GB at d_model 4096).
  *   n_tokens, ctx_len, domain_id, kv_slot: HOST arrays of n_req entries (n_tokens[b] >= 0;
  *     kv_slot NULL means slot b).
  *   tokens: the requests' tokens concatenated (sum(n_tokens) int32), DEVICE memory, or HOST

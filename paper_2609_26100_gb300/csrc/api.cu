@@ -145,6 +145,8 @@ struct tss_ctx {
   __nv_bfloat16 *pf_xh = nullptr, *pf_xl = nullptr, *pf_qh = nullptr, *pf_ql = nullptr, *pf_ah = nullptr,
                 *pf_al = nullptr, *pf_uh = nullptr, *pf_ul = nullptr;
   int* pf_tok = nullptr;
+  int *pf_pos = nullptr, *pf_slot = nullptr;
+  int4* pf_qt = nullptr;
   CUtensorMap pf_tm_xh, pf_tm_xl, pf_tm_qh, pf_tm_ql, pf_tm_ah, pf_tm_al, pf_tm_uh, pf_tm_ul;
   unsigned long long* trace = nullptr;  // persistent-kernel timeline when TSS_TRACE is set
   unsigned long long wait_ns = 2000000000ull;  // bound of the persistent kernel's waits (TSS_WAIT_LIMIT_MS)
@@ -1016,10 +1018,10 @@ tss_status prepare_step(const tss_ctx* c, const tss_verify_batch* bt, const tss_
   return TSS_OK;
 }
 
-// Workspaces of the compute-bound prefill, made at the first call: chunks of up to 1024 tokens.
+// Workspaces of the compute-bound prefill, made at the first call: passes of up to 4096 rows.
 tss_status pf_workspaces(tss_ctx* c) {
   if (c->pf_tmax) return TSS_OK;
-  const int T = 1024;
+  const int T = 4096;
   const size_t d = c->d, F = c->F_pad;
   TSS_TRY(c->alloc(&c->pf_h, T * d));
   TSS_TRY(c->alloc(&c->pf_xh, T * d));
@@ -1031,7 +1033,10 @@ tss_status pf_workspaces(tss_ctx* c) {
   TSS_TRY(c->alloc(&c->pf_uh, T * F));
   TSS_TRY(c->alloc(&c->pf_ul, T * F));
   TSS_TRY(c->alloc(&c->pf_tok, T));
-  // (rows past a chunk's tokens are read by the last tile of each GEMM and attention: finite)
+  TSS_TRY(c->alloc(&c->pf_pos, T));
+  TSS_TRY(c->alloc(&c->pf_slot, T));
+  TSS_TRY(c->alloc(&c->pf_qt, T / 128));
+  // (rows past a pass's rows are read by the last tile of each GEMM and attention: finite)
   TSS_CU(cudaMemset(c->pf_xh, 0, T * d * 2));
   TSS_CU(cudaMemset(c->pf_xl, 0, T * d * 2));
   TSS_CU(cudaMemset(c->pf_qh, 0, T * d * 2));
@@ -1053,20 +1058,20 @@ tss_status pf_workspaces(tss_ctx* c) {
   return TSS_OK;
 }
 
-// One request's chunk of T (<= pf_tmax) prompt tokens at positions pos0.. through every layer its
-// skip set keeps (Sec. "Domain-Aware Skip Controller": h_{l+1} = h_l for a skipped layer, which
-// writes no KV).  d_tokens: DEVICE, already in c->pf_tok.
-tss_status pf_chunk(tss_ctx* c, int slot, int pos0, int T, unsigned long long skip, const tss_kv_cache* kv,
-                    cudaStream_t s) {
+// One pass: T rows (the row tables and tokens already in place) through every layer the skip set
+// keeps (Sec. "Domain-Aware Skip Controller": h_{l+1} = h_l for a skipped layer, which writes no KV).
+tss_status pf_pass(tss_ctx* c, int T, int n_qtiles, unsigned long long skip, const tss_kv_cache* kv, cudaStream_t s) {
   PfParams p{};
   p.T = T;
-  p.pos0 = pos0;
-  p.slot = slot;
+  p.n_qtiles = n_qtiles;
   p.d_model = c->d;
   p.n_heads = c->H;
   p.head_dim = c->D;
   p.vocab = c->V;
   p.kv_cap = kv->cap;
+  p.row_pos = c->pf_pos;
+  p.row_slot = c->pf_slot;
+  p.qtiles = c->pf_qt;
   p.rms_eps = c->a.rms_eps;
   p.tokens = c->pf_tok;
   p.embed = c->embed;
@@ -1528,23 +1533,65 @@ tss_status tss_prefill(tss_ctx* c, int n_req, const int32_t* n_tokens, const int
     off[b + 1] = off[b] + n_tokens[b];
   }
   if (c->pf_enabled && c->D == 128) {
-    // compute-bound path: each request's tokens in chunks of up to pf_tmax, all at once per chunk
+    // compute-bound path: the requests of one skip set share passes of up to pf_tmax rows, each
+    // request's next chunk starting at a multiple of 128 rows
     for (int l = 0; l < c->L; ++l)
       if (kv->layer[l] && !aligned16(kv->layer[l])) return fail(TSS_ERR_INVALID_ARG, "KV buffers must be 16-byte aligned");
-    TSS_TRY(pf_workspaces(c));
+    std::vector<unsigned long long> skip(n_req);
     for (int b = 0; b < n_req; ++b) {
       const int dom = domain_id[b];
       const bool configured = dom >= 0 && dom < c->a.max_domains && c->phi_valid[dom];
-      const unsigned long long skip = configured ? c->phi[dom] : 0ull;
+      skip[b] = configured ? c->phi[dom] : 0ull;
       for (int l = 0; l < c->L; ++l)
-        if (!((skip >> l) & 1ull) && !kv->layer[l]) return fail(TSS_ERR_INVALID_ARG, "KV buffer of an active layer is NULL");
+        if (!((skip[b] >> l) & 1ull) && !kv->layer[l]) return fail(TSS_ERR_INVALID_ARG, "KV buffer of an active layer is NULL");
       const int slot = kv_slot ? kv_slot[b] : b;
       if (slot < 0 || slot >= kv->n_slots) return fail(TSS_ERR_INVALID_ARG, "kv_slot out of range");
-      for (int done = 0; done < n_tokens[b]; done += c->pf_tmax) {
-        const int T = std::min(c->pf_tmax, n_tokens[b] - done);
-        TSS_CU(cudaMemcpyAsync(c->pf_tok, tokens + off[b] + done, sizeof(int32_t) * T,
-                               io_host ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToDevice, s));
-        TSS_TRY(pf_chunk(c, slot, ctx_len[b] + done, T, skip, kv, s));
+    }
+    TSS_TRY(pf_workspaces(c));
+    std::vector<int> done(n_req, 0), pos, slt;
+    std::vector<int4> qt;
+    std::vector<char> grouped(n_req, 0);
+    for (int b0 = 0; b0 < n_req; ++b0) {
+      if (grouped[b0]) continue;
+      std::vector<int> grp;
+      for (int b = b0; b < n_req; ++b)
+        if (!grouped[b] && skip[b] == skip[b0]) {
+          grouped[b] = 1;
+          grp.push_back(b);
+        }
+      for (;;) {
+        int T = 0;
+        pos.assign(c->pf_tmax, -1);
+        slt.assign(c->pf_tmax, 0);
+        qt.clear();
+        bool any = false;
+        for (int b : grp) {
+          const int left = n_tokens[b] - done[b];
+          if (left <= 0) continue;
+          if (!any) TSS_CU(cudaMemsetAsync(c->pf_tok, 0, sizeof(int) * c->pf_tmax, s));
+          const int room = c->pf_tmax - T;
+          if (room < 128) break;
+          const int len = std::min(left, room);
+          const int slot = kv_slot ? kv_slot[b] : b;
+          const int p0 = ctx_len[b] + done[b];
+          TSS_CU(cudaMemcpyAsync(c->pf_tok + T, tokens + off[b] + done[b], sizeof(int32_t) * len,
+                                 io_host ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToDevice, s));
+          for (int i = 0; i < len; ++i) {
+            pos[T + i] = p0 + i;
+            slt[T + i] = slot;
+          }
+          for (int r = 0; r < len; r += 128) qt.push_back(make_int4(T + r, slot, p0 + r, std::min(128, len - r)));
+          done[b] += len;
+          T += (len + 127) / 128 * 128;
+          any = true;
+        }
+        if (!any) break;
+        // the attention's work items, the most keys first
+        std::stable_sort(qt.begin(), qt.end(), [](const int4& a, const int4& b2) { return a.z + a.w > b2.z + b2.w; });
+        TSS_CU(cudaMemcpyAsync(c->pf_pos, pos.data(), sizeof(int) * T, cudaMemcpyHostToDevice, s));
+        TSS_CU(cudaMemcpyAsync(c->pf_slot, slt.data(), sizeof(int) * T, cudaMemcpyHostToDevice, s));
+        TSS_CU(cudaMemcpyAsync(c->pf_qt, qt.data(), sizeof(int4) * qt.size(), cudaMemcpyHostToDevice, s));
+        TSS_TRY(pf_pass(c, T, static_cast<int>(qt.size()), skip[b0], kv, s));
       }
     }
     return TSS_OK;

@@ -95,11 +95,16 @@ struct AttnTcParams {
   int* status;
   int withhold;                  // fault injection: CTA 0 issues no MMA (its first wait runs out)
 };
-// Compute-bound prefill (prefill.cu): one request's chunk of T prompt tokens at positions
-// pos0 .. pos0 + T - 1 (head_dim 128).
+// Compute-bound prefill (prefill.cu; head_dim 128): one pass = T rows holding the prompt chunks
+// of requests with the same skip set, each chunk starting at a multiple of 128 rows (rows in the
+// gaps have position -1 and write nothing).
 constexpr int kPfEpiQkv = 0, kPfEpiResid = 1, kPfEpiSwiglu = 2;
 struct PfParams {
-  int T, pos0, slot, d_model, n_heads, head_dim, vocab, kv_cap;
+  int T, n_qtiles, d_model, n_heads, head_dim, vocab, kv_cap;
+  const int* row_pos;              // [T] position of each row's token, -1 for a gap row
+  const int* row_slot;             // [T] KV slot of each row's request
+  const int4* qtiles;              // [n_qtiles] (first row, slot, position of the first row, rows of the
+                                   // request in the tile), heaviest first: the attention's work items
   float rms_eps;
   const int* tokens;               // [T] device
   const __nv_bfloat16* embed;      // [vocab][d]

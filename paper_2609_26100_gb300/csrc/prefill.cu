@@ -1,8 +1,8 @@
 // Compute-bound prompt prefill under the skip mask (Sec. "Domain-Aware Skip Controller": the
 // mask is fixed for the whole request, prompt included; App. "Models": the LLaMA block).
 //
-// One request's chunk of T prompt tokens (positions pos0 .. pos0 + T - 1) runs through the
-// layers its skip set keeps, all T tokens at once: per layer RMSNorm, the fused QKV projection
+// The prompt chunks of requests with the same skip set (each at a multiple of 128 rows of one
+// pass) run through the layers the skip set keeps, all rows at once: per layer RMSNorm, the fused QKV projection
 // with RoPE whose K and V rows are appended to the cache, causal attention over the cache, the
 // O projection with the residual, RMSNorm, gate/up with SwiGLU and the down projection with the
 // residual.  Nothing past the last layer is computed (the prompt's logits are not needed).
@@ -129,9 +129,9 @@ __device__ __forceinline__ void pf_epilogue(const PfParams& p, const PfGemm& g, 
       const int pr = r ^ half, i = dim & (half - 1);
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) {
-        const int pos = p.pos0 + j0 + jj;
+        const int pos = j0 + jj < p.T ? p.row_pos[j0 + jj] : -1;
         out[jj] = 0.f;
-        if (j0 + jj < p.T) {
+        if (pos >= 0) {
           const float c = p.rope_cos[static_cast<size_t>(pos) * half + i];
           const float s = p.rope_sin[static_cast<size_t>(pos) * half + i];
           const float pv = xch[jj * 128 + pr];
@@ -147,11 +147,14 @@ __device__ __forceinline__ void pf_epilogue(const PfParams& p, const PfGemm& g, 
     for (int jj = 0; jj < 16; ++jj) {
       const int j = j0 + jj;
       if (j >= p.T) continue;
+      const int pos = p.row_pos[j];
+      if (pos < 0) continue;  // gap row
       if (sec == 0) {
         pf_split_store(p.qh, p.ql, static_cast<size_t>(j) * d + f, out[jj]);
       } else {
-        const size_t row = ((static_cast<size_t>(p.slot) * 2 + (sec - 1)) * p.n_heads + head) * static_cast<size_t>(p.kv_cap) +
-                           static_cast<size_t>(p.pos0 + j);
+        const size_t row =
+            ((static_cast<size_t>(p.row_slot[j]) * 2 + (sec - 1)) * p.n_heads + head) * static_cast<size_t>(p.kv_cap) +
+            static_cast<size_t>(pos);
         p.kv[row * D + dim] = __float2bfloat16_rn(out[jj]);
       }
     }
@@ -383,7 +386,9 @@ __device__ __forceinline__ bool pa_or(bool v) {
 
 }  // namespace
 
-// Grid (query tiles, heads); the KV map has 64-row boxes; tm_q: q hi / lo maps over [T_max][d].
+// Grid (heads, query tiles of p.qtiles, which the host orders heaviest first, so that the CTAs
+// with the most keys start first); the KV map has 64-row boxes; tm_q: q hi / lo maps over
+// [T_max][d].
 __global__ void __launch_bounds__(kPfThreads, 1) pf_attn_kernel(const __grid_constant__ CUtensorMap tm_qh,
                                                                 const __grid_constant__ CUtensorMap tm_ql,
                                                                 const __grid_constant__ CUtensorMap tm_kv,
@@ -399,10 +404,11 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_attn_kernel(const __grid_con
   __shared__ uint32_t tslot;
   __shared__ int abort_s;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int qt = blockIdx.x, h = blockIdx.y;
+  const int h = blockIdx.x;
+  const int4 qi = p.qtiles[blockIdx.y];  // (first row, slot, position of the first row, rows)
   const int H = p.n_heads, D = 128;
-  const int q0 = qt * 128;
-  const int key_end = p.pos0 + min(p.T, q0 + 128);  // keys any query of the tile may see
+  const int q0 = qi.x, slot = qi.y, pos_t0 = qi.z, nrow = qi.w;
+  const int key_end = pos_t0 + nrow;  // keys any query of the tile may see
   const int n = (key_end + kPaKeys - 1) / kPaKeys;
   if (tid == 0) {
     mbar_init(&qfull, 1);
@@ -433,7 +439,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_attn_kernel(const __grid_con
   const uint32_t tm = tslot;
   volatile int* abort = &abort_s;
   const size_t cap = static_cast<size_t>(p.kv_cap);
-  const int rowK = static_cast<int>(((static_cast<size_t>(p.slot) * 2) * H + h) * cap);
+  const int rowK = static_cast<int>(((static_cast<size_t>(slot) * 2) * H + h) * cap);
   const int rowV = rowK + static_cast<int>(static_cast<size_t>(H) * cap);
 
   if (warp == 0) {
@@ -518,9 +524,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_attn_kernel(const __grid_con
     // ---------------- softmax: thread = query row (TMEM lane) ----------------
     const int qg = warp & 3, qr = qg * 32 + lane, st = tid - 64;
     const uint32_t lanes = static_cast<uint32_t>(qg * 32) << 16;
-    const int j = q0 + qr;                  // token of this row
-    const bool valid = j < p.T;
-    const int pq = p.pos0 + j;              // its position: keys <= pq are visible
+    const int j = q0 + qr;                  // row of this query
+    const bool valid = qr < nrow;
+    const int pq = pos_t0 + qr;             // its position: keys <= pq are visible
     const float scale = 1.4426950408889634f / sqrtf(static_cast<float>(D));
     float m = -INFINITY, l = 0.f;
     bool ok = true;
@@ -668,7 +674,7 @@ cudaError_t launch_pf_gemm(int epi, const CUtensorMap& xh, const CUtensorMap& xl
 
 cudaError_t launch_pf_attn(const CUtensorMap& qh, const CUtensorMap& ql, const CUtensorMap& kv, const PfParams& p,
                            cudaStream_t s) {
-  const dim3 gr((p.T + 127) / 128, p.n_heads), blk(kPfThreads);
+  const dim3 gr(p.n_heads, p.n_qtiles), blk(kPfThreads);
   return launch_k(pf_attn_kernel, gr, blk, pf_attn_smem(), s, false, qh, ql, kv, p);
 }
 
