@@ -334,3 +334,44 @@ def test_7b_long_context_full_size():
         ref = refs[i][0]
         assert_logits(gl[q * n:(q + 1) * n], ref, f"7b long request {q}")
         check_greedy(ref, w.requests[q].tokens, w.requests[q].parents, res, q)
+
+
+def test_7b_prefill_full_size():
+    """The compute-bound prefill at 7B width (tokens-tiled tcgen05 GEMMs, causal tcgen05 attention):
+    a 130-token prompt appended to request 0's synthetic 1024-token context under the 7B chain's
+    skip set {20,24,27,30}; the K/V rows of every active layer against the oracle's (the same
+    prompt as a chain block over the same context), the skipped layers untouched, and a
+    verification step on top of the GPU-filled cache against the oracle."""
+    w = synth.workload_7b_chain()
+    from paper_2609_26100_gb300.runner import TssRunner
+    n_new = 130
+    run = TssRunner.for_workload(w, extra_cap=n_new + 8)
+    a_ = w.arch
+    r = w.requests[0]
+    wo = oracle_weights(w)
+    skip = skip_of(w, 0)
+    C0 = r.ctx_len
+    prompt = synth.uniform_ints(n_new, a_.vocab, w.seed, "full.prefill").tolist()
+    run.prefill([prompt], [C0], [0])
+    assert run.sync_status() == native.TSS_OK
+    torch.cuda.synchronize()
+    parents = [-1] + list(range(n_new - 1))
+    ref_logits, new_kv = O.verify_request(wo, a_, skip, prompt, parents, C0, LazyKV(a_, w.seed, 0, C0))
+    for l in range(a_.n_layers):
+        if l in skip:
+            assert run.kv[l] is None  # no request runs it: not even allocated
+            continue
+        gk = run.kv[l][0, 0, :, C0:C0 + n_new].float().cpu().numpy()
+        gv = run.kv[l][0, 1, :, C0:C0 + n_new].float().cpu().numpy()
+        k_ref, v_ref = np.transpose(new_kv[l][0], (1, 0, 2)), np.transpose(new_kv[l][1], (1, 0, 2))
+        np.testing.assert_allclose(gk, k_ref, atol=6e-2, rtol=3e-2, err_msg=f"K layer {l}")
+        np.testing.assert_allclose(gv, v_ref, atol=6e-2, rtol=3e-2, err_msg=f"V layer {l}")
+        assert float(np.abs(gk - k_ref).mean()) < 4e-3, f"K layer {l}"
+    # a verification step on the GPU-filled cache (context C0 + n_new)
+    kv = AppendedKV(a_, w.seed, 0, C0)
+    kv.append(new_kv, list(range(n_new)))
+    toks = synth.draft_tokens(r.parents, a_.vocab, w.seed, "full.after_prefill")
+    res = run_step(run, [synth.Request(C0 + n_new, r.parents, toks, 0)])
+    ref, _ = O.verify_request(wo, a_, skip, toks, r.parents, C0 + n_new, kv)
+    assert_logits(res["logits"].cpu().numpy(), ref, "7b verify after the tcgen05 prefill")
+    run.close()
