@@ -617,9 +617,21 @@ __global__ void __launch_bounds__(kPfThreads, 1) pf_attn_kernel(const __grid_con
           float o[16];
           tmem_ld16(tm + lanes + 128 + c * 16, o);
           if (valid) {
+            // this row's 16 outputs as bf16 hi and lo parts: two 16-byte stores per part
+            uint32_t hw[8], lw[8];
 #pragma unroll
-            for (int i = 0; i < 16; ++i)
-              pf_split_store(p.ah, p.al, static_cast<size_t>(j) * p.d_model + h * D + c * 16 + i, o[i] * inv);
+            for (int i = 0; i < 8; ++i) {
+              const float x0 = o[2 * i] * inv, x1 = o[2 * i + 1] * inv;
+              hw[i] = pack_bf16(x0, x1);
+              lw[i] = pack_bf16(x0 - __uint_as_float(hw[i] << 16), x1 - __uint_as_float(hw[i] & 0xffff0000u));
+            }
+            const size_t e = static_cast<size_t>(j) * p.d_model + h * D + c * 16;
+            uint4* ph = reinterpret_cast<uint4*>(p.ah + e);
+            uint4* pl = reinterpret_cast<uint4*>(p.al + e);
+            ph[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+            ph[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+            pl[0] = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+            pl[1] = make_uint4(lw[4], lw[5], lw[6], lw[7]);
           }
         }
         tc_fence_before();
