@@ -1532,7 +1532,7 @@ tss_status tss_prefill(tss_ctx* c, int n_req, const int32_t* n_tokens, const int
       return fail(TSS_ERR_KV_CAPACITY, "ctx_len + n_tokens exceeds KV capacity");
     off[b + 1] = off[b] + n_tokens[b];
   }
-  if (c->pf_enabled && c->D == 128) {
+  if (c->pf_enabled && c->D == 128 && c->d % 8 == 0 && c->d <= 256 * 8 * 4) {
     // compute-bound path: the requests of one skip set share passes of up to pf_tmax rows, each
     // request's next chunk starting at a multiple of 128 rows
     for (int l = 0; l < c->L; ++l)

@@ -61,13 +61,27 @@ __global__ void pf_embed_kernel(const PfParams p) {
   for (int c = threadIdx.x; c < p.d_model; c += blockDim.x) p.h[static_cast<size_t>(j) * p.d_model + c] = __bfloat162float(e[c]);
 }
 
-// x = h / sqrt(mean(h^2) + eps) * g, as bf16 hi + lo (one block per token row)
-__global__ void pf_norm_kernel(const PfParams p, const float* g) {
+// x = h / sqrt(mean(h^2) + eps) * g, as bf16 hi + lo (one block per token row): each thread holds
+// kPfNormV groups of 8 consecutive features in registers between the sum of squares and the scaling
+// (d_model <= 256 threads x 8 x kPfNormV).
+constexpr int kPfNormV = 4;
+__global__ void __launch_bounds__(256) pf_norm_kernel(const PfParams p, const float* g) {
   const int j = blockIdx.x;
   if (j >= p.T) return;
   const float* h = p.h + static_cast<size_t>(j) * p.d_model;
+  float x[kPfNormV][8];
   float ss = 0.f;
-  for (int c = threadIdx.x; c < p.d_model; c += blockDim.x) ss += h[c] * h[c];
+#pragma unroll
+  for (int v = 0; v < kPfNormV; ++v) {
+    const int c = (v * blockDim.x + threadIdx.x) * 8;
+    if (c < p.d_model) {
+      const float4 a = *reinterpret_cast<const float4*>(h + c), b = *reinterpret_cast<const float4*>(h + c + 4);
+      x[v][0] = a.x; x[v][1] = a.y; x[v][2] = a.z; x[v][3] = a.w;
+      x[v][4] = b.x; x[v][5] = b.y; x[v][6] = b.z; x[v][7] = b.w;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ss += x[v][i] * x[v][i];
+    }
+  }
   __shared__ float red[32];
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
@@ -79,8 +93,24 @@ __global__ void pf_norm_kernel(const PfParams p, const float* g) {
   }
   __syncthreads();
   const float inv = rsqrtf(red[0] / static_cast<float>(p.d_model) + p.rms_eps);
-  for (int c = threadIdx.x; c < p.d_model; c += blockDim.x)
-    pf_split_store(p.xh, p.xl, static_cast<size_t>(j) * p.x_ld + c, h[c] * inv * g[c]);
+#pragma unroll
+  for (int v = 0; v < kPfNormV; ++v) {
+    const int c = (v * blockDim.x + threadIdx.x) * 8;
+    if (c < p.d_model) {
+      const float4 ga = *reinterpret_cast<const float4*>(g + c), gb = *reinterpret_cast<const float4*>(g + c + 4);
+      const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
+      uint32_t hw[4], lw[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float y0 = x[v][2 * i] * inv * gg[2 * i], y1 = x[v][2 * i + 1] * inv * gg[2 * i + 1];
+        hw[i] = pack_bf16(y0, y1);
+        lw[i] = pack_bf16(y0 - __uint_as_float(hw[i] << 16), y1 - __uint_as_float(hw[i] & 0xffff0000u));
+      }
+      const size_t e = static_cast<size_t>(j) * p.x_ld + c;
+      *reinterpret_cast<uint4*>(p.xh + e) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+      *reinterpret_cast<uint4*>(p.xl + e) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------------------------
