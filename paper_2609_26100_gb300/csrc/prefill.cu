@@ -1,22 +1,24 @@
 // Compute-bound prompt prefill under the skip mask (Sec. "Domain-Aware Skip Controller": the
 // mask is fixed for the whole request, prompt included; App. "Models": the LLaMA block).
 //
-// The prompt chunks of requests with the same skip set (each at a multiple of 128 rows of one
-// pass) run through the layers the skip set keeps, all rows at once: per layer RMSNorm, the fused QKV projection
-// with RoPE whose K and V rows are appended to the cache, causal attention over the cache, the
-// O projection with the residual, RMSNorm, gate/up with SwiGLU and the down projection with the
-// residual.  Nothing past the last layer is computed (the prompt's logits are not needed).
+// The prompt chunks of requests with the same skip set (each starting at a multiple of 128 rows
+// of one pass of up to 4096 rows) run through the layers the skip set keeps, all rows at once: per
+// layer RMSNorm, the fused QKV projection with RoPE whose K and V rows are appended to the cache,
+// causal attention over the cache, the O projection with the residual, RMSNorm, gate/up with
+// SwiGLU and the down projection with the residual.  Nothing past the last layer is computed (the
+// prompt's logits are not needed).
 //
 // GEMMs (pf_gemm_kernel): out[t][o] = sum_k X[t][k] W[o][k] with the weights on the MMA's M side
 // (128-row tiles, the pre-tiled 128-byte-swizzled images the verification kernels stream) and
 // 128 tokens on the N side; a CTA takes two weight tiles against one token tile at a time (two
 // accumulators sharing the token operand) through its whole K loop (no split); items are taken
-// weight-row-major by a persistent grid so that the CTAs working at the same time share weight
-// tiles through L2.  X is held as two bf16 parts (hi = bf16(x), lo = bf16(x - hi)), both
-// multiplied by the weights into one fp32 accumulator in tensor memory, as on the verification
-// path.  Attention (pf_attn_kernel): one CTA per (128-query tile, head), queries on the MMA's M
-// side, 64-key tiles of the cache by TMA, S = Q K^T and O += P V in tensor memory, one thread
-// per query row for the online softmax; keys past a query's position are masked (causal).
+// weight-pair-major by a persistent grid so that the CTAs working at the same time share weight
+// tiles through L2; four groups of epilogue warps keep up with the MMAs.  X is held as two bf16
+// parts (hi = bf16(x), lo = bf16(x - hi)), both multiplied by the weights into one fp32
+// accumulator in tensor memory, as on the verification path.  Attention (pf_attn_kernel): one CTA
+// per (head, 128-query tile of one request), queries on the MMA's M side, 64-key tiles of the
+// cache by TMA, S = Q K^T and O += P V in tensor memory, one thread per query row for the online
+// softmax; keys past a query's position are masked (causal).
 #include "internal.h"
 
 namespace tss {
