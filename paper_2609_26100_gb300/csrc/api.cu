@@ -1530,6 +1530,8 @@ tss_status tss_prefill(tss_ctx* c, int n_req, const int32_t* n_tokens, const int
     if (n_tokens[b] < 0 || ctx_len[b] < 0) return fail(TSS_ERR_INVALID_ARG, "n_tokens and ctx_len must be >= 0");
     if (static_cast<long long>(ctx_len[b]) + n_tokens[b] > kv->cap)
       return fail(TSS_ERR_KV_CAPACITY, "ctx_len + n_tokens exceeds KV capacity");
+    if (static_cast<long long>(ctx_len[b]) + n_tokens[b] > c->a.max_positions)
+      return fail(TSS_ERR_INVALID_ARG, "position beyond max_positions");
     off[b + 1] = off[b] + n_tokens[b];
   }
   if (c->pf_enabled && c->D == 128 && c->d % 8 == 0 && c->d <= 256 * 8 * 4) {

@@ -115,3 +115,28 @@ def test_prefill_nan_tail_and_empty_prompt(weights):
         np.testing.assert_allclose(gv, ref[l][1], atol=5e-2, rtol=3e-2)
         assert bool(torch.isnan(run.kv[l][1]).all())  # slot 1: untouched
     run.close()
+
+
+def test_prefill_host_checks(weights):
+    """Host-detectable errors return before any launch: a prompt past the KV capacity, a slot out
+    of range, and positions past the context's max_positions (the RoPE tables' rows)."""
+    wo, wg = weights
+    run = make_runner(wg, n_slots=1, cap=256)
+    run.set_phi({0: 0})
+    with pytest.raises(native.TssError) as err:
+        run.prefill([list(range(100))], [200], [0])
+    assert err.value.status == native.TSS_ERR_KV_CAPACITY
+    with pytest.raises(native.TssError) as err:
+        run.prefill([list(range(10))], [0], [0], slots=[3])
+    assert err.value.status == native.TSS_ERR_INVALID_ARG
+    run.close()
+    v = native.Verifier(wg, ARCH, max_batch=8, max_rows=256, max_nodes=16, max_positions=64)
+    H, D = ARCH.n_heads, ARCH.head_dim
+    cache = [torch.zeros((1, 2, H, 256, D), dtype=torch.bfloat16, device="cuda") for _ in range(ARCH.n_layers)]
+    kv = v.make_kv([t.data_ptr() for t in cache], 1, 256)
+    toks = torch.zeros(100, dtype=torch.int32, device="cuda")
+    with pytest.raises(native.TssError) as err:
+        v.prefill([100], [0], [0], toks, kv)
+    assert err.value.status == native.TSS_ERR_INVALID_ARG
+    assert "max_positions" in str(err.value)
+    v.close()
