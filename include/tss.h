@@ -311,7 +311,9 @@ tss_status tss_sync_status(tss_ctx* ctx, void* stream);
  * withholds nothing.  n_steps = 0 cancels.  When the step's attention runs in the tcgen05 kernel
  * (tss_attention_kernel = 1), the first CTA of the step's first attention launch issues no MMA
  * instead, so that kernel's waits run out (after its fixed 2 s bound) and it takes the same
- * abort path; the next step's prologue resets its counters. */
+ * abort path; the next step's prologue resets its counters.  A tss_prefill call on the tcgen05
+ * path also counts as a step: the first CTA of its first GEMM launch issues no MMA (2 s bound);
+ * that call's cache rows are undefined. */
 tss_status tss_inject_timeout(tss_ctx* ctx, int n_steps);
 
 /* Diagnostic: the Philox4x32-10 stream that speculative sampling draws from when the batch gives

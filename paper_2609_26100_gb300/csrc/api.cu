@@ -1060,7 +1060,8 @@ tss_status pf_workspaces(tss_ctx* c) {
 
 // One pass: T rows (the row tables and tokens already in place) through every layer the skip set
 // keeps (Sec. "Domain-Aware Skip Controller": h_{l+1} = h_l for a skipped layer, which writes no KV).
-tss_status pf_pass(tss_ctx* c, int T, int n_qtiles, unsigned long long skip, const tss_kv_cache* kv, cudaStream_t s) {
+tss_status pf_pass(tss_ctx* c, int T, int n_qtiles, unsigned long long skip, const tss_kv_cache* kv, cudaStream_t s,
+                   bool inject) {
   PfParams p{};
   p.T = T;
   p.n_qtiles = n_qtiles;
@@ -1100,14 +1101,16 @@ tss_status pf_pass(tss_ctx* c, int T, int n_qtiles, unsigned long long skip, con
     if (!make_tmap(&tkv, kv->layer[l], 128, rows, 1, 64, 2)) return fail(TSS_ERR_CUDA, "cuTensorMapEncodeTiled failed (prefill KV)");
     p.kv = static_cast<__nv_bfloat16*>(kv->layer[l]);
     TSS_CU(launch_pf_norm(p, c->g_attn + static_cast<size_t>(l) * d, s));
-    TSS_CU(launch_pf_gemm(kPfEpiQkv, c->pf_tm_xh, c->pf_tm_xl, p, PfGemm{c->wqkv, static_cast<long long>(3 * dd), l, 3 * d / 128, kbd}, G, s));
+    TSS_CU(launch_pf_gemm(kPfEpiQkv, c->pf_tm_xh, c->pf_tm_xl, p,
+                          PfGemm{c->wqkv, static_cast<long long>(3 * dd), l, 3 * d / 128, kbd, inject ? 1 : 0}, G, s));
+    inject = false;
     TSS_CU(launch_pf_attn(c->pf_tm_qh, c->pf_tm_ql, tkv, p, s));
-    TSS_CU(launch_pf_gemm(kPfEpiResid, c->pf_tm_ah, c->pf_tm_al, p, PfGemm{c->wo, static_cast<long long>(dd), l, d / 128, kbd}, G, s));
+    TSS_CU(launch_pf_gemm(kPfEpiResid, c->pf_tm_ah, c->pf_tm_al, p, PfGemm{c->wo, static_cast<long long>(dd), l, d / 128, kbd, 0}, G, s));
     TSS_CU(launch_pf_norm(p, c->g_mlp + static_cast<size_t>(l) * d, s));
     TSS_CU(launch_pf_gemm(kPfEpiSwiglu, c->pf_tm_xh, c->pf_tm_xl, p,
-                          PfGemm{c->wgu, static_cast<long long>(c->Ft) * 128 * d, l, c->Ft, kbd}, G, s));
+                          PfGemm{c->wgu, static_cast<long long>(c->Ft) * 128 * d, l, c->Ft, kbd, 0}, G, s));
     TSS_CU(launch_pf_gemm(kPfEpiResid, c->pf_tm_uh, c->pf_tm_ul, p,
-                          PfGemm{c->wdown, static_cast<long long>(d) * c->F_pad, l, d / 128, c->F_pad / 64}, G, s));
+                          PfGemm{c->wdown, static_cast<long long>(d) * c->F_pad, l, d / 128, c->F_pad / 64, 0}, G, s));
   }
   return TSS_OK;
 }
@@ -1550,6 +1553,8 @@ tss_status tss_prefill(tss_ctx* c, int n_req, const int32_t* n_tokens, const int
       if (slot < 0 || slot >= kv->n_slots) return fail(TSS_ERR_INVALID_ARG, "kv_slot out of range");
     }
     TSS_TRY(pf_workspaces(c));
+    bool inject = c->inject_timeouts > 0;  // (tss_inject_timeout: the call's first GEMM)
+    if (inject) --c->inject_timeouts;
     std::vector<int> done(n_req, 0), pos, slt;
     std::vector<int4> qt;
     std::vector<char> grouped(n_req, 0);
@@ -1593,7 +1598,8 @@ tss_status tss_prefill(tss_ctx* c, int n_req, const int32_t* n_tokens, const int
         TSS_CU(cudaMemcpyAsync(c->pf_pos, pos.data(), sizeof(int) * T, cudaMemcpyHostToDevice, s));
         TSS_CU(cudaMemcpyAsync(c->pf_slot, slt.data(), sizeof(int) * T, cudaMemcpyHostToDevice, s));
         TSS_CU(cudaMemcpyAsync(c->pf_qt, qt.data(), sizeof(int4) * qt.size(), cudaMemcpyHostToDevice, s));
-        TSS_TRY(pf_pass(c, T, static_cast<int>(qt.size()), skip[b0], kv, s));
+        TSS_TRY(pf_pass(c, T, static_cast<int>(qt.size()), skip[b0], kv, s, inject));
+        inject = false;
       }
     }
     return TSS_OK;

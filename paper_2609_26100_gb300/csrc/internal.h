@@ -124,6 +124,7 @@ struct PfGemm {
   const __nv_bfloat16* w;          // pre-tiled weights (16 KiB blocks [layer][row tile][k-block])
   long long w_layer_elems;
   int layer, n_o, kb;              // layer, 128-row weight tiles, 64-column k-blocks
+  int withhold;                    // fault injection: CTA 0 issues no MMA (its waits run out)
 };
 cudaError_t pf_prepare();
 cudaError_t launch_pf_embed(const PfParams& p, cudaStream_t s);

@@ -291,7 +291,9 @@ __global__ void __launch_bounds__(kPgThreads, 1) pf_gemm_kernel(const __grid_con
       long long it = 0;
       int n = 0;
       bool ok = true;
-      for (long long item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++n) {
+      // fault injection: CTA 0 issues no MMA, so its epilogue's first wait runs out
+      const long long n_issue = g.withhold && blockIdx.x == 0 ? 0 : n_items;
+      for (long long item = blockIdx.x; item < n_issue && ok; item += gridDim.x, ++n) {
         const int w = static_cast<int>(item / n_u);
         const bool two = 2 * w + 1 < g.n_o;
         const int buf = n & 1;

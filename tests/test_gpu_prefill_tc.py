@@ -140,3 +140,25 @@ def test_prefill_host_checks(weights):
     assert err.value.status == native.TSS_ERR_INVALID_ARG
     assert "max_positions" in str(err.value)
     v.close()
+
+
+def test_prefill_bounded_wait_times_out_and_recovers(weights):
+    """Failure injection without a GPU fault, in the prefill GEMM: tss_inject_timeout makes CTA 0
+    of the call's first GEMM issue no MMA; the call ends with TSS_ERR_TIMEOUT from the bounded
+    waits (2 s), and the next prefill on the same context matches the oracle."""
+    wo, wg = weights
+    run = make_runner(wg, n_slots=1, cap=512)
+    run.set_phi({0: 0})
+    full = synth.uniform_ints(200, ARCH.vocab, SEED, "pft.to").tolist()
+    run.v.inject_timeout(1)
+    run.prefill([full], [0], [0])
+    assert run.sync_status() == native.TSS_ERR_TIMEOUT
+    assert run.sync_status() == native.TSS_OK  # reported once, then cleared
+    run.prefill([full], [0], [0])
+    assert run.sync_status() == native.TSS_OK
+    torch.cuda.synchronize()
+    ref = O.prefill(wo, ARCH, frozenset(), full)
+    for l in range(ARCH.n_layers):
+        np.testing.assert_allclose(run.kv[l][0, 0, :, :200].float().cpu().numpy(), ref[l][0], atol=5e-2, rtol=3e-2)
+        np.testing.assert_allclose(run.kv[l][0, 1, :, :200].float().cpu().numpy(), ref[l][1], atol=5e-2, rtol=3e-2)
+    run.close()
