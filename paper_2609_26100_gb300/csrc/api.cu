@@ -684,7 +684,7 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
       if (tc) {
         tp.slot = j;
         tp.withhold = j == 0 ? inject_attn : 0;
-        TSS_MK(2, TSS_CU(launch_attention_tc(tp, c->num_sms, s, false)));
+        TSS_MK(2, TSS_CU(launch_attention_tc(tp, c->num_sms, s, prof == nullptr)));
       } else {
         ap.slot = j;
         TSS_MK(2, TSS_CU(launch_attention(ap, sp.B, s, false)));
