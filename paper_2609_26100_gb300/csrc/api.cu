@@ -695,7 +695,7 @@ tss_status enqueue_step_mk(tss_ctx* c, const StepPlan& sp, cudaStream_t s, Prof*
     p.ph_end = 1 << 30;
     TSS_MK(8, TSS_CU(launch_verify_mk(p, c->num_sms, smem, s)));
   }
-  TSS_MK(7, TSS_CU(launch_finish(mp, sp.B, s, false)));
+  TSS_MK(7, TSS_CU(launch_finish(mp, sp.B, sp.mode == TSS_MODE_SAMPLE, s, false)));
 #undef TSS_MK
   return TSS_OK;
 }

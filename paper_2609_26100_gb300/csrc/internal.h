@@ -161,7 +161,14 @@ struct MiscParams {
 
 cudaError_t misc_prepare();
 cudaError_t launch_prologue(const MiscParams& p, float* ssp, int* zero_ints, int n_zero, int M, cudaStream_t s, bool pdl);
-cudaError_t launch_finish(const MiscParams& p, int B, cudaStream_t s, bool pdl);
+cudaError_t launch_finish(const MiscParams& p, int B, bool sample, cudaStream_t s, bool pdl);
+// Dynamic shared memory of the sampling acceptance's staged inverse CDF: the vocabulary's weights
+// with one skew word per 32 (0 when that exceeds kCdfStageMaxBytes: the unstaged pass runs).
+constexpr size_t kCdfStageMaxBytes = 200 * 1024;
+__host__ __device__ inline size_t cdf_stage_bytes(int vocab) {
+  const size_t n = (static_cast<size_t>(vocab) + vocab / 32 + 1) * sizeof(float);
+  return n <= kCdfStageMaxBytes ? n : 0;
+}
 cudaError_t launch_controller(const MiscParams& p, cudaStream_t s, bool pdl);
 cudaError_t launch_embed(const MiscParams& p, int M, cudaStream_t s, bool pdl);
 // which: 0 = attention norm of the slot's layer, 1 = MLP norm, 2 = final norm (slot ignored)

@@ -121,21 +121,36 @@ __global__ void rmsnorm_kernel(const MiscParams p, int slot, int which) {
 // lowest-index child whose token equals the argmax of the current row while one exists; the
 // bonus is the argmax of the last row reached.  Argmax ties go to the lowest token id.
 // ------------------------------------------------------------------------------------------
+// Request b's results, written by every thread of the block (a, bonus and path[0..a] are the
+// same in all of them; path is in shared memory).  The descriptor's fields are read once into
+// registers: read inside a loop of stores through the descriptor's pointers, each would be
+// reloaded from L2 after every store.
 __device__ void write_result(const MiscParams& p, int b, int a, int bonus, const int* path) {
   const StepDesc* st = p.step;
-  st->accept_len[b] = a;
-  st->bonus[b] = bonus;
-  st->new_ctx[b] = st->req_ctx[b] + 1 + a;
-  for (int i = 0; i < st->path_stride; ++i) st->path[static_cast<size_t>(b) * st->path_stride + i] = i <= a ? path[i] : -1;
-  p.plan->res_accept[b] = a;
-  for (int i = 0; i <= a; ++i) p.plan->res_path[b][i] = path[i];
+  PlanDev* pl = p.plan;
+  const int stride = st->path_stride;
+  int* out = st->path + static_cast<size_t>(b) * stride;
+  for (int i = threadIdx.x; i < stride; i += blockDim.x) out[i] = i <= a ? path[i] : -1;
+  for (int i = threadIdx.x; i <= a; i += blockDim.x) pl->res_path[b][i] = path[i];
+  if (threadIdx.x == 0) {
+    const int ctx = st->req_ctx[b];
+    int* accept_len = st->accept_len;
+    int* bonus_out = st->bonus;
+    int* new_ctx = st->new_ctx;
+    accept_len[b] = a;
+    bonus_out[b] = bonus;
+    new_ctx[b] = ctx + 1 + a;
+    pl->res_accept[b] = a;
+  }
 }
 
-__device__ void accept_greedy_body(const MiscParams& p, int b) {
+// Greedy acceptance of request b; returns the accept length (the same in every thread) and
+// leaves the accepted path in path[0..a].
+__device__ int accept_greedy_body(const MiscParams& p, int b, int* path) {
   const StepDesc* st = p.step;
   __shared__ int am[kMaxNodes];
-  __shared__ int path[kMaxNodes];
   __shared__ int s_par[kMaxNodes], s_tok[kMaxNodes];
+  __shared__ int s_a, s_bonus;
   const int N = st->req_nodes[b], off = st->req_rowoff[b];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
   for (int i = threadIdx.x; i < N; i += blockDim.x) {
@@ -198,15 +213,21 @@ __device__ void accept_greedy_body(const MiscParams& p, int b) {
       cur = nxt;
       path[++a] = cur;
     }
-    write_result(p, b, a, am[cur], path);
+    s_a = a;
+    s_bonus = am[cur];
   }
+  __syncthreads();
+  const int a = s_a;
+  write_result(p, b, a, s_bonus, path);
+  return a;
 }
 
 __global__ void accept_greedy_kernel(const MiscParams p) {
   griddep_wait();
   griddep_launch();
   if (blockIdx.x >= p.step->B) return;
-  accept_greedy_body(p, blockIdx.x);
+  __shared__ int path[kMaxNodes];
+  accept_greedy_body(p, blockIdx.x, path);
 }
 
 // Philox4x32-10 (Salmon et al., SC'11): 10 rounds of the 4x32 Philox round with key bumps.
@@ -361,21 +382,41 @@ __device__ int inverse_cdf_block(int V, float u, WFn w, float* scan) {
   return r;
 }
 
+// The same inverse CDF over weights staged in shared memory, when the launch gave the block
+// enough dynamic shared memory (cdf_stage_bytes): w(v) is computed once per token with coalesced
+// loads into a buffer indexed v + v / 32 (the skew puts the 32 consecutive tokens of each
+// thread's chunk in 32 different banks), then the chunk sums, scan and walk above read it there.
+// Without it each warp-wide load of the chunk pass touches 32 cache lines.
+__device__ __forceinline__ unsigned dyn_smem_bytes() {
+  unsigned n;
+  asm volatile("mov.u32 %0, %%dynamic_smem_size;" : "=r"(n));
+  return n;
+}
+
+template <typename WFn>
+__device__ int inverse_cdf_staged(int V, float u, WFn w, float* scan) {
+  extern __shared__ float cdf_stage[];
+  const size_t need = cdf_stage_bytes(V);
+  if (need == 0 || dyn_smem_bytes() < need) return inverse_cdf_block(V, u, w, scan);
+  for (int v = threadIdx.x; v < V; v += blockDim.x) cdf_stage[v + (v >> 5)] = w(v);
+  __syncthreads();
+  return inverse_cdf_block(V, u, [&](int v) { return cdf_stage[v + (v >> 5)]; }, scan);
+}
+
 // Speculative sampling on a chain draft (rule of the speculative-decoding works the paper cites
 // as its base methods): p_i = softmax(logits_i / T); accept draft x_i iff r_i * q_i(x_i) <
 // p_{i-1}(x_i); at the first rejection draw the bonus from normalise(max(0, p_{i-1} - q_i));
 // if every draft is accepted draw it from p_k.  Uniform slots: r_i at i-1, u_i at k+i-1.
-__device__ void accept_sample_body(const MiscParams& p, int b) {
+__device__ int accept_sample_body(const MiscParams& p, int b, int* path) {
   const StepDesc* st = p.step;
   __shared__ float scan[1025];
   __shared__ float redf[32];
-  __shared__ int path[kMaxNodes];
   const int N = st->req_nodes[b], off = st->req_rowoff[b], k = N - 1, V = p.vocab;
   const float invT = st->inv_temperature;
   auto fmx = [](float a, float c) { return a > c ? a : c; };
   auto fsum = [](float a, float c) { return a + c; };
   int a = 0, bonus = 0;
-  for (int i = 0; i < N; ++i) path[i] = i;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) path[i] = i;  // (read after the first barrier)
   for (int i = 1; i <= k + 1; ++i) {
     const float* lg = st->logits + static_cast<size_t>(off + i - 1) * V;
     const int nt = blockDim.x;
@@ -414,7 +455,7 @@ __device__ void accept_sample_body(const MiscParams& p, int b) {
       const float r = static_cast<float>(draw_uniform(st, b, i - 1));
       if (r * qx < pr(x)) continue;  // accept draft i
       const float u = static_cast<float>(draw_uniform(st, b, k + i - 1));
-      bonus = inverse_cdf_block(V, u, [&](int v) {
+      bonus = inverse_cdf_staged(V, u, [&](int v) {
         const float d = pr(v) - q[v];
         return d > 0.f ? d : 0.f;
       }, scan);
@@ -422,17 +463,20 @@ __device__ void accept_sample_body(const MiscParams& p, int b) {
       break;
     }
     const float u = static_cast<float>(draw_uniform(st, b, 2 * k));
-    bonus = inverse_cdf_block(V, u, pr, scan);
+    bonus = inverse_cdf_staged(V, u, pr, scan);
     a = k;
   }
-  if (threadIdx.x == 0) write_result(p, b, a, bonus, path);
+  __syncthreads();
+  write_result(p, b, a, bonus, path);
+  return a;
 }
 
 __global__ void __launch_bounds__(1024) accept_sample_kernel(const MiscParams p) {
   griddep_wait();
   griddep_launch();
   if (blockIdx.x >= p.step->B) return;
-  accept_sample_body(p, blockIdx.x);
+  __shared__ int path[kMaxNodes];
+  accept_sample_body(p, blockIdx.x, path);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -539,13 +583,8 @@ __global__ void __launch_bounds__(1024) finish_kernel(const MiscParams p) {
   const PlanDev* pl = p.plan;
   const int b = blockIdx.x;
   if (b >= st->B) return;
-  if (st->mode == TSS_MODE_SAMPLE) {
-    accept_sample_body(p, b);
-  } else {
-    accept_greedy_body(p, b);
-  }
-  __syncthreads();
-  const int a = pl->res_accept[b];
+  __shared__ int path[kMaxNodes];
+  const int a = st->mode == TSS_MODE_SAMPLE ? accept_sample_body(p, b, path) : accept_greedy_body(p, b, path);
   if (a <= 0) return;
   const int D = p.head_dim, H = p.n_heads;
   const size_t cap = static_cast<size_t>(st->kv_cap);
@@ -556,7 +595,7 @@ __global__ void __launch_bounds__(1024) finish_kernel(const MiscParams p) {
     // Element e = (kind, head, dim) stays with one thread across the path steps, and a later
     // step never reads a row an earlier step wrote, so the in-order copy needs no barrier.
     for (int jj = 1; jj <= a; ++jj) {
-      const int src = pl->res_path[b][jj];
+      const int src = path[jj];
       if (src == jj) continue;
       for (int e = threadIdx.x; e < 2 * H * D; e += blockDim.x) {
         const int kind_head = e / D, dd = e - kind_head * D;
@@ -611,6 +650,10 @@ cudaError_t misc_prepare() {
       (e = cudaFuncSetAttribute(accept_sample_kernel, a, c)) || (e = cudaFuncSetAttribute(compact_kernel, a, c)) ||
       (e = cudaFuncSetAttribute(prologue_kernel, a, c)) || (e = cudaFuncSetAttribute(finish_kernel, a, c)))
     return e;
+  const int dyn = static_cast<int>(kCdfStageMaxBytes);
+  const cudaFuncAttribute mx = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  if ((e = cudaFuncSetAttribute(finish_kernel, mx, dyn)) || (e = cudaFuncSetAttribute(accept_sample_kernel, mx, dyn)))
+    return e;
   return cudaSuccess;
 }
 
@@ -618,8 +661,8 @@ cudaError_t launch_prologue(const MiscParams& p, float* ssp, int* zero_ints, int
                             bool pdl) {
   return launch_k(prologue_kernel, dim3(M + 1), dim3(256), 0, s, pdl, p, ssp, zero_ints, n_zero);
 }
-cudaError_t launch_finish(const MiscParams& p, int B, cudaStream_t s, bool pdl) {
-  return launch_k(finish_kernel, dim3(B), dim3(1024), 0, s, pdl, p);
+cudaError_t launch_finish(const MiscParams& p, int B, bool sample, cudaStream_t s, bool pdl) {
+  return launch_k(finish_kernel, dim3(B), dim3(1024), sample ? cdf_stage_bytes(p.vocab) : 0, s, pdl, p);
 }
 
 cudaError_t launch_controller(const MiscParams& p, cudaStream_t s, bool pdl) {
@@ -635,7 +678,7 @@ cudaError_t launch_accept_greedy(const MiscParams& p, int B, cudaStream_t s, boo
   return launch_k(accept_greedy_kernel, dim3(B), dim3(256), 0, s, pdl, p);
 }
 cudaError_t launch_accept_sample(const MiscParams& p, int B, cudaStream_t s, bool pdl) {
-  return launch_k(accept_sample_kernel, dim3(B), dim3(1024), 0, s, pdl, p);
+  return launch_k(accept_sample_kernel, dim3(B), dim3(1024), cdf_stage_bytes(p.vocab), s, pdl, p);
 }
 cudaError_t launch_compact(const MiscParams& p, int B, int n_act, cudaStream_t s, bool pdl) {
   if (n_act <= 0) n_act = 1;
