@@ -152,49 +152,52 @@ __device__ int accept_greedy_body(const MiscParams& p, int b, int* path) {
   __shared__ int s_par[kMaxNodes], s_tok[kMaxNodes];
   __shared__ int s_a, s_bonus;
   const int N = st->req_nodes[b], off = st->req_rowoff[b];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
   for (int i = threadIdx.x; i < N; i += blockDim.x) {
     s_par[i] = st->row_parent[off + i];
     s_tok[i] = st->tokens[off + i];
   }
-  for (int i = warp; i < N; i += nw) {
-    float bv = -INFINITY;
-    int bi = 0x7fffffff;
-    constexpr int kPer = 16;  // tile partials per lane in one round of loads (vocab <= 65536)
-    float vv[kPer];
-    int vi[kPer];
+  // Argmax of every row over the vocabulary tiles' partials (laid out [tile][row]): thread
+  // (g, r), g < G = blockDim / RP, scans row r's tiles g, g + G, ..., so that a warp's loads
+  // cover consecutive rows of one tile; then the G results of each row are combined.  The
+  // maximum with ties to the lowest token id does not depend on the order of the comparisons.
+  auto better = [](float v, int ix, float& bv, int& bi) {
+    if (v > bv || (v == bv && ix < bi)) {
+      bv = v;
+      bi = ix;
+    }
+  };
+  const int RP = N > 32 ? (N + 31) & ~31 : 32, G = blockDim.x / RP;
+  const int r = threadIdx.x % RP, g = threadIdx.x / RP, n_vt = p.n_vtiles;
+  float bv = -INFINITY;
+  int bi = 0x7fffffff;
+  if (g < G && r < N) {
+    const float* pv = p.amax_val + off + r;
+    const int* pi = p.amax_idx + off + r;
+    constexpr int kPer = 8;  // tiles per thread in one round of loads
+    for (int t0 = g; t0 < n_vt; t0 += kPer * G) {
+      float vv[kPer];
+      int vi[kPer];
 #pragma unroll
-    for (int q = 0; q < kPer; ++q) {
-      const int t = lane + 32 * q;
-      const bool in = t < p.n_vtiles;
-      vv[q] = in ? p.amax_val[static_cast<size_t>(t) * kMaxRows + off + i] : -INFINITY;
-      vi[q] = in ? p.amax_idx[static_cast<size_t>(t) * kMaxRows + off + i] : 0x7fffffff;
-    }
+      for (int q = 0; q < kPer; ++q) {
+        const int t = t0 + q * G;
+        const bool in = t < n_vt;
+        vv[q] = in ? pv[static_cast<size_t>(t) * kMaxRows] : -INFINITY;
+        vi[q] = in ? pi[static_cast<size_t>(t) * kMaxRows] : 0x7fffffff;
+      }
 #pragma unroll
-    for (int q = 0; q < kPer; ++q) {
-      if (vv[q] > bv || (vv[q] == bv && vi[q] < bi)) {
-        bv = vv[q];
-        bi = vi[q];
-      }
+      for (int q = 0; q < kPer; ++q) better(vv[q], vi[q], bv, bi);
     }
-    for (int t = lane + 32 * kPer; t < p.n_vtiles; t += 32) {
-      const float v = p.amax_val[static_cast<size_t>(t) * kMaxRows + off + i];
-      const int ix = p.amax_idx[static_cast<size_t>(t) * kMaxRows + off + i];
-      if (v > bv || (v == bv && ix < bi)) {
-        bv = v;
-        bi = ix;
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-      if (ov > bv || (ov == bv && oi < bi)) {
-        bv = ov;
-        bi = oi;
-      }
-    }
-    if (lane == 0) am[i] = bi;
+  }
+  __shared__ float s_bv[1024];
+  __shared__ int s_bi[1024];
+  s_bv[threadIdx.x] = bv;
+  s_bi[threadIdx.x] = bi;
+  __syncthreads();
+  if (threadIdx.x < N) {
+    float v = -INFINITY;
+    int ix = 0x7fffffff;
+    for (int gg = 0; gg < G; ++gg) better(s_bv[gg * RP + threadIdx.x], s_bi[gg * RP + threadIdx.x], v, ix);
+    am[threadIdx.x] = ix;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -586,21 +589,35 @@ __global__ void __launch_bounds__(1024) finish_kernel(const MiscParams p) {
   __shared__ int path[kMaxNodes];
   const int a = st->mode == TSS_MODE_SAMPLE ? accept_sample_body(p, b, path) : accept_greedy_body(p, b, path);
   if (a <= 0) return;
+  // A chain's accepted rows are already in place (path[j] == j): nothing moves in any layer.
+  bool moved = false;
+  for (int jj = 1; jj <= a; ++jj) moved |= path[jj] != jj;
+  if (!moved) return;
   const int D = p.head_dim, H = p.n_heads;
   const size_t cap = static_cast<size_t>(st->kv_cap);
   const size_t ctx = static_cast<size_t>(st->req_ctx[b]);
-  for (int j = 0; j < pl->n_act; ++j) {
-    if (pl->slot_crow[j][b] < 0) continue;
-    __nv_bfloat16* base = st->kv_layer[pl->act_layer[j]] + static_cast<size_t>(st->req_slot[b]) * 2 * H * cap * D;
-    // Element e = (kind, head, dim) stays with one thread across the path steps, and a later
-    // step never reads a row an earlier step wrote, so the in-order copy needs no barrier.
+  const int n_act = pl->n_act;
+  // request b's cache region in every layer it ran, looked up by one thread per layer (null
+  // where it skipped the layer), so that the copies below wait on no descriptor loads
+  __shared__ __nv_bfloat16* s_base[kMaxLayers];
+  const size_t slot_off = static_cast<size_t>(st->req_slot[b]) * 2 * H * cap * D;
+  for (int j = threadIdx.x; j < n_act; j += blockDim.x)
+    s_base[j] = pl->slot_crow[j][b] < 0 ? nullptr : st->kv_layer[pl->act_layer[j]] + slot_off;
+  __syncthreads();
+  // 16-byte units (head_dim is 64 or 128): unit e = (kind, head, 8 dims) stays with one thread
+  // across the path steps, and a later step never reads a row an earlier step wrote, so the
+  // in-order copy needs no barrier.
+  const int vec = D / 8;
+  for (int j = 0; j < n_act; ++j) {
+    __nv_bfloat16* base = s_base[j];
+    if (!base) continue;
     for (int jj = 1; jj <= a; ++jj) {
       const int src = path[jj];
       if (src == jj) continue;
-      for (int e = threadIdx.x; e < 2 * H * D; e += blockDim.x) {
-        const int kind_head = e / D, dd = e - kind_head * D;
-        __nv_bfloat16* row = base + static_cast<size_t>(kind_head) * cap * D;
-        row[(ctx + jj) * D + dd] = row[(ctx + src) * D + dd];
+      for (int e = threadIdx.x; e < 2 * H * vec; e += blockDim.x) {
+        const int kind_head = e / vec, u = e - kind_head * vec;
+        uint4* row = reinterpret_cast<uint4*>(base + static_cast<size_t>(kind_head) * cap * D);
+        row[(ctx + jj) * vec + u] = row[(ctx + src) * vec + u];
       }
     }
   }
