@@ -401,7 +401,20 @@ __device__ int inverse_cdf_staged(int V, float u, WFn w, float* scan) {
   extern __shared__ float cdf_stage[];
   const size_t need = cdf_stage_bytes(V);
   if (need == 0 || dyn_smem_bytes() < need) return inverse_cdf_block(V, u, w, scan);
-  for (int v = threadIdx.x; v < V; v += blockDim.x) cdf_stage[v + (v >> 5)] = w(v);
+  // kStage weights per thread are computed before any is stored: the stores could alias the
+  // generic loads inside w, so a load after a store would wait for it
+  constexpr int kStage = 8;
+  const int nt = blockDim.x;
+  for (int v0 = threadIdx.x; v0 < V; v0 += kStage * nt) {
+    float x[kStage];
+#pragma unroll
+    for (int j = 0; j < kStage; ++j) x[j] = v0 + j * nt < V ? w(v0 + j * nt) : 0.f;
+#pragma unroll
+    for (int j = 0; j < kStage; ++j) {
+      const int v = v0 + j * nt;
+      if (v < V) cdf_stage[v + (v >> 5)] = x[j];
+    }
+  }
   __syncthreads();
   return inverse_cdf_block(V, u, [&](int v) { return cdf_stage[v + (v >> 5)]; }, scan);
 }
